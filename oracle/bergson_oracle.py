@@ -1,0 +1,247 @@
+"""Plain fp64 CPU oracle for Bergson's projected-gradient attribution path.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path imports this module:
+only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline /
+reference legs may call it.  It shares no code with the CUDA library.
+
+What it computes (Bergson, Sec. 3.1 and Fig. 1; App. "Gradients"):
+  1. the per-example gradient of an ``nn.Linear`` weight,
+     W_b = sum_t m_{b,t} g_{b,t} a_{b,t}^T   (d_out x d_in), explicitly;
+  2. optional Adafactor-style factored second-moment normalisation,
+     W~_b[i, j] = W_b[i, j] / sqrt(r_i c_j)   (r over d_out, c over d_in);
+  3. the double-sided per-module random projection
+     G^_b = P_out^T W~_b P_in                (k_out x k_in, row-major, k_out major);
+  4. concatenation over modules in call order and unit normalisation of the
+     whole per-example row (grad-cosine);
+  5. an fp16 gradient store, cosine scores against unit-normalised queries and
+     exact top-k, ordered by (score descending, index ascending).
+
+Readings taken where the paper is silent (each is listed in the design doc):
+  * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
+    stateless counter-based generator (SplitMix64 finaliser of Steele, Lea and
+    Flood 2014, then the Box-Muller transform of Box and Muller 1958), entry
+    e = i*k + j of the row-major [d, k] matrix, rounded once to fp32;
+  * second moments divide by sqrt(r c^T) with no 1/sum(r) and no epsilon;
+  * a masked token contributes nothing, whatever A and G hold there;
+  * a row whose norm is zero stays zero.
+
+Every function here is pinned by ``tests/test_oracle_pins.py`` against closed
+forms, finite differences, published generator outputs and brute force.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# SplitMix64 constants (Steele, Lea, Flood: "Fast splittable pseudorandom
+# number generators", OOPSLA 2014; finaliser variant "Mix13" by D. Stafford).
+_GOLDEN_GAMMA = np.uint64(0x9E3779B97F4A7C15)
+_M1 = np.uint64(0xBF58476D1CE4E5B9)
+_M2 = np.uint64(0x94D049BB133111EB)
+_TWO_M53 = 2.0 ** -53
+
+PROJ_GAUSSIAN = 0
+PROJ_IDENTITY = 1
+
+
+def mix64(x):
+    """SplitMix64 finaliser on a uint64 array (wrapping arithmetic)."""
+    x = np.asarray(x, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        z = (x ^ (x >> np.uint64(30))) * _M1
+        z = (z ^ (z >> np.uint64(27))) * _M2
+    return z ^ (z >> np.uint64(31))
+
+
+def splitmix64_sequence(seed: int, n: int) -> np.ndarray:
+    """The first ``n`` outputs of the SplitMix64 generator started at ``seed``."""
+    with np.errstate(over="ignore"):
+        states = np.uint64(seed) + _GOLDEN_GAMMA * np.arange(1, n + 1, dtype=np.uint64)
+    return mix64(states)
+
+
+def gaussian_counter(seed: int, n: int) -> np.ndarray:
+    """Standard normal draws z_0 .. z_{n-1} for counter e = 0 .. n-1 (fp64).
+
+    Pair p = e >> 1 takes two 64-bit hashes h1 = mix(seed ^ mix(2p)) and
+    h2 = mix(seed ^ mix(2p + 1)), turns them into u1 in (0, 1] and u2 in [0, 1)
+    with 53-bit resolution, and applies Box-Muller: even e takes the cosine
+    branch, odd e the sine branch.
+    """
+    e = np.arange(n, dtype=np.uint64)
+    p = e >> np.uint64(1)
+    s = np.uint64(seed)
+    h1 = mix64(s ^ mix64(np.uint64(2) * p))
+    h2 = mix64(s ^ mix64(np.uint64(2) * p + np.uint64(1)))
+    u1 = ((h1 >> np.uint64(11)) + np.uint64(1)).astype(np.float64) * _TWO_M53
+    u2 = (h2 >> np.uint64(11)).astype(np.float64) * _TWO_M53
+    rho = np.sqrt(-2.0 * np.log(u1))
+    theta = 2.0 * np.pi * u2
+    return np.where((e & np.uint64(1)) == 0, rho * np.cos(theta), rho * np.sin(theta))
+
+
+def projection_matrix(seed: int, d: int, k: int, kind: int = PROJ_GAUSSIAN) -> np.ndarray:
+    """Dense projection P in R^{d x k}, stored as fp32 values held in fp64.
+
+    Gaussian: P[i, j] = fl32(z(seed, i*k + j) / sqrt(k)), so E||P^T x||^2 = ||x||^2
+    (Johnson-Lindenstrauss scaling).  Identity (tests only): k == d and P = I.
+    """
+    if kind == PROJ_IDENTITY:
+        if k != d:
+            raise ValueError("identity projection needs k == d")
+        return np.eye(d, dtype=np.float64)
+    z = gaussian_counter(seed, d * k).reshape(d, k)
+    return (z / np.sqrt(k)).astype(np.float32).astype(np.float64)
+
+
+def module_seeds(base_seed: int, module_index: int) -> tuple[int, int]:
+    """Per-module seeds (s_in, s_out) derived from one base seed."""
+    b = np.uint64(base_seed)
+    m = np.uint64(module_index)
+    s_in = int(mix64(b ^ (np.uint64(2) * m)))
+    s_out = int(mix64(b ^ (np.uint64(2) * m + np.uint64(1))))
+    return s_in, s_out
+
+
+def per_example_gradient(a: np.ndarray, g: np.ndarray, m: np.ndarray | None) -> np.ndarray:
+    """W = sum over valid tokens t of g_t a_t^T, shape [d_out, d_in], fp64.
+
+    a: [T, d_in] layer inputs, g: [T, d_out] output gradients, m: [T] 0/1 mask
+    (None = every token valid).  Only valid tokens enter the sum.
+    """
+    a = np.asarray(a, dtype=np.float64)
+    g = np.asarray(g, dtype=np.float64)
+    if m is not None:
+        keep = np.asarray(m) != 0
+        a = a[keep]
+        g = g[keep]
+    return g.T @ a
+
+
+def adafactor_normalize(w: np.ndarray, r: np.ndarray | None, c: np.ndarray | None) -> np.ndarray:
+    """W~[i, j] = W[i, j] / sqrt(r_i c_j); identity when r and c are absent."""
+    if r is None and c is None:
+        return w
+    if r is None or c is None:
+        raise ValueError("r and c come together")
+    r = np.asarray(r, dtype=np.float64)
+    c = np.asarray(c, dtype=np.float64)
+    return w / np.sqrt(np.outer(r, c))
+
+
+def double_sided_projection(w: np.ndarray, p_out: np.ndarray, p_in: np.ndarray) -> np.ndarray:
+    """G^ = P_out^T W P_in, shape [k_out, k_in]."""
+    return p_out.T @ w @ p_in
+
+
+class Layer:
+    """One nn.Linear's captured tensors and projection settings (host arrays).
+
+    A: [B, T, d_in], G: [B, T, d_out] (any float dtype; bf16 values arrive as
+    exact fp32), r: [d_out] or None, c: [d_in] or None.
+    """
+
+    def __init__(self, A, G, k_in, k_out, seed_in, seed_out, r=None, c=None,
+                 col_offset=0, proj_kind=PROJ_GAUSSIAN):
+        self.A = np.asarray(A)
+        self.G = np.asarray(G)
+        self.k_in = int(k_in)
+        self.k_out = int(k_out)
+        self.seed_in = int(seed_in)
+        self.seed_out = int(seed_out)
+        self.r = None if r is None else np.asarray(r, dtype=np.float64)
+        self.c = None if c is None else np.asarray(c, dtype=np.float64)
+        self.col_offset = int(col_offset)
+        self.proj_kind = int(proj_kind)
+
+    @property
+    def d_in(self):
+        return self.A.shape[-1]
+
+    @property
+    def d_out(self):
+        return self.G.shape[-1]
+
+
+def project_module(layer: Layer, mask: np.ndarray | None, examples=None) -> np.ndarray:
+    """Projected per-example gradients of one module, [len(examples), k_out*k_in].
+
+    Steps 1-3 above for each example, flattened row-major (k_out major).
+    """
+    B = layer.A.shape[0]
+    examples = range(B) if examples is None else examples
+    p_in = projection_matrix(layer.seed_in, layer.d_in, layer.k_in, layer.proj_kind)
+    p_out = projection_matrix(layer.seed_out, layer.d_out, layer.k_out, layer.proj_kind)
+    rows = []
+    for b in examples:
+        m = None if mask is None else mask[b]
+        w = per_example_gradient(layer.A[b], layer.G[b], m)
+        w = adafactor_normalize(w, layer.r, layer.c)
+        rows.append(double_sided_projection(w, p_out, p_in).reshape(-1))
+    return np.stack(rows) if rows else np.zeros((0, layer.k_out * layer.k_in))
+
+
+def project_grads(layers, mask, ld_out: int | None = None, examples=None) -> np.ndarray:
+    """Unnormalised projected gradients of every module placed at its column offset.
+
+    Returns [len(examples), ld_out] fp64; columns no module covers are zero.
+    """
+    B = layers[0].A.shape[0]
+    examples = list(range(B)) if examples is None else list(examples)
+    if ld_out is None:
+        ld_out = max(l.col_offset + l.k_out * l.k_in for l in layers)
+    out = np.zeros((len(examples), ld_out), dtype=np.float64)
+    for layer in layers:
+        blk = layer.k_out * layer.k_in
+        out[:, layer.col_offset:layer.col_offset + blk] = project_module(layer, mask, examples)
+    return out
+
+
+def unit_normalize(x: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+    """Rows divided by their l2 norm; zero rows stay zero.  Returns (rows, norms)."""
+    x = np.asarray(x, dtype=np.float64)
+    norms = np.sqrt(np.sum(x * x, axis=1))
+    safe = np.where(norms > 0, norms, 1.0)
+    return x / safe[:, None], norms
+
+
+def build_store(proj: np.ndarray, unit: bool = True) -> tuple[np.ndarray, np.ndarray]:
+    """fp16 store rows (round to nearest even from fp64) and the row norms."""
+    rows, norms = unit_normalize(proj) if unit else (np.asarray(proj, np.float64), None)
+    if norms is None:
+        norms = np.sqrt(np.sum(rows * rows, axis=1))
+    return rows.astype(np.float16), norms
+
+
+def cosine_scores(store: np.ndarray, queries: np.ndarray, row_chunk: int = 1 << 18) -> np.ndarray:
+    """S[q, n] = (q / ||q||) . s_n in fp64 for every query and store row.
+
+    The store rows are used as stored (unit-norm up to fp16 rounding).  The
+    product is formed in slices of ``row_chunk`` rows only to bound host memory.
+    """
+    q, _ = unit_normalize(queries)
+    N = store.shape[0]
+    S = np.empty((q.shape[0], N), dtype=np.float64)
+    for n0 in range(0, N, row_chunk):
+        n1 = min(N, n0 + row_chunk)
+        S[:, n0:n1] = q @ np.asarray(store[n0:n1], dtype=np.float64).T
+    return S
+
+
+def topk_rows(S: np.ndarray, k: int) -> tuple[np.ndarray, np.ndarray]:
+    """Exact top-k of each row of S by full sort on key (-score, index)."""
+    Q, N = S.shape
+    if k > N:
+        raise ValueError("k > N")
+    idx = np.empty((Q, k), dtype=np.int64)
+    val = np.empty((Q, k), dtype=np.float64)
+    cols = np.arange(N)
+    for qi in range(Q):
+        order = np.lexsort((cols, -S[qi]))[:k]
+        idx[qi] = order
+        val[qi] = S[qi, order]
+    return val, idx
+
+
+def score_topk(store: np.ndarray, queries: np.ndarray, k: int):
+    """Cosine scores of queries against the store and their exact top-k."""
+    return topk_rows(cosine_scores(store, queries), k)
