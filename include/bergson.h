@@ -1,0 +1,220 @@
+/*
+ * bergson.h -- C ABI of the GB300 projected-gradient attribution library.
+ *
+ * The library implements the TrackStar-style gradient path of Bergson
+ * (Sec. 3.1 "Attribution Pipelines", Fig. 1, App. "Gradients"):
+ *   per-example gradients of every nn.Linear weight, optional Adafactor-style
+ *   factored second-moment normalisation, the double-sided per-module random
+ *   projection, unit normalisation into an fp16 gradient store, and exact
+ *   cosine top-k queries against that store.
+ *
+ * Conventions shared by every entry point
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *     never allocates.  Scratch memory comes in through `workspace`, sized by
+ *     the matching *_workspace query.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Every call only enqueues work on it; nothing synchronises.
+ *   - Arguments are validated on the host before anything is enqueued.  A
+ *     failing call returns a negative bergson_status, enqueues nothing and
+ *     leaves a message in bergson_last_error().  No call aborts the process.
+ *   - Device-side waits are bounded.  A wait that gives up records
+ *     BERGSON_EDEVICE_TIMEOUT in a device status word that
+ *     bergson_sync_status() reports.
+ *   - The device that executes the work is the one that owns `workspace` (or
+ *     the output buffer for calls without workspace).
+ */
+#ifndef BERGSON_H
+#define BERGSON_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(BERGSON_BUILD) && defined(__GNUC__)
+#define BERGSON_API __attribute__((visibility("default")))
+#else
+#define BERGSON_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  BERGSON_OK = 0,
+  BERGSON_EINVAL = -1,            /* bad size, null pointer or inconsistent arguments */
+  BERGSON_EALIGN = -2,            /* a pointer or leading dimension breaks an alignment rule */
+  BERGSON_EUNSUPPORTED = -3,      /* valid request outside what this build implements */
+  BERGSON_EWORKSPACE = -4,        /* workspace smaller than the *_workspace query */
+  BERGSON_ECUDA = -5,             /* a CUDA runtime/driver call failed */
+  BERGSON_EDEVICE_TIMEOUT = -6    /* a bounded device wait gave up (see bergson_sync_status) */
+} bergson_status;
+
+typedef enum {
+  BERGSON_PROJ_GAUSSIAN = 0,      /* seeded Gaussian, entries N(0, 1/k) */
+  BERGSON_PROJ_IDENTITY = 1       /* P = I, requires k == d (testing aid) */
+} bergson_proj_kind;
+
+/*
+ * One nn.Linear module's captured tensors (Bergson App. "Gradients": gradient
+ * collection from linear layers; Fig. 1: Adafactor normalisation and the
+ * double-sided per-module projection).
+ *
+ *   A      bf16 [B, T, d_in] layer inputs, contiguous, 16-byte aligned.
+ *   G      bf16 [B, T, d_out] gradients w.r.t. the layer output, contiguous,
+ *          16-byte aligned.
+ *   d_in, d_out   multiples of 8, >= 8.
+ *   k_in, k_out   projection sizes, each one of 16, 32, 64.
+ *   seed_in, seed_out   seeds of P_in [d_in, k_in] and P_out [d_out, k_out].
+ *          Entry (i, j) of P is z(seed, i*k + j) / sqrt(k), z the counter-based
+ *          SplitMix64 + Box-Muller normal draw, rounded to fp32.
+ *   proj_kind    bergson_proj_kind.
+ *   r, c   fp32 [d_out] and [d_in] factored second moments (> 0), or both
+ *          NULL for no normalisation.  The gradient is divided elementwise by
+ *          sqrt(r_i c_j).
+ *   out_col_offset   first column of this module's k_out*k_in block in `out`.
+ */
+typedef struct bergson_layer {
+  const void* A;
+  const void* G;
+  int64_t d_in;
+  int64_t d_out;
+  int64_t k_in;
+  int64_t k_out;
+  uint64_t seed_in;
+  uint64_t seed_out;
+  int32_t proj_kind;
+  int32_t reserved;               /* must be 0 */
+  const float* r;
+  const float* c;
+  int64_t out_col_offset;
+} bergson_layer;
+
+/* Bytes of workspace bergson_project_grads needs for these arguments. */
+BERGSON_API int bergson_project_grads_workspace(const bergson_layer* layers, int n_layers,
+                                    int64_t B, int64_t T, size_t* ws_bytes);
+
+/*
+ * Projected per-example gradients (Bergson Sec. 3.1 "processing ... down-
+ * projection"; Fig. 1 double-sided per-module random projection):
+ *
+ *   out[b, off + i*k_in + j] = ( P_out^T (W_b / sqrt(r c^T)) P_in )[i, j],
+ *   W_b = sum over valid tokens t of g_{b,t} a_{b,t}^T,
+ *
+ * computed without forming W_b, through the token-level projections
+ * (A diag(c^-1/2) P_in, G diag(r^-1/2) P_out) and a masked per-example
+ * contraction over tokens.  The result is NOT unit-normalised.
+ *
+ *   mask    u8 [B, T] (nonzero = valid token) or NULL (all valid).  A masked
+ *           token contributes nothing, whatever A and G hold there.
+ *   out     fp32 [B, ld_out]; only the layers' column blocks are written.
+ *           Blocks must lie inside [0, ld_out) and must not overlap.
+ *   B, T    >= 0.  T == 0 writes zero blocks.
+ *   workspace/ws_bytes   device scratch of at least the queried size,
+ *           256-byte aligned; contents on entry are ignored.
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                          const uint8_t* mask, float* out, int64_t ld_out,
+                          void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Gradient-store rows (Bergson Sec. 3.1 on-disk gradient store with unit
+ * normalisation; Fig. 1 "unit normalization"):
+ *
+ *   store[row_offset + b, 0:K] = fp16( proj[b, 0:K] / ||proj[b, 0:K]||_2 )
+ *
+ * (or fp16(proj) when unit_normalize == 0).  A zero row is stored as zeros.
+ *   proj      fp32 [B, ld_proj], 16-byte aligned, ld_proj % 4 == 0, ld_proj >= K.
+ *   K         > 0, K % 8 == 0.
+ *   store     fp16 [N_cap, ld_store], 16-byte aligned, ld_store % 8 == 0,
+ *             ld_store >= K.  Rows outside [row_offset, row_offset + B) are
+ *             untouched (stores are built by appending batches).
+ *   norms_out optional fp32 [B]: the l2 norms before normalisation.
+ * Errors: EINVAL, EALIGN, ECUDA.
+ */
+BERGSON_API int bergson_build_store(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
+                        int unit_normalize, void* store, int64_t ld_store,
+                        int64_t row_offset, int64_t N_cap, float* norms_out, void* stream);
+
+/* Bytes of workspace bergson_score_topk needs. */
+BERGSON_API int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes);
+
+/*
+ * Exact cosine top-k of queries against the store (Bergson Sec. 3.1: exact
+ * top-k nearest-neighbour lookup over the gradient store; grad-cosine):
+ *
+ *   S[q, n] = (query_q / ||query_q||) . store_n
+ *   out_scores[q, :], out_idx[q, :] = the topk largest S[q, n], ordered by
+ *   score descending, then index ascending.
+ *
+ * Store rows are taken as stored (unit norm when built by bergson_build_store).
+ * The N x Q score matrix is never materialised.
+ *   store     fp16 [N, ld_store], 16-byte aligned, ld_store % 8 == 0, ld_store >= K.
+ *   N         1 .. 2^31-1.   K > 0, K % 8 == 0.
+ *   queries   fp32 [Q, ld_q], ld_q >= K, 4-byte aligned; normalised inside
+ *             (a zero query scores 0 against every row).
+ *   Q         >= 0.   topk in 1 .. min(N, 1024).
+ *   out_scores fp32 [Q, topk]; out_idx int64 [Q, topk].
+ * NaN scores never enter the result; if fewer than topk scores are usable
+ * the tail holds score -inf and index -1.
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                       const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
+                       float* out_scores, int64_t* out_idx,
+                       void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * The projection actually used by bergson_project_grads (Fig. 1 random
+ * projection), materialised for inspection:
+ *   out[i, j] = scale_i * P[i, j]   (fp32 [d, k], row-major)
+ * with P as described for bergson_layer and scale_i = 1/sqrt(moment_i), or 1
+ * when `moment` is NULL.  k in 16, 32, 64; identity needs k == d.
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, ECUDA.
+ */
+BERGSON_API int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind,
+                              const float* moment, float* out, void* stream);
+
+/*
+ * Synchronises `stream`, then reports and clears the device status word:
+ * BERGSON_OK, BERGSON_EDEVICE_TIMEOUT (a bounded device wait gave up) or
+ * BERGSON_ECUDA (the stream carried a CUDA error).
+ */
+BERGSON_API int bergson_sync_status(void* stream);
+
+/* Message of the last failing call on this thread ("" if none). */
+BERGSON_API const char* bergson_last_error(void);
+
+/*
+ * Per-module projection seeds derived from one base seed, so that a model's
+ * modules get independent projections (reading of Fig. 1: every module has
+ * its own pair of random matrices):
+ *   seed_in = mix(base ^ 2m),  seed_out = mix(base ^ (2m + 1)),
+ * mix = the SplitMix64 finaliser, m = module index.  Pure host function.
+ */
+BERGSON_API void bergson_module_seeds(uint64_t base_seed, int64_t module_index, uint64_t* seed_in,
+                          uint64_t* seed_out);
+
+/* Library version, major*10000 + minor*100 + patch. */
+BERGSON_API int bergson_version(void);
+
+/*
+ * Test aid for the bounded-wait machinery: enqueues one kernel that waits on a
+ * barrier nothing will ever complete, for at most `timeout_ns`, then records
+ * BERGSON_EDEVICE_TIMEOUT in the device status word and returns.  The context
+ * stays usable.  timeout_ns in 1 .. 10^10.
+ */
+BERGSON_API int bergson_debug_wait_probe(uint64_t timeout_ns, void* stream);
+
+/*
+ * Test aid for host error paths: the next `count` calls of any entry point
+ * that would enqueue work return `status` (e.g. BERGSON_ECUDA) after argument
+ * validation, without enqueueing anything.  count = 0 clears it.
+ */
+BERGSON_API void bergson_debug_inject_status(int status, int count);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BERGSON_H */

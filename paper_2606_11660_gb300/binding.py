@@ -1,0 +1,223 @@
+"""Thin ctypes binding of the C ABI in include/bergson.h.
+
+Each ``bergson_*`` function here has the name of the C entry point it calls
+and only marshals arguments: torch tensors become device pointers and leading
+dimensions, ``stream=None`` becomes torch's current stream.  All computation
+happens in the CUDA library; if the library is missing, loading it raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Optional, Sequence
+
+_PKG_DIR = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG_DIR, "libbergson.so")
+
+BERGSON_OK = 0
+BERGSON_EINVAL = -1
+BERGSON_EALIGN = -2
+BERGSON_EUNSUPPORTED = -3
+BERGSON_EWORKSPACE = -4
+BERGSON_ECUDA = -5
+BERGSON_EDEVICE_TIMEOUT = -6
+
+BERGSON_PROJ_GAUSSIAN = 0
+BERGSON_PROJ_IDENTITY = 1
+
+STATUS_NAMES = {
+    0: "BERGSON_OK", -1: "BERGSON_EINVAL", -2: "BERGSON_EALIGN", -3: "BERGSON_EUNSUPPORTED",
+    -4: "BERGSON_EWORKSPACE", -5: "BERGSON_ECUDA", -6: "BERGSON_EDEVICE_TIMEOUT",
+}
+
+# Every symbol include/bergson.h declares.
+EXPORTED = (
+    "bergson_project_grads_workspace", "bergson_project_grads", "bergson_build_store",
+    "bergson_score_topk_workspace", "bergson_score_topk", "bergson_projection_matrix",
+    "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
+    "bergson_debug_wait_probe", "bergson_debug_inject_status",
+)
+
+
+class BergsonError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class bergson_layer(ctypes.Structure):
+    _fields_ = [
+        ("A", ctypes.c_void_p), ("G", ctypes.c_void_p),
+        ("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64),
+        ("k_in", ctypes.c_int64), ("k_out", ctypes.c_int64),
+        ("seed_in", ctypes.c_uint64), ("seed_out", ctypes.c_uint64),
+        ("proj_kind", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("r", ctypes.c_void_p), ("c", ctypes.c_void_p),
+        ("out_col_offset", ctypes.c_int64),
+    ]
+
+
+_LIB = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library (raises if it was not built)."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+    L = ctypes.CDLL(LIB_PATH)
+    i64, u64, vp, i32 = ctypes.c_int64, ctypes.c_uint64, ctypes.c_void_p, ctypes.c_int
+    szp = ctypes.POINTER(ctypes.c_size_t)
+    lp = ctypes.POINTER(bergson_layer)
+    sig = {
+        "bergson_project_grads_workspace": (i32, [lp, i32, i64, i64, szp]),
+        "bergson_project_grads": (i32, [lp, i32, i64, i64, vp, vp, i64, vp, ctypes.c_size_t, vp]),
+        "bergson_build_store": (i32, [vp, i64, i64, i64, i32, vp, i64, i64, i64, vp, vp]),
+        "bergson_score_topk_workspace": (i32, [i64, i64, i64, i64, szp]),
+        "bergson_score_topk": (i32, [vp, i64, i64, i64, vp, i64, i64, i64, vp, vp, vp,
+                                     ctypes.c_size_t, vp]),
+        "bergson_projection_matrix": (i32, [u64, i64, i64, i32, vp, vp, vp]),
+        "bergson_module_seeds": (None, [u64, i64, ctypes.POINTER(u64), ctypes.POINTER(u64)]),
+        "bergson_sync_status": (i32, [vp]),
+        "bergson_last_error": (ctypes.c_char_p, []),
+        "bergson_version": (i32, []),
+        "bergson_debug_wait_probe": (i32, [u64, vp]),
+        "bergson_debug_inject_status": (None, [i32, i32]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _LIB = L
+    return L
+
+
+def bergson_last_error() -> str:
+    return lib().bergson_last_error().decode()
+
+
+def _check(status: int) -> None:
+    if status != BERGSON_OK:
+        raise BergsonError(status, bergson_last_error())
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    return t.data_ptr() if hasattr(t, "data_ptr") else int(t)
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+@dataclasses.dataclass
+class Layer:
+    """One nn.Linear's captured tensors: A [B,T,d_in] bf16, G [B,T,d_out] bf16."""
+    A: object
+    G: object
+    k_in: int
+    k_out: int
+    seed_in: int
+    seed_out: int
+    r: object = None
+    c: object = None
+    out_col_offset: int = 0
+    proj_kind: int = BERGSON_PROJ_GAUSSIAN
+
+    def to_c(self) -> bergson_layer:
+        return bergson_layer(
+            A=_ptr(self.A), G=_ptr(self.G), d_in=int(self.A.shape[-1]), d_out=int(self.G.shape[-1]),
+            k_in=int(self.k_in), k_out=int(self.k_out), seed_in=int(self.seed_in),
+            seed_out=int(self.seed_out), proj_kind=int(self.proj_kind), reserved=0,
+            r=_ptr(self.r), c=_ptr(self.c), out_col_offset=int(self.out_col_offset))
+
+
+def _layer_array(layers: Sequence) -> "ctypes.Array":
+    arr = (bergson_layer * len(layers))()
+    for i, ly in enumerate(layers):
+        arr[i] = ly if isinstance(ly, bergson_layer) else ly.to_c()
+    return arr
+
+
+def bergson_module_seeds(base_seed: int, module_index: int) -> tuple[int, int]:
+    a, b = ctypes.c_uint64(), ctypes.c_uint64()
+    lib().bergson_module_seeds(int(base_seed), int(module_index), ctypes.byref(a), ctypes.byref(b))
+    return a.value, b.value
+
+
+def bergson_project_grads_workspace(layers: Sequence, B: int, T: int) -> int:
+    arr = _layer_array(layers)
+    n = ctypes.c_size_t()
+    _check(lib().bergson_project_grads_workspace(arr, len(layers), int(B), int(T), ctypes.byref(n)))
+    return n.value
+
+
+def bergson_project_grads(layers: Sequence, B: int, T: int, mask, out, workspace,
+                          stream=None, ld_out: Optional[int] = None) -> None:
+    arr = _layer_array(layers)
+    ld = int(out.stride(0)) if ld_out is None else int(ld_out)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().bergson_project_grads(arr, len(layers), int(B), int(T), _ptr(mask), _ptr(out), ld,
+                                       _ptr(workspace), ws_bytes, _stream(stream)))
+
+
+def bergson_build_store(proj, B: int, K: int, unit_normalize: bool, store, row_offset: int,
+                        norms_out=None, stream=None) -> None:
+    _check(lib().bergson_build_store(_ptr(proj), int(B), int(K), int(proj.stride(0)),
+                                     1 if unit_normalize else 0, _ptr(store), int(store.stride(0)),
+                                     int(row_offset), int(store.shape[0]), _ptr(norms_out),
+                                     _stream(stream)))
+
+
+def bergson_score_topk_workspace(N: int, K: int, Q: int, topk: int) -> int:
+    n = ctypes.c_size_t()
+    _check(lib().bergson_score_topk_workspace(int(N), int(K), int(Q), int(topk), ctypes.byref(n)))
+    return n.value
+
+
+def bergson_score_topk(store, N: int, K: int, queries, topk: int, out_scores, out_idx, workspace,
+                       stream=None) -> None:
+    Q = int(queries.shape[0])
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().bergson_score_topk(_ptr(store), int(N), int(K), int(store.stride(0)),
+                                    _ptr(queries), Q, int(queries.stride(0)), int(topk),
+                                    _ptr(out_scores), _ptr(out_idx), _ptr(workspace), ws_bytes,
+                                    _stream(stream)))
+
+
+def bergson_projection_matrix(seed: int, d: int, k: int, proj_kind: int, moment, out,
+                              stream=None) -> None:
+    _check(lib().bergson_projection_matrix(int(seed), int(d), int(k), int(proj_kind), _ptr(moment),
+                                           _ptr(out), _stream(stream)))
+
+
+def bergson_sync_status(stream=None) -> int:
+    """Returns the status code (does not raise)."""
+    return lib().bergson_sync_status(_stream(stream))
+
+
+def bergson_version() -> int:
+    return lib().bergson_version()
+
+
+def bergson_debug_wait_probe(timeout_ns: int, stream=None) -> None:
+    _check(lib().bergson_debug_wait_probe(int(timeout_ns), _stream(stream)))
+
+
+def bergson_debug_inject_status(status: int, count: int) -> None:
+    lib().bergson_debug_inject_status(int(status), int(count))
+
+
+# ------------------------------------------------------------------ helpers
+
+def workspace_tensor(nbytes: int, device="cuda"):
+    """A byte tensor usable as workspace (torch allocations are 512-byte aligned)."""
+    import torch
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)

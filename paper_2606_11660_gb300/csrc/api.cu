@@ -1,0 +1,635 @@
+// Host side of the C ABI declared in include/bergson.h: argument validation,
+// workspace layout, TMA descriptor encoding, kernel launches, error mapping.
+
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "bergson.h"
+#include "internal.h"
+
+namespace bergson {
+namespace {
+
+constexpr int kVersion = 100;                        // 0.1.0
+constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 s
+constexpr int kSchedTargetItems = 2048;              // work items per projection launch (target)
+constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
+constexpr int kMaxDevices = 64;
+
+__device__ int g_status_word;                        // device status word (one per device)
+
+thread_local std::string g_last_error;
+std::atomic<int> g_inject_status{0};
+std::atomic<int> g_inject_count{0};
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+int fail_cuda(cudaError_t e, const char* what) {
+  return fail(BERGSON_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+int injected() {
+  int n = g_inject_count.load();
+  while (n > 0) {
+    if (g_inject_count.compare_exchange_weak(n, n - 1)) {
+      const int st = g_inject_status.load();
+      return fail(st, "injected status %d (test hook)", st);
+    }
+  }
+  return BERGSON_OK;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Makes the device owning `ptr` current for the lifetime of the guard.
+struct DeviceGuard {
+  int prev = -1;
+  int dev = -1;
+  cudaError_t err = cudaSuccess;
+  explicit DeviceGuard(const void* ptr) {
+    cudaPointerAttributes at;
+    err = cudaPointerGetAttributes(&at, ptr);
+    if (err != cudaSuccess) return;
+    if (at.type != cudaMemoryTypeDevice && at.type != cudaMemoryTypeManaged) {
+      err = cudaErrorInvalidDevicePointer;
+      return;
+    }
+    err = cudaGetDevice(&prev);
+    if (err != cudaSuccess) return;
+    dev = at.device;
+    if (dev != prev) err = cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    if (prev >= 0 && dev >= 0 && prev != dev) cudaSetDevice(prev);
+  }
+};
+
+int* status_word(int dev) {
+  static std::mutex mu;
+  static int* ptrs[kMaxDevices] = {};
+  std::lock_guard<std::mutex> lk(mu);
+  if (dev < 0 || dev >= kMaxDevices) return nullptr;
+  if (ptrs[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    ptrs[dev] = static_cast<int*>(p);
+  }
+  return ptrs[dev];
+}
+
+int sm_count(int dev) {
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return n;
+}
+
+bool valid_k(int64_t k) { return k == 16 || k == 32 || k == 64; }
+
+// ----------------------------------------------------------- project_grads
+
+struct Group {
+  int k_in = 0, k_out = 0;
+  std::vector<int> layers;     // indices into the caller's array, call order
+  int first_mod = 0;           // index of its first ModDesc in workspace
+  int n_chunks = 0, tpc = 0, n_items = 0;
+  size_t partial_off = 0;
+};
+
+struct ProjLayout {
+  int n_tiles = 0;
+  std::vector<Group> groups;
+  std::vector<int> mod_slot;   // layer index -> ModDesc slot
+  size_t mods_off = 0, segs_off = 0, ctr_off = 0, tv_off = 0;
+  std::vector<size_t> pin_off, pout_off;
+  size_t total = 0;
+};
+
+int validate_layers(const bergson_layer* layers, int n_layers, int64_t B, int64_t T) {
+  if (layers == nullptr) return fail(BERGSON_EINVAL, "layers is NULL");
+  if (n_layers < 1) return fail(BERGSON_EINVAL, "n_layers must be >= 1 (got %d)", n_layers);
+  if (B < 0 || T < 0) return fail(BERGSON_EINVAL, "B and T must be >= 0 (B=%lld T=%lld)",
+                                  (long long)B, (long long)T);
+  if (B > (1ll << 30) || T > (1ll << 30) || B * T > (1ll << 37))
+    return fail(BERGSON_EUNSUPPORTED, "B*T too large");
+  for (int i = 0; i < n_layers; ++i) {
+    const bergson_layer& L = layers[i];
+    if (L.reserved != 0) return fail(BERGSON_EINVAL, "layer %d: reserved field must be 0", i);
+    if (L.d_in < 8 || L.d_out < 8 || L.d_in > (1 << 24) || L.d_out > (1 << 24))
+      return fail(BERGSON_EINVAL, "layer %d: d_in/d_out must be in [8, 2^24]", i);
+    if (L.d_in % 8 != 0 || L.d_out % 8 != 0)
+      return fail(BERGSON_EALIGN, "layer %d: d_in and d_out must be multiples of 8", i);
+    if (L.proj_kind != BERGSON_PROJ_GAUSSIAN && L.proj_kind != BERGSON_PROJ_IDENTITY)
+      return fail(BERGSON_EINVAL, "layer %d: unknown proj_kind %d", i, L.proj_kind);
+    if (!valid_k(L.k_in) || !valid_k(L.k_out))
+      return fail(BERGSON_EUNSUPPORTED, "layer %d: k_in and k_out must be 16, 32 or 64", i);
+    if (L.proj_kind == BERGSON_PROJ_IDENTITY && (L.k_in != L.d_in || L.k_out != L.d_out))
+      return fail(BERGSON_EINVAL, "layer %d: identity projection needs k == d", i);
+    if ((L.r == nullptr) != (L.c == nullptr))
+      return fail(BERGSON_EINVAL, "layer %d: r and c must both be given or both be NULL", i);
+    if ((L.r && !aligned(L.r, 4)) || (L.c && !aligned(L.c, 4)))
+      return fail(BERGSON_EALIGN, "layer %d: r/c must be 4-byte aligned", i);
+    if (B * T > 0) {
+      if (L.A == nullptr || L.G == nullptr) return fail(BERGSON_EINVAL, "layer %d: A or G is NULL", i);
+      if (!aligned(L.A, 16) || !aligned(L.G, 16))
+        return fail(BERGSON_EALIGN, "layer %d: A and G must be 16-byte aligned", i);
+    }
+    if (L.out_col_offset < 0) return fail(BERGSON_EINVAL, "layer %d: negative out_col_offset", i);
+  }
+  return BERGSON_OK;
+}
+
+int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out) {
+  std::vector<std::pair<int64_t, int64_t>> blk;
+  for (int i = 0; i < n_layers; ++i) {
+    const int64_t a = layers[i].out_col_offset;
+    const int64_t e = a + layers[i].k_in * layers[i].k_out;
+    if (e > ld_out)
+      return fail(BERGSON_EINVAL, "layer %d: block [%lld, %lld) exceeds ld_out=%lld", i,
+                  (long long)a, (long long)e, (long long)ld_out);
+    blk.emplace_back(a, e);
+  }
+  std::sort(blk.begin(), blk.end());
+  for (size_t i = 1; i < blk.size(); ++i)
+    if (blk[i].first < blk[i - 1].second)
+      return fail(BERGSON_EINVAL, "output column blocks overlap at column %lld",
+                  (long long)blk[i].first);
+  return BERGSON_OK;
+}
+
+ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, int64_t T) {
+  ProjLayout L;
+  L.n_tiles = static_cast<int>((T + kTileTokens - 1) / kTileTokens);
+  L.mod_slot.assign(n_layers, 0);
+  for (int i = 0; i < n_layers; ++i) {
+    const int ki = static_cast<int>(layers[i].k_in), ko = static_cast<int>(layers[i].k_out);
+    auto it = std::find_if(L.groups.begin(), L.groups.end(),
+                           [&](const Group& g) { return g.k_in == ki && g.k_out == ko; });
+    if (it == L.groups.end()) {
+      L.groups.push_back(Group());
+      it = L.groups.end() - 1;
+      it->k_in = ki;
+      it->k_out = ko;
+    }
+    it->layers.push_back(i);
+  }
+  int slot = 0;
+  for (Group& g : L.groups) {
+    g.first_mod = slot;
+    for (int li : g.layers) L.mod_slot[li] = slot++;
+    const int nt_per_group = (g.k_in + g.k_out <= 64) ? 2 : 1;
+    const int64_t mb = static_cast<int64_t>(g.layers.size()) * B;
+    if (L.n_tiles == 0 || mb == 0) {
+      g.n_chunks = 0;
+      g.tpc = 0;
+      g.n_items = 0;
+      continue;
+    }
+    const int max_chunks = (L.n_tiles + nt_per_group - 1) / nt_per_group;
+    int64_t want = (kSchedTargetItems + mb - 1) / mb;
+    if (want > max_chunks) want = max_chunks;
+    if (want < 1) want = 1;
+    int tpc = static_cast<int>((L.n_tiles + want - 1) / want);
+    tpc = (tpc + nt_per_group - 1) / nt_per_group * nt_per_group;
+    g.tpc = tpc;
+    g.n_chunks = (L.n_tiles + tpc - 1) / tpc;
+    g.n_items = static_cast<int>(mb * g.n_chunks);
+  }
+  size_t off = 0;
+  L.mods_off = off;
+  off += round_up(sizeof(ModDesc) * n_layers, 256);
+  L.segs_off = off;
+  off += round_up(sizeof(PrepSeg) * 2 * n_layers, 256);
+  L.ctr_off = off;
+  off += round_up(sizeof(int) * 32 * L.groups.size(), 256);
+  L.tv_off = off;
+  off += round_up(static_cast<size_t>(B) * L.n_tiles, 256);
+  L.pin_off.resize(n_layers);
+  L.pout_off.resize(n_layers);
+  for (int i = 0; i < n_layers; ++i) {
+    L.pin_off[i] = off;
+    off += round_up(2 * layers[i].k_in * layers[i].d_in * sizeof(__nv_bfloat16), 256);
+    L.pout_off[i] = off;
+    off += round_up(2 * layers[i].k_out * layers[i].d_out * sizeof(__nv_bfloat16), 256);
+  }
+  for (Group& g : L.groups) {
+    g.partial_off = off;
+    off += round_up(static_cast<size_t>(g.n_items) * g.k_in * g.k_out * sizeof(float), 256);
+  }
+  L.total = off;
+  return L;
+}
+
+CUresult encode_act(CUtensorMap* tm, const void* ptr, int64_t d, int64_t T, int64_t B) {
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T),
+                        static_cast<cuuint64_t>(B)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d * 2), static_cast<cuuint64_t>(T * d * 2)};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kChunk), static_cast<cuuint32_t>(kTileTokens), 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return encode_fn()(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+CUresult encode_2d(CUtensorMap* tm, CUtensorMapDataType dt, const void* ptr, int64_t inner,
+                   int64_t outer, int64_t row_bytes, int box_inner, int box_outer) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(row_bytes)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_outer)};
+  cuuint32_t es[2] = {1, 1};
+  return encode_fn()(tm, dt, 2, const_cast<void*>(ptr), dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+// ------------------------------------------------------------- score_topk
+
+struct ScoreLayout {
+  int qt = 1;
+  size_t qh_off = 0, heap_off = 0, total = 0;
+};
+
+ScoreLayout plan_score(int64_t K, int64_t Q, int64_t topk) {
+  ScoreLayout L;
+  L.qt = Q > kScoreQT ? 2 : 1;
+  L.qh_off = 0;
+  L.heap_off = round_up(static_cast<size_t>(Q) * K * sizeof(__half), 256);
+  L.total = L.heap_off + round_up(static_cast<size_t>(kMaxScoreCTAs) * topk * L.qt * kScoreQT *
+                                      sizeof(unsigned long long),
+                                  256);
+  return L;
+}
+
+int validate_score(const void* store, int64_t N, int64_t K, int64_t ld_store, const float* queries,
+                   int64_t Q, int64_t ld_q, int64_t topk) {
+  if (N < 1 || N >= (1ll << 31)) return fail(BERGSON_EINVAL, "N must be in [1, 2^31)");
+  if (K < 8 || K > (1ll << 24)) return fail(BERGSON_EINVAL, "K must be in [8, 2^24]");
+  if (K % 8 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 8");
+  if (Q < 0 || Q > (1ll << 24)) return fail(BERGSON_EINVAL, "Q must be in [0, 2^24]");
+  if (topk < 1 || topk > kMaxTopk)
+    return fail(BERGSON_EUNSUPPORTED, "topk must be in [1, %d]", kMaxTopk);
+  if (topk > N) return fail(BERGSON_EINVAL, "topk (%lld) > N (%lld)", (long long)topk, (long long)N);
+  if (ld_store < K || ld_store % 8 != 0)
+    return fail(ld_store < K ? BERGSON_EINVAL : BERGSON_EALIGN,
+                "ld_store must be >= K and a multiple of 8");
+  if (store == nullptr) return fail(BERGSON_EINVAL, "store is NULL");
+  if (!aligned(store, 16)) return fail(BERGSON_EALIGN, "store must be 16-byte aligned");
+  if (Q > 0) {
+    if (queries == nullptr) return fail(BERGSON_EINVAL, "queries is NULL");
+    if (!aligned(queries, 4)) return fail(BERGSON_EALIGN, "queries must be 4-byte aligned");
+    if (ld_q < K) return fail(BERGSON_EINVAL, "ld_q must be >= K");
+  }
+  return BERGSON_OK;
+}
+
+}  // namespace
+}  // namespace bergson
+
+using namespace bergson;
+
+extern "C" {
+
+int bergson_version(void) { return kVersion; }
+
+void bergson_module_seeds(uint64_t base_seed, int64_t module_index, uint64_t* seed_in,
+                          uint64_t* seed_out) {
+  auto mix = [](uint64_t x) {
+    x = (x ^ (x >> 30)) * 0xBF58476D1CE4E5B9ull;
+    x = (x ^ (x >> 27)) * 0x94D049BB133111EBull;
+    return x ^ (x >> 31);
+  };
+  const uint64_t m = static_cast<uint64_t>(module_index);
+  if (seed_in != nullptr) *seed_in = mix(base_seed ^ (2 * m));
+  if (seed_out != nullptr) *seed_out = mix(base_seed ^ (2 * m + 1));
+}
+
+const char* bergson_last_error(void) { return g_last_error.c_str(); }
+
+void bergson_debug_inject_status(int status, int count) {
+  g_inject_status.store(status);
+  g_inject_count.store(count > 0 ? count : 0);
+}
+
+int bergson_project_grads_workspace(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                                    size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  int st = validate_layers(layers, n_layers, B, T);
+  if (st != BERGSON_OK) return st;
+  *ws_bytes = plan_project(layers, n_layers, B, T).total;
+  return BERGSON_OK;
+}
+
+int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                          const uint8_t* mask, float* out, int64_t ld_out, void* workspace,
+                          size_t ws_bytes, void* stream) {
+  int st = validate_layers(layers, n_layers, B, T);
+  if (st != BERGSON_OK) return st;
+  if (ld_out < 0) return fail(BERGSON_EINVAL, "ld_out must be >= 0");
+  st = validate_blocks(layers, n_layers, ld_out);
+  if (st != BERGSON_OK) return st;
+  if (B > 0 && out == nullptr) return fail(BERGSON_EINVAL, "out is NULL");
+  if (out != nullptr && !aligned(out, 4)) return fail(BERGSON_EALIGN, "out must be 4-byte aligned");
+  const ProjLayout L = plan_project(layers, n_layers, B, T);
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < L.total)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, L.total);
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (B == 0) return BERGSON_OK;
+
+  DeviceGuard dg(workspace);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
+  if (T > 0 && encode_fn() == nullptr)
+    return fail(BERGSON_ECUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+  int* status = status_word(dg.dev);
+  if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+
+  // Host-built records: module descriptors, projection segments, zeroed counters.
+  std::vector<uint8_t> staging(L.tv_off, 0);
+  ModDesc* mods = reinterpret_cast<ModDesc*>(staging.data() + L.mods_off);
+  PrepSeg* segs = reinterpret_cast<PrepSeg*>(staging.data() + L.segs_off);
+  int64_t flat = 0;
+  for (int i = 0; i < n_layers; ++i) {
+    const bergson_layer& ly = layers[i];
+    ModDesc& md = mods[L.mod_slot[i]];
+    md.d_in = static_cast<int32_t>(ly.d_in);
+    md.d_out = static_cast<int32_t>(ly.d_out);
+    md.col_offset = ly.out_col_offset;
+    __nv_bfloat16* pin = reinterpret_cast<__nv_bfloat16*>(ws + L.pin_off[i]);
+    __nv_bfloat16* pout = reinterpret_cast<__nv_bfloat16*>(ws + L.pout_off[i]);
+    if (T > 0) {
+      CUresult r1 = encode_act(&md.tmA, ly.A, ly.d_in, T, B);
+      CUresult r2 = encode_act(&md.tmG, ly.G, ly.d_out, T, B);
+      CUresult r3 = encode_2d(&md.tmPin, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, pin, ly.d_in,
+                              2 * ly.k_in, ly.d_in * 2, kChunk, static_cast<int>(2 * ly.k_in));
+      CUresult r4 = encode_2d(&md.tmPout, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, pout, ly.d_out,
+                              2 * ly.k_out, ly.d_out * 2, kChunk, static_cast<int>(2 * ly.k_out));
+      if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS || r3 != CUDA_SUCCESS || r4 != CUDA_SUCCESS)
+        return fail(BERGSON_ECUDA, "layer %d: tensor map encoding failed (%d %d %d %d)", i,
+                    (int)r1, (int)r2, (int)r3, (int)r4);
+    }
+    PrepSeg& si = segs[2 * i];
+    si.seed = ly.seed_in;
+    si.moment = ly.c;
+    si.dst = pin;
+    si.begin = flat;
+    si.d = static_cast<int32_t>(ly.d_in);
+    si.k = static_cast<int32_t>(ly.k_in);
+    si.kind = ly.proj_kind;
+    flat += ly.d_in * ly.k_in;
+    PrepSeg& so = segs[2 * i + 1];
+    so.seed = ly.seed_out;
+    so.moment = ly.r;
+    so.dst = pout;
+    so.begin = flat;
+    so.d = static_cast<int32_t>(ly.d_out);
+    so.k = static_cast<int32_t>(ly.k_out);
+    so.kind = ly.proj_kind;
+    flat += ly.d_out * ly.k_out;
+  }
+  cudaError_t e = cudaMemcpyAsync(ws, staging.data(), staging.size(), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return fail_cuda(e, "staging copy");
+  const ModDesc* mods_dev = reinterpret_cast<const ModDesc*>(ws + L.mods_off);
+  const bool need_tiles = T > 0;
+  if (need_tiles) {
+    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, flat, s);
+    if (e != cudaSuccess) return fail_cuda(e, "prep launch");
+  }
+  uint8_t* tile_valid = nullptr;
+  if (mask != nullptr && need_tiles) {
+    tile_valid = ws + L.tv_off;
+    e = launch_tile_valid(mask, static_cast<int>(B), static_cast<int>(T), L.n_tiles, tile_valid, s);
+    if (e != cudaSuccess) return fail_cuda(e, "tile flag launch");
+  }
+  const int sms = sm_count(dg.dev);
+  for (size_t gi = 0; gi < L.groups.size(); ++gi) {
+    const Group& g = L.groups[gi];
+    float* partials = reinterpret_cast<float*>(ws + g.partial_off);
+    if (g.n_items > 0) {
+      ProjParams p;
+      p.mods = mods_dev + g.first_mod;
+      p.n_mods = static_cast<int>(g.layers.size());
+      p.B = static_cast<int>(B);
+      p.T = static_cast<int>(T);
+      p.n_tiles = L.n_tiles;
+      p.tpc = g.tpc;
+      p.n_chunks = g.n_chunks;
+      p.n_items = g.n_items;
+      p.mask = mask;
+      p.tile_valid = tile_valid;
+      p.partials = partials;
+      p.counter = reinterpret_cast<int*>(ws + L.ctr_off) + 32 * gi;
+      p.status = status;
+      p.timeout_ns = kWaitTimeoutNs;
+      const int grid = std::max(1, std::min(sms > 0 ? sms : 1, g.n_items));
+      e = launch_project(g.k_in, g.k_out, p, grid, s);
+      if (e != cudaSuccess) return fail_cuda(e, "projection kernel launch");
+    }
+    e = launch_reduce(mods_dev + g.first_mod, static_cast<int>(g.layers.size()), g.k_in, g.k_out,
+                      static_cast<int>(B), g.n_chunks, partials, out, ld_out, s);
+    if (e != cudaSuccess) return fail_cuda(e, "reduce launch");
+  }
+  return BERGSON_OK;
+}
+
+int bergson_build_store(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
+                        int unit_normalize, void* store, int64_t ld_store, int64_t row_offset,
+                        int64_t N_cap, float* norms_out, void* stream) {
+  if (B < 0 || B > (1ll << 31) - 1) return fail(BERGSON_EINVAL, "B must be in [0, 2^31)");
+  if (K < 8 || K > (1ll << 28)) return fail(BERGSON_EINVAL, "K must be in [8, 2^28]");
+  if (K % 8 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 8");
+  if (ld_proj < K) return fail(BERGSON_EINVAL, "ld_proj must be >= K");
+  if (ld_proj % 4 != 0) return fail(BERGSON_EALIGN, "ld_proj must be a multiple of 4");
+  if (ld_store < K) return fail(BERGSON_EINVAL, "ld_store must be >= K");
+  if (ld_store % 8 != 0) return fail(BERGSON_EALIGN, "ld_store must be a multiple of 8");
+  if (row_offset < 0 || N_cap < 0 || row_offset + B > N_cap)
+    return fail(BERGSON_EINVAL, "rows [%lld, %lld) do not fit N_cap=%lld", (long long)row_offset,
+                (long long)(row_offset + B), (long long)N_cap);
+  if (B > 0) {
+    if (proj == nullptr || store == nullptr) return fail(BERGSON_EINVAL, "proj or store is NULL");
+    if (!aligned(proj, 16) || !aligned(store, 16))
+      return fail(BERGSON_EALIGN, "proj and store must be 16-byte aligned");
+    if (norms_out != nullptr && !aligned(norms_out, 4))
+      return fail(BERGSON_EALIGN, "norms_out must be 4-byte aligned");
+  }
+  int st;
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (B == 0) return BERGSON_OK;
+  DeviceGuard dg(store);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "store device lookup");
+  __half* dst = static_cast<__half*>(store) + row_offset * ld_store;
+  cudaError_t e = launch_build_store(proj, static_cast<int>(B), static_cast<int>(K), ld_proj,
+                                     unit_normalize ? 1 : 0, dst, ld_store, norms_out,
+                                     static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "store kernel launch");
+  return BERGSON_OK;
+}
+
+int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (N < 1 || K < 8 || Q < 0 || topk < 1 || topk > kMaxTopk || topk > N || K % 8 != 0)
+    return fail(BERGSON_EINVAL, "invalid sizes for the score workspace");
+  *ws_bytes = plan_score(K, Q, topk).total;
+  return BERGSON_OK;
+}
+
+int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                       const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
+                       float* out_scores, int64_t* out_idx, void* workspace, size_t ws_bytes,
+                       void* stream) {
+  int st = validate_score(store, N, K, ld_store, queries, Q, ld_q, topk);
+  if (st != BERGSON_OK) return st;
+  if (Q > 0 && (out_scores == nullptr || out_idx == nullptr))
+    return fail(BERGSON_EINVAL, "out_scores or out_idx is NULL");
+  if ((out_scores && !aligned(out_scores, 4)) || (out_idx && !aligned(out_idx, 8)))
+    return fail(BERGSON_EALIGN, "outputs misaligned");
+  const ScoreLayout L = plan_score(K, Q, topk);
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < L.total)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, L.total);
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (Q == 0) return BERGSON_OK;
+
+  DeviceGuard dg(workspace);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
+  if (encode_fn() == nullptr)
+    return fail(BERGSON_ECUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+  int* status = status_word(dg.dev);
+  if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  __half* qh = reinterpret_cast<__half*>(ws + L.qh_off);
+  unsigned long long* heaps = reinterpret_cast<unsigned long long*>(ws + L.heap_off);
+
+  cudaError_t e = launch_normalize_queries(queries, static_cast<int>(Q), static_cast<int>(K), ld_q,
+                                           qh, s);
+  if (e != cudaSuccess) return fail_cuda(e, "query normalisation launch");
+
+  CUtensorMap tm_store, tm_q;
+  CUresult r1 = encode_2d(&tm_store, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, store, K, N, ld_store * 2,
+                          kChunk, kScoreBN);
+  CUresult r2 = encode_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, qh, K, Q, K * 2, kChunk, kScoreQT);
+  if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS)
+    return fail(BERGSON_ECUDA, "tensor map encoding failed (%d %d)", (int)r1, (int)r2);
+
+  const int sms = std::max(1, std::min(sm_count(dg.dev), kMaxScoreCTAs));
+  const int gsize = L.qt * kScoreQT;
+  const int n_qg_total = static_cast<int>((Q + gsize - 1) / gsize);
+  const int n_ntiles = static_cast<int>((N + kScoreBN - 1) / kScoreBN);
+  for (int pass = 0; pass < n_qg_total; pass += sms) {
+    const int n_qg = std::min(sms, n_qg_total - pass);
+    const int cpg = std::max(1, std::min(sms / n_qg, n_ntiles));
+    const int grid = n_qg * cpg;
+    ScoreParams p;
+    p.N = static_cast<int>(N);
+    p.K = static_cast<int>(K);
+    p.Q = static_cast<int>(Q);
+    p.topk = static_cast<int>(topk);
+    p.n_qg = n_qg;
+    p.qg_base = pass;
+    p.n_ntiles = n_ntiles;
+    p.heaps = heaps;
+    p.status = status;
+    p.timeout_ns = kWaitTimeoutNs;
+    e = launch_score(L.qt, tm_store, tm_q, p, grid, s);
+    if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
+    const int q_begin = pass * gsize;
+    const int q_end = static_cast<int>(std::min<int64_t>(Q, static_cast<int64_t>(pass + n_qg) * gsize));
+    e = launch_merge(heaps, grid, n_qg, L.qt, static_cast<int>(topk), q_begin, q_end, pass,
+                     out_scores, out_idx, s);
+    if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
+  }
+  return BERGSON_OK;
+}
+
+int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind,
+                              const float* moment, float* out, void* stream) {
+  if (d < 1 || d > (1 << 24)) return fail(BERGSON_EINVAL, "d must be in [1, 2^24]");
+  if (!valid_k(k)) return fail(BERGSON_EUNSUPPORTED, "k must be 16, 32 or 64");
+  if (proj_kind != BERGSON_PROJ_GAUSSIAN && proj_kind != BERGSON_PROJ_IDENTITY)
+    return fail(BERGSON_EINVAL, "unknown proj_kind %d", proj_kind);
+  if (proj_kind == BERGSON_PROJ_IDENTITY && k != d)
+    return fail(BERGSON_EINVAL, "identity projection needs k == d");
+  if (out == nullptr) return fail(BERGSON_EINVAL, "out is NULL");
+  if (!aligned(out, 4) || (moment && !aligned(moment, 4)))
+    return fail(BERGSON_EALIGN, "out/moment must be 4-byte aligned");
+  int st;
+  if ((st = injected()) != BERGSON_OK) return st;
+  DeviceGuard dg(out);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  cudaError_t e = launch_projection_matrix(seed, static_cast<int>(d), static_cast<int>(k),
+                                           proj_kind, moment, out,
+                                           static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "projection matrix launch");
+  return BERGSON_OK;
+}
+
+int bergson_sync_status(void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return fail_cuda(e, "stream synchronisation");
+  int dev = 0;
+  e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  int* w = status_word(dev);
+  if (w == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
+  int v = 0;
+  e = cudaMemcpy(&v, w, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail_cuda(e, "status word read");
+  if (v != 0) {
+    const int zero = 0;
+    cudaMemcpy(w, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    return fail(v, "a bounded device wait gave up (device status %d)", v);
+  }
+  return BERGSON_OK;
+}
+
+int bergson_debug_wait_probe(uint64_t timeout_ns, void* stream) {
+  if (timeout_ns < 1 || timeout_ns > 10000000000ull)
+    return fail(BERGSON_EINVAL, "timeout_ns must be in [1, 1e10]");
+  int st;
+  if ((st = injected()) != BERGSON_OK) return st;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail_cuda(e, "cudaGetDevice");
+  int* w = status_word(dev);
+  if (w == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
+  e = launch_wait_probe(w, timeout_ns, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "probe launch");
+  return BERGSON_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,102 @@
+// Structures shared between the host API (api.cu) and the kernel translation
+// units, and the launchers each kernel unit exports to the host API.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace bergson {
+
+constexpr int kTileTokens = 128;     // tokens per MMA tile (tcgen05 M)
+constexpr int kChunk = 64;           // bf16 elements per 128-byte swizzled row
+constexpr int kScoreBN = 256;        // store rows per score tile (tcgen05 N)
+constexpr int kScoreQT = 128;        // queries per query tile (tcgen05 M)
+constexpr int kMaxTopk = 1024;
+
+// Per-module launch record kept in workspace (global memory).  The tensor maps
+// are read by TMA straight from there, so the record is 64-byte aligned.
+struct ModDesc {
+  CUtensorMap tmA;      // bf16 {d_in, T, B}, box {64, 128, 1}, 128B swizzle
+  CUtensorMap tmG;      // bf16 {d_out, T, B}, box {64, 128, 1}, 128B swizzle
+  CUtensorMap tmPin;    // bf16 {d_in, 2 k_in} (hi rows then lo rows), box {64, 2 k_in}
+  CUtensorMap tmPout;   // bf16 {d_out, 2 k_out}, box {64, 2 k_out}
+  int32_t d_in;
+  int32_t d_out;
+  int64_t col_offset;
+  int64_t reserved[6];
+};
+static_assert(alignof(ModDesc) >= 64 && sizeof(ModDesc) % 64 == 0, "TMA needs 64-byte aligned maps");
+
+// One projection matrix to materialise: P'^T as bf16 hi rows [0, k) and lo rows
+// [k, 2k), each of length d, with P'[i, j] = scale_i * P[i, j].
+struct PrepSeg {
+  uint64_t seed;
+  const float* moment;      // r (output side) or c (input side), or nullptr
+  __nv_bfloat16* dst;       // [2k, d]
+  int64_t begin;            // first flat element of this segment (d*k elements)
+  int32_t d;
+  int32_t k;
+  int32_t kind;
+  int32_t reserved;
+};
+
+struct ProjParams {
+  const ModDesc* mods;
+  int n_mods;
+  int B;
+  int T;
+  int n_tiles;          // ceil(T / 128)
+  int tpc;              // tiles per work item
+  int n_chunks;         // work items per (module, example)
+  int n_items;          // n_mods * B * n_chunks
+  const uint8_t* mask;        // [B, T] or nullptr
+  const uint8_t* tile_valid;  // [B, n_tiles] or nullptr
+  float* partials;            // [n_items, k_out * k_in]
+  int* counter;               // dynamic scheduler, zero on entry
+  int* status;                // device status word
+  uint64_t timeout_ns;
+};
+
+struct ScoreParams {
+  int N;
+  int K;
+  int Q;
+  int topk;
+  int n_qg;             // query groups in this pass
+  int qg_base;          // first query group of this pass
+  int n_ntiles;         // ceil(N / 256)
+  unsigned long long* heaps;  // [grid, topk, QT*128]
+  int* status;
+  uint64_t timeout_ns;
+};
+
+// ---- launchers (return the launch error, if any) ----
+
+cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t total, cudaStream_t s);
+cudaError_t launch_projection_matrix(uint64_t seed, int d, int k, int kind, const float* moment,
+                                     float* out, cudaStream_t s);
+cudaError_t launch_tile_valid(const uint8_t* mask, int B, int T, int n_tiles, uint8_t* tile_valid,
+                              cudaStream_t s);
+cudaError_t launch_wait_probe(int* status, uint64_t timeout_ns, cudaStream_t s);
+
+cudaError_t launch_project(int k_in, int k_out, const ProjParams& p, int grid, cudaStream_t s);
+size_t project_smem_bytes(int k_in, int k_out);
+cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, int B,
+                          int n_chunks, const float* partials, float* out, int64_t ld_out,
+                          cudaStream_t s);
+
+cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj, int unit,
+                               __half* store, int64_t ld_store, float* norms, cudaStream_t s);
+cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, __half* qh,
+                                     cudaStream_t s);
+cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
+                         const ScoreParams& p, int grid, cudaStream_t s);
+size_t score_smem_bytes(int qt);
+cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
+                         int q_begin, int q_end, int qg_base, float* out_scores, int64_t* out_idx,
+                         cudaStream_t s);
+
+}  // namespace bergson

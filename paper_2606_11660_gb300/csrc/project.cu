@@ -1,0 +1,458 @@
+// Fused token projection + masked per-example contraction (Bergson Fig. 1:
+// Adafactor normalisation and the double-sided per-module random projection,
+// applied to per-example nn.Linear gradients as in App. "Gradients").
+//
+// For one module and example b the projected gradient is
+//   G^_b = P_out'^T (sum_t m_t g_t a_t^T) P_in' = sum_t m_t (P_out'^T g_t)(P_in'^T a_t)^T,
+// so the kernel never forms the d_out x d_in gradient.  Per 128-token tile:
+//   1. TMA streams 128 x 64 bf16 boxes of A and G (128-byte swizzle) and the
+//      matching 64-column slices of P'^T (hi and lo bf16 rows) into a ring of
+//      shared-memory stages;
+//   2. one thread issues tcgen05.mma (M = 128 tokens, N = k, K = 16) into TMEM:
+//      a~ = A P_in' (k_in columns) and g~ = G P_out' (k_out columns), each as
+//      A*hi + A*lo accumulated in fp32;
+//   3. four epilogue warps read a~ and g~ out of TMEM (one token per thread),
+//      zero masked tokens, stage them in shared memory and accumulate the
+//      k_out x k_in outer-product sum in fp32 registers.
+// Work items are (module, example, range of tiles); a global counter hands
+// them to persistent CTAs, and each item writes one k_out x k_in partial that
+// a second kernel sums in a fixed order (deterministic result).
+//
+// Warp roles: warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer,
+// warps 2..5 = epilogue.  Every wait is bounded (see ptx.cuh).
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace bergson {
+
+namespace {
+
+constexpr int kActBoxBytes = kTileTokens * 128;       // 128 rows x 64 bf16
+constexpr int kSmemBudget = 232448;                   // 227 KB opt-in per CTA
+constexpr uint64_t kDrainTimeoutNs = 2000000000ull;   // waits for own copies after an abort
+
+constexpr int pow2ceil(int x) {
+  int p = 32;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+template <int KI, int KO>
+struct ProjCfg {
+  static constexpr int NT = (KI + KO <= 64) ? 2 : 1;            // tiles sharing one P slice
+  static constexpr int kPRows = 2 * (KI > KO ? KI : KO);         // hi + lo rows
+  static constexpr int kPBytes = kPRows * 128;
+  static constexpr int kStageBytes = NT * kActBoxBytes + kPBytes;
+  static constexpr int kEpiBytes = kTileTokens * (KI + 4) * 4 + kTileTokens * (KO + 4) * 4;
+  static constexpr int kBarBytes = 512;
+  static constexpr int kStagesFit = (kSmemBudget - 1024 - kEpiBytes - kBarBytes) / kStageBytes;
+  static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kEpiBytes + kBarBytes;
+  static constexpr int kTmemPerBuf = NT * (KI + KO);
+  static constexpr int kTmemCols = pow2ceil(2 * kTmemPerBuf);
+  static constexpr int kOPT = KO * KI / kTileTokens;            // outputs per epilogue thread
+  static_assert(kStages >= 2, "shared memory budget too small");
+  static_assert(kTmemCols <= 512, "TMEM budget exceeded");
+  static_assert(kOPT >= 2 && kOPT % 2 == 0, "unsupported projection sizes");
+};
+
+struct ItemCoord {
+  int m, b, t_begin, t_end;
+};
+
+__device__ __forceinline__ ItemCoord decode_item(const ProjParams& p, int item) {
+  ItemCoord c;
+  const int chunk = item % p.n_chunks;
+  const int mb = item / p.n_chunks;
+  c.b = mb % p.B;
+  c.m = mb / p.B;
+  c.t_begin = chunk * p.tpc;
+  c.t_end = min(p.n_tiles, c.t_begin + p.tpc);
+  return c;
+}
+
+template <int NT>
+__device__ __forceinline__ uint32_t group_valid(const ProjParams& p, int b, int g, int t_end) {
+  uint32_t vm = 0;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    const int t = g + nt;
+    if (t < t_end && (p.tile_valid == nullptr || p.tile_valid[b * p.n_tiles + t] != 0))
+      vm |= 1u << nt;
+  }
+  return vm;
+}
+
+template <int KI, int KO>
+__global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
+  using C = ProjCfg<KI, KO>;
+  constexpr int NT = C::NT;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  float* sA = reinterpret_cast<float*>(smem + C::kStages * C::kStageBytes);
+  float* sG = sA + kTileTokens * (KI + 4);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sG + kTileTokens * (KO + 4));
+  uint64_t* empty = full + C::kStages;
+  uint64_t* tfull = empty + C::kStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* sfull = tempty + 2;
+  uint64_t* sempty = sfull + 2;
+  uint64_t* drain = sempty + 2;
+  int* s_item = reinterpret_cast<int*>(drain + 1);
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(s_item + 2);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+  volatile int* s_epi_stop = s_abort + 1;   // epilogue leader's broadcast of "stop"
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&tfull[i]), 1);
+      mbar_init(smem_u32(&tempty[i]), 4);
+      mbar_init(smem_u32(&sfull[i]), 1);
+      mbar_init(smem_u32(&sempty[i]), 2);
+    }
+    mbar_init(smem_u32(drain), 1);
+    *s_abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(s_tmem), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *s_tmem;
+  const uint64_t tmo = p.timeout_ns;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_act = policy_evict_first();
+      const uint64_t pol_p = policy_evict_last();
+      int stage = 0;
+      uint32_t ph = 0;
+      int ss = 0;
+      uint32_t sph = 0;
+      uint32_t issued = 0, issued_par = 0;      // per-stage: TMA in flight, its phase parity
+      bool ok = true;
+      for (;;) {
+        const int item = atomicAdd(p.counter, 1);
+        if (!mbar_wait(smem_u32(&sempty[ss]), sph ^ 1, tmo, s_abort)) { ok = false; break; }
+        s_item[ss] = item;
+        mbar_arrive(smem_u32(&sfull[ss]));
+        if (++ss == 2) { ss = 0; sph ^= 1; }
+        if (item >= p.n_items) break;
+        const ItemCoord ic = decode_item(p, item);
+        const ModDesc* md = p.mods + ic.m;
+        tmap_acquire(&md->tmA);
+        tmap_acquire(&md->tmG);
+        tmap_acquire(&md->tmPin);
+        tmap_acquire(&md->tmPout);
+        for (int g = ic.t_begin; g < ic.t_end && ok; g += NT) {
+          const uint32_t vm = group_valid<NT>(p, ic.b, g, ic.t_end);
+          if (vm == 0) continue;
+          const uint32_t act_bytes = __popc(vm) * kActBoxBytes;
+          for (int side = 0; side < 2 && ok; ++side) {
+            const void* tact = side ? static_cast<const void*>(&md->tmG) : &md->tmA;
+            const void* tp = side ? static_cast<const void*>(&md->tmPout) : &md->tmPin;
+            const int d = side ? md->d_out : md->d_in;
+            const uint32_t pbytes = (side ? 2 * KO : 2 * KI) * 128;
+            const int nch = (d + kChunk - 1) / kChunk;
+            for (int ch = 0; ch < nch; ++ch) {
+              if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
+              const uint32_t fb = smem_u32(&full[stage]);
+              mbar_arrive_expect_tx(fb, act_bytes + pbytes);
+              const uint32_t dst = sbase + stage * C::kStageBytes;
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt)
+                if (vm >> nt & 1)
+                  tma_load_3d_hint(dst + nt * kActBoxBytes, tact, fb, ch * kChunk,
+                                   (g + nt) * kTileTokens, ic.b, pol_act);
+              tma_load_2d_hint(dst + NT * kActBoxBytes, tp, fb, ch * kChunk, 0, pol_p);
+              issued |= 1u << stage;
+              issued_par = (issued_par & ~(1u << stage)) | (ph << stage);
+              if (++stage == C::kStages) { stage = 0; ph ^= 1; }
+            }
+          }
+        }
+        if (!ok) break;
+      }
+      if (!ok) {
+        raise_device_error(p.status, s_abort, kStatusTimeout);
+        // Let every copy this thread started land before the CTA can exit.
+        for (int s = 0; s < C::kStages; ++s)
+          if (issued >> s & 1)
+            mbar_wait(smem_u32(&full[s]), (issued_par >> s) & 1, kDrainTimeoutNs, nullptr);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0;
+      int ab = 0;
+      uint32_t aph = 0;
+      int ss = 0;
+      uint32_t sph = 0;
+      bool ok = true;
+      for (;;) {
+        if (!mbar_wait(smem_u32(&sfull[ss]), sph, tmo, s_abort)) { ok = false; break; }
+        const int item = s_item[ss];
+        mbar_arrive(smem_u32(&sempty[ss]));
+        if (++ss == 2) { ss = 0; sph ^= 1; }
+        if (item >= p.n_items) break;
+        const ItemCoord ic = decode_item(p, item);
+        const ModDesc* md = p.mods + ic.m;
+        for (int g = ic.t_begin; g < ic.t_end && ok; g += NT) {
+          const uint32_t vm = group_valid<NT>(p, ic.b, g, ic.t_end);
+          if (vm == 0) continue;
+          if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t dbuf = tmem + ab * C::kTmemPerBuf;
+          for (int side = 0; side < 2 && ok; ++side) {
+            const int N = side ? KO : KI;
+            const uint32_t idesc = make_idesc_f16(kTileTokens, N, true);
+            const int d = side ? md->d_out : md->d_in;
+            const int nch = (d + kChunk - 1) / kChunk;
+            for (int ch = 0; ch < nch; ++ch) {
+              if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) { ok = false; break; }
+              tc_fence_after();
+              const uint32_t act = sbase + stage * C::kStageBytes;
+              const uint32_t pp = act + NT * kActBoxBytes;
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                if (!(vm >> nt & 1)) continue;
+                const uint32_t dcol = dbuf + nt * (KI + KO) + (side ? KI : 0);
+#pragma unroll
+                for (int kk = 0; kk < kChunk / 16; ++kk) {
+                  const uint64_t ad = sw128_desc(act + nt * kActBoxBytes + kk * 32);
+                  umma_f16(dcol, ad, sw128_desc(pp + kk * 32), idesc, (ch | kk) != 0);
+                  umma_f16(dcol, ad, sw128_desc(pp + N * 128 + kk * 32), idesc, 1u);
+                }
+              }
+              umma_commit(smem_u32(&empty[stage]));
+              if (++stage == C::kStages) { stage = 0; ph ^= 1; }
+            }
+          }
+          if (!ok) break;
+          umma_commit(smem_u32(&tfull[ab]));
+          if (++ab == 2) { ab = 0; aph ^= 1; }
+        }
+        if (!ok) break;
+      }
+      if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
+      // Every MMA this thread issued must finish before TMEM is released.
+      umma_commit(smem_u32(drain));
+      mbar_wait(smem_u32(drain), 0, kDrainTimeoutNs, nullptr);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    constexpr int OPT = C::kOPT;
+    const int et = threadIdx.x - 64;                 // 0..127
+    const int quarter = warp & 3;                    // TMEM lanes 32*quarter ..
+    const int row = 32 * quarter + lane;             // token row within a tile
+    const int oi = et * KO / kTileTokens;            // output row (k_out index)
+    const int oj = (et % (kTileTokens / KO)) * OPT;  // first output column (k_in index)
+    int ab = 0;
+    uint32_t aph = 0;
+    int ss = 0;
+    uint32_t sph = 0;
+    float acc[OPT];
+    for (;;) {
+      if (et == 0) {
+        if (!mbar_wait(smem_u32(&sfull[ss]), sph, tmo, s_abort))
+          raise_device_error(p.status, s_abort, kStatusTimeout);
+        *s_epi_stop = *s_abort;
+      }
+      named_bar_sync(1, 128);
+      if (*s_epi_stop) break;
+      const int item = s_item[ss];
+      named_bar_sync(1, 128);
+      if (et == 0) mbar_arrive(smem_u32(&sempty[ss]));
+      if (++ss == 2) { ss = 0; sph ^= 1; }
+      if (item >= p.n_items) break;
+      const ItemCoord ic = decode_item(p, item);
+#pragma unroll
+      for (int x = 0; x < OPT; ++x) acc[x] = 0.0f;
+      bool aborted = false;
+      for (int g = ic.t_begin; g < ic.t_end; g += NT) {
+        const uint32_t vm = group_valid<NT>(p, ic.b, g, ic.t_end);
+        if (vm == 0) continue;
+        if (et == 0) {
+          if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
+            raise_device_error(p.status, s_abort, kStatusTimeout);
+          *s_epi_stop = *s_abort;
+        }
+        named_bar_sync(1, 128);
+        if (*s_epi_stop) { aborted = true; break; }
+        tc_fence_after();
+        float va[NT][KI];
+        float vg[NT][KO];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          if (!(vm >> nt & 1)) continue;
+          const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
+                                 ab * C::kTmemPerBuf + nt * (KI + KO);
+#pragma unroll
+          for (int c = 0; c < KI / 16; ++c) tmem_ld16(taddr + c * 16, &va[nt][c * 16]);
+#pragma unroll
+          for (int c = 0; c < KO / 16; ++c) tmem_ld16(taddr + KI + c * 16, &vg[nt][c * 16]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+        if (++ab == 2) { ab = 0; aph ^= 1; }
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          if (!(vm >> nt & 1)) continue;
+          const int t = (g + nt) * kTileTokens + row;
+          const bool valid = t < p.T &&
+              (p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0);
+          named_bar_sync(1, 128);                    // previous tile's readers are done
+          float4* ra = reinterpret_cast<float4*>(sA + row * (KI + 4));
+          float4* rg = reinterpret_cast<float4*>(sG + row * (KO + 4));
+          const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int x = 0; x < KI / 4; ++x)
+            ra[x] = valid ? make_float4(va[nt][4 * x], va[nt][4 * x + 1], va[nt][4 * x + 2],
+                                        va[nt][4 * x + 3])
+                          : z4;
+#pragma unroll
+          for (int x = 0; x < KO / 4; ++x)
+            rg[x] = valid ? make_float4(vg[nt][4 * x], vg[nt][4 * x + 1], vg[nt][4 * x + 2],
+                                        vg[nt][4 * x + 3])
+                          : z4;
+          named_bar_sync(1, 128);
+#pragma unroll 4
+          for (int t2 = 0; t2 < kTileTokens; ++t2) {
+            const float gv = sG[t2 * (KO + 4) + oi];
+            const float* ar = sA + t2 * (KI + 4) + oj;
+            if constexpr (OPT % 4 == 0) {
+#pragma unroll
+              for (int x = 0; x < OPT / 4; ++x) {
+                const float4 a4 = reinterpret_cast<const float4*>(ar)[x];
+                acc[4 * x] = fmaf(gv, a4.x, acc[4 * x]);
+                acc[4 * x + 1] = fmaf(gv, a4.y, acc[4 * x + 1]);
+                acc[4 * x + 2] = fmaf(gv, a4.z, acc[4 * x + 2]);
+                acc[4 * x + 3] = fmaf(gv, a4.w, acc[4 * x + 3]);
+              }
+            } else {
+#pragma unroll
+              for (int x = 0; x < OPT / 2; ++x) {
+                const float2 a2 = reinterpret_cast<const float2*>(ar)[x];
+                acc[2 * x] = fmaf(gv, a2.x, acc[2 * x]);
+                acc[2 * x + 1] = fmaf(gv, a2.y, acc[2 * x + 1]);
+              }
+            }
+          }
+        }
+      }
+      if (aborted) break;
+      float* dst = p.partials + static_cast<int64_t>(item) * (KO * KI) + et * OPT;
+#pragma unroll
+      for (int x = 0; x < OPT / 2; ++x)
+        reinterpret_cast<float2*>(dst)[x] = make_float2(acc[2 * x], acc[2 * x + 1]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+// out[b, off_m + e] = sum over chunks c (in order) of partials[(m*B + b)*n_chunks + c][e]
+__global__ void reduce_kernel(const ModDesc* __restrict__ mods, int B, int blk, int n_chunks,
+                              const float* __restrict__ partials, float* __restrict__ out,
+                              int64_t ld_out) {
+  const int mb = blockIdx.x;
+  const int m = mb / B;
+  const int b = mb % B;
+  float* dst = out + static_cast<int64_t>(b) * ld_out + mods[m].col_offset;
+  const float* src = partials + static_cast<int64_t>(mb) * n_chunks * blk;
+  for (int e = threadIdx.x; e < blk; e += blockDim.x) {
+    float s = 0.0f;
+    for (int c = 0; c < n_chunks; ++c) s += src[static_cast<int64_t>(c) * blk + e];
+    dst[e] = s;
+  }
+}
+
+template <int KI, int KO>
+cudaError_t launch_project_t(const ProjParams& p, int grid, cudaStream_t s) {
+  using C = ProjCfg<KI, KO>;
+  static bool attr_set = false;   // per process; the attribute is per function and device
+  cudaError_t e = cudaSuccess;
+  if (!attr_set) {
+    e = cudaFuncSetAttribute(project_kernel<KI, KO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  project_kernel<KI, KO><<<grid, 192, C::kSmemBytes, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int KI, int KO>
+constexpr size_t smem_of() {
+  return ProjCfg<KI, KO>::kSmemBytes;
+}
+
+}  // namespace
+
+#define BERGSON_PROJ_DISPATCH(KI_, KO_, EXPR)        \
+  if (k_in == KI_ && k_out == KO_) {                 \
+    return EXPR;                                     \
+  }
+
+cudaError_t launch_project(int k_in, int k_out, const ProjParams& p, int grid, cudaStream_t s) {
+  BERGSON_PROJ_DISPATCH(16, 16, (launch_project_t<16, 16>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(16, 32, (launch_project_t<16, 32>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(16, 64, (launch_project_t<16, 64>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(32, 16, (launch_project_t<32, 16>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(32, 32, (launch_project_t<32, 32>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(32, 64, (launch_project_t<32, 64>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(64, 16, (launch_project_t<64, 16>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(64, 32, (launch_project_t<64, 32>(p, grid, s)))
+  BERGSON_PROJ_DISPATCH(64, 64, (launch_project_t<64, 64>(p, grid, s)))
+  return cudaErrorInvalidValue;
+}
+
+size_t project_smem_bytes(int k_in, int k_out) {
+  BERGSON_PROJ_DISPATCH(16, 16, (smem_of<16, 16>()))
+  BERGSON_PROJ_DISPATCH(16, 32, (smem_of<16, 32>()))
+  BERGSON_PROJ_DISPATCH(16, 64, (smem_of<16, 64>()))
+  BERGSON_PROJ_DISPATCH(32, 16, (smem_of<32, 16>()))
+  BERGSON_PROJ_DISPATCH(32, 32, (smem_of<32, 32>()))
+  BERGSON_PROJ_DISPATCH(32, 64, (smem_of<32, 64>()))
+  BERGSON_PROJ_DISPATCH(64, 16, (smem_of<64, 16>()))
+  BERGSON_PROJ_DISPATCH(64, 32, (smem_of<64, 32>()))
+  BERGSON_PROJ_DISPATCH(64, 64, (smem_of<64, 64>()))
+  return 0;
+}
+
+cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, int B,
+                          int n_chunks, const float* partials, float* out, int64_t ld_out,
+                          cudaStream_t s) {
+  const int blocks = n_mods * B;
+  if (blocks == 0) return cudaSuccess;
+  const int blk = k_in * k_out;
+  reduce_kernel<<<blocks, blk < 1024 ? blk : 1024, 0, s>>>(mods, B, blk, n_chunks, partials, out,
+                                                          ld_out);
+  return cudaGetLastError();
+}
+
+}  // namespace bergson

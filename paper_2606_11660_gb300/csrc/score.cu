@@ -1,0 +1,371 @@
+// Exact cosine top-k over the gradient store (Bergson Sec. 3.1: exact top-k
+// nearest-neighbour lookup; queries score against unit-normalised rows).
+//
+// Score kernel (persistent, one CTA per SM): CTA c owns one query group of
+// QT x 128 normalised fp16 queries and streams every (grid / n_qg)-th tile of
+// 256 store rows.  TMA brings 64-column slices of the store tile and of the
+// query tiles into a shared-memory ring; one thread issues tcgen05.mma with
+// M = 128 queries, N = 256 store rows, K = 16 into TMEM (fp32), so that TMEM
+// lane = query and column = store row.  Epilogue warps read their query's 256
+// scores, drop everything not above the query's running k-th best, and keep a
+// per-(CTA, query) binary min-heap of the k best (score, row) pairs in global
+// memory.  The N x Q score matrix never exists.
+// Merge kernel: one CTA per query sorts the heaps of the CTAs that covered the
+// query (bitonic sort of 64-bit keys in shared memory) and writes the final
+// top-k ordered by score descending, then row ascending.
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace bergson {
+
+namespace {
+
+constexpr int kSmemBudget = 232448;
+constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
+constexpr int kStoreBoxBytes = kScoreBN * 128;      // 256 rows x 64 fp16
+constexpr int kQBoxBytes = kScoreQT * 128;          // 128 rows x 64 fp16
+constexpr unsigned long long kSentinelKey = 0x007FFFFF00000000ull;   // (-inf, row 0xFFFFFFFF)
+
+template <int QT>
+struct ScoreCfg {
+  static constexpr int kStageBytes = kStoreBoxBytes + QT * kQBoxBytes;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kStagesFit = (kSmemBudget - 1024 - kBarBytes) / kStageBytes;
+  static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
+  static constexpr int kNBuf = 512 / (QT * kScoreBN);   // TMEM accumulator buffers
+  static constexpr int kEpiThreads = QT * 128;
+  static constexpr int kThreads = 64 + kEpiThreads;
+  static_assert(kNBuf >= 1, "TMEM budget");
+};
+
+// Order-preserving map of a float onto uint32 (-0 is folded onto +0 first).
+__device__ __forceinline__ uint32_t float_order(float s) {
+  const uint32_t u = __float_as_uint(s + 0.0f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float order_to_float(uint32_t o) {
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
+
+// Larger key = better: higher score first, then lower row index.
+__device__ __forceinline__ unsigned long long make_key(float s, uint32_t row) {
+  return (static_cast<unsigned long long>(float_order(s)) << 32) | static_cast<uint32_t>(~row);
+}
+
+// Replace the root (worst kept entry) of a min-heap of `k` keys stored at
+// base[e * stride] and restore the heap property.
+__device__ __forceinline__ void heap_replace_root(unsigned long long* base, int stride, int k,
+                                                  unsigned long long key) {
+  int i = 0;
+  for (;;) {
+    const int l = 2 * i + 1;
+    if (l >= k) break;
+    int c = l;
+    unsigned long long kc = base[static_cast<int64_t>(l) * stride];
+    if (l + 1 < k) {
+      const unsigned long long kr = base[static_cast<int64_t>(l + 1) * stride];
+      if (kr < kc) { c = l + 1; kc = kr; }
+    }
+    if (kc >= key) break;
+    base[static_cast<int64_t>(i) * stride] = kc;
+    i = c;
+  }
+  base[static_cast<int64_t>(i) * stride] = key;
+}
+
+template <int QT>
+__global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
+    score_kernel(const __grid_constant__ CUtensorMap tm_store, const __grid_constant__ CUtensorMap tm_q,
+                 const ScoreParams p) {
+  using C = ScoreCfg<QT>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  uint64_t* empty = full + C::kStages;
+  uint64_t* tfull = empty + C::kStages;       // [kNBuf]
+  uint64_t* tempty = tfull + 2;               // [kNBuf]
+  uint64_t* drain = tempty + 2;
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+  volatile int* s_epi_stop = s_abort + 1;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int g_local = blockIdx.x % p.n_qg;
+  const int g = p.qg_base + g_local;
+  const int cpg = gridDim.x / p.n_qg;
+  const int nt0 = blockIdx.x / p.n_qg;
+  const int nK = (p.K + kChunk - 1) / kChunk;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int i = 0; i < C::kNBuf; ++i) {
+      mbar_init(smem_u32(&tfull[i]), 1);
+      mbar_init(smem_u32(&tempty[i]), QT * 4);
+    }
+    mbar_init(smem_u32(drain), 1);
+    *s_abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(s_tmem), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *s_tmem;
+  const uint64_t tmo = p.timeout_ns;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tmap(&tm_store);
+      prefetch_tmap(&tm_q);
+      const uint64_t pol_store = policy_evict_first();
+      const uint64_t pol_q = policy_evict_last();
+      int stage = 0;
+      uint32_t ph = 0;
+      uint32_t issued = 0, issued_par = 0;
+      bool ok = true;
+      for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
+        for (int kc = 0; kc < nK; ++kc) {
+          if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_arrive_expect_tx(fb, C::kStageBytes);
+          const uint32_t dst = sbase + stage * C::kStageBytes;
+          tma_load_2d_hint(dst, &tm_store, fb, kc * kChunk, nt * kScoreBN, pol_store);
+#pragma unroll
+          for (int qt = 0; qt < QT; ++qt)
+            tma_load_2d_hint(dst + kStoreBoxBytes + qt * kQBoxBytes, &tm_q, fb, kc * kChunk,
+                             (g * QT + qt) * kScoreQT, pol_q);
+          issued |= 1u << stage;
+          issued_par = (issued_par & ~(1u << stage)) | (ph << stage);
+          if (++stage == C::kStages) { stage = 0; ph ^= 1; }
+        }
+      }
+      if (!ok) {
+        raise_device_error(p.status, s_abort, kStatusTimeout);
+        for (int s = 0; s < C::kStages; ++s)
+          if (issued >> s & 1)
+            mbar_wait(smem_u32(&full[s]), (issued_par >> s) & 1, kDrainTimeoutNs, nullptr);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = make_idesc_f16(kScoreQT, kScoreBN, false);
+      int stage = 0;
+      uint32_t ph = 0;
+      int ab = 0;
+      uint32_t aph = 0;
+      bool ok = true;
+      for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
+        if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t dbuf = tmem + ab * QT * kScoreBN;
+        for (int kc = 0; kc < nK; ++kc) {
+          if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sd = sbase + stage * C::kStageBytes;
+          const uint32_t qd = sd + kStoreBoxBytes;
+#pragma unroll
+          for (int qt = 0; qt < QT; ++qt) {
+#pragma unroll
+            for (int kk = 0; kk < kChunk / 16; ++kk)
+              umma_f16(dbuf + qt * kScoreBN, sw128_desc(qd + qt * kQBoxBytes + kk * 32),
+                       sw128_desc(sd + kk * 32), idesc, (kc | kk) != 0);
+          }
+          umma_commit(smem_u32(&empty[stage]));
+          if (++stage == C::kStages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit(smem_u32(&tfull[ab]));
+        if (++ab == C::kNBuf) { ab = 0; aph ^= 1; }
+      }
+      if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
+      umma_commit(smem_u32(drain));
+      mbar_wait(smem_u32(drain), 0, kDrainTimeoutNs, nullptr);
+    }
+    __syncwarp();
+  } else {
+    const int et = threadIdx.x - 64;                 // 0 .. QT*128-1
+    const int qt = et >> 7;
+    const int quarter = warp & 3;
+    const int slot = qt * kScoreQT + 32 * quarter + lane;
+    const int stride = C::kEpiThreads;
+    unsigned long long* heap =
+        p.heaps + static_cast<int64_t>(blockIdx.x) * p.topk * stride + slot;
+    for (int e = 0; e < p.topk; ++e) heap[static_cast<int64_t>(e) * stride] = kSentinelKey;
+    unsigned long long tau_key = kSentinelKey;
+    float tau = -INFINITY;
+    int ab = 0;
+    uint32_t aph = 0;
+    for (int nt = nt0; nt < p.n_ntiles; nt += cpg) {
+      if (et == 0) {
+        if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
+          raise_device_error(p.status, s_abort, kStatusTimeout);
+        *s_epi_stop = *s_abort;
+      }
+      named_bar_sync(1, C::kEpiThreads);
+      if (*s_epi_stop) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
+                             ab * QT * kScoreBN + qt * kScoreBN;
+      const int row_base = nt * kScoreBN;
+#pragma unroll 1
+      for (int c = 0; c < kScoreBN / 32; ++c) {
+        float v[32];
+        tmem_ld32(tbase + c * 32, v);
+        const int r0 = row_base + c * 32;
+        const int nvalid = min(32, p.N - r0);
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < nvalid) mx = fmaxf(mx, v[j]);
+        if (mx >= tau) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            if (j < nvalid && v[j] >= tau) {         // the comparison also drops NaN
+              const unsigned long long key = make_key(v[j], static_cast<uint32_t>(r0 + j));
+              if (key > tau_key) {
+                heap_replace_root(heap, stride, p.topk, key);
+                tau_key = heap[0];
+                tau = order_to_float(static_cast<uint32_t>(tau_key >> 32));
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+      if (++ab == C::kNBuf) { ab = 0; aph ^= 1; }
+      named_bar_sync(1, C::kEpiThreads);   // keeps the stop broadcast single-writer
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// Final top-k of one query from the heaps of the CTAs that covered it.
+__global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __restrict__ heaps,
+                                                    int n_qg, int cpg, int gsize, int topk,
+                                                    int q_begin, int q_end, int sort_n,
+                                                    float* __restrict__ out_scores,
+                                                    int64_t* __restrict__ out_idx) {
+  extern __shared__ unsigned long long keys[];
+  const int q = q_begin + blockIdx.x;
+  if (q >= q_end) return;
+  const int local = q - q_begin;
+  const int gl = local / gsize;
+  const int slot = local % gsize;
+  const int64_t total = static_cast<int64_t>(cpg) * topk;
+  int64_t consumed = 0;
+  bool first = true;
+  while (first || consumed < total) {
+    const int start = first ? 0 : topk;
+    for (int i = start + threadIdx.x; i < sort_n; i += blockDim.x) {
+      const int64_t ci = consumed + (i - start);
+      unsigned long long k = 0ull;
+      if (ci < total) {
+        const int cta = gl + static_cast<int>(ci / topk) * n_qg;
+        const int e = static_cast<int>(ci % topk);
+        k = heaps[(static_cast<int64_t>(cta) * topk + e) * gsize + slot];
+      }
+      keys[i] = k;
+    }
+    consumed += sort_n - start;
+    first = false;
+    __syncthreads();
+    for (int kk = 2; kk <= sort_n; kk <<= 1) {
+      for (int j = kk >> 1; j > 0; j >>= 1) {
+        for (int i = threadIdx.x; i < sort_n; i += blockDim.x) {
+          const int ixj = i ^ j;
+          if (ixj > i) {
+            const unsigned long long a = keys[i];
+            const unsigned long long b = keys[ixj];
+            const bool desc = (i & kk) == 0;
+            if (desc ? (a < b) : (a > b)) {
+              keys[i] = b;
+              keys[ixj] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    }
+  }
+  for (int e = threadIdx.x; e < topk; e += blockDim.x) {
+    const unsigned long long k = keys[e];
+    const uint32_t lo = static_cast<uint32_t>(k);
+    const bool real = lo >= 0x80000000u;          // rows < 2^31 map to ~row >= 2^31
+    out_scores[static_cast<int64_t>(q) * topk + e] =
+        real ? order_to_float(static_cast<uint32_t>(k >> 32)) : -INFINITY;
+    out_idx[static_cast<int64_t>(q) * topk + e] = real ? static_cast<int64_t>(~lo) : -1;
+  }
+}
+
+template <int QT>
+cudaError_t launch_score_t(const CUtensorMap& tms, const CUtensorMap& tmq, const ScoreParams& p,
+                           int grid, cudaStream_t s) {
+  using C = ScoreCfg<QT>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(score_kernel<QT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  score_kernel<QT><<<grid, C::kThreads, C::kSmemBytes, s>>>(tms, tmq, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
+                         const ScoreParams& p, int grid, cudaStream_t s) {
+  if (qt == 1) return launch_score_t<1>(tm_store, tm_q, p, grid, s);
+  if (qt == 2) return launch_score_t<2>(tm_store, tm_q, p, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+size_t score_smem_bytes(int qt) {
+  return qt == 1 ? ScoreCfg<1>::kSmemBytes : ScoreCfg<2>::kSmemBytes;
+}
+
+cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
+                         int q_begin, int q_end, int /*qg_base*/, float* out_scores,
+                         int64_t* out_idx, cudaStream_t s) {
+  const int nq = q_end - q_begin;
+  if (nq <= 0) return cudaSuccess;
+  const int cpg = grid / n_qg;
+  const int64_t total = static_cast<int64_t>(cpg) * topk;
+  int sort_n = 2;
+  while (sort_n < total && sort_n < 8192) sort_n <<= 1;
+  const size_t smem = static_cast<size_t>(sort_n) * sizeof(unsigned long long);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         8192 * sizeof(unsigned long long));
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  merge_kernel<<<nq, 512, smem, s>>>(heaps, n_qg, cpg, qt * kScoreQT, topk, q_begin, q_end, sort_n,
+                                     out_scores, out_idx);
+  return cudaGetLastError();
+}
+
+}  // namespace bergson

@@ -1,0 +1,163 @@
+"""Host-side checks of the C ABI that need no GPU: load, exports, validation."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2606_11660_gb300 as bg
+from oracle import bergson_oracle as orc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built_library():
+    from paper_2606_11660_gb300 import _build
+    _build.build()
+    yield
+
+
+def _declared_symbols():
+    src = open(os.path.join(ROOT, "include", "bergson.h")).read()
+    return sorted(set(re.findall(r"BERGSON_API\s+[\w\s\*]*?\b(bergson_\w+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol():
+    declared = _declared_symbols()
+    assert len(declared) >= 12
+    assert sorted(bg.EXPORTED) == declared
+    L = ctypes.CDLL(bg.LIB_PATH)
+    for name in declared:
+        assert hasattr(L, name), name
+    assert bg.bergson_version() == 100
+
+
+def test_module_seeds_match_oracle_derivation():
+    for base, m in [(0, 0), (0, 47), (123456789, 3), (2**64 - 1, 159)]:
+        assert bg.bergson_module_seeds(base, m) == orc.module_seeds(base, m)
+
+
+FAKE = 0x7F0000000000  # aligned, never dereferenced: validation fails first or no device
+
+
+def _layer(**kw):
+    d = dict(A=FAKE, G=FAKE + 4096, d_in=64, d_out=64, k_in=16, k_out=16, seed_in=1, seed_out=2,
+             proj_kind=0, reserved=0, r=None, c=None, out_col_offset=0)
+    d.update(kw)
+    return bg.bergson_layer(**d)
+
+
+def _ws(layers, B=2, T=32):
+    arr = (bg.bergson_layer * len(layers))(*layers)
+    n = ctypes.c_size_t()
+    st = bg.lib().bergson_project_grads_workspace(arr, len(layers), B, T, ctypes.byref(n))
+    return st, n.value
+
+
+def _proj(layers, B=2, T=32, out=FAKE, ld_out=256, ws=FAKE, ws_bytes=1 << 30, mask=None):
+    arr = (bg.bergson_layer * len(layers))(*layers)
+    return bg.lib().bergson_project_grads(arr, len(layers), B, T, mask, out, ld_out, ws, ws_bytes,
+                                          None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(d_in=60), bg.BERGSON_EALIGN),
+    (dict(d_out=4), bg.BERGSON_EINVAL),
+    (dict(k_in=24), bg.BERGSON_EUNSUPPORTED),
+    (dict(k_out=128), bg.BERGSON_EUNSUPPORTED),
+    (dict(proj_kind=7), bg.BERGSON_EINVAL),
+    (dict(proj_kind=1), bg.BERGSON_EINVAL),            # identity needs k == d
+    (dict(r=FAKE), bg.BERGSON_EINVAL),                 # r without c
+    (dict(A=FAKE + 8), bg.BERGSON_EALIGN),
+    (dict(G=None), bg.BERGSON_EINVAL),
+    (dict(reserved=1), bg.BERGSON_EINVAL),
+    (dict(out_col_offset=-1), bg.BERGSON_EINVAL),
+])
+def test_layer_validation(kw, code):
+    st, _ = _ws([_layer(**kw)])
+    assert st == code
+    assert bg.bergson_last_error() != ""
+    assert _proj([_layer(**kw)]) == code
+
+
+def test_workspace_query_and_block_checks():
+    st, n = _ws([_layer(), _layer(out_col_offset=256, k_in=32)])
+    assert st == bg.BERGSON_OK and n > 0 and n % 256 == 0
+    st2, n2 = _ws([_layer(), _layer(out_col_offset=256, k_in=32)], B=64, T=4096)
+    assert st2 == bg.BERGSON_OK and n2 > n
+    # overlapping output blocks
+    assert _proj([_layer(), _layer(out_col_offset=128)], ld_out=512) == bg.BERGSON_EINVAL
+    assert "overlap" in bg.bergson_last_error()
+    # block past ld_out
+    assert _proj([_layer(out_col_offset=100)], ld_out=256) == bg.BERGSON_EINVAL
+    # workspace too small / misaligned / missing
+    assert _proj([_layer()], ws_bytes=16) == bg.BERGSON_EWORKSPACE
+    assert _proj([_layer()], ws=FAKE + 16) == bg.BERGSON_EALIGN
+    assert _proj([_layer()], ws=None) == bg.BERGSON_EINVAL
+    assert _proj([_layer()], B=-1) == bg.BERGSON_EINVAL
+    assert bg.lib().bergson_project_grads(None, 1, 2, 3, None, FAKE, 256, FAKE, 1 << 20, None) == bg.BERGSON_EINVAL
+
+
+def test_empty_batch_is_a_no_op_and_injection_hook():
+    assert _proj([_layer()], B=0) == bg.BERGSON_OK
+    bg.bergson_debug_inject_status(bg.BERGSON_ECUDA, 1)
+    assert _proj([_layer()], B=0) == bg.BERGSON_ECUDA
+    assert "injected" in bg.bergson_last_error()
+    assert _proj([_layer()], B=0) == bg.BERGSON_OK     # one-shot
+    bg.bergson_debug_inject_status(bg.BERGSON_ECUDA, 0)
+
+
+def test_store_validation():
+    f = bg.lib().bergson_build_store
+    ok_args = dict(proj=FAKE, B=4, K=64, ld_proj=64, unit=1, store=FAKE, ld_store=64, row_offset=0,
+                   N_cap=4, norms=None, stream=None)
+
+    def call(**kw):
+        a = dict(ok_args)
+        a.update(kw)
+        return f(*a.values())
+    assert call(K=60) == bg.BERGSON_EALIGN
+    assert call(ld_proj=32) == bg.BERGSON_EINVAL
+    assert call(ld_proj=66) == bg.BERGSON_EALIGN
+    assert call(ld_store=72 + 4) == bg.BERGSON_EALIGN
+    assert call(row_offset=1) == bg.BERGSON_EINVAL      # does not fit N_cap
+    assert call(store=FAKE + 8) == bg.BERGSON_EALIGN
+    assert call(B=0) == bg.BERGSON_OK
+
+
+def test_score_validation():
+    f = bg.lib().bergson_score_topk
+    n = ctypes.c_size_t()
+    assert bg.lib().bergson_score_topk_workspace(100, 64, 10, 5, ctypes.byref(n)) == bg.BERGSON_OK
+    ws = n.value
+
+    def call(N=100, K=64, ld=64, q=FAKE, Q=10, ldq=64, topk=5, ws_bytes=ws, store=FAKE):
+        return f(store, N, K, ld, q, Q, ldq, topk, FAKE, FAKE, FAKE, ws_bytes, None)
+    assert call(topk=101) == bg.BERGSON_EINVAL           # k > N
+    assert call(topk=0) == bg.BERGSON_EUNSUPPORTED
+    assert call(topk=2000, N=5000) == bg.BERGSON_EUNSUPPORTED
+    assert call(K=60, ld=64) == bg.BERGSON_EALIGN
+    assert call(ld=68) == bg.BERGSON_EALIGN
+    assert call(ldq=32) == bg.BERGSON_EINVAL
+    assert call(ws_bytes=ws - 1) == bg.BERGSON_EWORKSPACE
+    assert call(store=FAKE + 8) == bg.BERGSON_EALIGN
+    assert call(N=0) == bg.BERGSON_EINVAL
+    assert call(Q=0) == bg.BERGSON_OK
+
+
+def test_projection_matrix_validation():
+    f = bg.lib().bergson_projection_matrix
+    assert f(1, 64, 24, 0, None, FAKE, None) == bg.BERGSON_EUNSUPPORTED
+    assert f(1, 64, 16, 1, None, FAKE, None) == bg.BERGSON_EINVAL
+    assert f(1, 64, 16, 0, None, None, None) == bg.BERGSON_EINVAL
+    assert bg.lib().bergson_debug_wait_probe(0, None) == bg.BERGSON_EINVAL
+
+
+def test_calls_without_device_fail_cleanly():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("host without a GPU only")
+    st = _proj([_layer()])
+    assert st == bg.BERGSON_ECUDA
+    assert bg.bergson_last_error() != ""
