@@ -35,8 +35,8 @@ def test_projection_matrix_matches_generator(seed, d, k, moment):
     got = np32(out)
     # fp32 Box-Muller against the fp64 definition: a few fp32 ulps per entry
     assert np.max(np.abs(got - want)) < 5e-6
-    rel = np.abs(got - want) / np.maximum(np.abs(want), 1e-3)
-    assert np.median(rel) < 2e-7 and np.quantile(rel, 0.999) < 3e-6
+    err = np.abs(got - want) / np.sqrt(np.mean(want * want))   # relative to the entry scale
+    assert np.median(err) < 2e-7 and np.quantile(err, 0.999) < 2e-6
 
 
 def test_tiny_workload_parity():
