@@ -213,6 +213,30 @@ BERGSON_API int bergson_debug_wait_probe(uint64_t timeout_ns, void* stream);
  */
 BERGSON_API void bergson_debug_inject_status(int status, int count);
 
+/*
+ * Allocation-free variant of bergson_project_grads.  The paper has no
+ * counterpart: this exists for callers that cannot supply a workspace, such as
+ * plugin or callback interfaces that hand over only input and output buffers,
+ * runtimes that own all device memory through their own pool, or loops that
+ * must not call cudaMalloc (it can synchronise the device and can fail when
+ * memory is short).
+ *
+ * Same arguments and result as bergson_project_grads, minus the workspace.
+ * The scratch is a fixed static device array of BERGSON_NOALLOC_SCRATCH_BYTES
+ * that every GPU loading the library keeps until the process exits; requests
+ * needing more (see bergson_project_grads_workspace) fail with
+ * BERGSON_EWORKSPACE and enqueue nothing.  No allocation of any kind happens.
+ * All calls share the one array: calls that overlap on the GPU (e.g. on two
+ * streams) race and must be ordered by the caller.  The first call on each
+ * device looks up the array's device address; make that first call before any
+ * stream capture begins.
+ */
+#define BERGSON_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+BERGSON_API int bergson_project_grads_noalloc(const bergson_layer* layers, int n_layers,
+                                              int64_t B, int64_t T, const uint8_t* mask,
+                                              float* out, int64_t ld_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -36,7 +36,7 @@ EXPORTED = (
     "bergson_project_grads_workspace", "bergson_project_grads", "bergson_build_store",
     "bergson_score_topk_workspace", "bergson_score_topk", "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
-    "bergson_debug_wait_probe", "bergson_debug_inject_status",
+    "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_project_grads_noalloc",
 )
 
 
@@ -86,6 +86,7 @@ def lib() -> ctypes.CDLL:
         "bergson_version": (i32, []),
         "bergson_debug_wait_probe": (i32, [u64, vp]),
         "bergson_debug_inject_status": (None, [i32, i32]),
+        "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -166,6 +167,15 @@ def bergson_project_grads(layers: Sequence, B: int, T: int, mask, out, workspace
     ws_bytes = workspace.numel() * workspace.element_size()
     _check(lib().bergson_project_grads(arr, len(layers), int(B), int(T), _ptr(mask), _ptr(out), ld,
                                        _ptr(workspace), ws_bytes, _stream(stream)))
+
+
+def bergson_project_grads_noalloc(layers: Sequence, B: int, T: int, mask, out, stream=None,
+                                  ld_out: Optional[int] = None) -> None:
+    """Like bergson_project_grads, but on the library's fixed static scratch (no workspace)."""
+    arr = _layer_array(layers)
+    ld = int(out.stride(0)) if ld_out is None else int(ld_out)
+    _check(lib().bergson_project_grads_noalloc(arr, len(layers), int(B), int(T), _ptr(mask),
+                                               _ptr(out), ld, _stream(stream)))
 
 
 def bergson_build_store(proj, B: int, K: int, unit_normalize: bool, store, row_offset: int,

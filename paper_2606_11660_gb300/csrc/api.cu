@@ -313,6 +313,17 @@ int validate_score(const void* store, int64_t N, int64_t K, int64_t ld_store, co
 }
 
 }  // namespace
+
+int record_error(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
 }  // namespace bergson
 
 using namespace bergson;

@@ -73,6 +73,9 @@ struct ScoreParams {
   uint64_t timeout_ns;
 };
 
+// Sets this thread's bergson_last_error() message (printf format) and returns `code`.
+int record_error(int code, const char* fmt, ...);
+
 // ---- launchers (return the launch error, if any) ----
 
 cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t total, cudaStream_t s);
