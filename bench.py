@@ -403,7 +403,7 @@ def bench_scoring(args, world, dev, peaks, peak_kind):
                      "traffic": profiled_traffic("score_kernel_score4m.md", "score.cu"),
                      "peak_source": f"{peak_kind} bf16_tflops (fp16 dense runs at the bf16 rate)",
                      "hbm_gbs_achieved": round(N * K * 2 / (ms * 1e-3) / 1e9, 1)},
-        "gpu_launches": 3 * args.score_steps,   # query norm, score, merge
+        "gpu_launches": 5 * args.score_steps,   # query norm, 2 x (score, merge): prefix + full
         "clocks": sampler.summary(w0, w1),
     }
     del store

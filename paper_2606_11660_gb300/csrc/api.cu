@@ -23,6 +23,8 @@ constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 
 constexpr int kSchedTargetItems = 2048;              // work items per projection launch (target)
 constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
 constexpr int kMaxDevices = 64;
+constexpr int64_t kPrefixRowsPerTopk = 512;          // prefix pass: 512 * topk store rows
+constexpr int64_t kPrefixMinFactor = 8;              // ... only when N >= 8 * prefix
 
 __device__ int g_status_word;                        // device status word (one per device)
 
@@ -137,7 +139,8 @@ struct ProjLayout {
 
 int validate_layers(const bergson_layer* layers, int n_layers, int64_t B, int64_t T) {
   if (layers == nullptr) return fail(BERGSON_EINVAL, "layers is NULL");
-  if (n_layers < 1) return fail(BERGSON_EINVAL, "n_layers must be >= 1 (got %d)", n_layers);
+  if (n_layers < 1 || n_layers > 16384)
+    return fail(BERGSON_EINVAL, "n_layers must be in [1, 16384] (got %d)", n_layers);
   if (B < 0 || T < 0) return fail(BERGSON_EINVAL, "B and T must be >= 0 (B=%lld T=%lld)",
                                   (long long)B, (long long)T);
   if (B > (1ll << 30) || T > (1ll << 30) || B * T > (1ll << 37))
@@ -254,7 +257,7 @@ CUresult encode_act(CUtensorMap* tm, const void* ptr, int64_t d, int64_t T, int6
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(T),
                         static_cast<cuuint64_t>(B)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(d * 2), static_cast<cuuint64_t>(T * d * 2)};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(kChunk), static_cast<cuuint32_t>(kTileTokens), 1};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kChunk), 32, 1};   // 32-token slices
   cuuint32_t es[3] = {1, 1, 1};
   return encode_fn()(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims,
                      strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -391,7 +394,7 @@ int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, 
   std::vector<uint8_t> staging(L.tv_off, 0);
   ModDesc* mods = reinterpret_cast<ModDesc*>(staging.data() + L.mods_off);
   PrepSeg* segs = reinterpret_cast<PrepSeg*>(staging.data() + L.segs_off);
-  int64_t flat = 0;
+  int64_t max_pairs = 0;
   for (int i = 0; i < n_layers; ++i) {
     const bergson_layer& ly = layers[i];
     ModDesc& md = mods[L.mod_slot[i]];
@@ -415,27 +418,27 @@ int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, 
     si.seed = ly.seed_in;
     si.moment = ly.c;
     si.dst = pin;
-    si.begin = flat;
+    si.begin = 0;
     si.d = static_cast<int32_t>(ly.d_in);
     si.k = static_cast<int32_t>(ly.k_in);
     si.kind = ly.proj_kind;
-    flat += ly.d_in * ly.k_in;
+    max_pairs = std::max<int64_t>(max_pairs, ly.d_in * ly.k_in / 2);
     PrepSeg& so = segs[2 * i + 1];
     so.seed = ly.seed_out;
     so.moment = ly.r;
     so.dst = pout;
-    so.begin = flat;
+    so.begin = 0;
     so.d = static_cast<int32_t>(ly.d_out);
     so.k = static_cast<int32_t>(ly.k_out);
     so.kind = ly.proj_kind;
-    flat += ly.d_out * ly.k_out;
+    max_pairs = std::max<int64_t>(max_pairs, ly.d_out * ly.k_out / 2);
   }
   cudaError_t e = cudaMemcpyAsync(ws, staging.data(), staging.size(), cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return fail_cuda(e, "staging copy");
   const ModDesc* mods_dev = reinterpret_cast<const ModDesc*>(ws + L.mods_off);
   const bool need_tiles = T > 0;
   if (need_tiles) {
-    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, flat, s);
+    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, max_pairs, s);
     if (e != cudaSuccess) return fail_cuda(e, "prep launch");
   }
   uint8_t* tile_valid = nullptr;
@@ -559,29 +562,37 @@ int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store
   const int sms = std::max(1, std::min(sm_count(dg.dev), kMaxScoreCTAs));
   const int gsize = L.qt * kScoreQT;
   const int n_qg_total = static_cast<int>((Q + gsize - 1) / gsize);
-  const int n_ntiles = static_cast<int>((N + kScoreBN - 1) / kScoreBN);
+  // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
+  // lands in the outputs, and its k-th score seeds the full pass's threshold.
+  const int64_t prefix = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
+  const bool use_prefix = N >= kPrefixMinFactor * prefix;
   for (int pass = 0; pass < n_qg_total; pass += sms) {
     const int n_qg = std::min(sms, n_qg_total - pass);
-    const int cpg = std::max(1, std::min(sms / n_qg, n_ntiles));
-    const int grid = n_qg * cpg;
-    ScoreParams p;
-    p.N = static_cast<int>(N);
-    p.K = static_cast<int>(K);
-    p.Q = static_cast<int>(Q);
-    p.topk = static_cast<int>(topk);
-    p.n_qg = n_qg;
-    p.qg_base = pass;
-    p.n_ntiles = n_ntiles;
-    p.heaps = heaps;
-    p.status = status;
-    p.timeout_ns = kWaitTimeoutNs;
-    e = launch_score(L.qt, tm_store, tm_q, p, grid, s);
-    if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
     const int q_begin = pass * gsize;
     const int q_end = static_cast<int>(std::min<int64_t>(Q, static_cast<int64_t>(pass + n_qg) * gsize));
-    e = launch_merge(heaps, grid, n_qg, L.qt, static_cast<int>(topk), q_begin, q_end, pass,
-                     out_scores, out_idx, s);
-    if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
+    for (int stage = use_prefix ? 0 : 1; stage < 2; ++stage) {
+      const int64_t rows = stage == 0 ? prefix : N;
+      const int nt = static_cast<int>((rows + kScoreBN - 1) / kScoreBN);
+      const int cpg = std::max(1, std::min(sms / n_qg, nt));
+      const int grid = n_qg * cpg;
+      ScoreParams p;
+      p.N = static_cast<int>(rows);
+      p.K = static_cast<int>(K);
+      p.Q = static_cast<int>(Q);
+      p.topk = static_cast<int>(topk);
+      p.n_qg = n_qg;
+      p.qg_base = pass;
+      p.n_ntiles = nt;
+      p.heaps = heaps;
+      p.tau0 = stage == 1 && use_prefix ? out_scores : nullptr;
+      p.status = status;
+      p.timeout_ns = kWaitTimeoutNs;
+      e = launch_score(L.qt, tm_store, tm_q, p, grid, s);
+      if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
+      e = launch_merge(heaps, grid, n_qg, L.qt, static_cast<int>(topk), q_begin, q_end, pass,
+                       out_scores, out_idx, s);
+      if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
+    }
   }
   return BERGSON_OK;
 }

@@ -19,8 +19,8 @@ constexpr int kMaxTopk = 1024;
 // Per-module launch record kept in workspace (global memory).  The tensor maps
 // are read by TMA straight from there, so the record is 64-byte aligned.
 struct ModDesc {
-  CUtensorMap tmA;      // bf16 {d_in, T, B}, box {64, 128, 1}, 128B swizzle
-  CUtensorMap tmG;      // bf16 {d_out, T, B}, box {64, 128, 1}, 128B swizzle
+  CUtensorMap tmA;      // bf16 {d_in, T, B}, box {64, 32, 1}, 128B swizzle
+  CUtensorMap tmG;      // bf16 {d_out, T, B}, box {64, 32, 1}, 128B swizzle
   CUtensorMap tmPin;    // bf16 {d_in, 2 k_in} (hi rows then lo rows), box {64, 2 k_in}
   CUtensorMap tmPout;   // bf16 {d_out, 2 k_out}, box {64, 2 k_out}
   int32_t d_in;
@@ -36,7 +36,7 @@ struct PrepSeg {
   uint64_t seed;
   const float* moment;      // r (output side) or c (input side), or nullptr
   __nv_bfloat16* dst;       // [2k, d]
-  int64_t begin;            // first flat element of this segment (d*k elements)
+  int64_t begin;            // unused (kept zero)
   int32_t d;
   int32_t k;
   int32_t kind;
@@ -53,7 +53,7 @@ struct ProjParams {
   int n_chunks;         // work items per (module, example)
   int n_items;          // n_mods * B * n_chunks
   const uint8_t* mask;        // [B, T] or nullptr
-  const uint8_t* tile_valid;  // [B, n_tiles] or nullptr
+  const uint8_t* tile_valid;  // [B, n_tiles] 4-bit masks of valid 32-token slices, or nullptr
   float* partials;            // [n_items, k_out * k_in]
   int* counter;               // dynamic scheduler, zero on entry
   int* status;                // device status word
@@ -69,6 +69,7 @@ struct ScoreParams {
   int qg_base;          // first query group of this pass
   int n_ntiles;         // ceil(N / 256)
   unsigned long long* heaps;  // [grid, topk, QT*128]
+  const float* tau0;    // per query starting threshold at tau0[q * topk + topk - 1], or nullptr
   int* status;
   uint64_t timeout_ns;
 };
@@ -78,7 +79,7 @@ int record_error(int code, const char* fmt, ...);
 
 // ---- launchers (return the launch error, if any) ----
 
-cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t total, cudaStream_t s);
+cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, cudaStream_t s);
 cudaError_t launch_projection_matrix(uint64_t seed, int d, int k, int kind, const float* moment,
                                      float* out, cudaStream_t s);
 cudaError_t launch_tile_valid(const uint8_t* mask, int B, int T, int n_tiles, uint8_t* tile_valid,

@@ -28,9 +28,9 @@ __device__ __forceinline__ uint64_t mix64(uint64_t x) {
   return x ^ (x >> 31);
 }
 
-// Standard normal draw number `e` of stream `seed`.
-__device__ __forceinline__ float gaussian_draw(uint64_t seed, uint64_t e) {
-  const uint64_t p = e >> 1;
+// The two standard normal draws of pair `p` of stream `seed`: counter 2p takes
+// the cosine branch (*zc), counter 2p + 1 the sine branch (*zs).
+__device__ __forceinline__ void gaussian_pair(uint64_t seed, uint64_t p, float* zc, float* zs) {
   const uint64_t h1 = mix64(seed ^ mix64(2 * p));
   const uint64_t h2 = mix64(seed ^ mix64(2 * p + 1));
   const uint64_t n1 = (h1 >> 11) + 1;            // u1 = n1 * 2^-53 in (0, 1]
@@ -45,55 +45,71 @@ __device__ __forceinline__ float gaussian_draw(uint64_t seed, uint64_t e) {
   const float two_u2 = static_cast<float>(h2 >> 11) * 0x1p-52f;   // 2 u2 in [0, 2)
   float s, c;
   sincospif(two_u2, &s, &c);                                       // angle 2 pi u2
-  return (e & 1) ? rho * s : rho * c;
+  *zc = rho * c;
+  *zs = rho * s;
 }
 
-// Entry (i, j) of P' = diag(scale) P, fp32.
-__device__ __forceinline__ float projection_entry(uint64_t seed, int i, int j, int k, int kind,
-                                                  const float* moment) {
-  float v;
+// Entries (i, j) and (i, j + 1), j even, of P' = diag(scale) P, fp32.  They
+// are counters e = i*k + j and e + 1, i.e. both draws of pair e / 2.
+__device__ __forceinline__ void projection_pair(uint64_t seed, int i, int j, int k, int kind,
+                                                const float* moment, float* v0, float* v1) {
   if (kind == 1) {
-    v = (i == j) ? 1.0f : 0.0f;
+    *v0 = (i == j) ? 1.0f : 0.0f;
+    *v1 = (i == j + 1) ? 1.0f : 0.0f;
   } else {
     const float inv_sqrt_k = 1.0f / sqrtf(static_cast<float>(k));
-    v = gaussian_draw(seed, static_cast<uint64_t>(i) * k + j) * inv_sqrt_k;
+    float zc, zs;
+    gaussian_pair(seed, (static_cast<uint64_t>(i) * k + j) >> 1, &zc, &zs);
+    *v0 = zc * inv_sqrt_k;
+    *v1 = zs * inv_sqrt_k;
   }
-  if (moment != nullptr) v = v * (1.0f / sqrtf(moment[i]));
-  return v;
+  if (moment != nullptr) {
+    const float sc = 1.0f / sqrtf(moment[i]);
+    *v0 = *v0 * sc;
+    *v1 = *v1 * sc;
+  }
 }
 
-__global__ void prep_kernel(const PrepSeg* __restrict__ segs, int n_segs, int64_t total) {
-  for (int64_t f = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; f < total;
-       f += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    int lo = 0, hi = n_segs - 1;               // last segment with begin <= f
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (segs[mid].begin <= f) lo = mid; else hi = mid - 1;
-    }
-    const PrepSeg& sg = segs[lo];
-    const int64_t local = f - sg.begin;        // ordered (j, i): i fastest for coalesced stores
-    const int i = static_cast<int>(local % sg.d);
-    const int j = static_cast<int>(local / sg.d);
-    const float v = projection_entry(sg.seed, i, j, sg.k, sg.kind, sg.moment);
-    const __nv_bfloat16 h = __float2bfloat16_rn(v);
-    const __nv_bfloat16 l = __float2bfloat16_rn(v - __bfloat162float(h));
-    sg.dst[static_cast<int64_t>(j) * sg.d + i] = h;
-    sg.dst[static_cast<int64_t>(sg.k + j) * sg.d + i] = l;
+__device__ __forceinline__ void store_hi_lo(__nv_bfloat16* dst, int64_t hi_idx, int64_t lo_idx,
+                                            float v) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(v);
+  dst[hi_idx] = h;
+  dst[lo_idx] = __float2bfloat16_rn(v - __bfloat162float(h));
+}
+
+// blockIdx.y = segment; threads walk the segment's d*k/2 entry pairs with the
+// input index i fastest, so the transposed bf16 stores are coalesced.
+__global__ void prep_kernel(const PrepSeg* __restrict__ segs) {
+  const PrepSeg sg = segs[blockIdx.y];
+  const int64_t npairs = static_cast<int64_t>(sg.d) * sg.k / 2;
+  for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < npairs;
+       q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int i = static_cast<int>(q % sg.d);
+    const int j = 2 * static_cast<int>(q / sg.d);
+    float v0, v1;
+    projection_pair(sg.seed, i, j, sg.k, sg.kind, sg.moment, &v0, &v1);
+    const int64_t d = sg.d;
+    store_hi_lo(sg.dst, j * d + i, (sg.k + j) * d + i, v0);
+    store_hi_lo(sg.dst, (j + 1) * d + i, (sg.k + j + 1) * d + i, v1);
   }
 }
 
 __global__ void projection_matrix_kernel(uint64_t seed, int d, int k, int kind,
                                          const float* __restrict__ moment, float* __restrict__ out) {
-  const int64_t n = static_cast<int64_t>(d) * k;
-  for (int64_t f = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; f < n;
-       f += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int i = static_cast<int>(f / k);
-    const int j = static_cast<int>(f % k);
-    out[f] = projection_entry(seed, i, j, k, kind, moment);
+  const int64_t npairs = static_cast<int64_t>(d) * k / 2;
+  for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < npairs;
+       q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int i = static_cast<int>((2 * q) / k);
+    const int j = static_cast<int>((2 * q) % k);
+    float v0, v1;
+    projection_pair(seed, i, j, k, kind, moment, &v0, &v1);
+    out[2 * q] = v0;
+    out[2 * q + 1] = v1;
   }
 }
 
-// tile_valid[b, t] = 1 if any token of 128-token tile t of example b is valid.
+// tile_valid[b, t] bit q (q = 0..3) = 1 if any token of the 32-token slice
+// [128 t + 32 q, 128 t + 32 q + 32) of example b is valid.  One warp per tile.
 __global__ void tile_valid_kernel(const uint8_t* __restrict__ mask, int B, int T, int n_tiles,
                                   uint8_t* __restrict__ tile_valid) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -101,11 +117,14 @@ __global__ void tile_valid_kernel(const uint8_t* __restrict__ mask, int B, int T
   if (warp >= B * n_tiles) return;
   const int b = warp / n_tiles;
   const int t0 = (warp % n_tiles) * kTileTokens;
-  int any = 0;
-  for (int t = t0 + lane; t < min(T, t0 + kTileTokens); t += 32)
-    any |= mask[static_cast<int64_t>(b) * T + t] != 0;
-  any = __any_sync(0xffffffffu, any);
-  if (lane == 0) tile_valid[warp] = any ? 1 : 0;
+  uint32_t bits = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int t = t0 + 32 * q + lane;
+    const int v = t < T && mask[static_cast<int64_t>(b) * T + t] != 0;
+    if (__any_sync(0xffffffffu, v)) bits |= 1u << q;
+  }
+  if (lane == 0) tile_valid[warp] = static_cast<uint8_t>(bits);
 }
 
 // Waits on an mbarrier that nothing completes; exercises the timeout path.
@@ -121,20 +140,21 @@ __global__ void wait_probe_kernel(int* status, uint64_t timeout_ns) {
   }
 }
 
-cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t total, cudaStream_t s) {
-  if (total <= 0) return cudaSuccess;
+cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, cudaStream_t s) {
+  if (n_segs <= 0 || max_pairs <= 0) return cudaSuccess;
   const int threads = 256;
-  const int64_t blocks = (total + threads - 1) / threads;
-  prep_kernel<<<static_cast<unsigned>(blocks < 65535 * 8 ? blocks : 65535 * 8), threads, 0, s>>>(
-      segs, n_segs, total);
+  int64_t bx = (max_pairs + threads - 1) / threads;
+  if (bx > 4096) bx = 4096;
+  prep_kernel<<<dim3(static_cast<unsigned>(bx), static_cast<unsigned>(n_segs)), threads, 0, s>>>(
+      segs);
   return cudaGetLastError();
 }
 
 cudaError_t launch_projection_matrix(uint64_t seed, int d, int k, int kind, const float* moment,
                                      float* out, cudaStream_t s) {
-  const int64_t n = static_cast<int64_t>(d) * k;
+  const int64_t npairs = static_cast<int64_t>(d) * k / 2;
   const int threads = 256;
-  const int64_t blocks = (n + threads - 1) / threads;
+  const int64_t blocks = (npairs + threads - 1) / threads;
   projection_matrix_kernel<<<static_cast<unsigned>(blocks < 65535 ? blocks : 65535), threads, 0,
                              s>>>(seed, d, k, kind, moment, out);
   return cudaGetLastError();

@@ -5,7 +5,8 @@
 // For one module and example b the projected gradient is
 //   G^_b = P_out'^T (sum_t m_t g_t a_t^T) P_in' = sum_t m_t (P_out'^T g_t)(P_in'^T a_t)^T,
 // so the kernel never forms the d_out x d_in gradient.  Per 128-token tile:
-//   1. TMA streams 128 x 64 bf16 boxes of A and G (128-byte swizzle) and the
+//   1. TMA streams A and G in 32-token x 64-column bf16 boxes (128-byte
+//      swizzle; slices whose 32 tokens are all masked are not read) and the
 //      matching 64-column slices of P'^T (hi and lo bf16 rows) into a ring of
 //      shared-memory stages;
 //   2. one thread issues tcgen05.mma (M = 128 tokens, N = k, K = 16) into TMEM:
@@ -28,7 +29,8 @@ namespace bergson {
 
 namespace {
 
-constexpr int kActBoxBytes = kTileTokens * 128;       // 128 rows x 64 bf16
+constexpr int kActBoxBytes = kTileTokens * 128;       // 128 rows x 64 bf16 (one tile)
+constexpr int kSliceBytes = 32 * 128;                 // one 32-token TMA box
 constexpr int kSmemBudget = 232448;                   // 227 KB opt-in per CTA
 constexpr uint64_t kDrainTimeoutNs = 2000000000ull;   // waits for own copies after an abort
 
@@ -72,16 +74,36 @@ __device__ __forceinline__ ItemCoord decode_item(const ProjParams& p, int item) 
   return c;
 }
 
+// Valid 32-token slices of the NT tiles starting at tile g: bit 4*nt + q is set
+// when slice q of tile g + nt (inside the item) holds a valid token.  Without a
+// mask a slice is valid when it starts before T.
 template <int NT>
-__device__ __forceinline__ uint32_t group_valid(const ProjParams& p, int b, int g, int t_end) {
+__device__ __forceinline__ uint32_t group_slices(const ProjParams& p, int b, int g, int t_end) {
   uint32_t vm = 0;
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
     const int t = g + nt;
-    if (t < t_end && (p.tile_valid == nullptr || p.tile_valid[b * p.n_tiles + t] != 0))
-      vm |= 1u << nt;
+    if (t >= t_end) continue;
+    uint32_t q4;
+    if (p.tile_valid != nullptr) {
+      q4 = p.tile_valid[b * p.n_tiles + t] & 0xFu;
+    } else {
+      const int left = p.T - t * kTileTokens;          // > 0 inside the item
+      q4 = left >= kTileTokens ? 0xFu : (1u << ((left + 31) / 32)) - 1u;
+    }
+    vm |= q4 << (4 * nt);
   }
   return vm;
+}
+
+// Tiles (bit nt) that have at least one valid slice.
+template <int NT>
+__device__ __forceinline__ uint32_t tiles_of(uint32_t slices) {
+  uint32_t tm = 0;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt)
+    if ((slices >> (4 * nt)) & 0xFu) tm |= 1u << nt;
+  return tm;
 }
 
 template <int KI, int KO>
@@ -159,9 +181,9 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         tmap_acquire(&md->tmPin);
         tmap_acquire(&md->tmPout);
         for (int g = ic.t_begin; g < ic.t_end && ok; g += NT) {
-          const uint32_t vm = group_valid<NT>(p, ic.b, g, ic.t_end);
-          if (vm == 0) continue;
-          const uint32_t act_bytes = __popc(vm) * kActBoxBytes;
+          const uint32_t sl = group_slices<NT>(p, ic.b, g, ic.t_end);
+          if (sl == 0) continue;
+          const uint32_t act_bytes = __popc(sl) * kSliceBytes;
           for (int side = 0; side < 2 && ok; ++side) {
             const void* tact = side ? static_cast<const void*>(&md->tmG) : &md->tmA;
             const void* tp = side ? static_cast<const void*>(&md->tmPout) : &md->tmPin;
@@ -174,10 +196,10 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
               mbar_arrive_expect_tx(fb, act_bytes + pbytes);
               const uint32_t dst = sbase + stage * C::kStageBytes;
 #pragma unroll
-              for (int nt = 0; nt < NT; ++nt)
-                if (vm >> nt & 1)
-                  tma_load_3d_hint(dst + nt * kActBoxBytes, tact, fb, ch * kChunk,
-                                   (g + nt) * kTileTokens, ic.b, pol_act);
+              for (int x = 0; x < 4 * NT; ++x)
+                if (sl >> x & 1)
+                  tma_load_3d_hint(dst + x * kSliceBytes, tact, fb, ch * kChunk,
+                                   g * kTileTokens + 32 * x, ic.b, pol_act);
               tma_load_2d_hint(dst + NT * kActBoxBytes, tp, fb, ch * kChunk, 0, pol_p);
               issued |= 1u << stage;
               issued_par = (issued_par & ~(1u << stage)) | (ph << stage);
@@ -215,7 +237,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         const ItemCoord ic = decode_item(p, item);
         const ModDesc* md = p.mods + ic.m;
         for (int g = ic.t_begin; g < ic.t_end && ok; g += NT) {
-          const uint32_t vm = group_valid<NT>(p, ic.b, g, ic.t_end);
+          const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
           if (vm == 0) continue;
           if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
           tc_fence_after();
@@ -288,7 +310,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       for (int x = 0; x < OPT; ++x) acc[x] = 0.0f;
       bool aborted = false;
       for (int g = ic.t_begin; g < ic.t_end; g += NT) {
-        const uint32_t vm = group_valid<NT>(p, ic.b, g, ic.t_end);
+        const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
         if (vm == 0) continue;
         if (et == 0) {
           if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))

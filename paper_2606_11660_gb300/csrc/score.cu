@@ -13,6 +13,9 @@
 // Merge kernel: one CTA per query sorts the heaps of the CTAs that covered the
 // query (bitonic sort of 64-bit keys in shared memory) and writes the final
 // top-k ordered by score descending, then row ascending.
+// Large stores are scored twice: first a prefix of 512*topk rows, whose exact
+// per-query k-th best is a lower bound of the final k-th best; the full pass
+// then starts with that threshold, so few scores ever reach the heaps.
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -26,14 +29,25 @@ constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
 constexpr int kStoreBoxBytes = kScoreBN * 128;      // 256 rows x 64 fp16
 constexpr int kQBoxBytes = kScoreQT * 128;          // 128 rows x 64 fp16
 constexpr unsigned long long kSentinelKey = 0x007FFFFF00000000ull;   // (-inf, row 0xFFFFFFFF)
+// The first CTA of each group of CTAs that share store tiles pulls store chunks
+// into L2 this many chunks ahead of its own loads, so the shared-memory ring
+// sees L2 rather than DRAM latency (0 = no prefetch).
+constexpr int kStorePrefetchChunks = 0;
+// L2 policy of store-chunk loads: 0 = evict_normal, 1 = evict_first.
+constexpr int kStoreEvictFirst = 1;
+
+// Candidates a lane may park in shared memory per tile before inserting them
+// into its heap after the tile's TMEM buffer is released.
+constexpr int kQueueCap = 8;
 
 template <int QT>
 struct ScoreCfg {
   static constexpr int kStageBytes = kStoreBoxBytes + QT * kQBoxBytes;
   static constexpr int kBarBytes = 256;
-  static constexpr int kStagesFit = (kSmemBudget - 1024 - kBarBytes) / kStageBytes;
+  static constexpr int kQueueBytes = kQueueCap * QT * 128 * 8;
+  static constexpr int kStagesFit = (kSmemBudget - 1024 - kBarBytes - kQueueBytes) / kStageBytes;
   static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kBarBytes;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kQueueBytes + kBarBytes;
   static constexpr int kNBuf = 512 / (QT * kScoreBN);   // TMEM accumulator buffers
   static constexpr int kEpiThreads = QT * 128;
   static constexpr int kThreads = 64 + kEpiThreads;
@@ -55,25 +69,48 @@ __device__ __forceinline__ unsigned long long make_key(float s, uint32_t row) {
   return (static_cast<unsigned long long>(float_order(s)) << 32) | static_cast<uint32_t>(~row);
 }
 
-// Replace the root (worst kept entry) of a min-heap of `k` keys stored at
-// base[e * stride] and restore the heap property.
+// Children per node of the per-query min-heaps (a wider heap is shallower:
+// fewer dependent global-memory round trips per insertion).
+constexpr int kHeapArity = 4;
+
+// Replace the root (worst kept entry) of a kHeapArity-ary min-heap of `k` keys
+// stored at base[e * stride] and restore the heap property.  The children of
+// one node are loaded together, so each level costs one memory round trip.
 __device__ __forceinline__ void heap_replace_root(unsigned long long* base, int stride, int k,
                                                   unsigned long long key) {
   int i = 0;
   for (;;) {
-    const int l = 2 * i + 1;
-    if (l >= k) break;
-    int c = l;
-    unsigned long long kc = base[static_cast<int64_t>(l) * stride];
-    if (l + 1 < k) {
-      const unsigned long long kr = base[static_cast<int64_t>(l + 1) * stride];
-      if (kr < kc) { c = l + 1; kc = kr; }
+    const int c0 = kHeapArity * i + 1;
+    if (c0 >= k) break;
+    unsigned long long kc = base[static_cast<int64_t>(c0) * stride];
+    int c = c0;
+#pragma unroll
+    for (int t = 1; t < kHeapArity; ++t) {
+      if (c0 + t < k) {
+        const unsigned long long kt = base[static_cast<int64_t>(c0 + t) * stride];
+        if (kt < kc) { kc = kt; c = c0 + t; }
+      }
     }
     if (kc >= key) break;
     base[static_cast<int64_t>(i) * stride] = kc;
     i = c;
   }
   base[static_cast<int64_t>(i) * stride] = key;
+}
+
+// v[pos] for a run-time pos in [0, 32) without dynamic register indexing
+// (a 5-level select tree keeps v in registers).
+__device__ __forceinline__ float select32(const float* v, uint32_t pos) {
+  float t16[16], t8[8], t4[4], t2[2];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) t16[i] = (pos & 16u) ? v[i + 16] : v[i];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) t8[i] = (pos & 8u) ? t16[i + 8] : t16[i];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) t4[i] = (pos & 4u) ? t8[i + 4] : t8[i];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) t2[i] = (pos & 2u) ? t4[i + 2] : t4[i];
+  return (pos & 1u) ? t2[1] : t2[0];
 }
 
 template <int QT>
@@ -85,7 +122,9 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes);
+  unsigned long long* cand_queue =
+      reinterpret_cast<unsigned long long*>(smem + C::kStages * C::kStageBytes);  // [cap][lanes]
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes + C::kQueueBytes);
   uint64_t* empty = full + C::kStages;
   uint64_t* tfull = empty + C::kStages;       // [kNBuf]
   uint64_t* tempty = tfull + 2;               // [kNBuf]
@@ -129,14 +168,28 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
     if (lane == 0) {
       prefetch_tmap(&tm_store);
       prefetch_tmap(&tm_q);
-      const uint64_t pol_store = policy_evict_first();
+      const uint64_t pol_store = kStoreEvictFirst ? policy_evict_first() : policy_evict_normal();
       const uint64_t pol_q = policy_evict_last();
+      const bool prefetcher = kStorePrefetchChunks > 0 && g_local == 0;
+      const int my_tiles = nt0 < p.n_ntiles ? (p.n_ntiles - nt0 + cpg - 1) / cpg : 0;
+      const int64_t my_chunks = static_cast<int64_t>(my_tiles) * nK;
+      if (prefetcher) {
+        for (int64_t c = 0; c < kStorePrefetchChunks && c < my_chunks; ++c)
+          tma_prefetch_l2_2d(&tm_store, static_cast<int>(c % nK) * kChunk,
+                             (nt0 + static_cast<int>(c / nK) * cpg) * kScoreBN);
+      }
       int stage = 0;
       uint32_t ph = 0;
       uint32_t issued = 0, issued_par = 0;
       bool ok = true;
+      int64_t lin = 0;                       // this CTA's chunk counter
       for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
-        for (int kc = 0; kc < nK; ++kc) {
+        for (int kc = 0; kc < nK; ++kc, ++lin) {
+          if (prefetcher && lin + kStorePrefetchChunks < my_chunks) {
+            const int64_t c = lin + kStorePrefetchChunks;
+            tma_prefetch_l2_2d(&tm_store, static_cast<int>(c % nK) * kChunk,
+                               (nt0 + static_cast<int>(c / nK) * cpg) * kScoreBN);
+          }
           if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_arrive_expect_tx(fb, C::kStageBytes);
@@ -205,7 +258,14 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
         p.heaps + static_cast<int64_t>(blockIdx.x) * p.topk * stride + slot;
     for (int e = 0; e < p.topk; ++e) heap[static_cast<int64_t>(e) * stride] = kSentinelKey;
     unsigned long long tau_key = kSentinelKey;
-    float tau = -INFINITY;
+    // Scores below the k-th best of any subset of the rows can never reach the
+    // final top-k, so a threshold from a prefix pass (if any) filters from the start.
+    const int q_global = (g * QT + qt) * kScoreQT + 32 * quarter + lane;
+    const float tau0 = (p.tau0 != nullptr && q_global < p.Q)
+                           ? p.tau0[static_cast<int64_t>(q_global) * p.topk + p.topk - 1]
+                           : -INFINITY;
+    float tau = tau0;
+    int nq = 0;                                       // parked candidates of this lane
     int ab = 0;
     uint32_t aph = 0;
     for (int nt = nt0; nt < p.n_ntiles; nt += cpg) {
@@ -226,19 +286,26 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
         tmem_ld32(tbase + c * 32, v);
         const int r0 = row_base + c * 32;
         const int nvalid = min(32, p.N - r0);
-        float mx = -INFINITY;
+        // Candidate positions of this lane (the comparison also drops NaN).
+        uint32_t cand = 0;
 #pragma unroll
         for (int j = 0; j < 32; ++j)
-          if (j < nvalid) mx = fmaxf(mx, v[j]);
-        if (mx >= tau) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            if (j < nvalid && v[j] >= tau) {         // the comparison also drops NaN
-              const unsigned long long key = make_key(v[j], static_cast<uint32_t>(r0 + j));
-              if (key > tau_key) {
+          if (j < nvalid && v[j] >= tau) cand |= 1u << j;
+        // Warp-uniform rounds: in round r every lane inserts its r-th candidate,
+        // so a warp pays for its busiest lane, not for every distinct column.
+        while (__any_sync(0xffffffffu, cand != 0)) {
+          if (cand != 0) {
+            const uint32_t pos = __ffs(cand) - 1;
+            cand &= cand - 1;
+            const unsigned long long key = make_key(select32(v, pos), static_cast<uint32_t>(r0) + pos);
+            if (key > tau_key) {
+              if (nq < kQueueCap) {                 // park it; inserted after TMEM is released
+                cand_queue[nq * stride + slot] = key;
+                ++nq;
+              } else {                              // queue full: insert now
                 heap_replace_root(heap, stride, p.topk, key);
                 tau_key = heap[0];
-                tau = order_to_float(static_cast<uint32_t>(tau_key >> 32));
+                tau = fmaxf(tau0, order_to_float(static_cast<uint32_t>(tau_key >> 32)));
               }
             }
           }
@@ -248,6 +315,19 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
       if (++ab == C::kNBuf) { ab = 0; aph ^= 1; }
+      // The MMA warp is already filling TMEM for the next tile; drain the parked
+      // candidates meanwhile (warp-uniform rounds, as above).
+      while (__any_sync(0xffffffffu, nq > 0)) {
+        if (nq > 0) {
+          --nq;
+          const unsigned long long key = cand_queue[nq * stride + slot];
+          if (key > tau_key) {
+            heap_replace_root(heap, stride, p.topk, key);
+            tau_key = heap[0];
+            tau = fmaxf(tau0, order_to_float(static_cast<uint32_t>(tau_key >> 32)));
+          }
+        }
+      }
       named_bar_sync(1, C::kEpiThreads);   // keeps the stop broadcast single-writer
     }
   }

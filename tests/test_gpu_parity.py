@@ -223,6 +223,26 @@ def test_score_topk_random(N, K, Q, topk):
     check_topk(s, i, S, topk)
 
 
+@pytest.mark.parametrize("Q,topk", [(130, 5), (40, 3)])
+def test_score_prefix_threshold_pass(Q, topk):
+    # N >= 8 * 512 * topk: the scorer first takes the exact top-k of a prefix of
+    # the store and starts the full pass from its k-th score.
+    N, K = 30_000, 256
+    g = wl.generator(Q * 7 + topk, "cpu")
+    rows = torch.randn((N, K), generator=g)
+    queries = torch.randn((Q, K), generator=g)
+    rows[N - 5:] = rows[:5]                  # exact ties across the prefix boundary
+    queries[:5] = rows[:5]
+    rows[100:100 + Q] = queries + 0.3 * torch.randn((Q, K), generator=g)   # strong prefix hits
+    rows[N - 200:N - 200 + 20] = queries[:20] * 2.0 + torch.randn((20, K), generator=g)
+    store = _store_from_rows(rows)
+    s, i = _score(store, queries.to(DEV), topk)
+    S = orc.cosine_scores(store.cpu().numpy(), queries.numpy().astype(np.float64))
+    check_topk(s, i, S, topk)
+    for r in range(5):
+        assert set(i[r, :2].tolist()) == {r, N - 5 + r}
+
+
 def test_score_ties_prefer_lower_index():
     g = wl.generator(3, "cpu")
     base = torch.randn((50, 256), generator=g)
