@@ -436,11 +436,14 @@ def profile_case(args):
             bg.bergson_project_grads(layers, B, cfg.T, mask, out, ws)
         st = bg.bergson_sync_status()
     else:
-        # 262,144-row fp16 store x 8192 (4.3 GB), 1024 queries, top-100
-        N, K, Q, topk = 1 << 18, 8192, 1024, 100
+        # 409,600-row fp16 store x 8192 (6.7 GB, large enough for the prefix
+        # threshold pass), 1024 queries, top-100
+        N, K, Q, topk = 409_600, 8192, 1024, 100
         store = torch.empty((N, K), dtype=torch.float16, device=dev)
-        rows = wl.gaussian_rows(N, K, seed=7, device=dev)
-        bg.bergson_build_store(rows, N, K, True, store, 0)
+        for n0 in range(0, N, 1 << 16):
+            n1 = min(N, n0 + (1 << 16))
+            rows = wl.gaussian_rows(n1 - n0, K, seed=7 + n0, device=dev)
+            bg.bergson_build_store(rows, n1 - n0, K, True, store, n0)
         del rows
         queries = wl.gaussian_rows(Q, K, seed=8, device=dev)
         ws = bg.workspace_tensor(bg.bergson_score_topk_workspace(N, K, Q, topk), dev)
