@@ -296,6 +296,56 @@ def bench_collection(args, world, dev, peaks, peak_kind):
     return res, (cfg, layers, mask, ws, out, store)
 
 
+def bench_onthefly(args, world, dev, state):
+    """On-the-fly scoring step: project the batch, score it against 1024 fixed queries."""
+    import torch
+
+    import paper_2606_11660_gb300 as bg
+    from paper_2606_11660_gb300 import workloads as wl
+
+    cfg, layers, mask, ws, out, store = state
+    K = cfg.k_total
+    Q = 1024
+    queries = wl.gaussian_rows(Q, K, seed=12, device=dev)
+    sws = bg.workspace_tensor(bg.bergson_score_grads_workspace(cfg.B, K, Q), dev)
+    scores = torch.empty((cfg.B, Q), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+
+    def step(e=None):
+        bg.bergson_project_grads(layers, cfg.B, cfg.T, mask, out, ws, stream)
+        if e is not None:
+            e[0].record(stream)
+        bg.bergson_score_grads(out, cfg.B, K, queries, True, scores, sws, stream)
+        if e is not None:
+            e[1].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(args.steps):
+        step(ev[i])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(t0.elapsed_time(t1), world)
+    score_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    flops = 2.0 * cfg.B * K * Q
+    return {"value": round(cfg.B * world * args.steps / (ms * 1e-3), 2), "unit": "examples/s",
+            "ms_per_step": round(ms / args.steps, 4), "queries": Q,
+            "score_call_ms": round(score_ms, 4),
+            "score_gflops": round(flops / (score_ms * 1e-3) / 1e9, 1),
+            "gpu_launches": (5 + 4) * args.steps,
+            "what": "bergson_project_grads + bergson_score_grads (cosine vs 1024 fp32 queries, "
+                    "no store) per batch"}
+
+
 def bench_e2e(args, world, dev, state):
     """Same step through the public API with host (pinned) inputs copied in every step."""
     import torch
@@ -467,6 +517,7 @@ def main_ours(args):
     torch.cuda.set_device(dev)
     peaks, peak_kind = load_peaks()
     coll, state = bench_collection(args, world, dev, peaks, peak_kind)
+    onthefly = bench_onthefly(args, world, dev, state)
     e2e = bench_e2e(args, world, dev, state) if not args.no_e2e else None
     del state
     torch.cuda.empty_cache()
@@ -492,7 +543,7 @@ def main_ours(args):
                        "l2": "inputs 19.3 GB per step > 129 MB L2 (no flush needed)"},
             "roofline": coll["roofline"], "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": coll["gpu_launches"], "clocks": coll["clocks"],
-            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring,
+            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

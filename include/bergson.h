@@ -164,6 +164,30 @@ BERGSON_API int bergson_score_topk(const void* store, int64_t N, int64_t K, int6
                        float* out_scores, int64_t* out_idx,
                        void* workspace, size_t ws_bytes, void* stream);
 
+/* Bytes of workspace bergson_score_grads needs. */
+BERGSON_API int bergson_score_grads_workspace(int64_t B, int64_t K, int64_t Q, size_t* ws_bytes);
+
+/*
+ * On-the-fly attribution scores (Bergson Sec. 3.1, "bergson score": training
+ * gradients are streamed and only their influence on fixed queries is kept,
+ * with no gradient store; Table 3 grad-cosine / grad-dot):
+ *
+ *   scores[b, q] = <x_b, y_q> / (||x_b|| ||y_q||)   (unit_normalize != 0)
+ *   scores[b, q] = <x_b, y_q>                        (unit_normalize == 0)
+ *
+ * with x_b = proj[b, 0:K] (e.g. bergson_project_grads output) and
+ * y_q = queries[q, 0:K] (projected query gradients).  fp32 throughout; a zero
+ * row or query scores 0 under normalisation.  Deterministic.
+ *   proj      fp32 [B, ld_proj], queries fp32 [Q, ld_q]: 16-byte aligned,
+ *             ld % 4 == 0, ld >= K.   K > 0, K % 4 == 0.
+ *   scores    fp32 [B, ld_scores], ld_scores >= Q.
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_score_grads(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
+                                    const float* queries, int64_t Q, int64_t ld_q,
+                                    int unit_normalize, float* scores, int64_t ld_scores,
+                                    void* workspace, size_t ws_bytes, void* stream);
+
 /*
  * The projection actually used by bergson_project_grads (Fig. 1 random
  * projection), materialised for inspection:

@@ -14,7 +14,10 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. "Gradients"):
   4. concatenation over modules in call order and unit normalisation of the
      whole per-example row (grad-cosine);
   5. an fp16 gradient store, cosine scores against unit-normalised queries and
-     exact top-k, ordered by (score descending, index ascending).
+     exact top-k, ordered by (score descending, index ascending);
+  6. on-the-fly scores (Sec. 3.1, "bergson score"): training rows scored
+     directly against query rows without a store, as cosines (grad-cosine) or
+     plain inner products (grad-dot) -- Table 3's two identity-Hessian methods.
 
 Readings taken where the paper is silent (each is listed in the design doc):
   * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
@@ -245,3 +248,17 @@ def topk_rows(S: np.ndarray, k: int) -> tuple[np.ndarray, np.ndarray]:
 def score_topk(store: np.ndarray, queries: np.ndarray, k: int):
     """Cosine scores of queries against the store and their exact top-k."""
     return topk_rows(cosine_scores(store, queries), k)
+
+
+def onthefly_scores(rows: np.ndarray, queries: np.ndarray, unit: bool = True) -> np.ndarray:
+    """S[b, q] = <x_b, y_q>, with both sides unit-normalised when `unit` (fp64).
+
+    Rows and queries are projected gradients straight from the projection
+    step (no fp16 store in between); zero rows score 0 under normalisation.
+    """
+    x = np.asarray(rows, dtype=np.float64)
+    y = np.asarray(queries, dtype=np.float64)
+    if unit:
+        x, _ = unit_normalize(x)
+        y, _ = unit_normalize(y)
+    return x @ y.T

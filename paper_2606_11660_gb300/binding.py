@@ -37,6 +37,7 @@ EXPORTED = (
     "bergson_score_topk_workspace", "bergson_score_topk", "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
     "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_project_grads_noalloc",
+    "bergson_score_grads_workspace", "bergson_score_grads",
 )
 
 
@@ -87,6 +88,9 @@ def lib() -> ctypes.CDLL:
         "bergson_debug_wait_probe": (i32, [u64, vp]),
         "bergson_debug_inject_status": (None, [i32, i32]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
+        "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
+        "bergson_score_grads": (i32, [vp, i64, i64, i64, vp, i64, i64, i32, vp, i64, vp,
+                                      ctypes.c_size_t, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -200,6 +204,24 @@ def bergson_score_topk(store, N: int, K: int, queries, topk: int, out_scores, ou
                                     _ptr(queries), Q, int(queries.stride(0)), int(topk),
                                     _ptr(out_scores), _ptr(out_idx), _ptr(workspace), ws_bytes,
                                     _stream(stream)))
+
+
+def bergson_score_grads_workspace(B: int, K: int, Q: int) -> int:
+    n = ctypes.c_size_t()
+    _check(lib().bergson_score_grads_workspace(int(B), int(K), int(Q), ctypes.byref(n)))
+    return n.value
+
+
+def bergson_score_grads(proj, B: int, K: int, queries, unit_normalize: bool, scores, workspace,
+                        stream=None) -> None:
+    """On-the-fly scores of B projected rows against Q projected queries."""
+    Q = int(queries.shape[0])
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().bergson_score_grads(_ptr(proj), int(B), int(K), int(proj.stride(0)),
+                                     _ptr(queries), Q, int(queries.stride(0)),
+                                     1 if unit_normalize else 0, _ptr(scores),
+                                     int(scores.stride(0)), _ptr(workspace), ws_bytes,
+                                     _stream(stream)))
 
 
 def bergson_projection_matrix(seed: int, d: int, k: int, proj_kind: int, moment, out,

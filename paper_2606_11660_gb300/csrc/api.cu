@@ -597,6 +597,67 @@ int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store
   return BERGSON_OK;
 }
 
+static size_t onthefly_workspace(int64_t B, int64_t K, int64_t Q) {
+  const size_t S = static_cast<size_t>(onthefly_splits(B, Q, K));
+  return round_up(sizeof(float) * B, 256) + round_up(sizeof(float) * Q, 256) +
+         round_up(sizeof(float) * S * B * Q, 256);
+}
+
+static int validate_onthefly(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
+                             const float* queries, int64_t Q, int64_t ld_q, float* scores,
+                             int64_t ld_scores) {
+  if (B < 0 || B > (1 << 20) || Q < 0 || Q > (1 << 24))
+    return fail(BERGSON_EINVAL, "B must be in [0, 2^20] and Q in [0, 2^24]");
+  if (K < 4 || K > (1 << 26)) return fail(BERGSON_EINVAL, "K must be in [4, 2^26]");
+  if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
+  if (B * Q > (1ll << 34)) return fail(BERGSON_EUNSUPPORTED, "B*Q too large");
+  if (B > 0 && Q > 0) {
+    if (proj == nullptr || queries == nullptr || scores == nullptr)
+      return fail(BERGSON_EINVAL, "proj, queries or scores is NULL");
+    if (ld_proj < K || ld_q < K) return fail(BERGSON_EINVAL, "ld_proj and ld_q must be >= K");
+    if (ld_scores < Q) return fail(BERGSON_EINVAL, "ld_scores must be >= Q");
+    if (!aligned(proj, 16) || !aligned(queries, 16) || ld_proj % 4 != 0 || ld_q % 4 != 0)
+      return fail(BERGSON_EALIGN, "proj and queries need 16-byte aligned rows");
+    if (!aligned(scores, 4)) return fail(BERGSON_EALIGN, "scores must be 4-byte aligned");
+  }
+  return BERGSON_OK;
+}
+
+int bergson_score_grads_workspace(int64_t B, int64_t K, int64_t Q, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (B < 0 || B > (1 << 20) || Q < 0 || Q > (1 << 24) || K < 4 || K > (1 << 26))
+    return fail(BERGSON_EINVAL, "invalid sizes for the on-the-fly score workspace");
+  *ws_bytes = onthefly_workspace(B, K, Q);
+  return BERGSON_OK;
+}
+
+int bergson_score_grads(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
+                        const float* queries, int64_t Q, int64_t ld_q, int unit_normalize,
+                        float* scores, int64_t ld_scores, void* workspace, size_t ws_bytes,
+                        void* stream) {
+  int st = validate_onthefly(proj, B, K, ld_proj, queries, Q, ld_q, scores, ld_scores);
+  if (st != BERGSON_OK) return st;
+  const size_t need = onthefly_workspace(B, K, Q);
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (B == 0 || Q == 0) return BERGSON_OK;
+  DeviceGuard dg(workspace);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  float* sx = reinterpret_cast<float*>(ws);
+  float* sy = reinterpret_cast<float*>(ws + round_up(sizeof(float) * B, 256));
+  float* partial = reinterpret_cast<float*>(ws + round_up(sizeof(float) * B, 256) +
+                                            round_up(sizeof(float) * Q, 256));
+  cudaError_t e = launch_onthefly(proj, static_cast<int>(B), ld_proj, queries, static_cast<int>(Q),
+                                  ld_q, static_cast<int>(K), unit_normalize ? 1 : 0, sx, sy,
+                                  partial, scores, ld_scores, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "on-the-fly score launch");
+  return BERGSON_OK;
+}
+
 int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind,
                               const float* moment, float* out, void* stream) {
   if (d < 1 || d > (1 << 24)) return fail(BERGSON_EINVAL, "d must be in [1, 2^24]");

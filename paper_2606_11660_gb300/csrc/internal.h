@@ -15,6 +15,7 @@ constexpr int kChunk = 64;           // bf16 elements per 128-byte swizzled row
 constexpr int kScoreBN = 256;        // store rows per score tile (tcgen05 N)
 constexpr int kScoreQT = 128;        // queries per query tile (tcgen05 M)
 constexpr int kMaxTopk = 1024;
+constexpr int kOnTheFlyTargetCTAs = 1216;  // split-K target for on-the-fly scores
 
 // Per-module launch record kept in workspace (global memory).  The tensor maps
 // are read by TMA straight from there, so the record is 64-byte aligned.
@@ -102,5 +103,10 @@ size_t score_smem_bytes(int qt);
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
                          int q_begin, int q_end, int qg_base, float* out_scores, int64_t* out_idx,
                          cudaStream_t s);
+
+int onthefly_splits(int64_t B, int64_t Q, int64_t K);
+cudaError_t launch_onthefly(const float* x, int B, int64_t ldx, const float* y, int Q,
+                            int64_t ldy, int K, int unit, float* sx, float* sy, float* partial,
+                            float* scores, int64_t ld_scores, cudaStream_t s);
 
 }  // namespace bergson

@@ -143,7 +143,7 @@ __global__ void wait_probe_kernel(int* status, uint64_t timeout_ns) {
 cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, cudaStream_t s) {
   if (n_segs <= 0 || max_pairs <= 0) return cudaSuccess;
   const int threads = 256;
-  int64_t bx = (max_pairs + threads - 1) / threads;
+  int64_t bx = (max_pairs + 4 * threads - 1) / (4 * threads);   // ~4 pairs per thread
   if (bx > 4096) bx = 4096;
   prep_kernel<<<dim3(static_cast<unsigned>(bx), static_cast<unsigned>(n_segs)), threads, 0, s>>>(
       segs);

@@ -2,9 +2,10 @@
 // normalisation and the gradient store; grad-cosine = identity + unit norm).
 //
 // One CTA per row: the squared norm is accumulated from 16-byte vector loads
-// (fp64 partial sums, so a 10^5-long row keeps fp32-level accuracy), reduced
-// with warp shuffles, and the row is written back as fp16 (round to nearest
-// even) with 16-byte vector stores.
+// with compensated (Kahan) fp32 sums per thread -- fp64 arithmetic is slow on
+// this part and unnecessary at this accuracy -- reduced with warp shuffles,
+// and the row is written back as fp16 (round to nearest even) with 16-byte
+// vector stores.
 
 #include "internal.h"
 
@@ -14,7 +15,18 @@ namespace {
 
 constexpr int kRowThreads = 256;
 
-__device__ __forceinline__ double block_sum(double v, double* red) {
+// Kahan-compensated running sum.
+struct KahanSum {
+  float s = 0.0f, c = 0.0f;
+  __device__ __forceinline__ void add(float x) {
+    const float y = x - c;
+    const float t = s + y;
+    c = (t - s) - y;
+    s = t;
+  }
+};
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   const int warp = threadIdx.x >> 5;
@@ -22,7 +34,7 @@ __device__ __forceinline__ double block_sum(double v, double* red) {
   if (lane == 0) red[warp] = v;
   __syncthreads();
   if (warp == 0) {
-    v = lane < (blockDim.x >> 5) ? red[lane] : 0.0;
+    v = lane < (blockDim.x >> 5) ? red[lane] : 0.0f;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     if (lane == 0) red[0] = v;
@@ -48,18 +60,17 @@ __device__ __forceinline__ uint4 pack8(float4 a, float4 b, float s) {
 __global__ void __launch_bounds__(kRowThreads) normalize_rows_kernel(
     const float* __restrict__ x, int K, int64_t ldx, int unit, __half* __restrict__ y,
     int64_t ldy, float* __restrict__ norms) {
-  __shared__ double red[kRowThreads / 32];
+  __shared__ float red[kRowThreads / 32];
   const int64_t b = blockIdx.x;
   const float4* xr = reinterpret_cast<const float4*>(x + b * ldx);
-  double ss = 0.0;
+  KahanSum ss;
   for (int i = threadIdx.x; i < K / 4; i += kRowThreads) {
     const float4 v = xr[i];
-    ss += static_cast<double>(v.x) * v.x + static_cast<double>(v.y) * v.y +
-          static_cast<double>(v.z) * v.z + static_cast<double>(v.w) * v.w;
+    ss.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
   }
-  const double tot = block_sum(ss, red);
-  const float nrm = static_cast<float>(sqrt(tot));
-  const float scale = unit ? (tot > 0.0 ? static_cast<float>(1.0 / sqrt(tot)) : 0.0f) : 1.0f;
+  const float tot = block_sum(ss.s, red);
+  const float nrm = sqrtf(tot);
+  const float scale = unit ? (tot > 0.0f ? 1.0f / nrm : 0.0f) : 1.0f;
   uint4* yr = reinterpret_cast<uint4*>(y + b * ldy);
   for (int i = threadIdx.x; i < K / 8; i += kRowThreads) yr[i] = pack8(xr[2 * i], xr[2 * i + 1], scale);
   if (norms != nullptr && threadIdx.x == 0) norms[b] = nrm;
@@ -68,13 +79,13 @@ __global__ void __launch_bounds__(kRowThreads) normalize_rows_kernel(
 // Queries may have any row stride; they are read with scalar loads.
 __global__ void __launch_bounds__(kRowThreads) normalize_queries_kernel(
     const float* __restrict__ q, int K, int64_t ldq, __half* __restrict__ qh) {
-  __shared__ double red[kRowThreads / 32];
+  __shared__ float red[kRowThreads / 32];
   const int64_t r = blockIdx.x;
   const float* qr = q + r * ldq;
-  double ss = 0.0;
-  for (int i = threadIdx.x; i < K; i += kRowThreads) ss += static_cast<double>(qr[i]) * qr[i];
-  const double tot = block_sum(ss, red);
-  const float scale = tot > 0.0 ? static_cast<float>(1.0 / sqrt(tot)) : 0.0f;
+  KahanSum ss;
+  for (int i = threadIdx.x; i < K; i += kRowThreads) ss.add(qr[i] * qr[i]);
+  const float tot = block_sum(ss.s, red);
+  const float scale = tot > 0.0f ? 1.0f / sqrtf(tot) : 0.0f;
   __half* out = qh + r * K;
   for (int i = threadIdx.x; i < K; i += kRowThreads) out[i] = __float2half_rn(qr[i] * scale);
 }

@@ -161,3 +161,24 @@ def test_calls_without_device_fail_cleanly():
     st = _proj([_layer()])
     assert st == bg.BERGSON_ECUDA
     assert bg.bergson_last_error() != ""
+
+
+def test_onthefly_validation():
+    f = bg.lib().bergson_score_grads
+    n = ctypes.c_size_t()
+    assert bg.lib().bergson_score_grads_workspace(32, 12288, 1024, ctypes.byref(n)) == bg.BERGSON_OK
+    ws = n.value
+    assert ws >= 4 * 32 * 1024
+
+    def call(B=32, K=12288, ldp=12288, Q=1024, ldq=12288, lds=1024, ws_bytes=ws, proj=FAKE,
+             queries=FAKE, scores=FAKE, wsp=FAKE):
+        return f(proj, B, K, ldp, queries, Q, ldq, 1, scores, lds, wsp, ws_bytes, None)
+    assert call(K=10) == bg.BERGSON_EALIGN
+    assert call(ldp=100) == bg.BERGSON_EINVAL
+    assert call(ldq=12290) == bg.BERGSON_EALIGN
+    assert call(lds=10) == bg.BERGSON_EINVAL
+    assert call(proj=FAKE + 4) == bg.BERGSON_EALIGN
+    assert call(ws_bytes=ws - 1) == bg.BERGSON_EWORKSPACE
+    assert call(queries=None) == bg.BERGSON_EINVAL
+    assert call(B=0) == bg.BERGSON_OK
+    assert call(Q=0) == bg.BERGSON_OK

@@ -262,3 +262,28 @@ def test_topk_matches_sorted_with_ties():
         assert list(val[q]) == [S[q, n] for n in want]
     with pytest.raises(ValueError):
         orc.topk_rows(S, 41)
+
+
+# --- on-the-fly scores -------------------------------------------------------
+
+def test_onthefly_scores_definitions():
+    X = RNG.standard_normal((5, 40))
+    Y = RNG.standard_normal((3, 40))
+    X[2] = 0.0
+    S = orc.onthefly_scores(X, Y, unit=True)
+    D = orc.onthefly_scores(X, Y, unit=False)
+    for b in range(5):
+        for q in range(3):
+            dot = sum(float(X[b, i]) * float(Y[q, i]) for i in range(40))
+            assert abs(D[b, q] - dot) < 1e-12
+            nx = math.sqrt(sum(float(v) ** 2 for v in X[b]))
+            ny = math.sqrt(sum(float(v) ** 2 for v in Y[q]))
+            assert abs(S[b, q] - (dot / (nx * ny) if nx > 0 else 0.0)) < 1e-12
+    np.testing.assert_array_equal(S[2], 0.0)
+    # cosine: invariant to positive row/query scaling, bounded by 1, self-score 1
+    np.testing.assert_allclose(orc.onthefly_scores(3.0 * X, 0.5 * Y), S, atol=1e-14)
+    assert np.all(np.abs(S) <= 1 + 1e-12)
+    np.testing.assert_allclose(np.diag(orc.onthefly_scores(Y, Y)), 1.0, atol=1e-14)
+    # agrees with the store path up to the fp16 rounding of the rows
+    store, _ = orc.build_store(X)
+    np.testing.assert_allclose(orc.cosine_scores(store, Y).T, S, atol=2e-3)
