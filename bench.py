@@ -44,9 +44,13 @@ def load_peaks():
 
 
 def source_digest(name: str) -> str:
+    """First 16 hex digits of sha256 over a kernel source with comments and whitespace removed."""
     path = os.path.join(ROOT, "paper_2606_11660_gb300", "csrc", name)
-    with open(path, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    with open(path) as f:
+        src = f.read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    return hashlib.sha256("".join(src.split()).encode()).hexdigest()[:16]
 
 
 def profiled_traffic(profile: str, source: str):
@@ -57,7 +61,7 @@ def profiled_traffic(profile: str, source: str):
     except OSError:
         return None
     m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
-    s = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    s = re.search(r"kernel_code_digest:\s*([0-9a-f]+)", text)
     if not m or not s or s.group(1) != source_digest(source):
         return None
     return float(m.group(1))

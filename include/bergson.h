@@ -2,7 +2,7 @@
  * bergson.h -- C ABI of the GB300 projected-gradient attribution library.
  *
  * The library implements the TrackStar-style gradient path of Bergson
- * (Sec. 3.1 "Attribution Pipelines", Fig. 1, App. "Gradients"):
+ * (Sec. 3.1 "Attribution Pipelines", Fig. 1, App. B, "Gradients"):
  *   per-example gradients of every nn.Linear weight, optional Adafactor-style
  *   factored second-moment normalisation, the double-sided per-module random
  *   projection, unit normalisation into an fp16 gradient store, and exact
@@ -55,7 +55,7 @@ typedef enum {
 } bergson_proj_kind;
 
 /*
- * One nn.Linear module's captured tensors (Bergson App. "Gradients": gradient
+ * One nn.Linear module's captured tensors (Bergson App. B, "Gradients": gradient
  * collection from linear layers; Fig. 1: Adafactor normalisation and the
  * double-sided per-module projection).
  *

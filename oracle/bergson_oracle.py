@@ -4,7 +4,7 @@ TEST INFRASTRUCTURE ONLY.  Nothing in the product path imports this module:
 only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline /
 reference legs may call it.  It shares no code with the CUDA library.
 
-What it computes (Bergson, Sec. 3.1 and Fig. 1; App. "Gradients"):
+What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
   1. the per-example gradient of an ``nn.Linear`` weight,
      W_b = sum_t m_{b,t} g_{b,t} a_{b,t}^T   (d_out x d_in), explicitly;
   2. optional Adafactor-style factored second-moment normalisation,

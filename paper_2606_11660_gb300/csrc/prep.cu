@@ -1,4 +1,4 @@
-// Projection preparation (Fig. 1: random down-projection; App. "Gradients":
+// Projection preparation (Fig. 1: random down-projection; App. B, "Gradients":
 // double-sided projection), mask tile flags and the bounded-wait probe.
 //
 // The Gaussian projection is generated on the fly from its seed: entry

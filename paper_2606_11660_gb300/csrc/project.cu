@@ -1,6 +1,6 @@
 // Fused token projection + masked per-example contraction (Bergson Fig. 1:
 // Adafactor normalisation and the double-sided per-module random projection,
-// applied to per-example nn.Linear gradients as in App. "Gradients").
+// applied to per-example nn.Linear gradients as in App. B, "Gradients").
 //
 // For one module and example b the projected gradient is
 //   G^_b = P_out'^T (sum_t m_t g_t a_t^T) P_in' = sum_t m_t (P_out'^T g_t)(P_in'^T a_t)^T,
