@@ -350,6 +350,45 @@ def bench_onthefly(args, world, dev, state):
                     "no store) per batch"}
 
 
+def bench_tokens(args, world, dev, state, peaks):
+    """Per-token scores of the batch against 4 query rows (one fused pass over A and G)."""
+    import torch
+
+    import paper_2606_11660_gb300 as bg
+    from paper_2606_11660_gb300 import workloads as wl
+
+    cfg, layers, mask, ws, out, store = state
+    Q = 4
+    queries = wl.gaussian_rows(Q, cfg.k_total, seed=13, device=dev)
+    tws = bg.workspace_tensor(bg.bergson_token_scores_workspace(layers, cfg.B, cfg.T, Q), dev)
+    tout = torch.empty((Q, cfg.B, cfg.T), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        bg.bergson_token_scores(layers, cfg.B, cfg.T, mask, queries, tout, tws, stream)
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        bg.bergson_token_scores(layers, cfg.B, cfg.T, mask, queries, tout, tws, stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(t0.elapsed_time(t1), world) / args.steps
+    valid = int(mask.sum().item())
+    alg = 2 * sum(sp.d_in + sp.d_out for sp in cfg.modules) * valid
+    gbs = alg / (ms * 1e-3) / 1e9
+    return {"value": round(cfg.B * world / (ms * 1e-3), 2), "unit": "examples/s",
+            "ms_per_step": round(ms, 4), "queries": Q,
+            "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4)},
+            "gpu_launches": 5 * args.steps,
+            "what": "bergson_token_scores: per-token scores of all 65,536 tokens x 48 modules "
+                    "against 4 query rows"}
+
+
 def bench_e2e(args, world, dev, state):
     """Same step through the public API with host (pinned) inputs copied in every step."""
     import torch
@@ -522,6 +561,7 @@ def main_ours(args):
     peaks, peak_kind = load_peaks()
     coll, state = bench_collection(args, world, dev, peaks, peak_kind)
     onthefly = bench_onthefly(args, world, dev, state)
+    tokens = bench_tokens(args, world, dev, state, peaks)
     e2e = bench_e2e(args, world, dev, state) if not args.no_e2e else None
     del state
     torch.cuda.empty_cache()
@@ -547,7 +587,7 @@ def main_ours(args):
                        "l2": "inputs 19.3 GB per step > 129 MB L2 (no flush needed)"},
             "roofline": coll["roofline"], "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": coll["gpu_launches"], "clocks": coll["clocks"],
-            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly,
+            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly, "token_scores": tokens,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

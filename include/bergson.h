@@ -164,6 +164,35 @@ BERGSON_API int bergson_score_topk(const void* store, int64_t N, int64_t K, int6
                        float* out_scores, int64_t* out_idx,
                        void* workspace, size_t ws_bytes, void* stream);
 
+/* Bytes of workspace bergson_token_scores needs (n_queries in 1 .. 16). */
+BERGSON_API int bergson_token_scores_workspace(const bergson_layer* layers, int n_layers,
+                                               int64_t B, int64_t T, int64_t n_queries,
+                                               size_t* ws_bytes);
+
+/*
+ * Per-token attribution scores (Bergson Fig. 1: attribution scores per token
+ * or per sequence; Sec. 3.1 per-token gradient collection):
+ *
+ *   out[q, b, t] = sum over layers m of  g~_{b,t,m}^T  Q~_{q,m}  a~_{b,t,m}
+ *
+ * i.e. the Frobenius inner product of token t's own projected (and
+ * normalised) gradient P_out'^T g_t a_t^T P_in' with query q's k_out x k_in
+ * block Q~_{q,m} = queries[q, off_m : off_m + k_out*k_in] (row-major, the
+ * layout bergson_project_grads writes).  Summed over t, the scores give the
+ * per-sequence inner product <out_b, queries_q>.  Masked tokens score 0.
+ *   queries  fp32 [n_queries, ld_q], 4-byte aligned; the layers' column
+ *            blocks must fit in ld_q and must not overlap.
+ *   n_queries  1 .. 16, and at most what the layers' (k_in, k_out) allow
+ *            (16 for 16x16, 8 for 32x32, 4 for 64x64).
+ *   out      fp32 [n_queries, B, T] contiguous.
+ * Other arguments as for bergson_project_grads.  Deterministic.
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_token_scores(const bergson_layer* layers, int n_layers, int64_t B,
+                                     int64_t T, const uint8_t* mask, const float* queries,
+                                     int64_t n_queries, int64_t ld_q, float* out,
+                                     void* workspace, size_t ws_bytes, void* stream);
+
 /* Bytes of workspace bergson_score_grads needs. */
 BERGSON_API int bergson_score_grads_workspace(int64_t B, int64_t K, int64_t Q, size_t* ws_bytes);
 

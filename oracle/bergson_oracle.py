@@ -17,7 +17,9 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
      exact top-k, ordered by (score descending, index ascending);
   6. on-the-fly scores (Sec. 3.1, "bergson score"): training rows scored
      directly against query rows without a store, as cosines (grad-cosine) or
-     plain inner products (grad-dot) -- Table 3's two identity-Hessian methods.
+     plain inner products (grad-dot) -- Table 3's two identity-Hessian methods;
+  7. per-token scores (Fig. 1: attribution scores per token or per sequence):
+     the inner product of each token's own projected gradient with a query.
 
 Readings taken where the paper is silent (each is listed in the design doc):
   * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
@@ -262,3 +264,31 @@ def onthefly_scores(rows: np.ndarray, queries: np.ndarray, unit: bool = True) ->
         x, _ = unit_normalize(x)
         y, _ = unit_normalize(y)
     return x @ y.T
+
+
+def token_scores(layers, mask, queries: np.ndarray, examples=None) -> np.ndarray:
+    """Per-token scores s[q, b, t] = sum over modules of <G^_{b,t}, Q~_q,m>_F (fp64).
+
+    G^_{b,t} is the projected, normalised gradient of token t alone
+    (P_out^T (g_t a_t^T / sqrt(r c^T)) P_in) and Q~_q,m is module m's
+    k_out x k_in block of query row q (same column layout as project_grads).
+    Masked tokens score 0.  Returns [Q, len(examples), T].
+    """
+    queries = np.asarray(queries, dtype=np.float64)
+    B, T = layers[0].A.shape[0], layers[0].A.shape[1]
+    examples = list(range(B)) if examples is None else list(examples)
+    out = np.zeros((queries.shape[0], len(examples), T), dtype=np.float64)
+    for layer in layers:
+        p_in = projection_matrix(layer.seed_in, layer.d_in, layer.k_in, layer.proj_kind)
+        p_out = projection_matrix(layer.seed_out, layer.d_out, layer.k_out, layer.proj_kind)
+        blk = queries[:, layer.col_offset:layer.col_offset + layer.k_out * layer.k_in]
+        qm = blk.reshape(-1, layer.k_out, layer.k_in)
+        for bi, b in enumerate(examples):
+            for t in range(T):
+                if mask is not None and mask[b, t] == 0:
+                    continue
+                w = np.outer(np.asarray(layer.G[b, t], np.float64), np.asarray(layer.A[b, t], np.float64))
+                w = adafactor_normalize(w, layer.r, layer.c)
+                g_hat = double_sided_projection(w, p_out, p_in)
+                out[:, bi, t] += np.einsum("qij,ij->q", qm, g_hat)
+    return out

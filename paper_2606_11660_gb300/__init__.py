@@ -10,6 +10,6 @@ from .binding import (  # noqa: F401
     bergson_debug_wait_probe, bergson_last_error, bergson_module_seeds, bergson_project_grads,
     bergson_project_grads_noalloc, bergson_project_grads_workspace, bergson_projection_matrix, bergson_score_topk,
     bergson_score_topk_workspace, bergson_score_grads, bergson_score_grads_workspace,
-    bergson_sync_status, bergson_version, bergson_layer, lib,
+    bergson_sync_status, bergson_token_scores, bergson_token_scores_workspace, bergson_version, bergson_layer, lib,
     workspace_tensor,
 )

@@ -37,7 +37,8 @@ EXPORTED = (
     "bergson_score_topk_workspace", "bergson_score_topk", "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
     "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_project_grads_noalloc",
-    "bergson_score_grads_workspace", "bergson_score_grads",
+    "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
+    "bergson_token_scores",
 )
 
 
@@ -89,6 +90,9 @@ def lib() -> ctypes.CDLL:
         "bergson_debug_inject_status": (None, [i32, i32]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
+        "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
+        "bergson_token_scores": (i32, [lp, i32, i64, i64, vp, vp, i64, i64, vp, vp,
+                                       ctypes.c_size_t, vp]),
         "bergson_score_grads": (i32, [vp, i64, i64, i64, vp, i64, i64, i32, vp, i64, vp,
                                       ctypes.c_size_t, vp]),
     }
@@ -204,6 +208,24 @@ def bergson_score_topk(store, N: int, K: int, queries, topk: int, out_scores, ou
                                     _ptr(queries), Q, int(queries.stride(0)), int(topk),
                                     _ptr(out_scores), _ptr(out_idx), _ptr(workspace), ws_bytes,
                                     _stream(stream)))
+
+
+def bergson_token_scores_workspace(layers: Sequence, B: int, T: int, n_queries: int) -> int:
+    arr = _layer_array(layers)
+    n = ctypes.c_size_t()
+    _check(lib().bergson_token_scores_workspace(arr, len(layers), int(B), int(T), int(n_queries),
+                                                ctypes.byref(n)))
+    return n.value
+
+
+def bergson_token_scores(layers: Sequence, B: int, T: int, mask, queries, out, workspace,
+                         stream=None) -> None:
+    """Per-token scores out[q, b, t] of every token against each query row."""
+    arr = _layer_array(layers)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().bergson_token_scores(arr, len(layers), int(B), int(T), _ptr(mask), _ptr(queries),
+                                      int(queries.shape[0]), int(queries.stride(0)), _ptr(out),
+                                      _ptr(workspace), ws_bytes, _stream(stream)))
 
 
 def bergson_score_grads_workspace(B: int, K: int, Q: int) -> int:

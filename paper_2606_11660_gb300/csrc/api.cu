@@ -133,6 +133,7 @@ struct ProjLayout {
   std::vector<Group> groups;
   std::vector<int> mod_slot;   // layer index -> ModDesc slot
   size_t mods_off = 0, segs_off = 0, ctr_off = 0, tv_off = 0;
+  size_t token_off = 0;        // per-token score partials (token mode)
   std::vector<size_t> pin_off, pout_off;
   size_t total = 0;
 };
@@ -190,7 +191,10 @@ int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out) {
   return BERGSON_OK;
 }
 
-ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, int64_t T) {
+// n_queries > 0 lays out per-token score partials [n_layers, n_queries, B, T]
+// instead of per-item projection partials.
+ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                        int64_t n_queries = 0) {
   ProjLayout L;
   L.n_tiles = static_cast<int>((T + kTileTokens - 1) / kTileTokens);
   L.mod_slot.assign(n_layers, 0);
@@ -245,9 +249,16 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
     L.pout_off[i] = off;
     off += round_up(2 * layers[i].k_out * layers[i].d_out * sizeof(__nv_bfloat16), 256);
   }
-  for (Group& g : L.groups) {
-    g.partial_off = off;
-    off += round_up(static_cast<size_t>(g.n_items) * g.k_in * g.k_out * sizeof(float), 256);
+  if (n_queries > 0) {
+    const size_t per_mod = static_cast<size_t>(n_queries) * B * T * sizeof(float);
+    L.token_off = off;
+    for (Group& g : L.groups) g.partial_off = off + per_mod * g.first_mod;
+    off += round_up(per_mod * n_layers, 256);
+  } else {
+    for (Group& g : L.groups) {
+      g.partial_off = off;
+      off += round_up(static_cast<size_t>(g.n_items) * g.k_in * g.k_out * sizeof(float), 256);
+    }
   }
   L.total = off;
   return L;
@@ -363,23 +374,45 @@ int bergson_project_grads_workspace(const bergson_layer* layers, int n_layers, i
   return BERGSON_OK;
 }
 
-int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
-                          const uint8_t* mask, float* out, int64_t ld_out, void* workspace,
-                          size_t ws_bytes, void* stream) {
+// Projection mode (n_queries == 0): out = fp32 [B, ld_out] projected gradients.
+// Token mode (n_queries > 0): out = fp32 [n_queries, B, T] per-token scores
+// against queries [n_queries, ld_q] laid out like projection rows.
+static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                          const uint8_t* mask, float* out, int64_t ld_out, const float* queries,
+                          int64_t n_queries, int64_t ld_q, void* workspace, size_t ws_bytes,
+                          void* stream) {
+  const bool token = n_queries > 0;
   int st = validate_layers(layers, n_layers, B, T);
   if (st != BERGSON_OK) return st;
-  if (ld_out < 0) return fail(BERGSON_EINVAL, "ld_out must be >= 0");
-  st = validate_blocks(layers, n_layers, ld_out);
-  if (st != BERGSON_OK) return st;
-  if (B > 0 && out == nullptr) return fail(BERGSON_EINVAL, "out is NULL");
+  if (token) {
+    if (n_queries > 16) return fail(BERGSON_EUNSUPPORTED, "at most 16 queries per call");
+    for (int i = 0; i < n_layers; ++i) {
+      const int cap = token_query_capacity(static_cast<int>(layers[i].k_in),
+                                           static_cast<int>(layers[i].k_out));
+      if (n_queries > cap)
+        return fail(BERGSON_EUNSUPPORTED, "layer %d: at most %d queries for k_in=%lld, k_out=%lld",
+                    i, cap, (long long)layers[i].k_in, (long long)layers[i].k_out);
+    }
+    if (ld_q < 0) return fail(BERGSON_EINVAL, "ld_q must be >= 0");
+    st = validate_blocks(layers, n_layers, ld_q);
+    if (st != BERGSON_OK) return st;
+    if (queries == nullptr) return fail(BERGSON_EINVAL, "queries is NULL");
+    if (!aligned(queries, 4)) return fail(BERGSON_EALIGN, "queries must be 4-byte aligned");
+    if (B * T > 0 && out == nullptr) return fail(BERGSON_EINVAL, "out is NULL");
+  } else {
+    if (ld_out < 0) return fail(BERGSON_EINVAL, "ld_out must be >= 0");
+    st = validate_blocks(layers, n_layers, ld_out);
+    if (st != BERGSON_OK) return st;
+    if (B > 0 && out == nullptr) return fail(BERGSON_EINVAL, "out is NULL");
+  }
   if (out != nullptr && !aligned(out, 4)) return fail(BERGSON_EALIGN, "out must be 4-byte aligned");
-  const ProjLayout L = plan_project(layers, n_layers, B, T);
+  const ProjLayout L = plan_project(layers, n_layers, B, T, token ? n_queries : 0);
   if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
   if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
   if (ws_bytes < L.total)
     return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, L.total);
   if ((st = injected()) != BERGSON_OK) return st;
-  if (B == 0) return BERGSON_OK;
+  if (B == 0 || (token && T == 0)) return BERGSON_OK;
 
   DeviceGuard dg(workspace);
   if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
@@ -464,18 +497,56 @@ int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, 
       p.mask = mask;
       p.tile_valid = tile_valid;
       p.partials = partials;
+      p.queries = queries;
+      p.ld_q = ld_q;
+      p.n_queries = static_cast<int>(n_queries);
+      p.token_partials = partials;
       p.counter = reinterpret_cast<int*>(ws + L.ctr_off) + 32 * gi;
       p.status = status;
       p.timeout_ns = kWaitTimeoutNs;
       const int grid = std::max(1, std::min(sms > 0 ? sms : 1, g.n_items));
-      e = launch_project(g.k_in, g.k_out, p, grid, s);
+      e = launch_project(g.k_in, g.k_out, token, p, grid, s);
       if (e != cudaSuccess) return fail_cuda(e, "projection kernel launch");
     }
-    e = launch_reduce(mods_dev + g.first_mod, static_cast<int>(g.layers.size()), g.k_in, g.k_out,
-                      static_cast<int>(B), g.n_chunks, partials, out, ld_out, s);
-    if (e != cudaSuccess) return fail_cuda(e, "reduce launch");
+    if (!token) {
+      e = launch_reduce(mods_dev + g.first_mod, static_cast<int>(g.layers.size()), g.k_in,
+                        g.k_out, static_cast<int>(B), g.n_chunks, partials, out, ld_out, s);
+      if (e != cudaSuccess) return fail_cuda(e, "reduce launch");
+    }
+  }
+  if (token) {
+    e = launch_token_reduce(reinterpret_cast<const float*>(ws + L.token_off), n_layers, static_cast<int>(n_queries), static_cast<int>(B),
+                            static_cast<int>(T), mask, out, s);
+    if (e != cudaSuccess) return fail_cuda(e, "token reduce launch");
   }
   return BERGSON_OK;
+}
+
+int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                          const uint8_t* mask, float* out, int64_t ld_out, void* workspace,
+                          size_t ws_bytes, void* stream) {
+  return run_projection(layers, n_layers, B, T, mask, out, ld_out, nullptr, 0, 0, workspace,
+                        ws_bytes, stream);
+}
+
+int bergson_token_scores_workspace(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                                   int64_t n_queries, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (n_queries < 1 || n_queries > 16)
+    return fail(BERGSON_EUNSUPPORTED, "n_queries must be in [1, 16]");
+  int st = validate_layers(layers, n_layers, B, T);
+  if (st != BERGSON_OK) return st;
+  *ws_bytes = plan_project(layers, n_layers, B, T, n_queries).total;
+  return BERGSON_OK;
+}
+
+int bergson_token_scores(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                         const uint8_t* mask, const float* queries, int64_t n_queries,
+                         int64_t ld_q, float* out, void* workspace, size_t ws_bytes,
+                         void* stream) {
+  if (n_queries < 1) return fail(BERGSON_EINVAL, "n_queries must be >= 1");
+  return run_projection(layers, n_layers, B, T, mask, out, 0, queries, n_queries, ld_q, workspace,
+                        ws_bytes, stream);
 }
 
 int bergson_build_store(const float* proj, int64_t B, int64_t K, int64_t ld_proj,

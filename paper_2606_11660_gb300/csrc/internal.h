@@ -55,7 +55,11 @@ struct ProjParams {
   int n_items;          // n_mods * B * n_chunks
   const uint8_t* mask;        // [B, T] or nullptr
   const uint8_t* tile_valid;  // [B, n_tiles] 4-bit masks of valid 32-token slices, or nullptr
-  float* partials;            // [n_items, k_out * k_in]
+  float* partials;            // [n_items, k_out * k_in]   (projection mode)
+  const float* queries;       // [n_queries, ld_q] query rows          (token mode)
+  int64_t ld_q;
+  int n_queries;
+  float* token_partials;      // [n_mods, n_queries, B, T]             (token mode)
   int* counter;               // dynamic scheduler, zero on entry
   int* status;                // device status word
   uint64_t timeout_ns;
@@ -87,8 +91,14 @@ cudaError_t launch_tile_valid(const uint8_t* mask, int B, int T, int n_tiles, ui
                               cudaStream_t s);
 cudaError_t launch_wait_probe(int* status, uint64_t timeout_ns, cudaStream_t s);
 
-cudaError_t launch_project(int k_in, int k_out, const ProjParams& p, int grid, cudaStream_t s);
+// token = false: per-example projected gradients (partials); token = true:
+// per-token scores against p.queries (token_partials).
+cudaError_t launch_project(int k_in, int k_out, bool token, const ProjParams& p, int grid,
+                          cudaStream_t s);
 size_t project_smem_bytes(int k_in, int k_out);
+int token_query_capacity(int k_in, int k_out);
+cudaError_t launch_token_reduce(const float* token_partials, int n_mods, int Q, int B, int T,
+                                const uint8_t* mask, float* out, cudaStream_t s);
 cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, int B,
                           int n_chunks, const float* partials, float* out, int64_t ld_out,
                           cudaStream_t s);

@@ -106,7 +106,7 @@ __device__ __forceinline__ uint32_t tiles_of(uint32_t slices) {
   return tm;
 }
 
-template <int KI, int KO>
+template <int KI, int KO, bool TOKEN>
 __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   using C = ProjCfg<KI, KO>;
   constexpr int NT = C::NT;
@@ -308,6 +308,16 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       const ItemCoord ic = decode_item(p, item);
 #pragma unroll
       for (int x = 0; x < OPT; ++x) acc[x] = 0.0f;
+      if constexpr (TOKEN) {
+        // This module's k_out x k_in block of every query row, into the
+        // (otherwise unused) staging area.  All threads left the previous
+        // item behind the two barriers above.
+        const int blk = KO * KI;
+        const int64_t off = p.mods[ic.m].col_offset;
+        for (int e = et; e < p.n_queries * blk; e += 128)
+          sA[e] = p.queries[static_cast<int64_t>(e / blk) * p.ld_q + off + e % blk];
+        named_bar_sync(1, 128);
+      }
       bool aborted = false;
       for (int g = ic.t_begin; g < ic.t_end; g += NT) {
         const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
@@ -336,6 +346,37 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
         if (++ab == 2) { ab = 0; aph ^= 1; }
+        if constexpr (TOKEN) {
+          // s[q] = g~^T Q~_q a~ for this thread's token: its share of the
+          // query's score (masked tokens score 0).
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            if (!(vm >> nt & 1)) continue;
+            const int t = (g + nt) * kTileTokens + row;
+            if (t >= p.T) continue;
+            const bool valid =
+                p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0;
+            for (int q = 0; q < p.n_queries; ++q) {
+              const float* qm = sA + q * (KO * KI);
+              float sq = 0.0f;
+#pragma unroll
+              for (int i = 0; i < KO; ++i) {
+                float u = 0.0f;
+#pragma unroll
+                for (int j = 0; j < KI; j += 4) {
+                  const float4 w = *reinterpret_cast<const float4*>(qm + i * KI + j);
+                  u = fmaf(w.x, va[nt][j], u);
+                  u = fmaf(w.y, va[nt][j + 1], u);
+                  u = fmaf(w.z, va[nt][j + 2], u);
+                  u = fmaf(w.w, va[nt][j + 3], u);
+                }
+                sq = fmaf(vg[nt][i], u, sq);
+              }
+              p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q) * p.B + ic.b) *
+                                   p.T + t] = valid ? sq : 0.0f;
+            }
+          }
+        } else {
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
           if (!(vm >> nt & 1)) continue;
@@ -380,8 +421,10 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             }
           }
         }
+        }   // projection mode
       }
       if (aborted) break;
+      if constexpr (TOKEN) continue;
       float* dst = p.partials + static_cast<int64_t>(item) * (KO * KI) + et * OPT;
 #pragma unroll
       for (int x = 0; x < OPT / 2; ++x)
@@ -413,19 +456,46 @@ __global__ void reduce_kernel(const ModDesc* __restrict__ mods, int B, int blk, 
   }
 }
 
-template <int KI, int KO>
+// out[q, b, t] = sum over modules m (in order) of token_partials[m, q, b, t];
+// 0 for masked tokens (whose partials may never have been written).
+__global__ void token_reduce_kernel(const float* __restrict__ tp, int n_mods, int Q, int B, int T,
+                                    const uint8_t* __restrict__ mask, float* __restrict__ out) {
+  const int64_t bt = static_cast<int64_t>(B) * T;
+  const int64_t n = static_cast<int64_t>(Q) * bt;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i % bt;
+    float s = 0.0f;
+    for (int m = 0; m < n_mods; ++m) s += tp[static_cast<int64_t>(m) * n + i];
+    out[i] = (mask == nullptr || mask[r] != 0) ? s : 0.0f;
+  }
+}
+
+template <int KI, int KO, bool TOKEN>
 cudaError_t launch_project_t(const ProjParams& p, int grid, cudaStream_t s) {
   using C = ProjCfg<KI, KO>;
   static bool attr_set = false;   // per process; the attribute is per function and device
   cudaError_t e = cudaSuccess;
   if (!attr_set) {
-    e = cudaFuncSetAttribute(project_kernel<KI, KO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             C::kSmemBytes);
+    e = cudaFuncSetAttribute(project_kernel<KI, KO, TOKEN>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  project_kernel<KI, KO><<<grid, 192, C::kSmemBytes, s>>>(p);
+  project_kernel<KI, KO, TOKEN><<<grid, 192, C::kSmemBytes, s>>>(p);
   return cudaGetLastError();
+}
+
+template <int KI, int KO>
+cudaError_t launch_project_mode(bool token, const ProjParams& p, int grid, cudaStream_t s) {
+  return token ? launch_project_t<KI, KO, true>(p, grid, s)
+               : launch_project_t<KI, KO, false>(p, grid, s);
+}
+
+template <int KI, int KO>
+constexpr int token_capacity_of() {
+  const int cap = ProjCfg<KI, KO>::kEpiBytes / (4 * KI * KO);
+  return cap > 16 ? 16 : cap;
 }
 
 template <int KI, int KO>
@@ -440,17 +510,41 @@ constexpr size_t smem_of() {
     return EXPR;                                     \
   }
 
-cudaError_t launch_project(int k_in, int k_out, const ProjParams& p, int grid, cudaStream_t s) {
-  BERGSON_PROJ_DISPATCH(16, 16, (launch_project_t<16, 16>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(16, 32, (launch_project_t<16, 32>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(16, 64, (launch_project_t<16, 64>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(32, 16, (launch_project_t<32, 16>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(32, 32, (launch_project_t<32, 32>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(32, 64, (launch_project_t<32, 64>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(64, 16, (launch_project_t<64, 16>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(64, 32, (launch_project_t<64, 32>(p, grid, s)))
-  BERGSON_PROJ_DISPATCH(64, 64, (launch_project_t<64, 64>(p, grid, s)))
+cudaError_t launch_project(int k_in, int k_out, bool token, const ProjParams& p, int grid,
+                           cudaStream_t s) {
+  BERGSON_PROJ_DISPATCH(16, 16, (launch_project_mode<16, 16>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(16, 32, (launch_project_mode<16, 32>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(16, 64, (launch_project_mode<16, 64>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(32, 16, (launch_project_mode<32, 16>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(32, 32, (launch_project_mode<32, 32>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(32, 64, (launch_project_mode<32, 64>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(64, 16, (launch_project_mode<64, 16>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(64, 32, (launch_project_mode<64, 32>(token, p, grid, s)))
+  BERGSON_PROJ_DISPATCH(64, 64, (launch_project_mode<64, 64>(token, p, grid, s)))
   return cudaErrorInvalidValue;
+}
+
+int token_query_capacity(int k_in, int k_out) {
+  BERGSON_PROJ_DISPATCH(16, 16, (token_capacity_of<16, 16>()))
+  BERGSON_PROJ_DISPATCH(16, 32, (token_capacity_of<16, 32>()))
+  BERGSON_PROJ_DISPATCH(16, 64, (token_capacity_of<16, 64>()))
+  BERGSON_PROJ_DISPATCH(32, 16, (token_capacity_of<32, 16>()))
+  BERGSON_PROJ_DISPATCH(32, 32, (token_capacity_of<32, 32>()))
+  BERGSON_PROJ_DISPATCH(32, 64, (token_capacity_of<32, 64>()))
+  BERGSON_PROJ_DISPATCH(64, 16, (token_capacity_of<64, 16>()))
+  BERGSON_PROJ_DISPATCH(64, 32, (token_capacity_of<64, 32>()))
+  BERGSON_PROJ_DISPATCH(64, 64, (token_capacity_of<64, 64>()))
+  return 0;
+}
+
+cudaError_t launch_token_reduce(const float* token_partials, int n_mods, int Q, int B, int T,
+                                const uint8_t* mask, float* out, cudaStream_t s) {
+  const int64_t n = static_cast<int64_t>(Q) * B * T;
+  if (n == 0) return cudaSuccess;
+  const int64_t blocks = (n + 255) / 256;
+  token_reduce_kernel<<<static_cast<unsigned>(blocks < 8192 ? blocks : 8192), 256, 0, s>>>(
+      token_partials, n_mods, Q, B, T, mask, out);
+  return cudaGetLastError();
 }
 
 size_t project_smem_bytes(int k_in, int k_out) {

@@ -287,3 +287,44 @@ def test_onthefly_scores_definitions():
     # agrees with the store path up to the fp16 rounding of the rows
     store, _ = orc.build_store(X)
     np.testing.assert_allclose(orc.cosine_scores(store, Y).T, S, atol=2e-3)
+
+
+# --- per-token scores ---------------------------------------------------------
+
+def test_token_scores_sum_to_sequence_score():
+    B, T = 2, 9
+    L0 = _layer(B, T, 24, 16, 16, 16, rc=True)
+    L1 = _layer(B, T, 16, 40, 16, 16, rc=True, seed=5)
+    L1.col_offset = 256
+    mask = (RNG.random((B, T)) > 0.3).astype(np.uint8)
+    Qr = RNG.standard_normal((3, 512))
+    tok = orc.token_scores([L0, L1], mask, Qr)
+    seq = orc.project_grads([L0, L1], mask, 512)          # sums tokens before projecting
+    np.testing.assert_allclose(tok.sum(axis=2), Qr @ seq.T, rtol=1e-11, atol=1e-11)
+    assert np.all(tok[:, mask == 0] == 0.0)
+
+
+def test_token_score_equals_single_token_sequence():
+    B, T = 1, 6
+    L = _layer(B, T, 24, 16, 16, 16, rc=False)
+    Qr = RNG.standard_normal((2, 256))
+    tok = orc.token_scores([L], None, Qr)
+    for t in range(T):
+        m = np.zeros((1, T), np.uint8)
+        m[0, t] = 1
+        np.testing.assert_allclose(tok[:, 0, t], Qr @ orc.project_grads([L], m, 256)[0], rtol=1e-11)
+
+
+def test_token_scores_identity_closed_form():
+    # P = I, no moments: s[q, b, t] = g_t^T Q_q a_t
+    B, T, d_in, d_out = 1, 4, 16, 32
+    L = _layer(B, T, d_in, d_out, d_in, d_out, rc=False, kind=orc.PROJ_IDENTITY)
+    Qr = RNG.standard_normal((2, d_out * d_in))
+    tok = orc.token_scores([L], None, Qr)
+    for q in range(2):
+        Qm = Qr[q].reshape(d_out, d_in)
+        for t in range(T):
+            g = L.G[0, t].astype(np.float64)
+            a = L.A[0, t].astype(np.float64)
+            want = sum(g[i] * Qm[i, j] * a[j] for i in range(d_out) for j in range(d_in))
+            assert abs(tok[q, 0, t] - want) < 1e-10 * max(1.0, abs(want))
