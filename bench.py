@@ -389,6 +389,62 @@ def bench_tokens(args, world, dev, state, peaks):
                     "against 4 query rows"}
 
 
+def bench_fisher(args, world, dev, state):
+    """TrackStar-style preconditioning: fit R on 1024 rows, R^-1/2 once, apply per batch."""
+    import torch
+
+    import paper_2606_11660_gb300 as bg
+    from paper_2606_11660_gb300 import workloads as wl
+
+    cfg, layers, mask, ws, out, store = state
+    K = cfg.k_total
+    n_fit = 1024
+    fit_rows = wl.gaussian_rows(n_fit, K, seed=14, device=dev)
+    R = torch.empty((K, K), device=dev)
+    M = torch.empty((K, K), device=dev)
+    fws = bg.workspace_tensor(bg.bergson_fisher_fit_workspace(n_fit, K), dev)
+    pws = bg.workspace_tensor(bg.bergson_fisher_preconditioner_workspace(K), dev)
+    aws = bg.workspace_tensor(bg.bergson_score_grads_workspace(cfg.B, K, K), dev)
+    pre = torch.empty((cfg.B, K), device=dev)
+    stream = torch.cuda.current_stream()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+    bg.bergson_fisher_fit(fit_rows, n_fit, K, R, fws, stream)          # warm-up
+    ev[0].record(stream)
+    bg.bergson_fisher_fit(fit_rows, n_fit, K, R, fws, stream)
+    ev[1].record(stream)
+    bg.bergson_fisher_preconditioner(R, None, K, 1.0, 0.1, bg.BERGSON_FISHER_INV_SQRT,
+                                     args.fisher_iters, M, pws, stream)
+    ev[2].record(stream)
+    for _ in range(args.warmup):
+        bg.bergson_precondition_rows(out, cfg.B, K, M, pre, aws, stream)
+    ev[3].record(stream)
+    for _ in range(args.steps):
+        bg.bergson_project_grads(layers, cfg.B, cfg.T, mask, out, ws, stream)
+        bg.bergson_precondition_rows(out, cfg.B, K, M, pre, aws, stream)
+        bg.bergson_build_store(pre, cfg.B, K, True, store, 0, None, stream)
+    ev[4].record(stream)
+    for _ in range(args.steps):
+        bg.bergson_precondition_rows(out, cfg.B, K, M, pre, aws, stream)
+    ev[5].record(stream)
+    torch.cuda.synchronize()
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    fit_ms = ev[0].elapsed_time(ev[1])
+    pow_ms = ev[1].elapsed_time(ev[2])
+    step_ms = ev[3].elapsed_time(ev[4]) / args.steps
+    apply_ms = ev[4].elapsed_time(ev[5]) / args.steps
+    gemm_flops = 2.0 * K ** 3 * (3 * args.fisher_iters)
+    return {"value": round(cfg.B * world / (step_ms * 1e-3), 2), "unit": "examples/s",
+            "ms_per_step": round(step_ms, 4), "apply_ms": round(apply_ms, 4),
+            "apply_tflops": round(2.0 * cfg.B * K * K / (apply_ms * 1e-3) / 1e12, 2),
+            "fit_ms": round(fit_ms, 3), "fit_rows": n_fit,
+            "fit_tflops": round(2.0 * K * K * n_fit / (fit_ms * 1e-3) / 1e12, 2),
+            "preconditioner_ms": round(pow_ms, 1), "newton_schulz_iterations": args.fisher_iters,
+            "preconditioner_tflops": round(gemm_flops / (pow_ms * 1e-3) / 1e12, 2),
+            "what": "step = project_grads + precondition_rows (R^-1/2, K=12288) + build_store; "
+                    "fit and R^-1/2 are one-time costs (fp32 FFMA GEMMs)"}
+
+
 def bench_e2e(args, world, dev, state):
     """Same step through the public API with host (pinned) inputs copied in every step."""
     import torch
@@ -562,6 +618,7 @@ def main_ours(args):
     coll, state = bench_collection(args, world, dev, peaks, peak_kind)
     onthefly = bench_onthefly(args, world, dev, state)
     tokens = bench_tokens(args, world, dev, state, peaks)
+    fisher = bench_fisher(args, world, dev, state) if not args.no_fisher else None
     e2e = bench_e2e(args, world, dev, state) if not args.no_e2e else None
     del state
     torch.cuda.empty_cache()
@@ -587,7 +644,7 @@ def main_ours(args):
                        "l2": "inputs 19.3 GB per step > 129 MB L2 (no flush needed)"},
             "roofline": coll["roofline"], "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": coll["gpu_launches"], "clocks": coll["clocks"],
-            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly, "token_scores": tokens,
+            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly, "token_scores": tokens, "fisher": fisher,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -636,6 +693,8 @@ def parse(argv=None):
     ap.add_argument("--score-steps", type=int, default=5)
     ap.add_argument("--score-warmup", type=int, default=2)
     ap.add_argument("--cpu-examples", type=int, default=4)
+    ap.add_argument("--no-fisher", action="store_true")
+    ap.add_argument("--fisher-iters", type=int, default=20)
     ap.add_argument("--profile-case", choices=["collect", "score"], default=None,
                     help="run a small case of one kernel for ncu and exit")
     return ap.parse_args(argv)

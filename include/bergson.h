@@ -50,6 +50,16 @@ typedef enum {
 } bergson_status;
 
 typedef enum {
+  BERGSON_AGG_SUM = 0,
+  BERGSON_AGG_MEAN = 1
+} bergson_aggregation;
+
+typedef enum {
+  BERGSON_FISHER_INV_SQRT = 0,    /* M = R^-1/2 (whitening, TrackStar) */
+  BERGSON_FISHER_INV = 1          /* M = R^-1 */
+} bergson_fisher_power;
+
+typedef enum {
   BERGSON_PROJ_GAUSSIAN = 0,      /* seeded Gaussian, entries N(0, 1/k) */
   BERGSON_PROJ_IDENTITY = 1       /* P = I, requires k == d (testing aid) */
 } bergson_proj_kind;
@@ -192,6 +202,67 @@ BERGSON_API int bergson_token_scores(const bergson_layer* layers, int n_layers, 
                                      int64_t T, const uint8_t* mask, const float* queries,
                                      int64_t n_queries, int64_t ld_q, float* out,
                                      void* workspace, size_t ws_bytes, void* stream);
+
+/* Bytes of workspace bergson_aggregate_rows needs for n rows. */
+BERGSON_API int bergson_aggregate_rows_workspace(int64_t n, size_t* ws_bytes);
+
+/*
+ * Query aggregation (Bergson Sec. 3.2: queries formed as the mean or sum of
+ * the gradients of several generations or dataset items, as LESS builds its
+ * evaluation queries; Fig. 2 "unit_normalize: true, aggregation: mean"):
+ *
+ *   out[g, 0:K] = agg over r in [offsets[g], offsets[g+1]) of  w_r * rows[r, 0:K]
+ *
+ * with w_r = 1/||rows[r, 0:K]|| when normalize_each (0 for a zero row) else 1,
+ * and agg = sum (BERGSON_AGG_SUM) or mean (BERGSON_AGG_MEAN).  An empty group
+ * gives a zero row.  Rows are added in order (deterministic).
+ *   rows     fp32 [n, ld], out fp32 [G, ld_out]: 16-byte aligned, ld % 4 == 0.
+ *   K        multiple of 4.
+ *   offsets  DEVICE int64 [G + 1], non-decreasing within [0, n] (entries
+ *            outside are clamped; a decreasing pair is an empty group).
+ *   workspace  needed only when normalize_each (size from the query above).
+ * Errors: EINVAL, EALIGN, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_aggregate_rows(const float* rows, int64_t n, int64_t K, int64_t ld,
+                                       const int64_t* offsets, int64_t G, int mode,
+                                       int normalize_each, float* out, int64_t ld_out,
+                                       void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * TrackStar's empirical-Fisher preconditioner (Bergson Sec. 3.1: the
+ * empirical Fisher information matrix of TrackStar, stacked with optimizer
+ * normalisation and down-projection; Fig. 2: Fisher fitting and mixing).
+ * Three steps, all on the device, fp32:
+ *
+ *   bergson_fisher_fit:             R = (1/n) sum_i x_i x_i^T  over n rows x_i = rows[i, 0:K]
+ *   bergson_fisher_preconditioner:  R = lam R1 + (1 - lam) R2 (R2 = NULL: R = R1),
+ *                                   R += damping * (tr(R) / K) * I,
+ *                                   M = R^-1/2 (BERGSON_FISHER_INV_SQRT) or R^-1,
+ *                                   by `iterations` coupled Newton-Schulz steps
+ *                                   (20-30 reach fp32 accuracy for condition
+ *                                   numbers up to ~1e4-1e6; damping bounds it)
+ *   bergson_precondition_rows:      out[b] = M rows[b]   (M symmetric)
+ *
+ * Preconditioned rows then go through bergson_build_store / bergson_score_topk
+ * (or bergson_score_grads) as usual.  All matrices are fp32 row-major with
+ * 16-byte aligned rows (leading dimensions multiples of 4); K % 4 == 0,
+ * K <= 65536.  Workspaces: bergson_fisher_fit_workspace(n, K),
+ * bergson_fisher_preconditioner_workspace(K) (4 K^2 floats) and, for
+ * precondition_rows, bergson_score_grads_workspace(B, K, K).
+ * Errors: EINVAL, EALIGN, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_fisher_fit_workspace(int64_t n, int64_t K, size_t* ws_bytes);
+BERGSON_API int bergson_fisher_fit(const float* rows, int64_t n, int64_t K, int64_t ld, float* R,
+                                   int64_t ldr, void* workspace, size_t ws_bytes, void* stream);
+BERGSON_API int bergson_fisher_preconditioner_workspace(int64_t K, size_t* ws_bytes);
+BERGSON_API int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K,
+                                              int64_t ldr, float lam, float damping, int power,
+                                              int iterations, float* M, int64_t ldm,
+                                              void* workspace, size_t ws_bytes, void* stream);
+BERGSON_API int bergson_precondition_rows(const float* rows, int64_t B, int64_t K, int64_t ld,
+                                          const float* M, int64_t ldm, float* out,
+                                          int64_t ld_out, void* workspace, size_t ws_bytes,
+                                          void* stream);
 
 /* Bytes of workspace bergson_score_grads needs. */
 BERGSON_API int bergson_score_grads_workspace(int64_t B, int64_t K, int64_t Q, size_t* ws_bytes);

@@ -19,7 +19,13 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
      directly against query rows without a store, as cosines (grad-cosine) or
      plain inner products (grad-dot) -- Table 3's two identity-Hessian methods;
   7. per-token scores (Fig. 1: attribution scores per token or per sequence):
-     the inner product of each token's own projected gradient with a query.
+     the inner product of each token's own projected gradient with a query;
+  8. query aggregation (Sec. 3.2): a query row formed as the mean or sum of
+     several items' (optionally unit-normalised) projected gradients;
+  9. TrackStar's empirical-Fisher preconditioner (Sec. 3.1; Fig. 2 "empirical
+     Fisher information matrix fitting and mixing"): R = (1/n) sum_i x_i x_i^T
+     over projected gradients, a mix of two such matrices plus damping, and
+     its inverse square root (or inverse) applied to rows before unit norm.
 
 Readings taken where the paper is silent (each is listed in the design doc):
   * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
@@ -292,3 +298,50 @@ def token_scores(layers, mask, queries: np.ndarray, examples=None) -> np.ndarray
                 g_hat = double_sided_projection(w, p_out, p_in)
                 out[:, bi, t] += np.einsum("qij,ij->q", qm, g_hat)
     return out
+
+
+AGG_SUM = 0
+AGG_MEAN = 1
+
+
+def aggregate_rows(rows: np.ndarray, offsets, mode: int = AGG_MEAN,
+                   normalize_each: bool = True) -> np.ndarray:
+    """out[g] = sum or mean of rows[offsets[g]:offsets[g+1]] (each unit-normalised first
+    when normalize_each).  An empty group gives a zero row.  fp64."""
+    x = np.asarray(rows, dtype=np.float64)
+    if normalize_each:
+        x, _ = unit_normalize(x)
+    G = len(offsets) - 1
+    out = np.zeros((G, x.shape[1]), dtype=np.float64)
+    for g in range(G):
+        a, b = int(offsets[g]), int(offsets[g + 1])
+        if b > a:
+            acc = x[a:b].sum(axis=0)
+            out[g] = acc / (b - a) if mode == AGG_MEAN else acc
+    return out
+
+
+def fisher_fit(rows: np.ndarray) -> np.ndarray:
+    """Empirical Fisher (autocorrelation) R = (1/n) sum_i x_i x_i^T of n rows, fp64 [K, K]."""
+    x = np.asarray(rows, dtype=np.float64)
+    return x.T @ x / x.shape[0]
+
+
+def fisher_mix(r1: np.ndarray, r2: np.ndarray | None, lam: float, damping: float) -> np.ndarray:
+    """R = lam * R1 + (1 - lam) * R2 (R2 absent: R = R1), plus damping * (tr(R)/K) * I."""
+    r = np.asarray(r1, dtype=np.float64)
+    if r2 is not None:
+        r = lam * r + (1.0 - lam) * np.asarray(r2, dtype=np.float64)
+    K = r.shape[0]
+    return r + damping * (np.trace(r) / K) * np.eye(K)
+
+
+def fisher_power(r: np.ndarray, power: float) -> np.ndarray:
+    """R^power for symmetric positive definite R (power -1/2 or -1) by eigendecomposition."""
+    w, u = np.linalg.eigh(np.asarray(r, dtype=np.float64))
+    return (u * w ** power) @ u.T
+
+
+def precondition_rows(rows: np.ndarray, m: np.ndarray) -> np.ndarray:
+    """x' = M x for every row x (M symmetric): rows @ M."""
+    return np.asarray(rows, dtype=np.float64) @ np.asarray(m, dtype=np.float64)

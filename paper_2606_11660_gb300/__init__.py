@@ -4,6 +4,10 @@ The compute lives in ``libbergson.so`` (CUDA for sm_103a) behind the C ABI of
 ``include/bergson.h``; ``binding`` exposes the same entry points to Python.
 """
 from .binding import (  # noqa: F401
+    BERGSON_FISHER_INV, BERGSON_FISHER_INV_SQRT, bergson_fisher_fit, bergson_fisher_fit_workspace,
+    bergson_fisher_preconditioner, bergson_fisher_preconditioner_workspace,
+    bergson_precondition_rows,
+    BERGSON_AGG_MEAN, BERGSON_AGG_SUM, bergson_aggregate_rows, bergson_aggregate_rows_workspace,
     BERGSON_EALIGN, BERGSON_ECUDA, BERGSON_EDEVICE_TIMEOUT, BERGSON_EINVAL, BERGSON_EUNSUPPORTED,
     BERGSON_EWORKSPACE, BERGSON_OK, BERGSON_PROJ_GAUSSIAN, BERGSON_PROJ_IDENTITY, BergsonError,
     EXPORTED, LIB_PATH, Layer, bergson_build_store, bergson_debug_inject_status,

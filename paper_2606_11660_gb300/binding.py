@@ -26,6 +26,12 @@ BERGSON_EDEVICE_TIMEOUT = -6
 BERGSON_PROJ_GAUSSIAN = 0
 BERGSON_PROJ_IDENTITY = 1
 
+BERGSON_AGG_SUM = 0
+BERGSON_AGG_MEAN = 1
+
+BERGSON_FISHER_INV_SQRT = 0
+BERGSON_FISHER_INV = 1
+
 STATUS_NAMES = {
     0: "BERGSON_OK", -1: "BERGSON_EINVAL", -2: "BERGSON_EALIGN", -3: "BERGSON_EUNSUPPORTED",
     -4: "BERGSON_EWORKSPACE", -5: "BERGSON_ECUDA", -6: "BERGSON_EDEVICE_TIMEOUT",
@@ -38,7 +44,9 @@ EXPORTED = (
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
     "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_project_grads_noalloc",
     "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
-    "bergson_token_scores",
+    "bergson_token_scores", "bergson_aggregate_rows_workspace", "bergson_aggregate_rows",
+    "bergson_fisher_fit_workspace", "bergson_fisher_fit", "bergson_fisher_preconditioner_workspace",
+    "bergson_fisher_preconditioner", "bergson_precondition_rows",
 )
 
 
@@ -91,6 +99,16 @@ def lib() -> ctypes.CDLL:
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
+        "bergson_aggregate_rows_workspace": (i32, [i64, szp]),
+        "bergson_fisher_fit_workspace": (i32, [i64, i64, szp]),
+        "bergson_fisher_fit": (i32, [vp, i64, i64, i64, vp, i64, vp, ctypes.c_size_t, vp]),
+        "bergson_fisher_preconditioner_workspace": (i32, [i64, szp]),
+        "bergson_fisher_preconditioner": (i32, [vp, vp, i64, i64, ctypes.c_float, ctypes.c_float,
+                                                i32, i32, vp, i64, vp, ctypes.c_size_t, vp]),
+        "bergson_precondition_rows": (i32, [vp, i64, i64, i64, vp, i64, vp, i64, vp,
+                                            ctypes.c_size_t, vp]),
+        "bergson_aggregate_rows": (i32, [vp, i64, i64, i64, vp, i64, i32, i32, vp, i64, vp,
+                                         ctypes.c_size_t, vp]),
         "bergson_token_scores": (i32, [lp, i32, i64, i64, vp, vp, i64, i64, vp, vp,
                                        ctypes.c_size_t, vp]),
         "bergson_score_grads": (i32, [vp, i64, i64, i64, vp, i64, i64, i32, vp, i64, vp,
@@ -226,6 +244,60 @@ def bergson_token_scores(layers: Sequence, B: int, T: int, mask, queries, out, w
     _check(lib().bergson_token_scores(arr, len(layers), int(B), int(T), _ptr(mask), _ptr(queries),
                                       int(queries.shape[0]), int(queries.stride(0)), _ptr(out),
                                       _ptr(workspace), ws_bytes, _stream(stream)))
+
+
+def bergson_aggregate_rows_workspace(n: int) -> int:
+    m = ctypes.c_size_t()
+    _check(lib().bergson_aggregate_rows_workspace(int(n), ctypes.byref(m)))
+    return m.value
+
+
+def bergson_aggregate_rows(rows, n: int, K: int, offsets, mode: int, normalize_each: bool, out,
+                           workspace=None, stream=None) -> None:
+    """out[g] = sum/mean of rows[offsets[g]:offsets[g+1]] (offsets: device int64 [G+1])."""
+    G = int(offsets.shape[0]) - 1
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().bergson_aggregate_rows(_ptr(rows), int(n), int(K), int(rows.stride(0)),
+                                        _ptr(offsets), G, int(mode), 1 if normalize_each else 0,
+                                        _ptr(out), int(out.stride(0)), _ptr(workspace), ws_bytes,
+                                        _stream(stream)))
+
+
+def bergson_fisher_fit_workspace(n: int, K: int) -> int:
+    m = ctypes.c_size_t()
+    _check(lib().bergson_fisher_fit_workspace(int(n), int(K), ctypes.byref(m)))
+    return m.value
+
+
+def bergson_fisher_fit(rows, n: int, K: int, R, workspace, stream=None) -> None:
+    """R = (1/n) sum_i rows[i] rows[i]^T (empirical Fisher of projected gradients)."""
+    _check(lib().bergson_fisher_fit(_ptr(rows), int(n), int(K), int(rows.stride(0)), _ptr(R),
+                                    int(R.stride(0)), _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def bergson_fisher_preconditioner_workspace(K: int) -> int:
+    m = ctypes.c_size_t()
+    _check(lib().bergson_fisher_preconditioner_workspace(int(K), ctypes.byref(m)))
+    return m.value
+
+
+def bergson_fisher_preconditioner(R1, R2, K: int, lam: float, damping: float, power: int,
+                                  iterations: int, M, workspace, stream=None) -> None:
+    """M = (lam R1 + (1-lam) R2 + damping tr/K I)^-1/2 (or ^-1)."""
+    _check(lib().bergson_fisher_preconditioner(
+        _ptr(R1), _ptr(R2), int(K), int(R1.stride(0)), float(lam), float(damping), int(power),
+        int(iterations), _ptr(M), int(M.stride(0)), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def bergson_precondition_rows(rows, B: int, K: int, M, out, workspace, stream=None) -> None:
+    """out[b] = M rows[b] (M symmetric K x K)."""
+    _check(lib().bergson_precondition_rows(_ptr(rows), int(B), int(K), int(rows.stride(0)),
+                                           _ptr(M), int(M.stride(0)), _ptr(out),
+                                           int(out.stride(0)), _ptr(workspace),
+                                           workspace.numel() * workspace.element_size(),
+                                           _stream(stream)))
 
 
 def bergson_score_grads_workspace(B: int, K: int, Q: int) -> int:

@@ -729,6 +729,160 @@ int bergson_score_grads(const float* proj, int64_t B, int64_t K, int64_t ld_proj
   return BERGSON_OK;
 }
 
+int bergson_aggregate_rows_workspace(int64_t n, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (n < 0 || n > (1ll << 31) - 1) return fail(BERGSON_EINVAL, "n must be in [0, 2^31)");
+  *ws_bytes = round_up(sizeof(float) * static_cast<size_t>(n > 0 ? n : 1), 256);
+  return BERGSON_OK;
+}
+
+int bergson_aggregate_rows(const float* rows, int64_t n, int64_t K, int64_t ld,
+                           const int64_t* offsets, int64_t G, int mode, int normalize_each,
+                           float* out, int64_t ld_out, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  if (n < 0 || n > (1ll << 31) - 1 || G < 0 || G > (1ll << 31) - 1)
+    return fail(BERGSON_EINVAL, "n and G must be in [0, 2^31)");
+  if (K < 4 || K > (1 << 28)) return fail(BERGSON_EINVAL, "K must be in [4, 2^28]");
+  if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
+  if (mode != BERGSON_AGG_SUM && mode != BERGSON_AGG_MEAN)
+    return fail(BERGSON_EINVAL, "unknown aggregation mode %d", mode);
+  if (ld < K || ld_out < K) return fail(BERGSON_EINVAL, "ld and ld_out must be >= K");
+  if (G > 0) {
+    if (offsets == nullptr || out == nullptr)
+      return fail(BERGSON_EINVAL, "offsets or out is NULL");
+    if (n > 0 && rows == nullptr) return fail(BERGSON_EINVAL, "rows is NULL");
+    if ((rows && !aligned(rows, 16)) || !aligned(out, 16) || ld % 4 != 0 || ld_out % 4 != 0)
+      return fail(BERGSON_EALIGN, "rows and out need 16-byte aligned rows");
+    if (!aligned(offsets, 8)) return fail(BERGSON_EALIGN, "offsets must be 8-byte aligned");
+  }
+  const size_t need = round_up(sizeof(float) * static_cast<size_t>(n > 0 ? n : 1), 256);
+  if (normalize_each && n > 0) {
+    if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+    if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+    if (ws_bytes < need)
+      return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  }
+  int st;
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (G == 0) return BERGSON_OK;
+  DeviceGuard dg(out);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* scale = nullptr;
+  cudaError_t e = cudaSuccess;
+  if (normalize_each && n > 0) {
+    scale = static_cast<float*>(workspace);
+    e = launch_row_scales(rows, static_cast<int>(n), static_cast<int>(K), ld, 1, scale, s);
+    if (e != cudaSuccess) return fail_cuda(e, "row norm launch");
+  }
+  e = launch_aggregate(rows, n, static_cast<int>(K), ld, offsets, static_cast<int>(G), mode, scale,
+                       out, ld_out, s);
+  if (e != cudaSuccess) return fail_cuda(e, "aggregation launch");
+  return BERGSON_OK;
+}
+
+static int check_square(const float* r, int64_t K, int64_t ld, const char* name) {
+  if (r == nullptr) return fail(BERGSON_EINVAL, "%s is NULL", name);
+  if (ld < K) return fail(BERGSON_EINVAL, "%s: leading dimension < K", name);
+  if (!aligned(r, 16) || ld % 4 != 0)
+    return fail(BERGSON_EALIGN, "%s needs 16-byte aligned rows", name);
+  return BERGSON_OK;
+}
+
+int bergson_fisher_fit_workspace(int64_t n, int64_t K, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (n < 1 || n > (1 << 24) || K < 4 || K > (1 << 16))
+    return fail(BERGSON_EINVAL, "n must be in [1, 2^24] and K in [4, 65536]");
+  *ws_bytes = round_up(fisher_fit_workspace(n, K), 256);
+  return BERGSON_OK;
+}
+
+int bergson_fisher_fit(const float* rows, int64_t n, int64_t K, int64_t ld, float* R, int64_t ldr,
+                       void* workspace, size_t ws_bytes, void* stream) {
+  if (n < 1 || n > (1 << 24) || K < 4 || K > (1 << 16))
+    return fail(BERGSON_EINVAL, "n must be in [1, 2^24] and K in [4, 65536]");
+  if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
+  if (rows == nullptr) return fail(BERGSON_EINVAL, "rows is NULL");
+  if (ld < K) return fail(BERGSON_EINVAL, "ld must be >= K");
+  int st = check_square(R, K, ldr, "R");
+  if (st != BERGSON_OK) return st;
+  const size_t need = round_up(fisher_fit_workspace(n, K), 256);
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  if ((st = injected()) != BERGSON_OK) return st;
+  DeviceGuard dg(R);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  cudaError_t e = launch_fisher_fit(rows, static_cast<int>(n), static_cast<int>(K), ld, R, ldr,
+                                    static_cast<float*>(workspace),
+                                    static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "Fisher fit launch");
+  return BERGSON_OK;
+}
+
+int bergson_fisher_preconditioner_workspace(int64_t K, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (K < 4 || K > (1 << 16)) return fail(BERGSON_EINVAL, "K must be in [4, 65536]");
+  *ws_bytes = round_up(fisher_power_workspace(K), 256);
+  return BERGSON_OK;
+}
+
+int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K, int64_t ldr,
+                                  float lam, float damping, int power, int iterations, float* M,
+                                  int64_t ldm, void* workspace, size_t ws_bytes, void* stream) {
+  if (K < 4 || K > (1 << 16)) return fail(BERGSON_EINVAL, "K must be in [4, 65536]");
+  if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
+  int st = check_square(R1, K, ldr, "R1");
+  if (st != BERGSON_OK) return st;
+  if (R2 != nullptr && (st = check_square(R2, K, ldr, "R2")) != BERGSON_OK) return st;
+  if ((st = check_square(M, K, ldm, "M")) != BERGSON_OK) return st;
+  if (!(lam >= 0.0f && lam <= 1.0f)) return fail(BERGSON_EINVAL, "lam must be in [0, 1]");
+  if (!(damping >= 0.0f)) return fail(BERGSON_EINVAL, "damping must be >= 0");
+  if (power != BERGSON_FISHER_INV_SQRT && power != BERGSON_FISHER_INV)
+    return fail(BERGSON_EINVAL, "unknown power %d", power);
+  if (iterations < 1 || iterations > 100) return fail(BERGSON_EINVAL, "iterations in [1, 100]");
+  const size_t need = round_up(fisher_power_workspace(K), 256);
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  if ((st = injected()) != BERGSON_OK) return st;
+  DeviceGuard dg(M);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  cudaError_t e = launch_fisher_power(R1, R2, static_cast<int>(K), ldr, lam, damping,
+                                      power == BERGSON_FISHER_INV ? 1 : 0, iterations, M, ldm,
+                                      static_cast<float*>(workspace),
+                                      static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "Fisher preconditioner launch");
+  return BERGSON_OK;
+}
+
+int bergson_precondition_rows(const float* rows, int64_t B, int64_t K, int64_t ld, const float* M,
+                              int64_t ldm, float* out, int64_t ld_out, void* workspace,
+                              size_t ws_bytes, void* stream) {
+  int st = validate_onthefly(rows, B, K, ld, M, K, ldm, out, ld_out);
+  if (st != BERGSON_OK) return st;
+  if (B > 0 && !aligned(out, 4)) return fail(BERGSON_EALIGN, "out must be 4-byte aligned");
+  const size_t need = onthefly_workspace(B, K, K);
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (B == 0) return BERGSON_OK;
+  DeviceGuard dg(workspace);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  float* partial = reinterpret_cast<float*>(ws + round_up(sizeof(float) * B, 256) +
+                                            round_up(sizeof(float) * K, 256));
+  cudaError_t e = launch_onthefly(rows, static_cast<int>(B), ld, M, static_cast<int>(K), ldm,
+                                  static_cast<int>(K), 0, nullptr, nullptr, partial, out, ld_out,
+                                  static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "preconditioning launch");
+  return BERGSON_OK;
+}
+
 int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind,
                               const float* moment, float* out, void* stream) {
   if (d < 1 || d > (1 << 24)) return fail(BERGSON_EINVAL, "d must be in [1, 2^24]");

@@ -114,7 +114,19 @@ cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, in
                          int q_begin, int q_end, int qg_base, float* out_scores, int64_t* out_idx,
                          cudaStream_t s);
 
+cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit, float* scale,
+                              cudaStream_t s);
+cudaError_t launch_aggregate(const float* rows, int64_t n, int K, int64_t ld,
+                             const int64_t* offsets, int G, int mode, const float* scale,
+                             float* out, int64_t ld_out, cudaStream_t s);
 int onthefly_splits(int64_t B, int64_t Q, int64_t K);
+size_t fisher_fit_workspace(int64_t n, int64_t K);
+cudaError_t launch_fisher_fit(const float* x, int n, int K, int64_t ldx, float* r, int64_t ldr,
+                              float* ws, cudaStream_t s);
+size_t fisher_power_workspace(int64_t K);
+cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
+                                float damping, int inverse, int iterations, float* m, int64_t ldm,
+                                float* ws, cudaStream_t s);
 cudaError_t launch_onthefly(const float* x, int B, int64_t ldx, const float* y, int Q,
                             int64_t ldy, int K, int unit, float* sx, float* sy, float* partial,
                             float* scores, int64_t ld_scores, cudaStream_t s);

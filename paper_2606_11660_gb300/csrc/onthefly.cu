@@ -143,11 +143,18 @@ __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, i
     float s = 0.0f;
     for (int z = 0; z < S; ++z) s += partial[z * n + i];
     const int b = static_cast<int>(i / Q), q = static_cast<int>(i % Q);
-    scores[b * ld + q] = s * sx[b] * sy[q];
+    scores[b * ld + q] = sx != nullptr ? s * sx[b] * sy[q] : s;
   }
 }
 
 }  // namespace
+
+cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit, float* scale,
+                              cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  row_scales_kernel<<<n, kRowThreads, 0, s>>>(x, K, ld, unit, scale);
+  return cudaGetLastError();
+}
 
 int onthefly_splits(int64_t B, int64_t Q, int64_t K) {
   const int64_t tiles = ((Q + kBN - 1) / kBN) * ((B + kBM - 1) / kBM);
@@ -166,8 +173,12 @@ cudaError_t launch_onthefly(const float* x, int B, int64_t ldx, const float* y, 
   if (B == 0 || Q == 0) return cudaSuccess;
   const int S = onthefly_splits(B, Q, K);
   const int slice = ((K + S - 1) / S + kBK - 1) / kBK * kBK;
-  row_scales_kernel<<<B, kRowThreads, 0, s>>>(x, K, ldx, unit, sx);
-  row_scales_kernel<<<Q, kRowThreads, 0, s>>>(y, K, ldy, unit, sy);
+  if (unit) {                  // plain products need no norms
+    row_scales_kernel<<<B, kRowThreads, 0, s>>>(x, K, ldx, unit, sx);
+    row_scales_kernel<<<Q, kRowThreads, 0, s>>>(y, K, ldy, unit, sy);
+  } else {
+    sx = sy = nullptr;
+  }
   dim3 grid((Q + kBN - 1) / kBN, (B + kBM - 1) / kBM, S);
   dot_partials_kernel<<<grid, kThreads, 0, s>>>(x, B, ldx, y, Q, ldy, K, slice, partial);
   const int64_t n = static_cast<int64_t>(B) * Q;

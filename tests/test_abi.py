@@ -182,3 +182,44 @@ def test_onthefly_validation():
     assert call(queries=None) == bg.BERGSON_EINVAL
     assert call(B=0) == bg.BERGSON_OK
     assert call(Q=0) == bg.BERGSON_OK
+
+
+def test_aggregate_validation():
+    f = bg.lib().bergson_aggregate_rows
+
+    def call(rows=FAKE, n=10, K=64, ld=64, offsets=FAKE, G=3, mode=1, norm=1, out=FAKE,
+             ld_out=64, ws=FAKE, ws_bytes=1 << 20):
+        return f(rows, n, K, ld, offsets, G, mode, norm, out, ld_out, ws, ws_bytes, None)
+    assert call(K=62) == bg.BERGSON_EALIGN
+    assert call(mode=5) == bg.BERGSON_EINVAL
+    assert call(ld=60) == bg.BERGSON_EINVAL
+    assert call(offsets=None) == bg.BERGSON_EINVAL
+    assert call(offsets=FAKE + 4) == bg.BERGSON_EALIGN
+    assert call(ws_bytes=8) == bg.BERGSON_EWORKSPACE
+    assert call(G=0) == bg.BERGSON_OK
+
+
+def test_fisher_validation():
+    L = bg.lib()
+    n = ctypes.c_size_t()
+    assert L.bergson_fisher_preconditioner_workspace(256, ctypes.byref(n)) == bg.BERGSON_OK
+    assert n.value >= 4 * 256 * 256 * 4
+    f = L.bergson_fisher_preconditioner
+    ok = dict(R1=FAKE, R2=None, K=256, ldr=256, lam=0.5, damping=0.1, power=0, iters=20, M=FAKE,
+              ldm=256, ws=FAKE, wsb=n.value)
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        return f(*a.values(), None)
+    assert call(K=254) == bg.BERGSON_EALIGN
+    assert call(lam=1.5) == bg.BERGSON_EINVAL
+    assert call(damping=-1.0) == bg.BERGSON_EINVAL
+    assert call(power=7) == bg.BERGSON_EINVAL
+    assert call(iters=0) == bg.BERGSON_EINVAL
+    assert call(R1=None) == bg.BERGSON_EINVAL
+    assert call(M=FAKE + 4) == bg.BERGSON_EALIGN
+    assert call(wsb=16) == bg.BERGSON_EWORKSPACE
+    fit = L.bergson_fisher_fit
+    assert fit(FAKE, 0, 256, 256, FAKE, 256, FAKE, 1 << 30, None) == bg.BERGSON_EINVAL
+    assert fit(FAKE, 10, 256, 200, FAKE, 256, FAKE, 1 << 30, None) == bg.BERGSON_EINVAL

@@ -328,3 +328,48 @@ def test_token_scores_identity_closed_form():
             a = L.A[0, t].astype(np.float64)
             want = sum(g[i] * Qm[i, j] * a[j] for i in range(d_out) for j in range(d_in))
             assert abs(tok[q, 0, t] - want) < 1e-10 * max(1.0, abs(want))
+
+
+# --- query aggregation --------------------------------------------------------
+
+def test_aggregate_rows_closed_forms():
+    r = RNG.standard_normal(30)
+    X = np.stack([r, 2 * r, 5 * r, RNG.standard_normal(30), RNG.standard_normal(30)])
+    offs = [0, 3, 3, 5]                                   # groups: 3 rows, empty, 2 rows
+    mean_n = orc.aggregate_rows(X, offs, orc.AGG_MEAN, True)
+    np.testing.assert_allclose(mean_n[0], r / np.linalg.norm(r), atol=1e-14)   # same direction
+    np.testing.assert_array_equal(mean_n[1], 0.0)
+    sum_raw = orc.aggregate_rows(X, offs, orc.AGG_SUM, False)
+    np.testing.assert_allclose(sum_raw[0], 8 * r, atol=1e-13)
+    np.testing.assert_allclose(sum_raw[2], X[3] + X[4], atol=1e-14)
+    mean_raw = orc.aggregate_rows(X, offs, orc.AGG_MEAN, False)
+    np.testing.assert_allclose(mean_raw[2], 0.5 * (X[3] + X[4]), atol=1e-14)
+    # scores of a mean-aggregated query are the mean of the members' scores
+    store, _ = orc.build_store(RNG.standard_normal((7, 30)))
+    S_members = store.astype(np.float64) @ orc.unit_normalize(X[3:5])[0].T
+    np.testing.assert_allclose(store.astype(np.float64) @ mean_n[2], S_members.mean(axis=1), atol=1e-13)
+
+
+# --- empirical-Fisher preconditioner ------------------------------------------
+
+def test_fisher_fit_mix_power_apply():
+    n, K = 40, 12
+    X = RNG.standard_normal((n, K)) @ np.diag(np.linspace(0.2, 3.0, K))
+    R = orc.fisher_fit(X)
+    want = np.zeros((K, K))
+    for i in range(n):
+        want += np.outer(X[i], X[i])
+    np.testing.assert_allclose(R, want / n, atol=1e-13)
+    assert np.all(np.linalg.eigvalsh(R) > 0)
+    R2 = orc.fisher_fit(RNG.standard_normal((n, K)))
+    Rm = orc.fisher_mix(R, R2, 0.25, 0.1)
+    np.testing.assert_allclose(Rm, 0.25 * R + 0.75 * R2 + 0.1 * np.trace(0.25 * R + 0.75 * R2) / K * np.eye(K),
+                               atol=1e-13)
+    M = orc.fisher_power(Rm, -0.5)
+    np.testing.assert_allclose(M @ Rm @ M, np.eye(K), atol=1e-10)       # whitening
+    np.testing.assert_allclose(M, M.T, atol=1e-12)
+    Minv = orc.fisher_power(Rm, -1.0)
+    np.testing.assert_allclose(Minv @ Rm, np.eye(K), atol=1e-10)
+    # preconditioned rows are whitened: their Fisher under M is the identity
+    Xp = orc.precondition_rows(X, orc.fisher_power(orc.fisher_mix(R, None, 1.0, 0.0), -0.5))
+    np.testing.assert_allclose(orc.fisher_fit(Xp), np.eye(K), atol=1e-10)
