@@ -383,7 +383,8 @@ def bench_tokens(args, world, dev, state, peaks):
     return {"value": round(cfg.B * world / (ms * 1e-3), 2), "unit": "examples/s",
             "ms_per_step": round(ms, 4), "queries": Q,
             "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"],
-                         "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4)},
+                         "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4),
+                         "traffic": profiled_traffic("project_kernel_pythia160m.md", "project.cu")},
             "gpu_launches": 5 * args.steps,
             "what": "bergson_token_scores: per-token scores of all 65,536 tokens x 48 modules "
                     "against 4 query rows"}
@@ -569,7 +570,44 @@ def profile_case(args):
     from paper_2606_11660_gb300 import workloads as wl
     __graft_entry__.build()
     dev = torch.device("cuda", 0)
-    if args.profile_case == "collect":
+    if args.profile_case == "tokens":
+        # one block of the Pythia-160M-shaped workload, B=8, T=2048, 4 query rows
+        cfg = wl.PYTHIA160M
+        B = 8
+        mask = wl.right_padding_mask(B, cfg.T, cfg.max_pad, seed=1, device=dev)
+        layers = []
+        for m, spec in enumerate(cfg.block_modules(0)):
+            A, G = wl.layer_inputs(spec, B, cfg.T, seed=10_000 + m, device=dev, input_scale=True)
+            s_in, s_out = bg.bergson_module_seeds(0, m)
+            layers.append(bg.Layer(A, G, cfg.k, cfg.k, s_in, s_out, None, None, cfg.col_offset(m)))
+        queries = wl.gaussian_rows(4, 4 * cfg.k * cfg.k, seed=13, device=dev)
+        ws = bg.workspace_tensor(bg.bergson_token_scores_workspace(layers, B, cfg.T, 4), dev)
+        out = torch.empty((4, B, cfg.T), dtype=torch.float32, device=dev)
+        for _ in range(2):
+            bg.bergson_token_scores(layers, B, cfg.T, mask, queries, out, ws)
+        st = bg.bergson_sync_status()
+    elif args.profile_case == "onthefly":
+        # 32 rows x 12288 against 4096 queries (201 MB of queries, > L2)
+        B, K, Q = 32, 12288, 4096
+        x = wl.gaussian_rows(B, K, seed=15, device=dev)
+        y = wl.gaussian_rows(Q, K, seed=16, device=dev)
+        ws = bg.workspace_tensor(bg.bergson_score_grads_workspace(B, K, Q), dev)
+        out = torch.empty((B, Q), dtype=torch.float32, device=dev)
+        for _ in range(2):
+            bg.bergson_score_grads(x, B, K, y, True, out, ws)
+        st = bg.bergson_sync_status()
+    elif args.profile_case == "fisher":
+        # one Newton-Schulz iteration at K = 8192 (256 MB per matrix)
+        K = 8192
+        x = wl.gaussian_rows(2048, K, seed=17, device=dev)
+        R = torch.empty((K, K), device=dev)
+        M = torch.empty((K, K), device=dev)
+        fws = bg.workspace_tensor(bg.bergson_fisher_fit_workspace(2048, K), dev)
+        bg.bergson_fisher_fit(x, 2048, K, R, fws)
+        pws = bg.workspace_tensor(bg.bergson_fisher_preconditioner_workspace(K), dev)
+        bg.bergson_fisher_preconditioner(R, None, K, 1.0, 0.1, bg.BERGSON_FISHER_INV_SQRT, 1, M, pws)
+        st = bg.bergson_sync_status()
+    elif args.profile_case == "collect":
         # one block (4 modules) of the Pythia-160M-shaped workload, B=8, T=2048: 403 MB
         cfg = wl.PYTHIA160M
         B = 8
@@ -695,7 +733,8 @@ def parse(argv=None):
     ap.add_argument("--cpu-examples", type=int, default=4)
     ap.add_argument("--no-fisher", action="store_true")
     ap.add_argument("--fisher-iters", type=int, default=20)
-    ap.add_argument("--profile-case", choices=["collect", "score"], default=None,
+    ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "fisher"],
+                    default=None,
                     help="run a small case of one kernel for ncu and exit")
     return ap.parse_args(argv)
 

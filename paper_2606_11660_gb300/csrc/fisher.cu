@@ -162,12 +162,16 @@ __global__ void mix_kernel(const float* __restrict__ r1, const float* __restrict
   }
 }
 
-// scal[1] = ||R||_F, scal[2] = 1/||R||_F, scal[3] = 1/sqrt(||R||_F), scal[4] = 1/||R||_F
-__global__ void frob_kernel(const float* __restrict__ r, int64_t ld, int K, float* __restrict__ scal) {
+constexpr int kFrobBlocks = 512;
+
+// part[blockIdx] = compensated sum of squares over a grid-stride slice of R.
+__global__ void frob_partial_kernel(const float* __restrict__ r, int64_t ld, int K,
+                                    float* __restrict__ part) {
   __shared__ float red[32];
   float s = 0.0f, comp = 0.0f;
   const int64_t n = static_cast<int64_t>(K) * K;
-  for (int64_t e = threadIdx.x; e < n; e += blockDim.x) {
+  for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n;
+       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const float x = r[(e / K) * ld + e % K];
     const float y = x * x - comp;
     const float t = s + y;
@@ -181,12 +185,26 @@ __global__ void frob_kernel(const float* __restrict__ r, int64_t ld, int K, floa
   if (threadIdx.x == 0) {
     float t = 0.0f;
     for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += red[w];
-    const float c = sqrtf(t);
-    scal[1] = c;
-    scal[2] = 1.0f / c;
-    scal[3] = 1.0f / sqrtf(c);
-    scal[4] = 1.0f / c;
+    part[blockIdx.x] = t;
   }
+}
+
+// scal[1] = ||R||_F, scal[2] = 1/c, scal[3] = 1/sqrt(c), scal[4] = 1/c  (fixed-order sum)
+__global__ void frob_final_kernel(const float* __restrict__ part, int n_part,
+                                  float* __restrict__ scal) {
+  if (threadIdx.x != 0) return;
+  float t = 0.0f, comp = 0.0f;
+  for (int i = 0; i < n_part; ++i) {
+    const float y = part[i] - comp;
+    const float u = t + y;
+    comp = (u - t) - y;
+    t = u;
+  }
+  const float c = sqrtf(t);
+  scal[1] = c;
+  scal[2] = 1.0f / c;
+  scal[3] = 1.0f / sqrtf(c);
+  scal[4] = 1.0f / c;
 }
 
 // y = r * scal[2] (R / c); z = I
@@ -263,7 +281,7 @@ cudaError_t launch_fisher_fit(const float* x, int n, int K, int64_t ldx, float* 
 }
 
 size_t fisher_power_workspace(int64_t K) {
-  return (4 * static_cast<size_t>(K) * K + 64) * sizeof(float);
+  return (4 * static_cast<size_t>(K) * K + 64 + kFrobBlocks) * sizeof(float);
 }
 
 cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
@@ -274,10 +292,11 @@ cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t
   float* y = a + kk;
   float* z = y + kk;
   float* t = z + kk;
-  float* scal = t + kk;     // trace, ||R||_F, 1/c, 1/sqrt(c), 1/c
+  float* scal = t + kk;     // trace, ||R||_F, 1/c, 1/sqrt(c), 1/c; [64, 64 + 512): partial sums
   mixed_trace_kernel<<<1, 1024, 0, s>>>(r1, r2, ldr, K, lam, scal);
   mix_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(r1, r2, ldr, K, lam, damping, scal, a, K);
-  frob_kernel<<<1, 1024, 0, s>>>(a, K, K, scal);
+  frob_partial_kernel<<<kFrobBlocks, 256, 0, s>>>(a, K, K, scal + 64);
+  frob_final_kernel<<<1, 32, 0, s>>>(scal + 64, kFrobBlocks, scal);
   ns_init_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(a, K, K, scal, y, z);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
