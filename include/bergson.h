@@ -60,6 +60,10 @@ typedef enum {
 } bergson_fisher_power;
 
 typedef enum {
+  BERGSON_LAYER_BIAS = 1          /* also write the layer's projected bias gradient */
+} bergson_layer_flags;
+
+typedef enum {
   BERGSON_PROJ_GAUSSIAN = 0,      /* seeded Gaussian, entries N(0, 1/k) */
   BERGSON_PROJ_IDENTITY = 1       /* P = I, requires k == d (testing aid) */
 } bergson_proj_kind;
@@ -82,6 +86,11 @@ typedef enum {
  *          NULL for no normalisation.  The gradient is divided elementwise by
  *          sqrt(r_i c_j).
  *   out_col_offset   first column of this module's k_out*k_in block in `out`.
+ *   flags  0 or BERGSON_LAYER_BIAS.  With BERGSON_LAYER_BIAS the projected
+ *          bias gradient P_out^T (sum over valid tokens of g_t / sqrt(r)) --
+ *          App. B, gradients of linear "weight and bias" -- is written as
+ *          k_out values at bias_col_offset (bergson_project_grads only; the
+ *          per-token scores cover the weight blocks).
  */
 typedef struct bergson_layer {
   const void* A;
@@ -93,10 +102,11 @@ typedef struct bergson_layer {
   uint64_t seed_in;
   uint64_t seed_out;
   int32_t proj_kind;
-  int32_t reserved;               /* must be 0 */
+  int32_t flags;                  /* bergson_layer_flags */
   const float* r;
   const float* c;
   int64_t out_col_offset;
+  int64_t bias_col_offset;        /* used with BERGSON_LAYER_BIAS */
 } bergson_layer;
 
 /* Bytes of workspace bergson_project_grads needs for these arguments. */

@@ -25,7 +25,9 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
   9. TrackStar's empirical-Fisher preconditioner (Sec. 3.1; Fig. 2 "empirical
      Fisher information matrix fitting and mixing"): R = (1/n) sum_i x_i x_i^T
      over projected gradients, a mix of two such matrices plus damping, and
-     its inverse square root (or inverse) applied to rows before unit norm.
+     its inverse square root (or inverse) applied to rows before unit norm;
+ 10. bias gradients (App. B, "linear (weight and bias) parameters"):
+     sum_t m_t g_t, scaled by r^-1/2 and projected with P_out (k_out values).
 
 Readings taken where the paper is silent (each is listed in the design doc):
   * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
@@ -144,15 +146,24 @@ def double_sided_projection(w: np.ndarray, p_out: np.ndarray, p_in: np.ndarray) 
     return p_out.T @ w @ p_in
 
 
+def bias_gradient(g: np.ndarray, m: np.ndarray | None) -> np.ndarray:
+    """Per-example bias gradient sum over valid tokens t of g_t, shape [d_out], fp64."""
+    g = np.asarray(g, dtype=np.float64)
+    if m is not None:
+        g = g[np.asarray(m) != 0]
+    return g.sum(axis=0)
+
+
 class Layer:
     """One nn.Linear's captured tensors and projection settings (host arrays).
 
     A: [B, T, d_in], G: [B, T, d_out] (any float dtype; bf16 values arrive as
-    exact fp32), r: [d_out] or None, c: [d_in] or None.
+    exact fp32), r: [d_out] or None, c: [d_in] or None.  bias_col_offset >= 0
+    also places the projected bias gradient (k_out values) at that column.
     """
 
     def __init__(self, A, G, k_in, k_out, seed_in, seed_out, r=None, c=None,
-                 col_offset=0, proj_kind=PROJ_GAUSSIAN):
+                 col_offset=0, proj_kind=PROJ_GAUSSIAN, bias_col_offset=-1):
         self.A = np.asarray(A)
         self.G = np.asarray(G)
         self.k_in = int(k_in)
@@ -163,6 +174,7 @@ class Layer:
         self.c = None if c is None else np.asarray(c, dtype=np.float64)
         self.col_offset = int(col_offset)
         self.proj_kind = int(proj_kind)
+        self.bias_col_offset = int(bias_col_offset)
 
     @property
     def d_in(self):
@@ -199,12 +211,30 @@ def project_grads(layers, mask, ld_out: int | None = None, examples=None) -> np.
     B = layers[0].A.shape[0]
     examples = list(range(B)) if examples is None else list(examples)
     if ld_out is None:
-        ld_out = max(l.col_offset + l.k_out * l.k_in for l in layers)
+        ld_out = max(max(l.col_offset + l.k_out * l.k_in, l.bias_col_offset + l.k_out)
+                     for l in layers)
     out = np.zeros((len(examples), ld_out), dtype=np.float64)
     for layer in layers:
         blk = layer.k_out * layer.k_in
         out[:, layer.col_offset:layer.col_offset + blk] = project_module(layer, mask, examples)
+        if layer.bias_col_offset >= 0:
+            out[:, layer.bias_col_offset:layer.bias_col_offset + layer.k_out] = \
+                project_bias(layer, mask, examples)
     return out
+
+
+def project_bias(layer: Layer, mask: np.ndarray | None, examples=None) -> np.ndarray:
+    """P_out^T (bias gradient / sqrt(r)) per example, [len(examples), k_out]."""
+    B = layer.A.shape[0]
+    examples = range(B) if examples is None else examples
+    p_out = projection_matrix(layer.seed_out, layer.d_out, layer.k_out, layer.proj_kind)
+    rows = []
+    for b in examples:
+        gb = bias_gradient(layer.G[b], None if mask is None else mask[b])
+        if layer.r is not None:
+            gb = gb / np.sqrt(layer.r)
+        rows.append(p_out.T @ gb)
+    return np.stack(rows) if rows else np.zeros((0, layer.k_out))
 
 
 def unit_normalize(x: np.ndarray) -> tuple[np.ndarray, np.ndarray]:

@@ -26,6 +26,8 @@ BERGSON_EDEVICE_TIMEOUT = -6
 BERGSON_PROJ_GAUSSIAN = 0
 BERGSON_PROJ_IDENTITY = 1
 
+BERGSON_LAYER_BIAS = 1
+
 BERGSON_AGG_SUM = 0
 BERGSON_AGG_MEAN = 1
 
@@ -62,9 +64,9 @@ class bergson_layer(ctypes.Structure):
         ("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64),
         ("k_in", ctypes.c_int64), ("k_out", ctypes.c_int64),
         ("seed_in", ctypes.c_uint64), ("seed_out", ctypes.c_uint64),
-        ("proj_kind", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("proj_kind", ctypes.c_int32), ("flags", ctypes.c_int32),
         ("r", ctypes.c_void_p), ("c", ctypes.c_void_p),
-        ("out_col_offset", ctypes.c_int64),
+        ("out_col_offset", ctypes.c_int64), ("bias_col_offset", ctypes.c_int64),
     ]
 
 
@@ -157,13 +159,17 @@ class Layer:
     c: object = None
     out_col_offset: int = 0
     proj_kind: int = BERGSON_PROJ_GAUSSIAN
+    bias_col_offset: Optional[int] = None     # set to also write the projected bias gradient
 
     def to_c(self) -> bergson_layer:
+        bias = self.bias_col_offset is not None
         return bergson_layer(
             A=_ptr(self.A), G=_ptr(self.G), d_in=int(self.A.shape[-1]), d_out=int(self.G.shape[-1]),
             k_in=int(self.k_in), k_out=int(self.k_out), seed_in=int(self.seed_in),
-            seed_out=int(self.seed_out), proj_kind=int(self.proj_kind), reserved=0,
-            r=_ptr(self.r), c=_ptr(self.c), out_col_offset=int(self.out_col_offset))
+            seed_out=int(self.seed_out), proj_kind=int(self.proj_kind),
+            flags=BERGSON_LAYER_BIAS if bias else 0, r=_ptr(self.r), c=_ptr(self.c),
+            out_col_offset=int(self.out_col_offset),
+            bias_col_offset=int(self.bias_col_offset) if bias else 0)
 
 
 def _layer_array(layers: Sequence) -> "ctypes.Array":

@@ -125,7 +125,9 @@ struct Group {
   std::vector<int> layers;     // indices into the caller's array, call order
   int first_mod = 0;           // index of its first ModDesc in workspace
   int n_chunks = 0, tpc = 0, n_items = 0;
+  bool has_bias = false;
   size_t partial_off = 0;
+  size_t bias_off = 0;
 };
 
 struct ProjLayout {
@@ -148,7 +150,10 @@ int validate_layers(const bergson_layer* layers, int n_layers, int64_t B, int64_
     return fail(BERGSON_EUNSUPPORTED, "B*T too large");
   for (int i = 0; i < n_layers; ++i) {
     const bergson_layer& L = layers[i];
-    if (L.reserved != 0) return fail(BERGSON_EINVAL, "layer %d: reserved field must be 0", i);
+    if ((L.flags & ~BERGSON_LAYER_BIAS) != 0)
+      return fail(BERGSON_EINVAL, "layer %d: unknown flags 0x%x", i, L.flags);
+    if ((L.flags & BERGSON_LAYER_BIAS) && L.bias_col_offset < 0)
+      return fail(BERGSON_EINVAL, "layer %d: negative bias_col_offset", i);
     if (L.d_in < 8 || L.d_out < 8 || L.d_in > (1 << 24) || L.d_out > (1 << 24))
       return fail(BERGSON_EINVAL, "layer %d: d_in/d_out must be in [8, 2^24]", i);
     if (L.d_in % 8 != 0 || L.d_out % 8 != 0)
@@ -173,7 +178,8 @@ int validate_layers(const bergson_layer* layers, int n_layers, int64_t B, int64_
   return BERGSON_OK;
 }
 
-int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out) {
+int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out,
+                    bool with_bias = true) {
   std::vector<std::pair<int64_t, int64_t>> blk;
   for (int i = 0; i < n_layers; ++i) {
     const int64_t a = layers[i].out_col_offset;
@@ -182,6 +188,13 @@ int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out) {
       return fail(BERGSON_EINVAL, "layer %d: block [%lld, %lld) exceeds ld_out=%lld", i,
                   (long long)a, (long long)e, (long long)ld_out);
     blk.emplace_back(a, e);
+    if (with_bias && (layers[i].flags & BERGSON_LAYER_BIAS)) {
+      const int64_t ba = layers[i].bias_col_offset, be = ba + layers[i].k_out;
+      if (be > ld_out)
+        return fail(BERGSON_EINVAL, "layer %d: bias block [%lld, %lld) exceeds ld_out=%lld", i,
+                    (long long)ba, (long long)be, (long long)ld_out);
+      blk.emplace_back(ba, be);
+    }
   }
   std::sort(blk.begin(), blk.end());
   for (size_t i = 1; i < blk.size(); ++i)
@@ -209,6 +222,7 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
       it->k_out = ko;
     }
     it->layers.push_back(i);
+    if (layers[i].flags & BERGSON_LAYER_BIAS) it->has_bias = true;
   }
   int slot = 0;
   for (Group& g : L.groups) {
@@ -258,6 +272,10 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
     for (Group& g : L.groups) {
       g.partial_off = off;
       off += round_up(static_cast<size_t>(g.n_items) * g.k_in * g.k_out * sizeof(float), 256);
+      if (g.has_bias) {
+        g.bias_off = off;
+        off += round_up(static_cast<size_t>(g.n_items) * kTileTokens * sizeof(float), 256);
+      }
     }
   }
   L.total = off;
@@ -394,7 +412,7 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
                     i, cap, (long long)layers[i].k_in, (long long)layers[i].k_out);
     }
     if (ld_q < 0) return fail(BERGSON_EINVAL, "ld_q must be >= 0");
-    st = validate_blocks(layers, n_layers, ld_q);
+    st = validate_blocks(layers, n_layers, ld_q, false);
     if (st != BERGSON_OK) return st;
     if (queries == nullptr) return fail(BERGSON_EINVAL, "queries is NULL");
     if (!aligned(queries, 4)) return fail(BERGSON_EALIGN, "queries must be 4-byte aligned");
@@ -434,6 +452,7 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
     md.d_in = static_cast<int32_t>(ly.d_in);
     md.d_out = static_cast<int32_t>(ly.d_out);
     md.col_offset = ly.out_col_offset;
+    md.bias_col_offset = (ly.flags & BERGSON_LAYER_BIAS) ? ly.bias_col_offset : -1;
     __nv_bfloat16* pin = reinterpret_cast<__nv_bfloat16*>(ws + L.pin_off[i]);
     __nv_bfloat16* pout = reinterpret_cast<__nv_bfloat16*>(ws + L.pout_off[i]);
     if (T > 0) {
@@ -497,6 +516,7 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
       p.mask = mask;
       p.tile_valid = tile_valid;
       p.partials = partials;
+      p.bias_partials = (g.has_bias && !token) ? reinterpret_cast<float*>(ws + g.bias_off) : nullptr;
       p.queries = queries;
       p.ld_q = ld_q;
       p.n_queries = static_cast<int>(n_queries);
@@ -510,7 +530,9 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
     }
     if (!token) {
       e = launch_reduce(mods_dev + g.first_mod, static_cast<int>(g.layers.size()), g.k_in,
-                        g.k_out, static_cast<int>(B), g.n_chunks, partials, out, ld_out, s);
+                        g.k_out, static_cast<int>(B), g.n_chunks, partials,
+                        g.has_bias ? reinterpret_cast<const float*>(ws + g.bias_off) : nullptr,
+                        out, ld_out, s);
       if (e != cudaSuccess) return fail_cuda(e, "reduce launch");
     }
   }

@@ -27,7 +27,8 @@ struct ModDesc {
   int32_t d_in;
   int32_t d_out;
   int64_t col_offset;
-  int64_t reserved[6];
+  int64_t bias_col_offset;   // -1: no bias block
+  int64_t reserved[5];
 };
 static_assert(alignof(ModDesc) >= 64 && sizeof(ModDesc) % 64 == 0, "TMA needs 64-byte aligned maps");
 
@@ -56,6 +57,7 @@ struct ProjParams {
   const uint8_t* mask;        // [B, T] or nullptr
   const uint8_t* tile_valid;  // [B, n_tiles] 4-bit masks of valid 32-token slices, or nullptr
   float* partials;            // [n_items, k_out * k_in]   (projection mode)
+  float* bias_partials;       // [n_items, 128] column sums of g~, or nullptr (no bias)
   const float* queries;       // [n_queries, ld_q] query rows          (token mode)
   int64_t ld_q;
   int n_queries;
@@ -100,8 +102,8 @@ int token_query_capacity(int k_in, int k_out);
 cudaError_t launch_token_reduce(const float* token_partials, int n_mods, int Q, int B, int T,
                                 const uint8_t* mask, float* out, cudaStream_t s);
 cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, int B,
-                          int n_chunks, const float* partials, float* out, int64_t ld_out,
-                          cudaStream_t s);
+                          int n_chunks, const float* partials, const float* bias_partials,
+                          float* out, int64_t ld_out, cudaStream_t s);
 
 cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj, int unit,
                                __half* store, int64_t ld_store, float* norms, cudaStream_t s);

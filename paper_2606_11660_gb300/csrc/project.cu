@@ -292,6 +292,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
     int ss = 0;
     uint32_t sph = 0;
     float acc[OPT];
+    float bias_acc = 0.0f;   // column (et % KO) of g~ summed over rows (et / KO)*KO .. +KO
     for (;;) {
       if (et == 0) {
         if (!mbar_wait(smem_u32(&sfull[ss]), sph, tmo, s_abort))
@@ -308,6 +309,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       const ItemCoord ic = decode_item(p, item);
 #pragma unroll
       for (int x = 0; x < OPT; ++x) acc[x] = 0.0f;
+      bias_acc = 0.0f;
       if constexpr (TOKEN) {
         // This module's k_out x k_in block of every query row, into the
         // (otherwise unused) staging area.  All threads left the previous
@@ -398,6 +400,11 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
                                         vg[nt][4 * x + 3])
                           : z4;
           named_bar_sync(1, 128);
+          if (p.bias_partials != nullptr) {      // projected bias gradient: sum_t g~_t
+            const int col = et % KO, r0 = (et / KO) * KO;
+#pragma unroll 4
+            for (int i = 0; i < KO; ++i) bias_acc += sG[(r0 + i) * (KO + 4) + col];
+          }
 #pragma unroll 4
           for (int t2 = 0; t2 < kTileTokens; ++t2) {
             const float gv = sG[t2 * (KO + 4) + oi];
@@ -429,6 +436,8 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
 #pragma unroll
       for (int x = 0; x < OPT / 2; ++x)
         reinterpret_cast<float2*>(dst)[x] = make_float2(acc[2 * x], acc[2 * x + 1]);
+      if (p.bias_partials != nullptr)
+        p.bias_partials[static_cast<int64_t>(item) * kTileTokens + et] = bias_acc;
     }
   }
 
@@ -441,8 +450,11 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
 }
 
 // out[b, off_m + e] = sum over chunks c (in order) of partials[(m*B + b)*n_chunks + c][e]
-__global__ void reduce_kernel(const ModDesc* __restrict__ mods, int B, int blk, int n_chunks,
-                              const float* __restrict__ partials, float* __restrict__ out,
+// and, for layers with a bias block, out[b, bias_off + i] = sum over chunks and
+// row groups (in order) of the items' column sums of g~.
+__global__ void reduce_kernel(const ModDesc* __restrict__ mods, int B, int blk, int k_out,
+                              int n_chunks, const float* __restrict__ partials,
+                              const float* __restrict__ bias_partials, float* __restrict__ out,
                               int64_t ld_out) {
   const int mb = blockIdx.x;
   const int m = mb / B;
@@ -453,6 +465,17 @@ __global__ void reduce_kernel(const ModDesc* __restrict__ mods, int B, int blk, 
     float s = 0.0f;
     for (int c = 0; c < n_chunks; ++c) s += src[static_cast<int64_t>(c) * blk + e];
     dst[e] = s;
+  }
+  const int64_t boff = mods[m].bias_col_offset;
+  if (bias_partials != nullptr && boff >= 0) {
+    const float* bsrc = bias_partials + static_cast<int64_t>(mb) * n_chunks * kTileTokens;
+    for (int i = threadIdx.x; i < k_out; i += blockDim.x) {
+      float s = 0.0f;
+      for (int c = 0; c < n_chunks; ++c)
+        for (int rg = 0; rg < kTileTokens / k_out; ++rg)
+          s += bsrc[static_cast<int64_t>(c) * kTileTokens + rg * k_out + i];
+      out[static_cast<int64_t>(b) * ld_out + boff + i] = s;
+    }
   }
 }
 
@@ -561,13 +584,13 @@ size_t project_smem_bytes(int k_in, int k_out) {
 }
 
 cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, int B,
-                          int n_chunks, const float* partials, float* out, int64_t ld_out,
-                          cudaStream_t s) {
+                          int n_chunks, const float* partials, const float* bias_partials,
+                          float* out, int64_t ld_out, cudaStream_t s) {
   const int blocks = n_mods * B;
   if (blocks == 0) return cudaSuccess;
   const int blk = k_in * k_out;
-  reduce_kernel<<<blocks, blk < 1024 ? blk : 1024, 0, s>>>(mods, B, blk, n_chunks, partials, out,
-                                                          ld_out);
+  reduce_kernel<<<blocks, blk < 1024 ? blk : 1024, 0, s>>>(mods, B, blk, k_out, n_chunks, partials,
+                                                          bias_partials, out, ld_out);
   return cudaGetLastError();
 }
 

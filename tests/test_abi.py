@@ -43,7 +43,7 @@ FAKE = 0x7F0000000000  # aligned, never dereferenced: validation fails first or 
 
 def _layer(**kw):
     d = dict(A=FAKE, G=FAKE + 4096, d_in=64, d_out=64, k_in=16, k_out=16, seed_in=1, seed_out=2,
-             proj_kind=0, reserved=0, r=None, c=None, out_col_offset=0)
+             proj_kind=0, flags=0, r=None, c=None, out_col_offset=0)
     d.update(kw)
     return bg.bergson_layer(**d)
 
@@ -71,7 +71,8 @@ def _proj(layers, B=2, T=32, out=FAKE, ld_out=256, ws=FAKE, ws_bytes=1 << 30, ma
     (dict(r=FAKE), bg.BERGSON_EINVAL),                 # r without c
     (dict(A=FAKE + 8), bg.BERGSON_EALIGN),
     (dict(G=None), bg.BERGSON_EINVAL),
-    (dict(reserved=1), bg.BERGSON_EINVAL),
+    (dict(flags=2), bg.BERGSON_EINVAL),
+    (dict(flags=1, bias_col_offset=-3), bg.BERGSON_EINVAL),
     (dict(out_col_offset=-1), bg.BERGSON_EINVAL),
 ])
 def test_layer_validation(kw, code):

@@ -289,3 +289,30 @@ def test_bounded_wait_reports_timeout_and_context_survives():
     assert bg.bergson_sync_status() == bg.BERGSON_EDEVICE_TIMEOUT
     assert bg.bergson_sync_status() == bg.BERGSON_OK  # cleared
     test_tiny_workload_parity()                      # the context still works
+
+
+def test_bias_blocks_with_mask_and_moments():
+    specs = [wl.ModuleSpec("a", 64, 200), wl.ModuleSpec("b", 136, 64), wl.ModuleSpec("c", 96, 72)]
+    kp = [(16, 16), (32, 32), (16, 32)]
+    B, T = 3, 300
+    gl, ol, ld = make_layers(specs, B, T, kp, base_seed=9, data_seed=4, rc=True)
+    # bias blocks after the weight blocks, for layers 0 and 2 only
+    gl[0].bias_col_offset = ol[0].bias_col_offset = ld
+    gl[2].bias_col_offset = ol[2].bias_col_offset = ld + 16
+    ld_b = ld + 16 + 32
+    g = wl.generator(10, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.3).to(torch.uint8)
+    mask[1, 128:256] = 0
+    out = run_project(gl, B, T, mask.to(DEV), ld_b)
+    want = orc.project_grads(ol, mask.numpy(), ld_b)
+    got = np32(out).astype(np.float64)
+    assert rel_frobenius(got, want).max() <= TIGHT
+    for off, k in ((ld, 16), (ld + 16, 32)):
+        blk_g, blk_w = got[:, off:off + k], want[:, off:off + k]
+        assert rel_frobenius(blk_g, blk_w).max() <= TIGHT
+    # overlapping a bias block with a weight block is rejected
+    gl[2].bias_col_offset = 8
+    ws = bg.workspace_tensor(1 << 24, DEV)
+    with pytest.raises(bg.BergsonError) as e:
+        bg.bergson_project_grads(gl, B, T, None, out, ws)
+    assert e.value.status == bg.BERGSON_EINVAL

@@ -373,3 +373,38 @@ def test_fisher_fit_mix_power_apply():
     # preconditioned rows are whitened: their Fisher under M is the identity
     Xp = orc.precondition_rows(X, orc.fisher_power(orc.fisher_mix(R, None, 1.0, 0.0), -0.5))
     np.testing.assert_allclose(orc.fisher_fit(Xp), np.eye(K), atol=1e-10)
+
+
+# --- bias gradients -----------------------------------------------------------
+
+def test_bias_gradient_finite_differences_and_augmented_input():
+    T, d_in, d_out = 8, 5, 4
+    W = RNG.standard_normal((d_out, d_in))
+    bias = RNG.standard_normal(d_out)
+    a = RNG.standard_normal((T, d_in))
+    u = RNG.standard_normal((T, d_out))
+    m = (RNG.random(T) > 0.3).astype(np.float64)
+
+    def loss(bv):
+        y = a @ W.T + bv
+        return float(np.sum(m[:, None] * (u * y + 0.5 * y * y)))
+    g = u + a @ W.T + bias                       # dL/dy_t
+    gb = orc.bias_gradient(g, m)
+    h = 1e-6
+    fd = np.array([(loss(bias + h * np.eye(d_out)[i]) - loss(bias - h * np.eye(d_out)[i])) / (2 * h)
+                   for i in range(d_out)])
+    assert np.max(np.abs(gb - fd)) / np.max(np.abs(fd)) < 1e-7
+    # the bias is the weight of a constant-one input feature
+    a_aug = np.concatenate([a, np.ones((T, 1))], axis=1)
+    np.testing.assert_allclose(orc.per_example_gradient(a_aug, g, m)[:, -1], gb, rtol=1e-13)
+
+
+def test_projected_bias_identity_and_offsets():
+    B, T, d = 2, 6, 16
+    L = _layer(B, T, d, d, d, d, rc=True, kind=orc.PROJ_IDENTITY)
+    L.bias_col_offset = d * d
+    out = orc.project_grads([L], None)
+    assert out.shape == (B, d * d + d)
+    for b in range(B):
+        want = L.G[b].astype(np.float64).sum(axis=0) / np.sqrt(L.r)
+        np.testing.assert_allclose(out[b, d * d:], want, rtol=1e-12)

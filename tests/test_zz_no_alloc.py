@@ -61,7 +61,7 @@ def test_noalloc_rejects_requests_larger_than_its_scratch():
     # projection slices alone, more than the fixed scratch; nothing is enqueued.
     fake = 0x7F0000000000
     L = bg.bergson_layer(A=fake, G=fake, d_in=8192, d_out=8192, k_in=64, k_out=64, seed_in=1,
-                         seed_out=2, proj_kind=0, reserved=0, r=None, c=None, out_col_offset=0)
+                         seed_out=2, proj_kind=0, flags=0, r=None, c=None, out_col_offset=0)
     arr = (bg.bergson_layer * 8)()
     for m in range(8):
         arr[m] = L
