@@ -348,6 +348,22 @@ BERGSON_API int bergson_debug_wait_probe(uint64_t timeout_ns, void* stream);
 BERGSON_API void bergson_debug_inject_status(int status, int count);
 
 /*
+ * On-disk gradient store (Bergson Sec. 3.1: gradient stores persisted to disk,
+ * read back as memory maps).  The file is N rows of K fp16 values, row-major,
+ * with no header (numpy.memmap(path, dtype=float16, shape=(N, K)) opens it).
+ *   bergson_store_save: rows [0, rows) of the device store -> file rows
+ *     [file_row_offset, file_row_offset + rows); creates or extends the file.
+ *   bergson_store_load: file rows [file_row_offset, +rows) -> device store rows [0, rows).
+ * Both synchronise `stream` first and return when the data has moved (host
+ * I/O through a bounce buffer; not a hot-path call).
+ * Errors: EINVAL (bad arguments, I/O failure, file too short), ECUDA.
+ */
+BERGSON_API int bergson_store_save(const void* store, int64_t rows, int64_t K, int64_t ld_store,
+                                   const char* path, int64_t file_row_offset, void* stream);
+BERGSON_API int bergson_store_load(const char* path, int64_t file_row_offset, int64_t rows,
+                                   int64_t K, void* store, int64_t ld_store, void* stream);
+
+/*
  * Allocation-free variant of bergson_project_grads.  The paper has no
  * counterpart: this exists for callers that cannot supply a workspace, such as
  * plugin or callback interfaces that hand over only input and output buffers,

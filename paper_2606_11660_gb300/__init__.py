@@ -4,6 +4,7 @@ The compute lives in ``libbergson.so`` (CUDA for sm_103a) behind the C ABI of
 ``include/bergson.h``; ``binding`` exposes the same entry points to Python.
 """
 from .binding import (  # noqa: F401
+    bergson_store_load, bergson_store_save,
     BERGSON_LAYER_BIAS,
     BERGSON_FISHER_INV, BERGSON_FISHER_INV_SQRT, bergson_fisher_fit, bergson_fisher_fit_workspace,
     bergson_fisher_preconditioner, bergson_fisher_preconditioner_workspace,

@@ -48,7 +48,8 @@ EXPORTED = (
     "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
     "bergson_token_scores", "bergson_aggregate_rows_workspace", "bergson_aggregate_rows",
     "bergson_fisher_fit_workspace", "bergson_fisher_fit", "bergson_fisher_preconditioner_workspace",
-    "bergson_fisher_preconditioner", "bergson_precondition_rows",
+    "bergson_fisher_preconditioner", "bergson_precondition_rows", "bergson_store_save",
+    "bergson_store_load",
 )
 
 
@@ -102,6 +103,8 @@ def lib() -> ctypes.CDLL:
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
         "bergson_aggregate_rows_workspace": (i32, [i64, szp]),
+        "bergson_store_save": (i32, [vp, i64, i64, i64, ctypes.c_char_p, i64, vp]),
+        "bergson_store_load": (i32, [ctypes.c_char_p, i64, i64, i64, vp, i64, vp]),
         "bergson_fisher_fit_workspace": (i32, [i64, i64, szp]),
         "bergson_fisher_fit": (i32, [vp, i64, i64, i64, vp, i64, vp, ctypes.c_size_t, vp]),
         "bergson_fisher_preconditioner_workspace": (i32, [i64, szp]),
@@ -304,6 +307,20 @@ def bergson_precondition_rows(rows, B: int, K: int, M, out, workspace, stream=No
                                            int(out.stride(0)), _ptr(workspace),
                                            workspace.numel() * workspace.element_size(),
                                            _stream(stream)))
+
+
+def bergson_store_save(store, rows: int, K: int, path: str, file_row_offset: int = 0,
+                       stream=None) -> None:
+    """Write device store rows [0, rows) to the raw fp16 store file at path."""
+    _check(lib().bergson_store_save(_ptr(store), int(rows), int(K), int(store.stride(0)),
+                                    os.fsencode(path), int(file_row_offset), _stream(stream)))
+
+
+def bergson_store_load(path: str, file_row_offset: int, rows: int, K: int, store,
+                       stream=None) -> None:
+    """Read file rows [file_row_offset, +rows) into device store rows [0, rows)."""
+    _check(lib().bergson_store_load(os.fsencode(path), int(file_row_offset), int(rows), int(K),
+                                    _ptr(store), int(store.stride(0)), _stream(stream)))
 
 
 def bergson_score_grads_workspace(B: int, K: int, Q: int) -> int:

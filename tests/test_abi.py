@@ -224,3 +224,10 @@ def test_fisher_validation():
     fit = L.bergson_fisher_fit
     assert fit(FAKE, 0, 256, 256, FAKE, 256, FAKE, 1 << 30, None) == bg.BERGSON_EINVAL
     assert fit(FAKE, 10, 256, 200, FAKE, 256, FAKE, 1 << 30, None) == bg.BERGSON_EINVAL
+
+
+def test_store_io_validation(tmp_path):
+    L = bg.lib()
+    assert L.bergson_store_save(FAKE, 10, 64, 32, b"/tmp/x", 0, None) == bg.BERGSON_EINVAL
+    assert L.bergson_store_save(FAKE, 10, 64, 64, b"", 0, None) == bg.BERGSON_EINVAL
+    assert L.bergson_store_load(str(tmp_path / "missing").encode(), 0, 1, 64, FAKE, 64, None) == bg.BERGSON_EINVAL
