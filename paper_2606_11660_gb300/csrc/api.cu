@@ -20,7 +20,7 @@ namespace {
 
 constexpr int kVersion = 100;                        // 0.1.0
 constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 s
-constexpr int kSchedTargetItems = 2048;              // work items per projection launch (target)
+constexpr int kSchedTargetItems = 8192;              // work items per projection launch (target)
 constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
 constexpr int kMaxDevices = 64;
 constexpr int64_t kPrefixRowsPerTopk = 512;          // prefix pass: 512 * topk store rows
@@ -228,7 +228,7 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
   for (Group& g : L.groups) {
     g.first_mod = slot;
     for (int li : g.layers) L.mod_slot[li] = slot++;
-    const int nt_per_group = (g.k_in + g.k_out <= 64) ? 2 : 1;
+    const int nt_per_group = (g.k_in + g.k_out <= 32) ? 4 : ((g.k_in + g.k_out <= 64) ? 2 : 1);
     const int64_t mb = static_cast<int64_t>(g.layers.size()) * B;
     if (L.n_tiles == 0 || mb == 0) {
       g.n_chunks = 0;
