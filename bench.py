@@ -446,6 +446,68 @@ def bench_fisher(args, world, dev, state):
                     "fit and R^-1/2 are one-time costs (fp32 FFMA GEMMs)"}
 
 
+def bench_streamed(args, world, dev, name, peaks):
+    """A streamed workload: one transformer block per bergson_project_grads call, all
+    blocks of one batch, then the store rows.  One block's inputs are generated
+    and reused for every block (each call still reads them from HBM)."""
+    import torch
+
+    import paper_2606_11660_gb300 as bg
+    from paper_2606_11660_gb300 import workloads as wl
+
+    cfg = wl.COLLECT_WORKLOADS[name]
+    nmod = cfg.modules_per_block
+    specs = cfg.block_modules(0)
+    tensors = []
+    for j, spec in enumerate(specs):
+        A, G = wl.layer_inputs(spec, cfg.B, cfg.T, seed=20_000 + j, device=dev, input_scale=True)
+        r = c = None
+        if cfg.second_moments:
+            r, c = wl.second_moments(spec.d_out, spec.d_in, seed=30_000 + j, device=dev)
+        tensors.append((A, G, r, c))
+    calls = []
+    for blk in range(cfg.blocks):
+        layers = []
+        for j, (A, G, r, c) in enumerate(tensors):
+            m = blk * nmod + j
+            s_in, s_out = bg.bergson_module_seeds(0, m)
+            layers.append(bg.Layer(A, G, cfg.k, cfg.k, s_in, s_out, r, c, cfg.col_offset(m)))
+        calls.append(layers)
+    ws = bg.workspace_tensor(bg.bergson_project_grads_workspace(calls[0], cfg.B, cfg.T), dev)
+    out = torch.empty((cfg.B, cfg.k_total), dtype=torch.float32, device=dev)
+    store = torch.empty((cfg.B, cfg.k_total), dtype=torch.float16, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        for layers in calls:
+            bg.bergson_project_grads(layers, cfg.B, cfg.T, None, out, ws, stream)
+        bg.bergson_build_store(out, cfg.B, cfg.k_total, True, store, 0, None, stream)
+
+    step()
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    steps = max(1, min(args.steps, 5))
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1), world) / steps
+    alg = 2 * sum(sp.d_in + sp.d_out for sp in cfg.modules) * cfg.B * cfg.T
+    gbs = alg / (ms * 1e-3) / 1e9
+    del tensors, calls
+    torch.cuda.empty_cache()
+    return {"value": round(cfg.B * world / (ms * 1e-3), 2), "unit": "examples/s",
+            "ms_per_step": round(ms, 3), "calls_per_step": cfg.blocks,
+            "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4),
+                         "algorithmic_bytes_per_step": alg},
+            "config": cfg.name}
+
+
 def bench_e2e(args, world, dev, state):
     """Same step through the public API with host (pinned) inputs copied in every step."""
     import torch
@@ -679,6 +741,9 @@ def main_ours(args):
     del state
     torch.cuda.empty_cache()
     scoring = bench_scoring(args, world, dev, peaks, peak_kind) if not args.no_score else None
+    streamed = None
+    if not args.no_streamed:
+        streamed = {n: bench_streamed(args, world, dev, n, peaks) for n in ("pythia1b4", "llama8b")}
     coll["roofline"]["read_ceiling_gbs"] = read_ceiling(dev)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -701,7 +766,7 @@ def main_ours(args):
                        "l2": "inputs 19.3 GB per step > 129 MB L2 (no flush needed)"},
             "roofline": coll["roofline"], "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": coll["gpu_launches"], "clocks": coll["clocks"],
-            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly, "token_scores": tokens, "fisher": fisher,
+            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly, "token_scores": tokens, "fisher": fisher, "streamed": streamed,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -751,6 +816,7 @@ def parse(argv=None):
     ap.add_argument("--score-warmup", type=int, default=2)
     ap.add_argument("--cpu-examples", type=int, default=4)
     ap.add_argument("--no-fisher", action="store_true")
+    ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--fisher-iters", type=int, default=20)
     ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "fisher"],
                     default=None,
