@@ -122,7 +122,7 @@ bool valid_k(int64_t k) { return k == 16 || k == 32 || k == 64; }
 
 struct Group {
   int k_in = 0, k_out = 0;
-  std::vector<int> layers;     // indices into the caller's array, call order
+  std::vector<int> layers;     // indices into the caller's array, largest module first
   int first_mod = 0;           // index of its first ModDesc in workspace
   int n_chunks = 0, tpc = 0, n_items = 0;
   bool has_bias = false;
@@ -226,6 +226,12 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
   }
   int slot = 0;
   for (Group& g : L.groups) {
+    // Largest modules first: the scheduler hands items out in slot order, so
+    // the last items a launch waits on are the cheapest ones (longest
+    // processing time first).  Cost of one tile is proportional to d_in + d_out.
+    std::stable_sort(g.layers.begin(), g.layers.end(), [&](int a, int b) {
+      return layers[a].d_in + layers[a].d_out > layers[b].d_in + layers[b].d_out;
+    });
     g.first_mod = slot;
     for (int li : g.layers) L.mod_slot[li] = slot++;
     const int nt_per_group = (g.k_in + g.k_out <= 32) ? 4 : ((g.k_in + g.k_out <= 64) ? 2 : 1);
