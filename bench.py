@@ -669,6 +669,24 @@ def profile_case(args):
         pws = bg.workspace_tensor(bg.bergson_fisher_preconditioner_workspace(K), dev)
         bg.bergson_fisher_preconditioner(R, None, K, 1.0, 0.1, bg.BERGSON_FISHER_INV_SQRT, 1, M, pws)
         st = bg.bergson_sync_status()
+    elif args.profile_case in ("streamed_pythia1b4", "streamed_llama8b"):
+        # block 0 of a streamed workload at its full B and T, one call per block
+        # (Pythia-1.4B shape: 2.1 GB of A/G; Llama-8B shape: 4.8 GB)
+        cfg = wl.COLLECT_WORKLOADS[args.profile_case.split("_", 1)[1]]
+        layers = []
+        for m, spec in enumerate(cfg.block_modules(0)):
+            A, G = wl.layer_inputs(spec, cfg.B, cfg.T, seed=20_000 + m, device=dev,
+                                   input_scale=True)
+            r = c = None
+            if cfg.second_moments:
+                r, c = wl.second_moments(spec.d_out, spec.d_in, seed=30_000 + m, device=dev)
+            s_in, s_out = bg.bergson_module_seeds(0, m)
+            layers.append(bg.Layer(A, G, cfg.k, cfg.k, s_in, s_out, r, c, cfg.col_offset(m)))
+        ws = bg.workspace_tensor(bg.bergson_project_grads_workspace(layers, cfg.B, cfg.T), dev)
+        out = torch.empty((cfg.B, cfg.k_total), dtype=torch.float32, device=dev)
+        for _ in range(2):
+            bg.bergson_project_grads(layers, cfg.B, cfg.T, None, out, ws)
+        st = bg.bergson_sync_status()
     elif args.profile_case == "collect":
         # one block (4 modules) of the Pythia-160M-shaped workload, B=8, T=2048: 403 MB
         cfg = wl.PYTHIA160M
@@ -818,7 +836,8 @@ def parse(argv=None):
     ap.add_argument("--no-fisher", action="store_true")
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--fisher-iters", type=int, default=20)
-    ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "fisher"],
+    ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "fisher",
+                             "streamed_pythia1b4", "streamed_llama8b"],
                     default=None,
                     help="run a small case of one kernel for ncu and exit")
     return ap.parse_args(argv)

@@ -44,7 +44,7 @@ EXPORTED = (
     "bergson_project_grads_workspace", "bergson_project_grads", "bergson_build_store",
     "bergson_score_topk_workspace", "bergson_score_topk", "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
-    "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_project_grads_noalloc",
+    "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_debug_project_plan", "bergson_project_grads_noalloc",
     "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
     "bergson_token_scores", "bergson_aggregate_rows_workspace", "bergson_aggregate_rows",
     "bergson_fisher_fit_workspace", "bergson_fisher_fit", "bergson_fisher_preconditioner_workspace",
@@ -84,6 +84,7 @@ def lib() -> ctypes.CDLL:
     L = ctypes.CDLL(LIB_PATH)
     i64, u64, vp, i32 = ctypes.c_int64, ctypes.c_uint64, ctypes.c_void_p, ctypes.c_int
     szp = ctypes.POINTER(ctypes.c_size_t)
+    i64p = ctypes.POINTER(ctypes.c_int64)
     lp = ctypes.POINTER(bergson_layer)
     sig = {
         "bergson_project_grads_workspace": (i32, [lp, i32, i64, i64, szp]),
@@ -99,6 +100,7 @@ def lib() -> ctypes.CDLL:
         "bergson_version": (i32, []),
         "bergson_debug_wait_probe": (i32, [u64, vp]),
         "bergson_debug_inject_status": (None, [i32, i32]),
+        "bergson_debug_project_plan": (i32, [lp, i32, i64, i64, i64p, i64p, i64p]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
@@ -362,6 +364,15 @@ def bergson_debug_wait_probe(timeout_ns: int, stream=None) -> None:
 
 def bergson_debug_inject_status(status: int, count: int) -> None:
     lib().bergson_debug_inject_status(int(status), int(count))
+
+
+def bergson_debug_project_plan(layers, B: int, T: int) -> tuple[int, int, int]:
+    """(slots, work items, pieces) the projection planner chooses; host only."""
+    arr = _layer_array(layers)
+    n = [ctypes.c_int64() for _ in range(3)]
+    _check(lib().bergson_debug_project_plan(arr, len(layers), int(B), int(T),
+                                            *(ctypes.byref(x) for x in n)))
+    return tuple(x.value for x in n)
 
 
 # ------------------------------------------------------------------ helpers

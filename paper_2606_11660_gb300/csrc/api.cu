@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <cstdarg>
 #include <cstdio>
@@ -21,6 +22,13 @@ namespace {
 constexpr int kVersion = 100;                        // 0.1.0
 constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 s
 constexpr int kSchedTargetItems = 8192;              // work items per projection launch (target)
+// Piece splitting of projection slots.  The planner assumes kBalanceCTAs
+// persistent CTAs (one per SM of this part; the launch uses the real count).
+// A launch is split when its largest slot exceeds kSplitShare of one CTA's
+// share of the work, into pieces of about 1/kPiecesPerShare of a share.
+constexpr int kBalanceCTAs = 152;
+constexpr double kSplitShare = 0.4;
+constexpr int kPiecesPerShare = 4;
 constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
 constexpr int kMaxDevices = 64;
 constexpr int64_t kPrefixRowsPerTopk = 512;          // prefix pass: 512 * topk store rows
@@ -124,10 +132,16 @@ struct Group {
   int k_in = 0, k_out = 0;
   std::vector<int> layers;     // indices into the caller's array, largest module first
   int first_mod = 0;           // index of its first ModDesc in workspace
-  int n_chunks = 0, tpc = 0, n_items = 0;
+  int n_chunks = 0, tpc = 0;
+  int n_slots = 0;             // layers * B * n_chunks partials
+  int n_items = 0;             // work items of the launch (= n_slots without a table)
   bool has_bias = false;
   size_t partial_off = 0;
   size_t bias_off = 0;
+  std::vector<WorkItem> table; // work table (empty: item i is fused slot i)
+  int n_split = 0;             // slots cut into pieces
+  int64_t piece_floats = 0;    // token projections stored by pieces
+  size_t table_off = 0, split_cnt_off = 0, piece_off = 0;
 };
 
 struct ProjLayout {
@@ -204,6 +218,71 @@ int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out,
   return BERGSON_OK;
 }
 
+int chunks_of(int64_t d) { return static_cast<int>((d + kChunk - 1) / kChunk); }
+
+// Cuts a group's large slots into pieces when the launch is too coarse for
+// the SMs to finish together (see kSplitShare).  Cost unit: one 64-column
+// chunk of one tile.  The table lists fused slots and pieces largest first.
+void plan_pieces(const bergson_layer* layers, int64_t B, int n_tiles, Group& g) {
+  int64_t total = 0, max_slot = 0;
+  for (int li : g.layers) {
+    const int64_t c = chunks_of(layers[li].d_in) + chunks_of(layers[li].d_out);
+    total += c * n_tiles * B;
+    max_slot = std::max<int64_t>(max_slot, c * std::min(g.tpc, n_tiles));
+  }
+  const double share = static_cast<double>(total) / kBalanceCTAs;
+  if (g.n_slots == 0 || static_cast<double>(max_slot) <= kSplitShare * share) return;
+  const double target = share / kPiecesPerShare;
+  struct Entry {
+    WorkItem w;
+    int64_t cost;
+  };
+  std::vector<Entry> es;
+  int64_t base = 0;
+  int split = 0;
+  for (size_t mi = 0; mi < g.layers.size(); ++mi) {
+    const bergson_layer& ly = layers[g.layers[mi]];
+    const int ca = chunks_of(ly.d_in), cg = chunks_of(ly.d_out);
+    const bool cut = static_cast<double>(ca + cg) * g.tpc > target;
+    // A piece stores and its slot's finisher reloads 4k fp32 bytes per token,
+    // against 128 bytes per token and chunk streamed: pieces of at least k
+    // chunks keep that under 1/16 of the piece's traffic.
+    auto pieces = [&](int ch, int k) {
+      const int n = static_cast<int>(std::ceil(static_cast<double>(ch) * g.tpc / target));
+      return std::max(1, std::min(n, ch / k));
+    };
+    const int n_a = cut ? pieces(ca, g.k_in) : 0, n_g = cut ? pieces(cg, g.k_out) : 0;
+    for (int64_t b = 0; b < B; ++b) {
+      for (int c = 0; c < g.n_chunks; ++c) {
+        const int slot = static_cast<int>((static_cast<int64_t>(mi) * B + b) * g.n_chunks + c);
+        const int tiles = std::min(n_tiles, (c + 1) * g.tpc) - c * g.tpc;
+        if (!cut) {
+          es.push_back({WorkItem{slot, 0, 0, 0, 0, 0, 0, 0, 0}, int64_t{ca + cg} * tiles});
+          continue;
+        }
+        for (int side = 1; side <= 2; ++side) {
+          const int nch = side == 1 ? ca : cg, n = side == 1 ? n_a : n_g;
+          for (int q = 0; q < n; ++q) {
+            const int c0 = static_cast<int>(static_cast<int64_t>(q) * nch / n);
+            const int c1 = static_cast<int>(static_cast<int64_t>(q + 1) * nch / n);
+            es.push_back({WorkItem{slot, side, c0, c1, split, n_a, n_g, q, base},
+                          int64_t{c1 - c0} * tiles});
+          }
+        }
+        base += (int64_t{n_a} * g.k_in + int64_t{n_g} * g.k_out) * g.tpc * kTileTokens;
+        ++split;
+      }
+    }
+  }
+  std::stable_sort(es.begin(), es.end(),
+                   [](const Entry& x, const Entry& y) { return x.cost > y.cost; });
+  g.table.resize(es.size());
+  for (size_t i = 0; i < es.size(); ++i) g.table[i] = es[i].w;
+  g.n_items = static_cast<int>(es.size());
+  g.n_split = split;
+  g.piece_floats = base;
+}
+
 // n_queries > 0 lays out per-token score partials [n_layers, n_queries, B, T]
 // instead of per-item projection partials.
 ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
@@ -250,7 +329,9 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
     tpc = (tpc + nt_per_group - 1) / nt_per_group * nt_per_group;
     g.tpc = tpc;
     g.n_chunks = (L.n_tiles + tpc - 1) / tpc;
-    g.n_items = static_cast<int>(mb * g.n_chunks);
+    g.n_slots = static_cast<int>(mb * g.n_chunks);
+    g.n_items = g.n_slots;
+    if (n_queries == 0) plan_pieces(layers, B, L.n_tiles, g);
   }
   size_t off = 0;
   L.mods_off = off;
@@ -259,7 +340,14 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
   off += round_up(sizeof(PrepSeg) * 2 * n_layers, 256);
   L.ctr_off = off;
   off += round_up(sizeof(int) * 32 * L.groups.size(), 256);
-  L.tv_off = off;
+  for (Group& g : L.groups) {
+    if (g.table.empty()) continue;
+    g.table_off = off;
+    off += round_up(sizeof(WorkItem) * g.table.size(), 256);
+    g.split_cnt_off = off;
+    off += round_up(sizeof(int) * g.n_split, 256);
+  }
+  L.tv_off = off;        // everything before this offset is host-staged each call
   off += round_up(static_cast<size_t>(B) * L.n_tiles, 256);
   L.pin_off.resize(n_layers);
   L.pout_off.resize(n_layers);
@@ -277,10 +365,14 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
   } else {
     for (Group& g : L.groups) {
       g.partial_off = off;
-      off += round_up(static_cast<size_t>(g.n_items) * g.k_in * g.k_out * sizeof(float), 256);
+      off += round_up(static_cast<size_t>(g.n_slots) * g.k_in * g.k_out * sizeof(float), 256);
       if (g.has_bias) {
         g.bias_off = off;
-        off += round_up(static_cast<size_t>(g.n_items) * kTileTokens * sizeof(float), 256);
+        off += round_up(static_cast<size_t>(g.n_slots) * kTileTokens * sizeof(float), 256);
+      }
+      if (g.piece_floats > 0) {
+        g.piece_off = off;
+        off += round_up(static_cast<size_t>(g.piece_floats) * sizeof(float), 256);
       }
     }
   }
@@ -383,6 +475,23 @@ void bergson_module_seeds(uint64_t base_seed, int64_t module_index, uint64_t* se
 }
 
 const char* bergson_last_error(void) { return g_last_error.c_str(); }
+
+int bergson_debug_project_plan(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
+                               int64_t* n_slots, int64_t* n_items, int64_t* n_pieces) {
+  const int st = validate_layers(layers, n_layers, B, T);
+  if (st != BERGSON_OK) return st;
+  const ProjLayout L = plan_project(layers, n_layers, B, T);
+  int64_t slots = 0, items = 0, pieces = 0;
+  for (const Group& g : L.groups) {
+    slots += g.n_slots;
+    items += g.n_items;
+    for (const WorkItem& w : g.table) pieces += w.side != 0;
+  }
+  if (n_slots != nullptr) *n_slots = slots;
+  if (n_items != nullptr) *n_items = items;
+  if (n_pieces != nullptr) *n_pieces = pieces;
+  return BERGSON_OK;
+}
 
 void bergson_debug_inject_status(int status, int count) {
   g_inject_status.store(status);
@@ -491,6 +600,9 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
     so.kind = ly.proj_kind;
     max_pairs = std::max<int64_t>(max_pairs, ly.d_out * ly.k_out / 2);
   }
+  for (const Group& g : L.groups)
+    if (!g.table.empty())
+      std::memcpy(staging.data() + g.table_off, g.table.data(), sizeof(WorkItem) * g.table.size());
   cudaError_t e = cudaMemcpyAsync(ws, staging.data(), staging.size(), cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return fail_cuda(e, "staging copy");
   const ModDesc* mods_dev = reinterpret_cast<const ModDesc*>(ws + L.mods_off);
@@ -519,6 +631,9 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
       p.tpc = g.tpc;
       p.n_chunks = g.n_chunks;
       p.n_items = g.n_items;
+      p.items = g.table.empty() ? nullptr : reinterpret_cast<const WorkItem*>(ws + g.table_off);
+      p.piece_buf = g.piece_floats > 0 ? reinterpret_cast<float*>(ws + g.piece_off) : nullptr;
+      p.split_cnt = g.table.empty() ? nullptr : reinterpret_cast<int*>(ws + g.split_cnt_off);
       p.mask = mask;
       p.tile_valid = tile_valid;
       p.partials = partials;

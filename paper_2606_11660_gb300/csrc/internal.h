@@ -45,6 +45,21 @@ struct PrepSeg {
   int32_t reserved;
 };
 
+// One entry of a projection launch's work table.  A fused item projects both
+// sides of every tile of its slot and contracts them; a piece projects one
+// side over a range of 64-column chunks and stores the fp32 token
+// projections, and the last piece of a slot to finish sums them and contracts.
+struct WorkItem {
+  int32_t slot;              // partial index (m * B + b) * n_chunks + chunk
+  int32_t side;              // 0: fused; 1: A-side piece; 2: G-side piece
+  int32_t ch_begin, ch_end;  // chunk range of a piece
+  int32_t split;             // piece counter index of the slot
+  int32_t n_a, n_g;          // pieces of the slot on the A and G side
+  int32_t piece;             // index of this piece on its side
+  int64_t base;              // float offset of the slot's pieces in piece_buf
+};
+static_assert(sizeof(WorkItem) == 40, "WorkItem layout");
+
 struct ProjParams {
   const ModDesc* mods;
   int n_mods;
@@ -53,7 +68,7 @@ struct ProjParams {
   int n_tiles;          // ceil(T / 128)
   int tpc;              // tiles per work item
   int n_chunks;         // work items per (module, example)
-  int n_items;          // n_mods * B * n_chunks
+  int n_items;          // work items (n_mods * B * n_chunks without a work table)
   const uint8_t* mask;        // [B, T] or nullptr
   const uint8_t* tile_valid;  // [B, n_tiles] 4-bit masks of valid 32-token slices, or nullptr
   float* partials;            // [n_items, k_out * k_in]   (projection mode)
@@ -62,6 +77,9 @@ struct ProjParams {
   int64_t ld_q;
   int n_queries;
   float* token_partials;      // [n_mods, n_queries, B, T]             (token mode)
+  const WorkItem* items;      // [n_items] work table, or nullptr: item i is fused slot i
+  float* piece_buf;           // token projections of pieces (see WorkItem)
+  int* split_cnt;             // per split slot: pieces finished, zero on entry
   int* counter;               // dynamic scheduler, zero on entry
   int* status;                // device status word
   uint64_t timeout_ns;

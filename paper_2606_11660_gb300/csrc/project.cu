@@ -15,9 +15,14 @@
 //   3. four epilogue warps read a~ and g~ out of TMEM (one token per thread),
 //      zero masked tokens, stage them in shared memory and accumulate the
 //      k_out x k_in outer-product sum in fp32 registers.
-// Work items are (module, example, range of tiles); a global counter hands
-// them to persistent CTAs, and each item writes one k_out x k_in partial that
-// a second kernel sums in a fixed order (deterministic result).
+// Slots are (module, example, range of tiles); a global counter hands work
+// items to persistent CTAs, and each slot writes one k_out x k_in partial that
+// a second kernel sums in a fixed order (deterministic result).  Normally one
+// item is one slot.  When a launch has too few slots for the SMs to finish
+// together, the host cuts large slots into pieces (one side, a range of
+// 64-column chunks) listed in a work table: a piece stores its fp32 token
+// projections, and the slot's last piece to finish sums them in piece order and
+// contracts, so the result does not depend on which CTA finished last.
 //
 // Warp roles: warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer,
 // warps 2..5 = epilogue.  Every wait is bounded (see ptx.cuh).
@@ -64,12 +69,34 @@ struct ProjCfg {
 
 struct ItemCoord {
   int m, b, t_begin, t_end;
+  int slot;                 // partial index of the (module, example, tile range)
+  int side;                 // 0: fused; 1 / 2: A / G side piece
+  int ch_begin, ch_end;     // chunk range of a piece
+  int split, n_a, n_g, piece;
+  int64_t base;
 };
 
 __device__ __forceinline__ ItemCoord decode_item(const ProjParams& p, int item) {
   ItemCoord c;
-  const int chunk = item % p.n_chunks;
-  const int mb = item / p.n_chunks;
+  c.slot = item;
+  c.side = 0;
+  c.ch_begin = c.ch_end = 0;
+  c.split = c.n_a = c.n_g = c.piece = 0;
+  c.base = 0;
+  if (p.items != nullptr) {
+    const WorkItem& w = p.items[item];
+    c.slot = w.slot;
+    c.side = w.side;
+    c.ch_begin = w.ch_begin;
+    c.ch_end = w.ch_end;
+    c.split = w.split;
+    c.n_a = w.n_a;
+    c.n_g = w.n_g;
+    c.piece = w.piece;
+    c.base = w.base;
+  }
+  const int chunk = c.slot % p.n_chunks;
+  const int mb = c.slot / p.n_chunks;
   c.b = mb % p.B;
   c.m = mb / p.B;
   c.t_begin = chunk * p.tpc;
@@ -97,6 +124,36 @@ __device__ __forceinline__ uint32_t group_slices(const ProjParams& p, int b, int
     vm |= q4 << (4 * nt);
   }
   return vm;
+}
+
+// Copies this thread's TMEM lane (one token) of N columns to dst (fp32, 16-byte aligned).
+template <int N>
+__device__ __forceinline__ void store_token_row(uint32_t taddr, float* dst) {
+  float v[N];
+#pragma unroll
+  for (int c = 0; c < N / 16; ++c) tmem_ld16(taddr + c * 16, &v[c * 16]);
+#pragma unroll
+  for (int x = 0; x < N / 4; ++x)
+    reinterpret_cast<float4*>(dst)[x] = make_float4(v[4 * x], v[4 * x + 1], v[4 * x + 2], v[4 * x + 3]);
+}
+
+// v = sum over pieces q = 0..n-1 (in order) of the token row src + q * stride.
+// Other CTAs wrote the rows during this launch: the loads bypass L1.
+template <int N>
+__device__ __forceinline__ void sum_token_rows(const float* src, int64_t stride, int n, float (&v)[N]) {
+#pragma unroll
+  for (int x = 0; x < N; ++x) v[x] = 0.0f;
+  for (int q = 0; q < n; ++q) {
+    const float4* s4 = reinterpret_cast<const float4*>(src + q * stride);
+#pragma unroll
+    for (int x = 0; x < N / 4; ++x) {
+      const float4 w = __ldcg(s4 + x);
+      v[4 * x] += w.x;
+      v[4 * x + 1] += w.y;
+      v[4 * x + 2] += w.z;
+      v[4 * x + 3] += w.w;
+    }
+  }
 }
 
 // Tiles (bit nt) that have at least one valid slice.
@@ -130,6 +187,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(s_item + 2);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   volatile int* s_epi_stop = s_abort + 1;   // epilogue leader's broadcast of "stop"
+  volatile int* s_last = s_epi_stop + 1;     // epilogue leader's broadcast of "last piece"
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -188,12 +246,14 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           if (sl == 0) continue;
           const uint32_t act_bytes = __popc(sl) * kSliceBytes;
           for (int side = 0; side < 2 && ok; ++side) {
+            if (ic.side != 0 && side != ic.side - 1) continue;
             const void* tact = side ? static_cast<const void*>(&md->tmG) : &md->tmA;
             const void* tp = side ? static_cast<const void*>(&md->tmPout) : &md->tmPin;
             const int d = side ? md->d_out : md->d_in;
             const uint32_t pbytes = (side ? 2 * KO : 2 * KI) * 128;
-            const int nch = (d + kChunk - 1) / kChunk;
-            for (int ch = 0; ch < nch; ++ch) {
+            const int c0 = ic.side != 0 ? ic.ch_begin : 0;
+            const int c1 = ic.side != 0 ? ic.ch_end : (d + kChunk - 1) / kChunk;
+            for (int ch = c0; ch < c1; ++ch) {
               if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
               const uint32_t fb = smem_u32(&full[stage]);
               mbar_arrive_expect_tx(fb, act_bytes + pbytes);
@@ -246,11 +306,13 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           tc_fence_after();
           const uint32_t dbuf = tmem + ab * C::kTmemPerBuf;
           for (int side = 0; side < 2 && ok; ++side) {
+            if (ic.side != 0 && side != ic.side - 1) continue;
             const int N = side ? KO : KI;
             const uint32_t idesc = make_idesc_f16(kTileTokens, N, true);
             const int d = side ? md->d_out : md->d_in;
-            const int nch = (d + kChunk - 1) / kChunk;
-            for (int ch = 0; ch < nch; ++ch) {
+            const int c0 = ic.side != 0 ? ic.ch_begin : 0;
+            const int c1 = ic.side != 0 ? ic.ch_end : (d + kChunk - 1) / kChunk;
+            for (int ch = c0; ch < c1; ++ch) {
               if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) { ok = false; break; }
               tc_fence_after();
               const uint32_t act = sbase + stage * C::kStageBytes;
@@ -262,7 +324,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
 #pragma unroll
                 for (int kk = 0; kk < kChunk / 16; ++kk) {
                   const uint64_t ad = sw128_desc(act + nt * kActBoxBytes + kk * 32);
-                  umma_f16(dcol, ad, sw128_desc(pp + kk * 32), idesc, (ch | kk) != 0);
+                  umma_f16(dcol, ad, sw128_desc(pp + kk * 32), idesc, ch != c0 || kk != 0);
                   umma_f16(dcol, ad, sw128_desc(pp + N * 128 + kk * 32), idesc, 1u);
                 }
               }
@@ -310,6 +372,53 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       if (++ss == 2) { ss = 0; sph ^= 1; }
       if (item >= p.n_items) break;
       const ItemCoord ic = decode_item(p, item);
+      bool aborted = false;
+      bool finisher = false;       // last piece of its slot: contracts the summed pieces
+      const int64_t stride_a = static_cast<int64_t>(p.tpc) * kTileTokens * KI;
+      const int64_t stride_g = static_cast<int64_t>(p.tpc) * kTileTokens * KO;
+      if constexpr (!TOKEN) {
+        if (ic.side != 0) {
+          // A piece: store this side's token projections of the slot's tiles.
+          float* dst = p.piece_buf + ic.base +
+                       (ic.side == 1 ? ic.piece * stride_a : ic.n_a * stride_a + ic.piece * stride_g);
+          for (int g = ic.t_begin; g < ic.t_end; g += NT) {
+            const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
+            if (vm == 0) continue;
+            if (et == 0) {
+              if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
+                raise_device_error(p.status, s_abort, kStatusTimeout);
+              *s_epi_stop = *s_abort;
+            }
+            named_bar_sync(1, 128);
+            if (*s_epi_stop) { aborted = true; break; }
+            tc_fence_after();
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              if (!(vm >> nt & 1)) continue;
+              const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
+                                     ab * C::kTmemPerBuf + nt * (KI + KO);
+              const int64_t tok = static_cast<int64_t>(g - ic.t_begin + nt) * kTileTokens + row;
+              if (ic.side == 1)
+                store_token_row<KI>(taddr, dst + tok * KI);
+              else
+                store_token_row<KO>(taddr + KI, dst + tok * KO);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+            if (++ab == 2) { ab = 0; aph ^= 1; }
+          }
+          if (aborted) break;
+          // Count the piece; the slot's last piece to finish contracts them all.
+          __threadfence();
+          named_bar_sync(1, 128);
+          if (et == 0) *s_last = atomicAdd(p.split_cnt + ic.split, 1) == ic.n_a + ic.n_g - 1;
+          named_bar_sync(1, 128);
+          if (!*s_last) continue;
+          __threadfence();
+          finisher = true;
+        }
+      }
 #pragma unroll
       for (int x = 0; x < OPT; ++x) acc[x] = 0.0f;
       bias_acc = 0.0f;
@@ -323,34 +432,44 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           sA[e] = p.queries[static_cast<int64_t>(e / blk) * p.ld_q + off + e % blk];
         named_bar_sync(1, 128);
       }
-      bool aborted = false;
       for (int g = ic.t_begin; g < ic.t_end; g += NT) {
         const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
         if (vm == 0) continue;
-        if (et == 0) {
-          if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
-            raise_device_error(p.status, s_abort, kStatusTimeout);
-          *s_epi_stop = *s_abort;
-        }
-        named_bar_sync(1, 128);
-        if (*s_epi_stop) { aborted = true; break; }
-        tc_fence_after();
         float va[NT][KI];
         float vg[NT][KO];
+        if (finisher) {
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          if (!(vm >> nt & 1)) continue;
-          const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
-                                 ab * C::kTmemPerBuf + nt * (KI + KO);
+          for (int nt = 0; nt < NT; ++nt) {
+            if (!(vm >> nt & 1)) continue;
+            const int64_t tok = static_cast<int64_t>(g - ic.t_begin + nt) * kTileTokens + row;
+            sum_token_rows<KI>(p.piece_buf + ic.base + tok * KI, stride_a, ic.n_a, va[nt]);
+            sum_token_rows<KO>(p.piece_buf + ic.base + ic.n_a * stride_a + tok * KO, stride_g,
+                               ic.n_g, vg[nt]);
+          }
+        } else {
+          if (et == 0) {
+            if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
+              raise_device_error(p.status, s_abort, kStatusTimeout);
+            *s_epi_stop = *s_abort;
+          }
+          named_bar_sync(1, 128);
+          if (*s_epi_stop) { aborted = true; break; }
+          tc_fence_after();
 #pragma unroll
-          for (int c = 0; c < KI / 16; ++c) tmem_ld16(taddr + c * 16, &va[nt][c * 16]);
+          for (int nt = 0; nt < NT; ++nt) {
+            if (!(vm >> nt & 1)) continue;
+            const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
+                                   ab * C::kTmemPerBuf + nt * (KI + KO);
 #pragma unroll
-          for (int c = 0; c < KO / 16; ++c) tmem_ld16(taddr + KI + c * 16, &vg[nt][c * 16]);
+            for (int c = 0; c < KI / 16; ++c) tmem_ld16(taddr + c * 16, &va[nt][c * 16]);
+#pragma unroll
+            for (int c = 0; c < KO / 16; ++c) tmem_ld16(taddr + KI + c * 16, &vg[nt][c * 16]);
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+          if (++ab == 2) { ab = 0; aph ^= 1; }
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
-        if (++ab == 2) { ab = 0; aph ^= 1; }
         if constexpr (TOKEN) {
           // s[q] = g~^T Q~_q a~ for this thread's token: its share of the
           // query's score (masked tokens score 0).
@@ -435,12 +554,12 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       }
       if (aborted) break;
       if constexpr (TOKEN) continue;
-      float* dst = p.partials + static_cast<int64_t>(item) * (KO * KI) + et * OPT;
+      float* dst = p.partials + static_cast<int64_t>(ic.slot) * (KO * KI) + et * OPT;
 #pragma unroll
       for (int x = 0; x < OPT / 2; ++x)
         reinterpret_cast<float2*>(dst)[x] = make_float2(acc[2 * x], acc[2 * x + 1]);
       if (p.bias_partials != nullptr)
-        p.bias_partials[static_cast<int64_t>(item) * kTileTokens + et] = bias_acc;
+        p.bias_partials[static_cast<int64_t>(ic.slot) * kTileTokens + et] = bias_acc;
     }
   }
 

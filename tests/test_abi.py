@@ -7,6 +7,7 @@ import pytest
 
 import paper_2606_11660_gb300 as bg
 from oracle import bergson_oracle as orc
+from paper_2606_11660_gb300 import workloads as wl
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -231,3 +232,45 @@ def test_store_io_validation(tmp_path):
     assert L.bergson_store_save(FAKE, 10, 64, 32, b"/tmp/x", 0, None) == bg.BERGSON_EINVAL
     assert L.bergson_store_save(FAKE, 10, 64, 64, b"", 0, None) == bg.BERGSON_EINVAL
     assert L.bergson_store_load(str(tmp_path / "missing").encode(), 0, 1, 64, FAKE, 64, None) == bg.BERGSON_EINVAL
+
+
+def _plan(layers, B, T):
+    return bg.bergson_debug_project_plan(layers, B, T)
+
+
+def _block_layers(specs, k):
+    out, off = [], 0
+    for s in specs:
+        out.append(_layer(d_in=s.d_in, d_out=s.d_out, k_in=k, k_out=k, out_col_offset=off))
+        off += k * k
+    return out
+
+
+def test_planner_keeps_fine_launches_fused():
+    """48 modules x 32 examples x 4 slots: enough work items, no pieces."""
+    cfg = wl.PYTHIA160M
+    slots, items, pieces = _plan(_block_layers(cfg.modules, 16), cfg.B, cfg.T)
+    assert (slots, items, pieces) == (48 * 32 * 4, 48 * 32 * 4, 0)
+    cfg = wl.PYTHIA1B4                  # one block per call: 512 slots, still balanced enough
+    slots, items, pieces = _plan(_block_layers(cfg.block_modules(0), 32), cfg.B, cfg.T)
+    assert (slots, items, pieces) == (4 * 16 * 8, 4 * 16 * 8, 0)
+
+
+@pytest.mark.parametrize("name,B,T,k", [("llama8b", 8, 4096, 16), ("tiny", 8, 32, 16),
+                                        ("llama8b", 1, 160, 16), ("pythia1b4", 2, 256, 32)])
+def test_planner_cuts_coarse_launches_into_pieces(name, B, T, k):
+    cfg = wl.COLLECT_WORKLOADS[name]
+    specs = cfg.block_modules(0)
+    slots, items, pieces = _plan(_block_layers(specs, k), B, T)
+    fused = items - pieces
+    split = slots - fused
+    assert pieces > 0 and split > 0
+    assert pieces >= 2 * split          # every cut slot has pieces on both sides
+    st, n = _ws(_block_layers(specs, k), B, T)
+    assert st == bg.BERGSON_OK and n % 256 == 0
+
+
+def test_planner_validates_like_the_workspace_query():
+    with pytest.raises(bg.BergsonError) as e:
+        _plan([_layer(k_in=24)], 2, 32)
+    assert e.value.status == bg.BERGSON_EUNSUPPORTED

@@ -116,9 +116,57 @@ def test_empty_token_axis_writes_zero_blocks():
 def test_deterministic_bitwise():
     specs = [wl.ModuleSpec("a", 256, 768), wl.ModuleSpec("b", 768, 256)]
     gl, _, ld = make_layers(specs, 6, 1024, [(16, 16), (16, 16)], input_scale=True)
+    assert bg.bergson_debug_project_plan(gl, 6, 1024)[2] > 0     # pieces: last finisher varies
     a = run_project(gl, 6, 1024, None, ld)
     b = run_project(gl, 6, 1024, None, ld)
     assert torch.equal(a, b)
+
+
+def test_piece_path_wide_modules_mask_bias_moments():
+    """Few examples, wide modules: slots are cut into per-side pieces whose
+    token projections the last piece sums; ragged tail, masked tiles, bias."""
+    specs = [wl.ModuleSpec("up", 1024, 4096), wl.ModuleSpec("down", 3072, 1024),
+             wl.ModuleSpec("small", 256, 264)]
+    B, T = 3, 700                       # 6 tiles, the last one ragged
+    gl, ol, ld = make_layers(specs, B, T, [(16, 16)] * 3, base_seed=21, data_seed=8, rc=True,
+                             input_scale=True)
+    gl[1].bias_col_offset = ol[1].bias_col_offset = ld
+    ld_b = ld + 16
+    slots, items, pieces = bg.bergson_debug_project_plan(gl, B, T)
+    assert pieces > 0 and items > slots
+    g = wl.generator(12, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.25).to(torch.uint8)
+    mask[1, 128:384] = 0                # two fully masked tiles
+    mask[2, 650:] = 0
+    out = run_project(gl, B, T, mask.to(DEV), ld_b)
+    want = orc.project_grads(ol, mask.numpy(), ld_b)
+    got = np32(out).astype(np.float64)
+    assert rel_frobenius(got, want).max() <= TIGHT
+    assert rel_frobenius(got[:, ld:ld_b], want[:, ld:ld_b]).max() <= TIGHT
+
+
+@pytest.mark.parametrize("kp", [[(16, 32), (32, 16)], [(32, 32), (64, 64)]])
+def test_piece_path_mixed_k_groups(kp):
+    specs = [wl.ModuleSpec("a", 2048, 512), wl.ModuleSpec("b", 512, 1536)]
+    B, T = 2, 520
+    gl, ol, ld = make_layers(specs, B, T, kp, base_seed=5, data_seed=9, rc=True, input_scale=True)
+    assert bg.bergson_debug_project_plan(gl, B, T)[2] > 0
+    out = run_project(gl, B, T, None, ld)
+    want = orc.project_grads(ol, None, ld)
+    assert rel_frobenius(np32(out).astype(np.float64), want).max() <= TIGHT
+
+
+def test_fused_path_many_slots():
+    """Enough (module, example) slots that the planner keeps every item fused."""
+    specs = [wl.ModuleSpec("a", 64, 128), wl.ModuleSpec("b", 128, 64)]
+    B, T = 200, 500
+    gl, ol, ld = make_layers(specs, B, T, [(16, 16), (16, 16)], base_seed=3, data_seed=6, rc=True)
+    assert bg.bergson_debug_project_plan(gl, B, T)[2] == 0
+    g = wl.generator(14, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.1).to(torch.uint8)
+    out = run_project(gl, B, T, mask.to(DEV), ld)
+    want = orc.project_grads(ol, mask.numpy(), ld)
+    assert rel_frobenius(np32(out).astype(np.float64), want).max() <= TIGHT
 
 
 @pytest.mark.parametrize("blk", [0, 11])
