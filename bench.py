@@ -345,7 +345,7 @@ def bench_onthefly(args, world, dev, state):
             "ms_per_step": round(ms / args.steps, 4), "queries": Q,
             "score_call_ms": round(score_ms, 4),
             "score_gflops": round(flops / (score_ms * 1e-3) / 1e9, 1),
-            "gpu_launches": (5 + 4) * args.steps,
+            "gpu_launches": (5 + 3) * args.steps,
             "what": "bergson_project_grads + bergson_score_grads (cosine vs 1024 fp32 queries, "
                     "no store) per batch"}
 

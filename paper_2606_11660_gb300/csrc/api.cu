@@ -22,13 +22,12 @@ namespace {
 constexpr int kVersion = 100;                        // 0.1.0
 constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 s
 constexpr int kSchedTargetItems = 8192;              // work items per projection launch (target)
-// Piece splitting of projection slots.  The planner assumes kBalanceCTAs
+// Piece splitting of projection slots.  The planner assumes kPlanCTAs
 // persistent CTAs (one per SM of this part; the launch uses the real count).
 // A launch is split when its largest slot exceeds kSplitShare of one CTA's
 // share of the work, into pieces of about 1/kPiecesPerShare of a share.
-constexpr int kBalanceCTAs = 152;
 constexpr double kSplitShare = 0.4;
-constexpr int kPiecesPerShare = 4;
+constexpr int kPiecesPerShare = 2;
 constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
 constexpr int kMaxDevices = 64;
 constexpr int64_t kPrefixRowsPerTopk = 512;          // prefix pass: 512 * topk store rows
@@ -230,7 +229,7 @@ void plan_pieces(const bergson_layer* layers, int64_t B, int n_tiles, Group& g) 
     total += c * n_tiles * B;
     max_slot = std::max<int64_t>(max_slot, c * std::min(g.tpc, n_tiles));
   }
-  const double share = static_cast<double>(total) / kBalanceCTAs;
+  const double share = static_cast<double>(total) / kPlanCTAs;
   if (g.n_slots == 0 || static_cast<double>(max_slot) <= kSplitShare * share) return;
   const double target = share / kPiecesPerShare;
   struct Entry {
@@ -245,11 +244,13 @@ void plan_pieces(const bergson_layer* layers, int64_t B, int n_tiles, Group& g) 
     const int ca = chunks_of(ly.d_in), cg = chunks_of(ly.d_out);
     const bool cut = static_cast<double>(ca + cg) * g.tpc > target;
     // A piece stores and its slot's finisher reloads 4k fp32 bytes per token,
-    // against 128 bytes per token and chunk streamed: pieces of at least k
-    // chunks keep that under 1/16 of the piece's traffic.
+    // against 128 bytes per token and chunk streamed: pieces of at least 2k
+    // chunks keep that under 1/32 of the piece's traffic.  (Fewer, larger
+    // pieces measured faster: Llama-8B-shaped block 0.790 ms at a quarter of a
+    // share per piece, 0.770 ms at half.)
     auto pieces = [&](int ch, int k) {
       const int n = static_cast<int>(std::ceil(static_cast<double>(ch) * g.tpc / target));
-      return std::max(1, std::min(n, ch / k));
+      return std::max(1, std::min(n, ch / (2 * k)));
     };
     const int n_a = cut ? pieces(ca, g.k_in) : 0, n_g = cut ? pieces(cg, g.k_out) : 0;
     for (int64_t b = 0; b < B; ++b) {
@@ -812,9 +813,47 @@ int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store
 }
 
 static size_t onthefly_workspace(int64_t B, int64_t K, int64_t Q) {
-  const size_t S = static_cast<size_t>(onthefly_splits(B, Q, K));
-  return round_up(sizeof(float) * B, 256) + round_up(sizeof(float) * Q, 256) +
-         round_up(sizeof(float) * S * B * Q, 256);
+  return xgemm_plan(B, Q, K).total;
+}
+
+// C[b, q] = <x_b, y_q> (scaled to cosines when unit) into out; x [B, ldx] and
+// y [Q, ldy] validated by validate_onthefly.
+static int run_xgemm(const float* x, int64_t B, int64_t ldx, const float* y, int64_t Q,
+                     int64_t ldy, int64_t K, int unit, float* out, int64_t ld_out,
+                     void* workspace, void* stream, const char* what) {
+  DeviceGuard dg(workspace);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
+  if (encode_fn() == nullptr)
+    return fail(BERGSON_ECUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
+  int* status = status_word(dg.dev);
+  if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
+  const XGemmPlan pl = xgemm_plan(B, Q, K);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  CUtensorMap tm_y, tm_xh, tm_xl;
+  CUresult r1 = encode_2d(&tm_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, y, K, Q, ldy * 4, 32, 128);
+  CUresult r2 = encode_2d(&tm_xh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, ws + pl.xh_off, K, B, K * 4, 32,
+                          pl.n_pad);
+  CUresult r3 = encode_2d(&tm_xl, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, ws + pl.xl_off, K, B, K * 4, 32,
+                          pl.n_pad);
+  if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS || r3 != CUDA_SUCCESS)
+    return fail(BERGSON_ECUDA, "%s: tensor map encoding failed (%d %d %d)", what, (int)r1,
+                (int)r2, (int)r3);
+  XGemmArgs a;
+  a.x = x;
+  a.ldx = ldx;
+  a.B = static_cast<int>(B);
+  a.Q = static_cast<int>(Q);
+  a.K = static_cast<int>(K);
+  a.unit = unit;
+  a.scores = out;
+  a.ld_scores = ld_out;
+  a.ws = ws;
+  a.status = status;
+  a.timeout_ns = kWaitTimeoutNs;
+  cudaError_t e = launch_xgemm(tm_y, tm_xh, tm_xl, pl, a, sm_count(dg.dev),
+                               static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, what);
+  return BERGSON_OK;
 }
 
 static int validate_onthefly(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
@@ -858,18 +897,8 @@ int bergson_score_grads(const float* proj, int64_t B, int64_t K, int64_t ld_proj
     return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
   if ((st = injected()) != BERGSON_OK) return st;
   if (B == 0 || Q == 0) return BERGSON_OK;
-  DeviceGuard dg(workspace);
-  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  float* sx = reinterpret_cast<float*>(ws);
-  float* sy = reinterpret_cast<float*>(ws + round_up(sizeof(float) * B, 256));
-  float* partial = reinterpret_cast<float*>(ws + round_up(sizeof(float) * B, 256) +
-                                            round_up(sizeof(float) * Q, 256));
-  cudaError_t e = launch_onthefly(proj, static_cast<int>(B), ld_proj, queries, static_cast<int>(Q),
-                                  ld_q, static_cast<int>(K), unit_normalize ? 1 : 0, sx, sy,
-                                  partial, scores, ld_scores, static_cast<cudaStream_t>(stream));
-  if (e != cudaSuccess) return fail_cuda(e, "on-the-fly score launch");
-  return BERGSON_OK;
+  return run_xgemm(proj, B, ld_proj, queries, Q, ld_q, K, unit_normalize ? 1 : 0, scores,
+                   ld_scores, workspace, stream, "on-the-fly score launch");
 }
 
 int bergson_aggregate_rows_workspace(int64_t n, size_t* ws_bytes) {
@@ -1014,16 +1043,8 @@ int bergson_precondition_rows(const float* rows, int64_t B, int64_t K, int64_t l
     return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
   if ((st = injected()) != BERGSON_OK) return st;
   if (B == 0) return BERGSON_OK;
-  DeviceGuard dg(workspace);
-  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  float* partial = reinterpret_cast<float*>(ws + round_up(sizeof(float) * B, 256) +
-                                            round_up(sizeof(float) * K, 256));
-  cudaError_t e = launch_onthefly(rows, static_cast<int>(B), ld, M, static_cast<int>(K), ldm,
-                                  static_cast<int>(K), 0, nullptr, nullptr, partial, out, ld_out,
-                                  static_cast<cudaStream_t>(stream));
-  if (e != cudaSuccess) return fail_cuda(e, "preconditioning launch");
-  return BERGSON_OK;
+  return run_xgemm(rows, B, ld, M, K, ldm, K, 0, out, ld_out, workspace, stream,
+                   "preconditioning launch");
 }
 
 int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind,

@@ -15,7 +15,7 @@ constexpr int kChunk = 64;           // bf16 elements per 128-byte swizzled row
 constexpr int kScoreBN = 256;        // store rows per score tile (tcgen05 N)
 constexpr int kScoreQT = 128;        // queries per query tile (tcgen05 M)
 constexpr int kMaxTopk = 1024;
-constexpr int kOnTheFlyTargetCTAs = 1216;  // split-K target for on-the-fly scores
+constexpr int kPlanCTAs = 152;   // persistent CTAs work planners assume (one per SM of this part)
 
 // Per-module launch record kept in workspace (global memory).  The tensor maps
 // are read by TMA straight from there, so the record is 64-byte aligned.
@@ -139,7 +139,6 @@ cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit
 cudaError_t launch_aggregate(const float* rows, int64_t n, int K, int64_t ld,
                              const int64_t* offsets, int G, int mode, const float* scale,
                              float* out, int64_t ld_out, cudaStream_t s);
-int onthefly_splits(int64_t B, int64_t Q, int64_t K);
 size_t fisher_fit_workspace(int64_t n, int64_t K);
 cudaError_t launch_fisher_fit(const float* x, int n, int K, int64_t ldx, float* r, int64_t ldr,
                               float* ws, cudaStream_t s);
@@ -147,8 +146,35 @@ size_t fisher_power_workspace(int64_t K);
 cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
                                 float damping, int inverse, int iterations, float* m, int64_t ldm,
                                 float* ws, cudaStream_t s);
-cudaError_t launch_onthefly(const float* x, int B, int64_t ldx, const float* y, int Q,
-                            int64_t ldy, int K, int unit, float* sx, float* sy, float* partial,
-                            float* scores, int64_t ld_scores, cudaStream_t s);
+
+// Skinny fp32 product C[b, q] = <x_b, y_q> on the tensor cores (on-the-fly
+// scores, preconditioner application): plan and workspace layout.
+struct XGemmPlan {
+  int n_pad = 16;          // batch rows per tile (multiple of 16, <= 128)
+  int n_ntiles = 1;        // ceil(B / n_pad)
+  int n_mtiles = 1;        // ceil(Q / 128)
+  int steps = 1;           // ceil(K / 32)
+  int S = 1;               // K slices
+  int stages = 2;          // shared-memory pipeline depth
+  size_t sx_off = 0, ynorm_off = 0, partial_off = 0, xh_off = 0, xl_off = 0, total = 0;
+};
+XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K);
+
+struct XGemmArgs {
+  const float* x;          // [B, ldx] fp32, 16-byte aligned rows
+  int64_t ldx;
+  int B, Q, K;
+  int unit;                // 1: cosine (scale by both norms), 0: plain products
+  float* scores;           // [B, ld_scores]
+  int64_t ld_scores;
+  uint8_t* ws;             // workspace laid out by the plan
+  int* status;
+  uint64_t timeout_ns;
+};
+// tm_y: y [Q, K] fp32, box 32 x 128; tm_xh / tm_xl: the plan's x_hi / x_lo
+// regions [B, K], box 32 x n_pad; all with the 128-byte swizzle.
+cudaError_t launch_xgemm(const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
+                         const CUtensorMap& tm_xl, const XGemmPlan& plan, const XGemmArgs& a,
+                         int sms, cudaStream_t s);
 
 }  // namespace bergson

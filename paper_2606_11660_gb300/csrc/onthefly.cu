@@ -3,24 +3,90 @@
 // store in between.  Table 3's grad-cosine (unit-normalised rows and queries)
 // and grad-dot (raw inner products) are both served:
 //   scores[b, q] = <x_b, y_q> * s_b * t_q,  s = 1/||x||, t = 1/||y|| (cosine) or 1.
+// The same skinny product applies the preconditioner (Sec. 3.2): there y is
+// the K x K matrix M and the outputs are the preconditioned rows M x_b.
 //
-// The inner products are a small fp32 GEMM [B x K] x [K x Q] (for a batch of
-// 32 examples and 1024 queries at K = 12288, 0.8 GFLOP: ~0.5% of the batch's
-// projection time), computed with CUDA-core FFMA in fp32 for full accuracy.
-// Split-K gives enough CTAs for a 32-row batch; the partial sums are added in
-// a fixed order, so the result is deterministic.
+// The product C[b, q] = <x_b, y_q> runs on the tensor cores (tcgen05,
+// kind::tf32) at fp32 accuracy.  tf32 keeps 10 of fp32's 23 mantissa bits, so
+// every operand is split into two tf32 values, each rounded to nearest:
+//   y ~= y_hi + y_lo,  y_lo = tf32(y - y_hi)   (error <= 2^-22 |y|),
+//   <x, y> ~= <x_hi, y_hi> + <x_lo, y_hi> + <x_hi, y_lo> (+ <x_lo, y_lo>, which
+// comes free here): the 3xTF32 scheme of Ootomo and Yokota (2022).
+// Round-to-nearest splitting keeps the per-product errors unbiased, so they
+// grow like sqrt(K) rather than K.
+//
+// y (queries, or M) is the large operand and is streamed from HBM once: TMA
+// loads 128-row x 32-column fp32 tiles (128-byte swizzle) into a shared-memory
+// ring; the tile itself is y_hi (the tensor cores truncate it), and four
+// converter warps write its y_lo (the swizzle permutes 16-byte chunks, so an
+// elementwise map keeps the layout) and, for cosine scores, accumulate the
+// rows' squared norms from the same tile; one thread issues two MMAs per 8 columns into TMEM (M = 128 rows
+// of y; N = x_hi and x_lo stacked, twice the batch padded to 16), which reads
+// each y part from shared memory once (shared-memory bandwidth, not the
+// tensor pipe, bounds this kernel); four epilogue warps add the four partial
+// products up.  x is small: a pre-pass splits it into x_hi and x_lo
+// (and its norms) in workspace, and its tiles come from L2.
+//
+// Work items are (128-row tile of y, batch tile, K slice), handed out
+// round-robin to persistent CTAs (all items have the same cost); every item
+// writes an fp32 partial that a finishing kernel sums over the K slices in
+// order and scales (deterministic result).  Every wait is bounded.
+
+#include <algorithm>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace bergson {
 
 namespace {
 
-constexpr int kBM = 32;        // rows (examples) per CTA tile
-constexpr int kBN = 128;       // queries per CTA tile
-constexpr int kBK = 32;        // K per shared-memory step
-constexpr int kThreads = 128;  // thread tile: 4 rows x 8 queries
 constexpr int kRowThreads = 256;
+constexpr int kXM = 128;                   // rows of y per tile (MMA M)
+constexpr int kXK = 32;                    // fp32 columns per stage: one 128-byte row
+constexpr int kYBytes = kXM * 128;         // one y tile
+constexpr int kXThreads = 320;             // producer, MMA, 4 converter, 4 epilogue warps
+constexpr int kXSmemBudget = 232448;       // 227 KB opt-in per CTA
+constexpr int kXBarBytes = 512;
+constexpr int kMaxSlices = 64;
+constexpr uint64_t kXDrainTimeoutNs = 2000000000ull;
+
+struct KahanSum {
+  float s = 0.0f, c = 0.0f;
+  __device__ __forceinline__ void add(float x) {
+    const float y = x - c;
+    const float t = s + y;
+    c = (t - s) - y;
+    s = t;
+  }
+};
+
+// v rounded to the nearest tf32 value (10 explicit mantissa bits; ties away
+// from zero), as an fp32 bit pattern whose low 13 bits are zero.
+__device__ __forceinline__ float tf32_round(float v) {
+  return __uint_as_float((__float_as_uint(v) + 0x1000u) & 0xFFFFE000u);
+}
+
+// v = hi + lo + e with hi, lo exact tf32 values and |e| <= 2^-22 |v|: the
+// tensor cores read both parts exactly.
+__device__ __forceinline__ void tf32_split(float4 v, float4& hi, float4& lo) {
+  hi = make_float4(tf32_round(v.x), tf32_round(v.y), tf32_round(v.z), tf32_round(v.w));
+  lo = make_float4(tf32_round(v.x - hi.x), tf32_round(v.y - hi.y), tf32_round(v.z - hi.z),
+                   tf32_round(v.w - hi.w));
+}
+
+__device__ __forceinline__ float tf32_trunc(float v) {
+  return __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
+}
+
+// The tensor cores read an fp32 operand of kind::tf32 as tf32 by dropping its
+// low 13 mantissa bits (truncation; the fp64 checks of the tests would show
+// errors near 2^-12 otherwise).  So y itself serves as y_hi = trunc(y), and
+// y_lo = tf32(y - trunc(y)) is what truncation leaves out, rounded to nearest.
+__device__ __forceinline__ float4 tf32_remainder(float4 v) {
+  return make_float4(tf32_round(v.x - tf32_trunc(v.x)), tf32_round(v.y - tf32_trunc(v.y)),
+                     tf32_round(v.z - tf32_trunc(v.z)), tf32_round(v.w - tf32_trunc(v.w)));
+}
 
 // scale[i] = 1/||row_i|| (unit, 0 for a zero row) or 1.  One CTA per row,
 // 16-byte loads, compensated fp32 sums per thread (fp64 is slow on this part).
@@ -28,14 +94,12 @@ __global__ void __launch_bounds__(kRowThreads) row_scales_kernel(
     const float* __restrict__ x, int K, int64_t ld, int unit, float* __restrict__ scale) {
   __shared__ float red[kRowThreads / 32];
   const float4* xr = reinterpret_cast<const float4*>(x + blockIdx.x * ld);
-  float s = 0.0f, comp = 0.0f;
+  KahanSum ks;
   for (int i = threadIdx.x; i < K / 4; i += kRowThreads) {
     const float4 v = xr[i];
-    const float y = (v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w) - comp;
-    const float t = s + y;
-    comp = (t - s) - y;
-    s = t;
+    ks.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
   }
+  float s = ks.s;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
@@ -47,95 +111,302 @@ __global__ void __launch_bounds__(kRowThreads) row_scales_kernel(
   }
 }
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool valid) {
-  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
-  const int n = valid ? 16 : 0;                      // 0 source bytes -> zero fill
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(gmem), "r"(n)
-               : "memory");
+// Row b of x -> rows of x_hi and x_lo ([B, K], contiguous) and scale[b] as above.
+__global__ void __launch_bounds__(kRowThreads) split_rows_kernel(
+    const float* __restrict__ x, int K, int64_t ld, int unit, float* __restrict__ xh,
+    float* __restrict__ xl, float* __restrict__ scale) {
+  __shared__ float red[kRowThreads / 32];
+  const int64_t b = blockIdx.x;
+  const float4* xr = reinterpret_cast<const float4*>(x + b * ld);
+  float4* hr = reinterpret_cast<float4*>(xh + b * K);
+  float4* lr = reinterpret_cast<float4*>(xl + b * K);
+  KahanSum ks;
+  for (int i = threadIdx.x; i < K / 4; i += kRowThreads) {
+    const float4 v = xr[i];
+    float4 h, l;
+    tf32_split(v, h, l);
+    hr[i] = h;
+    lr[i] = l;
+    ks.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
+  }
+  float s = ks.s;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float tot = 0.0f;
+    for (int w = 0; w < kRowThreads / 32; ++w) tot += red[w];
+    scale[b] = unit ? (tot > 0.0f ? 1.0f / sqrtf(tot) : 0.0f) : 1.0f;
+  }
 }
 
-// partial[z, b, q] = sum over k in slice z of x[b, k] * y[q, k].
-// Two shared-memory stages filled with cp.async; thread (tx, ty) owns rows
-// 4ty..4ty+3 and queries tx + 16j (j < 8), which keeps the 16-byte shared
-// loads of one warp on distinct banks.
-__global__ void __launch_bounds__(kThreads) dot_partials_kernel(
-    const float* __restrict__ x, int B, int64_t ldx, const float* __restrict__ y, int Q,
-    int64_t ldy, int K, int kslice, float* __restrict__ partial) {
-  __shared__ __align__(16) float xs[2][kBM][kBK + 4];
-  __shared__ __align__(16) float ys[2][kBN][kBK + 4];
-  const int tid = threadIdx.x;
-  const int tx = tid % 16;
-  const int ty = tid / 16;
-  const int q0 = blockIdx.x * kBN;
-  const int b0 = blockIdx.y * kBM;
-  const int k_begin = blockIdx.z * kslice;
-  const int k_end = min(K, k_begin + kslice);
-  const int nsteps = (k_end - k_begin + kBK - 1) / kBK;
+struct XGemmParams {
+  int B, Q;
+  int n_pad, n_mtiles, S, steps, stages;
+  int n_buf;          // TMEM accumulator sets (2: epilogue overlaps the next item)
+  int n_items;
+  int tmem_cols;
+  int unit;
+  float* partial;     // [S, B, Q]
+  float* ynorm;       // [S, Q] squared norms of y rows over each slice (unit only)
+  int* status;
+  uint64_t timeout_ns;
+};
 
-  auto load = [&](int st, int k0) {
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {   // x: 32 rows x 8 chunks of 16 B
-      const int idx = tid + h * kThreads;
-      const int r = idx / 8, c = (idx % 8) * 4;
-      const bool ok = b0 + r < B && k0 + c < k_end;
-      cp_async16(&xs[st][r][c], ok ? x + (b0 + r) * ldx + k0 + c : x, ok);
-    }
-#pragma unroll
-    for (int h = 0; h < 8; ++h) {   // y: 128 rows x 8 chunks of 16 B
-      const int idx = tid + h * kThreads;
-      const int r = idx / 8, c = (idx % 8) * 4;
-      const bool ok = q0 + r < Q && k0 + c < k_end;
-      cp_async16(&ys[st][r][c], ok ? y + (q0 + r) * ldy + k0 + c : y, ok);
-    }
-    asm volatile("cp.async.commit_group;" ::: "memory");
-  };
+struct XItem {
+  int mt, nt, z, s0, s1;
+};
 
-  float acc[4][8] = {};
-  if (nsteps > 0) load(0, k_begin);
-  for (int step = 0; step < nsteps; ++step) {
-    const int st = step & 1;
-    if (step + 1 < nsteps) {
-      load(st ^ 1, k_begin + (step + 1) * kBK);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
+__device__ __forceinline__ XItem decode_xitem(const XGemmParams& p, int item) {
+  XItem it;
+  it.z = item % p.S;
+  const int t = item / p.S;
+  it.mt = t % p.n_mtiles;
+  it.nt = t / p.n_mtiles;
+  it.s0 = static_cast<int>(static_cast<int64_t>(it.z) * p.steps / p.S);
+  it.s1 = static_cast<int>(static_cast<int64_t>(it.z + 1) * p.steps / p.S);
+  return it;
+}
+
+// Lane 0 waits, the warp takes its answer (keeps the warp's control flow uniform).
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint64_t tmo,
+                                          const volatile int* abort_flag) {
+  bool ok = true;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, tmo, abort_flag);
+  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
+
+__global__ void __launch_bounds__(kXThreads, 1)
+    xgemm_kernel(const __grid_constant__ CUtensorMap tm_y, const __grid_constant__ CUtensorMap tm_xh,
+                 const __grid_constant__ CUtensorMap tm_xl, const XGemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const int xbytes = p.n_pad * 128;
+  const int stage_bytes = 2 * kYBytes + 2 * xbytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
+  uint64_t* empty = full + p.stages;
+  uint64_t* conv = empty + p.stages;
+  uint64_t* tfull = conv + p.stages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+      mbar_init(smem_u32(&conv[s]), 128);
     }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < kBK; kk += 4) {
-      float4 a[4], c[8];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = *reinterpret_cast<const float4*>(&xs[st][4 * ty + i][kk]);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) c[j] = *reinterpret_cast<const float4*>(&ys[st][tx + 16 * j][kk]);
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          acc[i][j] = fmaf(a[i].x, c[j].x, acc[i][j]);
-          acc[i][j] = fmaf(a[i].y, c[j].y, acc[i][j]);
-          acc[i][j] = fmaf(a[i].z, c[j].z, acc[i][j]);
-          acc[i][j] = fmaf(a[i].w, c[j].w, acc[i][j]);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&tfull[i]), 1);
+      mbar_init(smem_u32(&tempty[i]), 4);
+    }
+    mbar_init(smem_u32(drain), 1);
+    *s_abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(s_tmem), p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *s_tmem;
+  const uint64_t tmo = p.timeout_ns;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      prefetch_tmap(&tm_y);
+      prefetch_tmap(&tm_xh);
+      prefetch_tmap(&tm_xl);
+      const uint64_t pol_y = policy_evict_first();    // streamed once
+      const uint64_t pol_x = policy_evict_last();     // re-read by every tile
+      int stage = 0;
+      uint32_t ph = 0;
+      uint32_t issued = 0, issued_par = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
+        const XItem it = decode_xitem(p, item);
+        for (int st = it.s0; st < it.s1; ++st) {
+          if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_arrive_expect_tx(fb, kYBytes + 2 * xbytes);
+          const uint32_t dst = sbase + stage * stage_bytes;
+          tma_load_2d_hint(dst, &tm_y, fb, st * kXK, it.mt * kXM, pol_y);
+          tma_load_2d_hint(dst + 2 * kYBytes, &tm_xh, fb, st * kXK, it.nt * p.n_pad, pol_x);
+          tma_load_2d_hint(dst + 2 * kYBytes + xbytes, &tm_xl, fb, st * kXK, it.nt * p.n_pad,
+                           pol_x);
+          issued |= 1u << stage;
+          issued_par = (issued_par & ~(1u << stage)) | (ph << stage);
+          if (++stage == p.stages) { stage = 0; ph ^= 1; }
         }
+      }
+      if (!ok) {
+        raise_device_error(p.status, s_abort, kStatusTimeout);
+        for (int s = 0; s < p.stages; ++s)
+          if (issued >> s & 1)
+            mbar_wait(smem_u32(&full[s]), (issued_par >> s) & 1, kXDrainTimeoutNs, nullptr);
+      }
     }
-    __syncthreads();
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = make_idesc_tf32(kXM, 2 * p.n_pad);
+      int stage = 0;
+      uint32_t ph = 0;
+      int ab = 0;
+      uint32_t aph = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
+        const XItem it = decode_xitem(p, item);
+        if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+        tc_fence_after();
+        // Set ab: D_hi = y_hi [x_hi; x_lo]^T in columns [0, 2 n_pad), D_lo =
+        // y_lo [x_hi; x_lo]^T in [2 n_pad, 4 n_pad).  x_hi and x_lo land next to
+        // each other, so one B operand of 2 n_pad rows serves both, and y_hi and
+        // y_lo are each read once per K step.
+        const uint32_t d_hi = tmem + ab * 4 * p.n_pad;
+        const uint32_t d_lo = d_hi + 2 * p.n_pad;
+        for (int st = it.s0; st < it.s1; ++st) {
+          if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
+              !mbar_wait(smem_u32(&conv[stage]), ph, tmo, s_abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t yh = sbase + stage * stage_bytes;
+          const uint64_t dyh = sw128_desc(yh);
+          const uint64_t dyl = sw128_desc(yh + kYBytes);
+          const uint64_t dx = sw128_desc(yh + 2 * kYBytes);
+#pragma unroll
+          for (int kk = 0; kk < kXK / 8; ++kk) {       // 8 tf32 = 32 bytes: +2 in the address field
+            const uint64_t o = 2 * kk;
+            const uint32_t acc = st != it.s0 || kk != 0;
+            umma_tf32(d_hi, dyh + o, dx + o, idesc, acc);
+            umma_tf32(d_lo, dyl + o, dx + o, idesc, acc);
+          }
+          umma_commit(smem_u32(&empty[stage]));
+          if (++stage == p.stages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit(smem_u32(&tfull[ab]));
+        if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
+      }
+      if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
+      umma_commit(smem_u32(drain));
+      mbar_wait(smem_u32(drain), 0, kXDrainTimeoutNs, nullptr);
+    }
+    __syncwarp();
+  } else if (warp < 6) {
+    // ------------------------------------------------------------ converter
+    // Thread ct owns 16-byte chunks ct + 128 i (i < 8) of each tile: rows
+    // ct / 8 + 16 i, whatever the swizzle did to their columns.
+    const int ct = threadIdx.x - 64;
+    int stage = 0;
+    uint32_t ph = 0;
+    for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
+      const XItem it = decode_xitem(p, item);
+      KahanSum nrm[8];
+      bool aborted = false;
+      for (int st = it.s0; st < it.s1; ++st) {
+        if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) {
+          raise_device_error(p.status, s_abort, kStatusTimeout);
+          aborted = true;
+          break;
+        }
+        float4* yb = reinterpret_cast<float4*>(smem + stage * stage_bytes);
+        float4* lb = yb + kYBytes / 16;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int idx = ct + 128 * i;
+          const float4 v = yb[idx];
+          lb[idx] = tf32_remainder(v);
+          if (p.unit) nrm[i].add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(smem_u32(&conv[stage]));
+        if (++stage == p.stages) { stage = 0; ph ^= 1; }
+      }
+      if (aborted) break;
+      if (p.unit && it.nt == 0) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float s = nrm[i].s;                        // the 8 lanes of a row, in a fixed order
+          s += __shfl_xor_sync(0xffffffffu, s, 1);
+          s += __shfl_xor_sync(0xffffffffu, s, 2);
+          s += __shfl_xor_sync(0xffffffffu, s, 4);
+          const int q = it.mt * kXM + ct / 8 + 16 * i;
+          if ((ct & 7) == 0 && q < p.Q) p.ynorm[static_cast<int64_t>(it.z) * p.Q + q] = s;
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quarter = warp & 3;                    // TMEM lanes 32*quarter ..
+    const int row = 32 * quarter + lane;
+    int ab = 0;
+    uint32_t aph = 0;
+    for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
+      const XItem it = decode_xitem(p, item);
+      if (!warp_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort)) {
+        raise_device_error(p.status, s_abort, kStatusTimeout);
+        break;
+      }
+      tc_fence_after();
+      const int q = it.mt * kXM + row;
+      float* dst = p.partial + static_cast<int64_t>(it.z) * p.B * p.Q + q;
+      const uint32_t tbase =
+          tmem + (static_cast<uint32_t>(32 * quarter) << 16) + ab * 4 * p.n_pad;
+      for (int c = 0; c < p.n_pad; c += 16) {
+        // <x_b, y_q> ~= y_hi x_hi + y_hi x_lo + y_lo x_hi (+ y_lo x_lo), in this order
+        float v[16], w[16];
+        tmem_ld16(tbase + c, v);
+        tmem_ld16(tbase + p.n_pad + c, w);
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
+        tmem_ld16(tbase + 2 * p.n_pad + c, w);
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
+        tmem_ld16(tbase + 3 * p.n_pad + c, w);
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
+        if (q < p.Q) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int b = it.nt * p.n_pad + c + j;
+            if (b < p.B) dst[static_cast<int64_t>(b) * p.Q] = v[j];
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+      if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
+    }
   }
-  float* dst = partial + static_cast<int64_t>(blockIdx.z) * B * Q;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int b = b0 + 4 * ty + i;
-    if (b >= B) continue;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int q = q0 + tx + 16 * j;
-      if (q < Q) dst[static_cast<int64_t>(b) * Q + q] = acc[i][j];
-    }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, p.tmem_cols);
   }
 }
 
-// scores[b, q] = (sum over slices, in order) * sx[b] * sy[q]
+// scores[b, q] = (sum over slices z, in order, of partial[z, b, q]) * sx[b] * t_q
+// with t_q = 1/sqrt(sum over z of ynorm[z, q]) (0 for a zero row); unscaled
+// when sx is null.
 __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, int Q,
-                              const float* __restrict__ sx, const float* __restrict__ sy,
+                              const float* __restrict__ sx, const float* __restrict__ ynorm,
                               float* __restrict__ scores, int64_t ld) {
   const int64_t n = static_cast<int64_t>(B) * Q;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
@@ -143,9 +414,16 @@ __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, i
     float s = 0.0f;
     for (int z = 0; z < S; ++z) s += partial[z * n + i];
     const int b = static_cast<int>(i / Q), q = static_cast<int>(i % Q);
-    scores[b * ld + q] = sx != nullptr ? s * sx[b] * sy[q] : s;
+    if (sx != nullptr) {
+      float ny = 0.0f;
+      for (int z = 0; z < S; ++z) ny += ynorm[static_cast<int64_t>(z) * Q + q];
+      s *= sx[b] * (ny > 0.0f ? 1.0f / sqrtf(ny) : 0.0f);
+    }
+    scores[b * ld + q] = s;
   }
 }
+
+size_t round_up256(size_t x) { return (x + 255) / 256 * 256; }
 
 }  // namespace
 
@@ -156,35 +434,93 @@ cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit
   return cudaGetLastError();
 }
 
-int onthefly_splits(int64_t B, int64_t Q, int64_t K) {
-  const int64_t tiles = ((Q + kBN - 1) / kBN) * ((B + kBM - 1) / kBM);
-  if (tiles == 0) return 1;                       // empty problem: nothing to split
-  int64_t s = (kOnTheFlyTargetCTAs + tiles - 1) / tiles;
-  const int64_t max_s = (K + kBK - 1) / kBK;
-  if (s > max_s) s = max_s;
-  if (s < 1) s = 1;
-  const int64_t slice = ((K + s - 1) / s + kBK - 1) / kBK * kBK;
-  return static_cast<int>((K + slice - 1) / slice);
+XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
+  XGemmPlan pl;
+  const int64_t b1 = B > 0 ? B : 1;
+  pl.n_pad = static_cast<int>(std::min<int64_t>(128, (b1 + 15) / 16 * 16));
+  pl.n_ntiles = static_cast<int>((b1 + pl.n_pad - 1) / pl.n_pad);
+  pl.n_mtiles = static_cast<int>(std::max<int64_t>(1, (Q + kXM - 1) / kXM));
+  pl.steps = static_cast<int>(std::max<int64_t>(1, (K + kXK - 1) / kXK));
+  const int stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
+  pl.stages = std::min(8, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
+  // K slices: fewest waves of persistent CTAs for the y stream, plus the
+  // partials each slice adds (written and read back once).
+  const int64_t tiles = static_cast<int64_t>(pl.n_mtiles) * pl.n_ntiles;
+  double best = -1.0;
+  pl.S = 1;
+  for (int S = 1; S <= std::min(pl.steps, kMaxSlices); ++S) {
+    if (tiles * S > (1ll << 30)) break;
+    const int64_t waves = (tiles * S + kPlanCTAs - 1) / kPlanCTAs;
+    const int64_t per_item = (pl.steps + S - 1) / S;
+    const double cost = static_cast<double>(waves) * (per_item + 2) * stage_bytes +
+                        8.0 * S * static_cast<double>(b1) * static_cast<double>(Q) / kPlanCTAs;
+    if (best < 0.0 || cost < best) {
+      best = cost;
+      pl.S = S;
+    }
+  }
+  size_t off = 0;
+  pl.sx_off = off;
+  off += round_up256(sizeof(float) * static_cast<size_t>(b1));
+  pl.ynorm_off = off;
+  off += round_up256(sizeof(float) * static_cast<size_t>(pl.S) * std::max<int64_t>(Q, 1));
+  pl.partial_off = off;
+  off += round_up256(sizeof(float) * static_cast<size_t>(pl.S) * b1 * std::max<int64_t>(Q, 1));
+  pl.xh_off = off;
+  off += round_up256(sizeof(float) * static_cast<size_t>(b1) * K);
+  pl.xl_off = off;
+  off += round_up256(sizeof(float) * static_cast<size_t>(b1) * K);
+  pl.total = off;
+  return pl;
 }
 
-cudaError_t launch_onthefly(const float* x, int B, int64_t ldx, const float* y, int Q,
-                            int64_t ldy, int K, int unit, float* sx, float* sy, float* partial,
-                            float* scores, int64_t ld_scores, cudaStream_t s) {
-  if (B == 0 || Q == 0) return cudaSuccess;
-  const int S = onthefly_splits(B, Q, K);
-  const int slice = ((K + S - 1) / S + kBK - 1) / kBK * kBK;
-  if (unit) {                  // plain products need no norms
-    row_scales_kernel<<<B, kRowThreads, 0, s>>>(x, K, ldx, unit, sx);
-    row_scales_kernel<<<Q, kRowThreads, 0, s>>>(y, K, ldy, unit, sy);
-  } else {
-    sx = sy = nullptr;
+cudaError_t launch_xgemm(const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
+                         const CUtensorMap& tm_xl, const XGemmPlan& pl, const XGemmArgs& a,
+                         int sms, cudaStream_t s) {
+  if (a.B == 0 || a.Q == 0) return cudaSuccess;
+  float* sx = reinterpret_cast<float*>(a.ws + pl.sx_off);
+  float* xh = reinterpret_cast<float*>(a.ws + pl.xh_off);
+  float* xl = reinterpret_cast<float*>(a.ws + pl.xl_off);
+  split_rows_kernel<<<a.B, kRowThreads, 0, s>>>(a.x, a.K, a.ldx, a.unit, xh, xl, sx);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+
+  XGemmParams p;
+  p.B = a.B;
+  p.Q = a.Q;
+  p.n_pad = pl.n_pad;
+  p.n_mtiles = pl.n_mtiles;
+  p.S = pl.S;
+  p.steps = pl.steps;
+  p.stages = pl.stages;
+  p.n_items = pl.n_mtiles * pl.n_ntiles * pl.S;
+  p.n_buf = 8 * pl.n_pad <= 512 ? 2 : 1;
+  int cols = 32;
+  while (cols < p.n_buf * 4 * pl.n_pad) cols <<= 1;
+  p.tmem_cols = cols;
+  p.unit = a.unit;
+  p.partial = reinterpret_cast<float*>(a.ws + pl.partial_off);
+  p.ynorm = reinterpret_cast<float*>(a.ws + pl.ynorm_off);
+  p.status = a.status;
+  p.timeout_ns = a.timeout_ns;
+  static bool attr_set = false;   // per process; the attribute is per function and device
+  if (!attr_set) {
+    e = cudaFuncSetAttribute(xgemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kXSmemBudget);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
   }
-  dim3 grid((Q + kBN - 1) / kBN, (B + kBM - 1) / kBM, S);
-  dot_partials_kernel<<<grid, kThreads, 0, s>>>(x, B, ldx, y, Q, ldy, K, slice, partial);
-  const int64_t n = static_cast<int64_t>(B) * Q;
+  const size_t smem = 1024 + static_cast<size_t>(pl.stages) * (2 * kYBytes + 2 * pl.n_pad * 128) +
+                      kXBarBytes;
+  const int grid = std::max(1, std::min(sms > 0 ? sms : 1, p.n_items));
+  xgemm_kernel<<<grid, kXThreads, smem, s>>>(tm_y, tm_xh, tm_xl, p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+
+  const int64_t n = static_cast<int64_t>(a.B) * a.Q;
   const int64_t blocks = (n + 255) / 256;
   finish_kernel<<<static_cast<unsigned>(blocks < 4096 ? blocks : 4096), 256, 0, s>>>(
-      partial, S, B, Q, sx, sy, scores, ld_scores);
+      p.partial, pl.S, a.B, a.Q, a.unit ? sx : nullptr, p.ynorm, a.scores, a.ld_scores);
   return cudaGetLastError();
 }
 

@@ -22,7 +22,8 @@ def _scores(x, y, unit, ld_pad=0):
     return np32(out)
 
 
-@pytest.mark.parametrize("B,K,Q", [(37, 12288, 130), (1, 36, 1), (64, 520, 1000), (3, 4096, 7)])
+@pytest.mark.parametrize("B,K,Q", [(37, 12288, 130), (1, 36, 1), (64, 520, 1000), (3, 4096, 7),
+                                   (300, 1000, 200), (16, 4, 129)])
 @pytest.mark.parametrize("unit", [True, False])
 def test_random_rows(B, K, Q, unit):
     g = wl.generator(B * 31 + K + Q, "cpu")
@@ -69,3 +70,18 @@ def test_deterministic():
     a = _scores(x, y, True)
     b = _scores(x, y, True)
     assert np.array_equal(a, b)
+
+
+@pytest.mark.parametrize("B,K", [(40, 1000), (1, 128), (257, 520)])
+def test_precondition_rows_random_matrix(B, K):
+    """M x_b for a dense random M, against fp64: the same skinny product with y = M."""
+    g = wl.generator(B + K, "cpu")
+    x = torch.randn((B, K), generator=g)
+    M = torch.randn((K, K), generator=g) / np.sqrt(K)
+    M = (M + M.T) / 2                       # the entry point's contract: M symmetric
+    ws = bg.workspace_tensor(bg.bergson_score_grads_workspace(B, K, K), DEV)
+    out = torch.full((B, K), float("nan"), dtype=torch.float32, device=DEV)
+    bg.bergson_precondition_rows(x.to(DEV), B, K, M.to(DEV), out, ws)
+    assert bg.bergson_sync_status() == bg.BERGSON_OK, bg.bergson_last_error()
+    want = x.numpy().astype(np.float64) @ M.numpy().astype(np.float64).T
+    np.testing.assert_allclose(np32(out), want, atol=2e-6 * np.abs(want).max(), rtol=0)
