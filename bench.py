@@ -688,9 +688,10 @@ def profile_case(args):
             bg.bergson_project_grads(layers, cfg.B, cfg.T, None, out, ws)
         st = bg.bergson_sync_status()
     elif args.profile_case == "collect":
-        # one block (4 modules) of the Pythia-160M-shaped workload, B=8, T=2048: 403 MB
+        # one block (4 modules) of the Pythia-160M-shaped workload at the bench's
+        # B=32, T=2048 and padding mask: 1.6 GB of A/G, the fused launch path
         cfg = wl.PYTHIA160M
-        B = 8
+        B = cfg.B
         mask = wl.right_padding_mask(B, cfg.T, cfg.max_pad, seed=1, device=dev)
         layers = []
         for m, spec in enumerate(cfg.block_modules(0)):
