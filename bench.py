@@ -725,24 +725,6 @@ def profile_case(args):
     print("profile case done:", args.profile_case)
 
 
-def read_ceiling(dev):
-    """Read-only streaming bandwidth (GB/s) of a 16 GiB bf16 sum (torch reduction kernel)."""
-    import torch
-    x = torch.ones((8 << 30,), dtype=torch.bfloat16, device=dev)
-    torch.sum(x, dtype=torch.float32)
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(5):
-        torch.sum(x, dtype=torch.float32)
-    e1.record()
-    torch.cuda.synchronize()
-    gbs = 5 * x.numel() * 2 / (e0.elapsed_time(e1) * 1e6)
-    del x
-    torch.cuda.empty_cache()
-    return round(gbs, 1)
-
-
 def main_ours(args):
     import torch
 
@@ -763,7 +745,6 @@ def main_ours(args):
     streamed = None
     if not args.no_streamed:
         streamed = {n: bench_streamed(args, world, dev, n, peaks) for n in ("pythia1b4", "llama8b")}
-    coll["roofline"]["read_ceiling_gbs"] = read_ceiling(dev)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         times, cores = run_cpu_oracle(args.cpu_examples, 1)
