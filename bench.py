@@ -459,8 +459,9 @@ def bench_streamed(args, world, dev, name, peaks):
     nmod = cfg.modules_per_block
     specs = cfg.block_modules(0)
     tensors = []
-    for j, spec in enumerate(specs):
-        A, G = wl.layer_inputs(spec, cfg.B, cfg.T, seed=20_000 + j, device=dev, input_scale=True)
+    ins = wl.module_inputs(specs, cfg.B, cfg.T, [20_000 + j for j in range(len(specs))],
+                           device=dev, input_scale=True)
+    for j, (spec, (A, G)) in enumerate(zip(specs, ins)):
         r = c = None
         if cfg.second_moments:
             r, c = wl.second_moments(spec.d_out, spec.d_in, seed=30_000 + j, device=dev)
@@ -496,9 +497,9 @@ def bench_streamed(args, world, dev, name, peaks):
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1), world) / steps
-    alg = 2 * sum(sp.d_in + sp.d_out for sp in cfg.modules) * cfg.B * cfg.T
+    alg = wl.input_bytes(cfg.modules, cfg.B * cfg.T)      # a shared input counts once
     gbs = alg / (ms * 1e-3) / 1e9
-    del tensors, calls
+    del tensors, calls, ins
     torch.cuda.empty_cache()
     return {"value": round(cfg.B * world / (ms * 1e-3), 2), "unit": "examples/s",
             "ms_per_step": round(ms, 3), "calls_per_step": cfg.blocks,
@@ -674,9 +675,10 @@ def profile_case(args):
         # (Pythia-1.4B shape: 2.1 GB of A/G; Llama-8B shape: 4.8 GB)
         cfg = wl.COLLECT_WORKLOADS[args.profile_case.split("_", 1)[1]]
         layers = []
-        for m, spec in enumerate(cfg.block_modules(0)):
-            A, G = wl.layer_inputs(spec, cfg.B, cfg.T, seed=20_000 + m, device=dev,
-                                   input_scale=True)
+        specs = cfg.block_modules(0)
+        ins = wl.module_inputs(specs, cfg.B, cfg.T, [20_000 + m for m in range(len(specs))],
+                               device=dev, input_scale=True)
+        for m, (spec, (A, G)) in enumerate(zip(specs, ins)):
             r = c = None
             if cfg.second_moments:
                 r, c = wl.second_moments(spec.d_out, spec.d_in, seed=30_000 + m, device=dev)

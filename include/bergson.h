@@ -351,14 +351,17 @@ BERGSON_API void bergson_debug_inject_status(int status, int count);
  * Test aid for the projection work planner: for the same arguments as
  * bergson_project_grads_workspace, reports the (module, example, tile range)
  * partial slots of all launches (*n_slots), the work items the launches hand
- * out (*n_items) and how many of those items are pieces (*n_pieces; a piece
+ * out (*n_items), how many of those items are pieces (*n_pieces; a piece
  * projects one side of a slot over a range of 64-column chunks, and the
- * slot's last piece contracts them).  Host only: enqueues nothing.  Returns
- * the validation status; NULL outputs are skipped.
+ * slot's last piece contracts them) and how many layers share their input
+ * tensor A with another layer of the same (k_in, k_out) (*n_shared; their
+ * items are scheduled side by side).
+ * Host only: enqueues nothing.  Returns the validation status; NULL outputs
+ * are skipped.
  */
 BERGSON_API int bergson_debug_project_plan(const bergson_layer* layers, int n_layers, int64_t B,
                                            int64_t T, int64_t* n_slots, int64_t* n_items,
-                                           int64_t* n_pieces);
+                                           int64_t* n_pieces, int64_t* n_shared);
 
 /*
  * On-disk gradient store (Bergson Sec. 3.1: gradient stores persisted to disk,

@@ -100,7 +100,7 @@ def lib() -> ctypes.CDLL:
         "bergson_version": (i32, []),
         "bergson_debug_wait_probe": (i32, [u64, vp]),
         "bergson_debug_inject_status": (None, [i32, i32]),
-        "bergson_debug_project_plan": (i32, [lp, i32, i64, i64, i64p, i64p, i64p]),
+        "bergson_debug_project_plan": (i32, [lp, i32, i64, i64, i64p, i64p, i64p, i64p]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
@@ -366,10 +366,11 @@ def bergson_debug_inject_status(status: int, count: int) -> None:
     lib().bergson_debug_inject_status(int(status), int(count))
 
 
-def bergson_debug_project_plan(layers, B: int, T: int) -> tuple[int, int, int]:
-    """(slots, work items, pieces) the projection planner chooses; host only."""
+def bergson_debug_project_plan(layers, B: int, T: int) -> tuple[int, int, int, int]:
+    """(slots, work items, pieces, layers sharing their A) the projection planner
+    chooses; host only."""
     arr = _layer_array(layers)
-    n = [ctypes.c_int64() for _ in range(3)]
+    n = [ctypes.c_int64() for _ in range(4)]
     _check(lib().bergson_debug_project_plan(arr, len(layers), int(B), int(T),
                                             *(ctypes.byref(x) for x in n)))
     return tuple(x.value for x in n)

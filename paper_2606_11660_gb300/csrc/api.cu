@@ -129,7 +129,9 @@ bool valid_k(int64_t k) { return k == 16 || k == 32 || k == 64; }
 
 struct Group {
   int k_in = 0, k_out = 0;
-  std::vector<int> layers;     // indices into the caller's array, largest module first
+  std::vector<int> layers;     // indices into the caller's array, largest unit first
+  std::vector<std::pair<int, int>> units;   // (first position in layers, count): layers that
+                                            // read one A tensor, scheduled side by side
   int first_mod = 0;           // index of its first ModDesc in workspace
   int n_chunks = 0, tpc = 0;
   int n_slots = 0;             // layers * B * n_chunks partials
@@ -147,6 +149,7 @@ struct ProjLayout {
   int n_tiles = 0;
   std::vector<Group> groups;
   std::vector<int> mod_slot;   // layer index -> ModDesc slot
+  std::vector<uint8_t> shared; // layer index -> 1 if another layer of its group reads its A
   size_t mods_off = 0, segs_off = 0, ctr_off = 0, tv_off = 0;
   size_t token_off = 0;        // per-token score partials (token mode)
   std::vector<size_t> pin_off, pout_off;
@@ -219,10 +222,15 @@ int validate_blocks(const bergson_layer* layers, int n_layers, int64_t ld_out,
 
 int chunks_of(int64_t d) { return static_cast<int>((d + kChunk - 1) / kChunk); }
 
-// Cuts a group's large slots into pieces when the launch is too coarse for
-// the SMs to finish together (see kSplitShare).  Cost unit: one 64-column
-// chunk of one tile.  The table lists fused slots and pieces largest first.
-void plan_pieces(const bergson_layer* layers, int64_t B, int n_tiles, Group& g) {
+// Builds a group's work table when its slots need more than "item i is slot i":
+// (1) cutting: when the launch is too coarse for the SMs to finish together
+// (largest slot above kSplitShare of one CTA's share), large slots are cut
+// into pieces (split = allowed only in projection mode); (2) shared inputs:
+// the items of a unit's layers for the same example and tiles are listed next
+// to each other (A-side pieces too), so the scheduler starts them together.
+// Cost unit: one 64-column chunk of one tile; the table runs largest first.
+void plan_work(const bergson_layer* layers, int64_t B, int n_tiles, Group& g, bool allow_split) {
+  if (g.n_slots == 0) return;
   int64_t total = 0, max_slot = 0;
   for (int li : g.layers) {
     const int64_t c = chunks_of(layers[li].d_in) + chunks_of(layers[li].d_out);
@@ -230,57 +238,83 @@ void plan_pieces(const bergson_layer* layers, int64_t B, int n_tiles, Group& g) 
     max_slot = std::max<int64_t>(max_slot, c * std::min(g.tpc, n_tiles));
   }
   const double share = static_cast<double>(total) / kPlanCTAs;
-  if (g.n_slots == 0 || static_cast<double>(max_slot) <= kSplitShare * share) return;
+  const bool split = allow_split && static_cast<double>(max_slot) > kSplitShare * share;
+  bool shared = false;
+  for (const auto& u : g.units) shared = shared || u.second > 1;
+  if (!split && !shared) return;
   const double target = share / kPiecesPerShare;
+  // A piece stores and its slot's finisher reloads 4k fp32 bytes per token,
+  // against 128 bytes per token and chunk streamed: pieces of at least 2k
+  // chunks keep that under 1/32 of the piece's traffic.  (Fewer, larger
+  // pieces measured faster: Llama-8B-shaped block 0.790 ms at a quarter of a
+  // share per piece, 0.770 ms at half.)
+  auto pieces = [&](int ch, int k) {
+    const int n = static_cast<int>(std::ceil(static_cast<double>(ch) * g.tpc / target));
+    return std::max(1, std::min(n, ch / (2 * k)));
+  };
   struct Entry {
     WorkItem w;
-    int64_t cost;
+    int64_t key;
   };
   std::vector<Entry> es;
   int64_t base = 0;
-  int split = 0;
-  for (size_t mi = 0; mi < g.layers.size(); ++mi) {
-    const bergson_layer& ly = layers[g.layers[mi]];
-    const int ca = chunks_of(ly.d_in), cg = chunks_of(ly.d_out);
-    const bool cut = static_cast<double>(ca + cg) * g.tpc > target;
-    // A piece stores and its slot's finisher reloads 4k fp32 bytes per token,
-    // against 128 bytes per token and chunk streamed: pieces of at least 2k
-    // chunks keep that under 1/32 of the piece's traffic.  (Fewer, larger
-    // pieces measured faster: Llama-8B-shaped block 0.790 ms at a quarter of a
-    // share per piece, 0.770 ms at half.)
-    auto pieces = [&](int ch, int k) {
-      const int n = static_cast<int>(std::ceil(static_cast<double>(ch) * g.tpc / target));
-      return std::max(1, std::min(n, ch / (2 * k)));
-    };
-    const int n_a = cut ? pieces(ca, g.k_in) : 0, n_g = cut ? pieces(cg, g.k_out) : 0;
+  int n_split = 0;
+  for (const auto& u : g.units) {
+    const int m0 = u.first, cnt = u.second;
+    const int ca = chunks_of(layers[g.layers[m0]].d_in);
+    bool cut = false;
+    int64_t worst = 0;
+    std::vector<int> cg(cnt), n_g(cnt, 0);
+    for (int j = 0; j < cnt; ++j) {
+      cg[j] = chunks_of(layers[g.layers[m0 + j]].d_out);
+      worst = std::max<int64_t>(worst, ca + cg[j]);
+      cut = cut || (split && static_cast<double>(ca + cg[j]) * g.tpc > target);
+    }
+    const int n_a = cut ? pieces(ca, g.k_in) : 0;
+    if (cut)
+      for (int j = 0; j < cnt; ++j) n_g[j] = pieces(cg[j], g.k_out);
+    std::vector<int> sid(cnt);
+    std::vector<int64_t> sbase(cnt);
     for (int64_t b = 0; b < B; ++b) {
       for (int c = 0; c < g.n_chunks; ++c) {
-        const int slot = static_cast<int>((static_cast<int64_t>(mi) * B + b) * g.n_chunks + c);
         const int tiles = std::min(n_tiles, (c + 1) * g.tpc) - c * g.tpc;
+        auto slot_of = [&](int j) {
+          return static_cast<int>((static_cast<int64_t>(m0 + j) * B + b) * g.n_chunks + c);
+        };
         if (!cut) {
-          es.push_back({WorkItem{slot, 0, 0, 0, 0, 0, 0, 0, 0}, int64_t{ca + cg} * tiles});
+          for (int j = 0; j < cnt; ++j)
+            es.push_back({WorkItem{slot_of(j), 0, 0, 0, 0, 0, 0, 0, 0}, worst * tiles});
           continue;
         }
-        for (int side = 1; side <= 2; ++side) {
-          const int nch = side == 1 ? ca : cg, n = side == 1 ? n_a : n_g;
-          for (int q = 0; q < n; ++q) {
-            const int c0 = static_cast<int>(static_cast<int64_t>(q) * nch / n);
-            const int c1 = static_cast<int>(static_cast<int64_t>(q + 1) * nch / n);
-            es.push_back({WorkItem{slot, side, c0, c1, split, n_a, n_g, q, base},
+        for (int j = 0; j < cnt; ++j) {
+          sid[j] = n_split++;
+          sbase[j] = base;
+          base += (int64_t{n_a} * g.k_in + int64_t{n_g[j]} * g.k_out) * g.tpc * kTileTokens;
+        }
+        for (int q = 0; q < n_a; ++q) {             // A side: the unit's layers together
+          const int c0 = static_cast<int>(static_cast<int64_t>(q) * ca / n_a);
+          const int c1 = static_cast<int>(static_cast<int64_t>(q + 1) * ca / n_a);
+          for (int j = 0; j < cnt; ++j)
+            es.push_back({WorkItem{slot_of(j), 1, c0, c1, sid[j], n_a, n_g[j], q, sbase[j]},
+                          int64_t{c1 - c0} * tiles});
+        }
+        for (int j = 0; j < cnt; ++j) {
+          for (int q = 0; q < n_g[j]; ++q) {
+            const int c0 = static_cast<int>(static_cast<int64_t>(q) * cg[j] / n_g[j]);
+            const int c1 = static_cast<int>(static_cast<int64_t>(q + 1) * cg[j] / n_g[j]);
+            es.push_back({WorkItem{slot_of(j), 2, c0, c1, sid[j], n_a, n_g[j], q, sbase[j]},
                           int64_t{c1 - c0} * tiles});
           }
         }
-        base += (int64_t{n_a} * g.k_in + int64_t{n_g} * g.k_out) * g.tpc * kTileTokens;
-        ++split;
       }
     }
   }
   std::stable_sort(es.begin(), es.end(),
-                   [](const Entry& x, const Entry& y) { return x.cost > y.cost; });
+                   [](const Entry& x, const Entry& y) { return x.key > y.key; });
   g.table.resize(es.size());
   for (size_t i = 0; i < es.size(); ++i) g.table[i] = es[i].w;
   g.n_items = static_cast<int>(es.size());
-  g.n_split = split;
+  g.n_split = n_split;
   g.piece_floats = base;
 }
 
@@ -291,6 +325,7 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
   ProjLayout L;
   L.n_tiles = static_cast<int>((T + kTileTokens - 1) / kTileTokens);
   L.mod_slot.assign(n_layers, 0);
+  L.shared.assign(n_layers, 0);
   for (int i = 0; i < n_layers; ++i) {
     const int ki = static_cast<int>(layers[i].k_in), ko = static_cast<int>(layers[i].k_out);
     auto it = std::find_if(L.groups.begin(), L.groups.end(),
@@ -306,12 +341,39 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
   }
   int slot = 0;
   for (Group& g : L.groups) {
-    // Largest modules first: the scheduler hands items out in slot order, so
-    // the last items a launch waits on are the cheapest ones (longest
-    // processing time first).  Cost of one tile is proportional to d_in + d_out.
-    std::stable_sort(g.layers.begin(), g.layers.end(), [&](int a, int b) {
-      return layers[a].d_in + layers[a].d_out > layers[b].d_in + layers[b].d_out;
-    });
+    // Units: layers that read the same A tensor (same pointer and d_in, e.g. a
+    // gate and an up projection) are scheduled side by side, so that the second
+    // reader of an A tile can find it in L2 (the saving is small: the lines
+    // are streamed with evict_first, and L2 turns over in tens of
+    // microseconds; keeping them measured slower).  Largest unit first: the scheduler
+    // hands items out in order, so the last items a launch waits on are the
+    // cheapest ones (longest processing time first); a tile costs d_in + d_out.
+    std::vector<std::vector<int>> units;
+    for (int li : g.layers) {
+      auto u = std::find_if(units.begin(), units.end(), [&](const std::vector<int>& v) {
+        return layers[li].A != nullptr && layers[v[0]].A == layers[li].A &&
+               layers[v[0]].d_in == layers[li].d_in;
+      });
+      if (u == units.end()) units.push_back({li});
+      else u->push_back(li);
+    }
+    auto unit_cost = [&](const std::vector<int>& v) {
+      int64_t c = 0;
+      for (int li : v) c = std::max<int64_t>(c, layers[li].d_in + layers[li].d_out);
+      return c;
+    };
+    std::stable_sort(units.begin(), units.end(),
+                     [&](const std::vector<int>& x, const std::vector<int>& y) {
+                       return unit_cost(x) > unit_cost(y);
+                     });
+    g.layers.clear();
+    g.units.clear();
+    for (const auto& v : units) {
+      g.units.emplace_back(static_cast<int>(g.layers.size()), static_cast<int>(v.size()));
+      g.layers.insert(g.layers.end(), v.begin(), v.end());
+      if (v.size() > 1)
+        for (int li : v) L.shared[li] = 1;
+    }
     g.first_mod = slot;
     for (int li : g.layers) L.mod_slot[li] = slot++;
     const int nt_per_group = (g.k_in + g.k_out <= 32) ? 4 : ((g.k_in + g.k_out <= 64) ? 2 : 1);
@@ -332,7 +394,7 @@ ProjLayout plan_project(const bergson_layer* layers, int n_layers, int64_t B, in
     g.n_chunks = (L.n_tiles + tpc - 1) / tpc;
     g.n_slots = static_cast<int>(mb * g.n_chunks);
     g.n_items = g.n_slots;
-    if (n_queries == 0) plan_pieces(layers, B, L.n_tiles, g);
+    plan_work(layers, B, L.n_tiles, g, n_queries == 0);
   }
   size_t off = 0;
   L.mods_off = off;
@@ -478,7 +540,8 @@ void bergson_module_seeds(uint64_t base_seed, int64_t module_index, uint64_t* se
 const char* bergson_last_error(void) { return g_last_error.c_str(); }
 
 int bergson_debug_project_plan(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
-                               int64_t* n_slots, int64_t* n_items, int64_t* n_pieces) {
+                               int64_t* n_slots, int64_t* n_items, int64_t* n_pieces,
+                               int64_t* n_shared) {
   const int st = validate_layers(layers, n_layers, B, T);
   if (st != BERGSON_OK) return st;
   const ProjLayout L = plan_project(layers, n_layers, B, T);
@@ -491,6 +554,11 @@ int bergson_debug_project_plan(const bergson_layer* layers, int n_layers, int64_
   if (n_slots != nullptr) *n_slots = slots;
   if (n_items != nullptr) *n_items = items;
   if (n_pieces != nullptr) *n_pieces = pieces;
+  if (n_shared != nullptr) {
+    int64_t sh = 0;
+    for (uint8_t f : L.shared) sh += f;
+    *n_shared = sh;
+  }
   return BERGSON_OK;
 }
 

@@ -13,7 +13,7 @@ Workloads (module lists follow the Pythia and Llama layer shapes):
               a time
   llama8b     32 blocks x {4096->6144, 4096->4096, 4096->14336 (gate),
               4096->14336 (up), 14336->4096}, B=8, T=4096, k=16, one block at
-              a time
+              a time; gate and up read the same input (one A tensor)
   score4m     fp16 store 4,000,000 x 8192, 1024 queries, top-100
 """
 from __future__ import annotations
@@ -28,6 +28,7 @@ class ModuleSpec:
     name: str
     d_in: int
     d_out: int
+    shares_input: bool = False   # reads the same input tensor as the module before it
 
 
 @dataclasses.dataclass(frozen=True)
@@ -61,9 +62,16 @@ class CollectWorkload:
 def _blocks(n_blocks, shapes):
     mods = []
     for b in range(n_blocks):
-        for name, di, do in shapes:
-            mods.append(ModuleSpec(f"h{b}.{name}", di, do))
+        for shape in shapes:
+            name, di, do = shape[:3]
+            mods.append(ModuleSpec(f"h{b}.{name}", di, do, *shape[3:]))
     return tuple(mods)
+
+
+def input_bytes(specs, tokens: int) -> int:
+    """bf16 bytes of distinct A and G tensors of `tokens` tokens (a shared input counts once)."""
+    dims = sum(s.d_out + (0 if s.shares_input else s.d_in) for s in specs)
+    return 2 * dims * tokens
 
 
 TINY = CollectWorkload("tiny: Linear 64->64, B=8, T=32, k=16, Adafactor r,c",
@@ -85,9 +93,9 @@ PYTHIA1B4 = CollectWorkload(
 
 LLAMA8B = CollectWorkload(
     "llama8b-shaped: 32 blocks x {4096->6144, 4096->4096, 4096->14336 x2, 14336->4096}, "
-    "B=8, T=4096, k=16, one block per call",
+    "B=8, T=4096, k=16, one block per call, gate and up share their input",
     _blocks(32, [("qkv", 4096, 6144), ("attn_out", 4096, 4096), ("gate", 4096, 14336),
-                 ("up", 4096, 14336), ("down", 14336, 4096)]),
+                 ("up", 4096, 14336, True), ("down", 14336, 4096)]),
     8, 4096, 16, 0, False, 32, True)
 
 COLLECT_WORKLOADS = {"tiny": TINY, "pythia160m": PYTHIA160M, "pythia1b4": PYTHIA1B4,
@@ -123,6 +131,20 @@ def layer_inputs(spec: ModuleSpec, B: int, T: int, seed: int, device="cpu",
         A.mul_(spec.d_in ** -0.5)
         G.mul_(spec.d_out ** -0.5)
     return A.to(torch.bfloat16), G.to(torch.bfloat16)
+
+
+def module_inputs(specs, B: int, T: int, seeds, device="cpu", input_scale: bool = False):
+    """[(A, G)] per module as layer_inputs draws them, except that a module with
+    shares_input takes the previous module's A tensor itself (same storage)."""
+    out = []
+    for spec, seed in zip(specs, seeds):
+        A, G = layer_inputs(spec, B, T, seed=seed, device=device, input_scale=input_scale)
+        if spec.shares_input:
+            if not out or out[-1][0].shape[-1] != spec.d_in:
+                raise ValueError(f"{spec.name}: no preceding module with d_in={spec.d_in}")
+            A = out[-1][0]
+        out.append((A, G))
+    return out
 
 
 def right_padding_mask(B: int, T: int, max_pad: int, seed: int, device="cpu"):

@@ -18,13 +18,15 @@ def make_layers(specs, B, T, k_pairs, base_seed=0, data_seed=0, rc=False, input_
     """Seeded inputs for several modules; returns (gpu Layers, oracle Layers, ld_out)."""
     gl, ol = [], []
     off = 0
-    for m, (spec, (ki, ko)) in enumerate(zip(specs, k_pairs)):
-        A, G = wl.layer_inputs(spec, B, T, seed=data_seed * 1000 + m, input_scale=input_scale)
+    ins = wl.module_inputs(specs, B, T, [data_seed * 1000 + m for m in range(len(specs))],
+                           input_scale=input_scale)
+    for m, (spec, (ki, ko), (A, G)) in enumerate(zip(specs, k_pairs, ins)):
         r = c = None
         if rc:
             r, c = wl.second_moments(spec.d_out, spec.d_in, seed=data_seed * 1000 + 500 + m)
         s_in, s_out = orc.module_seeds(base_seed, m)
-        gl.append(bg.Layer(A.to(device), G.to(device), ki, ko, s_in, s_out,
+        A_dev = gl[-1].A if spec.shares_input else A.to(device)   # one device tensor when shared
+        gl.append(bg.Layer(A_dev, G.to(device), ki, ko, s_in, s_out,
                            None if r is None else r.to(device), None if c is None else c.to(device),
                            off, kind))
         ol.append(orc.Layer(np32(A), np32(G), ki, ko, s_in, s_out,

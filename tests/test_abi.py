@@ -240,8 +240,9 @@ def _plan(layers, B, T):
 
 def _block_layers(specs, k):
     out, off = [], 0
-    for s in specs:
-        out.append(_layer(d_in=s.d_in, d_out=s.d_out, k_in=k, k_out=k, out_col_offset=off))
+    for i, s in enumerate(specs):
+        a = out[-1].A if s.shares_input else FAKE + 8192 * i       # a shared input: one pointer
+        out.append(_layer(A=a, d_in=s.d_in, d_out=s.d_out, k_in=k, k_out=k, out_col_offset=off))
         off += k * k
     return out
 
@@ -249,11 +250,9 @@ def _block_layers(specs, k):
 def test_planner_keeps_fine_launches_fused():
     """48 modules x 32 examples x 4 slots: enough work items, no pieces."""
     cfg = wl.PYTHIA160M
-    slots, items, pieces = _plan(_block_layers(cfg.modules, 16), cfg.B, cfg.T)
-    assert (slots, items, pieces) == (48 * 32 * 4, 48 * 32 * 4, 0)
+    assert _plan(_block_layers(cfg.modules, 16), cfg.B, cfg.T) == (48 * 32 * 4, 48 * 32 * 4, 0, 0)
     cfg = wl.PYTHIA1B4                  # one block per call: 512 slots, still balanced enough
-    slots, items, pieces = _plan(_block_layers(cfg.block_modules(0), 32), cfg.B, cfg.T)
-    assert (slots, items, pieces) == (4 * 16 * 8, 4 * 16 * 8, 0)
+    assert _plan(_block_layers(cfg.block_modules(0), 32), cfg.B, cfg.T) == (512, 512, 0, 0)
 
 
 @pytest.mark.parametrize("name,B,T,k", [("llama8b", 8, 4096, 16), ("tiny", 8, 32, 16),
@@ -261,7 +260,7 @@ def test_planner_keeps_fine_launches_fused():
 def test_planner_cuts_coarse_launches_into_pieces(name, B, T, k):
     cfg = wl.COLLECT_WORKLOADS[name]
     specs = cfg.block_modules(0)
-    slots, items, pieces = _plan(_block_layers(specs, k), B, T)
+    slots, items, pieces, _ = _plan(_block_layers(specs, k), B, T)
     fused = items - pieces
     split = slots - fused
     assert pieces > 0 and split > 0
@@ -274,3 +273,20 @@ def test_planner_validates_like_the_workspace_query():
     with pytest.raises(bg.BergsonError) as e:
         _plan([_layer(k_in=24)], 2, 32)
     assert e.value.status == bg.BERGSON_EUNSUPPORTED
+
+
+def test_planner_groups_layers_that_share_an_input():
+    """Llama-shaped block: gate and up read one A tensor."""
+    cfg = wl.LLAMA8B
+    layers = _block_layers(cfg.block_modules(0), 16)
+    slots, items, pieces, shared = _plan(layers, cfg.B, cfg.T)
+    assert shared == 2 and pieces > 0
+    # many examples: no pieces, but a work table lists the shared layers' items together
+    slots, items, pieces, shared = _plan(layers, 256, cfg.T)
+    assert shared == 2 and pieces == 0 and items == slots
+    # different d_in, or different k, is not sharing
+    a = _layer(d_in=64, d_out=128)
+    b = _layer(A=a.A, d_in=128, d_out=64, out_col_offset=256)
+    c = _layer(A=a.A, d_in=64, d_out=64, k_in=32, out_col_offset=512)
+    assert _plan([a, b, c], 2, 32)[3] == 0
+    assert _plan([a, _layer(A=a.A, d_in=64, d_out=64, out_col_offset=256)], 2, 32)[3] == 2

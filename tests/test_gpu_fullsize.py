@@ -79,10 +79,11 @@ def test_streamed_block_calls_sampled_blocks(name, blocks, samples):
     ws = None
     for bi in blocks:
         specs = cfg.block_modules(bi)
-        layers, held = [], []
-        for j, spec in enumerate(specs):
+        layers = []
+        ins = wl.module_inputs(specs, cfg.B, cfg.T, [20_000 + bi * nmod + j for j in range(nmod)],
+                               device=DEV, input_scale=True)
+        for j, (spec, (A, G)) in enumerate(zip(specs, ins)):
             m = bi * nmod + j
-            A, G = wl.layer_inputs(spec, cfg.B, cfg.T, seed=20_000 + m, device=DEV, input_scale=True)
             r = c = None
             if cfg.second_moments:
                 r, c = wl.second_moments(spec.d_out, spec.d_in, seed=30_000 + m, device=DEV)
@@ -100,7 +101,7 @@ def test_streamed_block_calls_sampled_blocks(name, blocks, samples):
             want = _oracle_block(ly.A[b], ly.G[b], None, k, k, ly.seed_in, ly.seed_out, ly.r, ly.c)
             g = got[b, m * blk:(m + 1) * blk]
             assert np.linalg.norm(g - want) / np.linalg.norm(want) <= TIGHT, (name, bi, b, j)
-        del layers
+        del layers, ins
         torch.cuda.empty_cache()
     # the written blocks form rows that the store normalises to unit length
     cols = np.concatenate([np.arange(bi * nmod * blk, (bi + 1) * nmod * blk) for bi in blocks])

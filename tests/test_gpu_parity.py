@@ -132,7 +132,7 @@ def test_piece_path_wide_modules_mask_bias_moments():
                              input_scale=True)
     gl[1].bias_col_offset = ol[1].bias_col_offset = ld
     ld_b = ld + 16
-    slots, items, pieces = bg.bergson_debug_project_plan(gl, B, T)
+    slots, items, pieces, _ = bg.bergson_debug_project_plan(gl, B, T)
     assert pieces > 0 and items > slots
     g = wl.generator(12, "cpu")
     mask = (torch.rand((B, T), generator=g) > 0.25).to(torch.uint8)
@@ -364,3 +364,22 @@ def test_bias_blocks_with_mask_and_moments():
     with pytest.raises(bg.BergsonError) as e:
         bg.bergson_project_grads(gl, B, T, None, out, ws)
     assert e.value.status == bg.BERGSON_EINVAL
+
+
+@pytest.mark.parametrize("B,T,d,f", [(2, 700, 1024, 2048), (200, 256, 128, 256)])
+def test_shared_input_layers(B, T, d, f):
+    """Layers reading one A tensor (a gate and an up projection) are scheduled
+    side by side; results match the oracle on the piece path (few examples)
+    and on the fused path (many)."""
+    specs = [wl.ModuleSpec("gate", d, f), wl.ModuleSpec("up", d, f, True),
+             wl.ModuleSpec("down", f, d)]
+    gl, ol, ld = make_layers(specs, B, T, [(16, 16)] * 3, base_seed=4, data_seed=2, rc=True,
+                             input_scale=True)
+    assert gl[1].A.data_ptr() == gl[0].A.data_ptr()
+    slots, items, pieces, shared = bg.bergson_debug_project_plan(gl, B, T)
+    assert shared == 2 and (pieces > 0) == (B == 2)
+    g = wl.generator(15, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.2).to(torch.uint8)
+    out = run_project(gl, B, T, mask.to(DEV), ld)
+    want = orc.project_grads(ol, mask.numpy(), ld)
+    assert rel_frobenius(np32(out).astype(np.float64), want).max() <= TIGHT
