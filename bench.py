@@ -443,7 +443,7 @@ def bench_fisher(args, world, dev, state):
             "preconditioner_ms": round(pow_ms, 1), "newton_schulz_iterations": args.fisher_iters,
             "preconditioner_tflops": round(gemm_flops / (pow_ms * 1e-3) / 1e12, 2),
             "what": "step = project_grads + precondition_rows (R^-1/2, K=12288) + build_store; "
-                    "fit and R^-1/2 are one-time costs (fp32 FFMA GEMMs)"}
+                    "fit and R^-1/2 are one-time costs (3xTF32 tcgen05 GEMMs)"}
 
 
 def bench_streamed(args, world, dev, name, peaks):

@@ -20,7 +20,6 @@ namespace bergson {
 namespace {
 
 constexpr int kVersion = 100;                        // 0.1.0
-constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 s
 constexpr int kSchedTargetItems = 8192;              // work items per projection launch (target)
 // Piece splitting of projection slots.  The planner assumes kPlanCTAs
 // persistent CTAs (one per SM of this part; the launch uses the real count).
@@ -517,6 +516,12 @@ int record_error(int code, const char* fmt, ...) {
   return code;
 }
 
+CUresult encode_tmap_2d(CUtensorMap* tm, CUtensorMapDataType dt, const void* ptr, int64_t inner,
+                        int64_t outer, int64_t row_bytes, int box_inner, int box_outer) {
+  if (encode_fn() == nullptr) return CUDA_ERROR_NOT_SUPPORTED;
+  return encode_2d(tm, dt, ptr, inner, outer, row_bytes, box_inner, box_outer);
+}
+
 }  // namespace bergson
 
 using namespace bergson;
@@ -895,31 +900,21 @@ static int run_xgemm(const float* x, int64_t B, int64_t ldx, const float* y, int
     return fail(BERGSON_ECUDA, "cuTensorMapEncodeTiled is unavailable from the driver");
   int* status = status_word(dg.dev);
   if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
-  const XGemmPlan pl = xgemm_plan(B, Q, K);
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  CUtensorMap tm_y, tm_xh, tm_xl;
-  CUresult r1 = encode_2d(&tm_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, y, K, Q, ldy * 4, 32, 128);
-  CUresult r2 = encode_2d(&tm_xh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, ws + pl.xh_off, K, B, K * 4, 32,
-                          pl.n_pad);
-  CUresult r3 = encode_2d(&tm_xl, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, ws + pl.xl_off, K, B, K * 4, 32,
-                          pl.n_pad);
-  if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS || r3 != CUDA_SUCCESS)
-    return fail(BERGSON_ECUDA, "%s: tensor map encoding failed (%d %d %d)", what, (int)r1,
-                (int)r2, (int)r3);
   XGemmArgs a;
   a.x = x;
   a.ldx = ldx;
+  a.y = y;
+  a.ldy = ldy;
   a.B = static_cast<int>(B);
   a.Q = static_cast<int>(Q);
   a.K = static_cast<int>(K);
   a.unit = unit;
   a.scores = out;
   a.ld_scores = ld_out;
-  a.ws = ws;
+  a.ws = static_cast<uint8_t*>(workspace);
   a.status = status;
   a.timeout_ns = kWaitTimeoutNs;
-  cudaError_t e = launch_xgemm(tm_y, tm_xh, tm_xl, pl, a, sm_count(dg.dev),
-                               static_cast<cudaStream_t>(stream));
+  cudaError_t e = xgemm_run(a, sm_count(dg.dev), static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return fail_cuda(e, what);
   return BERGSON_OK;
 }
@@ -1054,8 +1049,10 @@ int bergson_fisher_fit(const float* rows, int64_t n, int64_t K, int64_t ld, floa
   if ((st = injected()) != BERGSON_OK) return st;
   DeviceGuard dg(R);
   if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  int* status = status_word(dg.dev);
+  if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
   cudaError_t e = launch_fisher_fit(rows, static_cast<int>(n), static_cast<int>(K), ld, R, ldr,
-                                    static_cast<float*>(workspace),
+                                    static_cast<float*>(workspace), status, sm_count(dg.dev),
                                     static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return fail_cuda(e, "Fisher fit launch");
   return BERGSON_OK;
@@ -1090,9 +1087,11 @@ int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K, i
   if ((st = injected()) != BERGSON_OK) return st;
   DeviceGuard dg(M);
   if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  int* status = status_word(dg.dev);
+  if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
   cudaError_t e = launch_fisher_power(R1, R2, static_cast<int>(K), ldr, lam, damping,
                                       power == BERGSON_FISHER_INV ? 1 : 0, iterations, M, ldm,
-                                      static_cast<float*>(workspace),
+                                      static_cast<float*>(workspace), status, sm_count(dg.dev),
                                       static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return fail_cuda(e, "Fisher preconditioner launch");
   return BERGSON_OK;

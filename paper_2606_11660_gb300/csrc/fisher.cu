@@ -11,11 +11,11 @@
 //   apply:  x' = M x for each row (bergson_precondition_rows, same GEMM as
 //           the on-the-fly scores).
 //
-// All products are fp32 "NT" GEMMs C = alpha A B^T + beta C + gamma I, with A
-// and B row-major and the reduction index contiguous: a 128 x 128 CTA tile,
-// 8 x 8 outputs per thread over strided rows/columns (conflict-free 16-byte
-// shared loads) and cp.async double buffering.  Products of the iteration
-// are symmetric in exact arithmetic, so B^T = B there; each update is
+// All products are "NT" GEMMs C = alpha A B^T + beta C + gamma I with A and B
+// row-major and the reduction index contiguous, run by the tcgen05 skinny
+// product of onthefly.cu (3xTF32: fp32 accuracy from tf32 tensor-core MMAs)
+// with 128-row tiles on both sides.  Products of the iteration are
+// symmetric in exact arithmetic, so B^T = B there; each update is
 // re-symmetrised so that rounding cannot build up an antisymmetric part.
 
 #include "internal.h"
@@ -23,92 +23,6 @@
 namespace bergson {
 
 namespace {
-
-constexpr int kTile = 128;
-constexpr int kBK = 16;
-constexpr int kThreads = 256;
-
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool valid) {
-  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(gmem),
-               "r"(valid ? 16 : 0)
-               : "memory");
-}
-
-// C[m, n] = alpha * sum_k A[m, k] B[n, k] + beta * C[m, n] + (m == n ? gamma : 0),
-// alpha and gamma optionally scaled by a device scalar: alpha * (*alpha_s), gamma * (*gamma_s).
-__global__ void __launch_bounds__(kThreads) gemm_nt_kernel(
-    const float* __restrict__ A, int64_t lda, const float* __restrict__ B, int64_t ldb,
-    float* C, int64_t ldc, int M, int N, int K, float alpha, float beta, float gamma,
-    const float* __restrict__ alpha_s) {
-  __shared__ __align__(16) float as[2][kTile][kBK + 4];
-  __shared__ __align__(16) float bs[2][kTile][kBK + 4];
-  const int tid = threadIdx.x;
-  const int tx = tid % 16;
-  const int ty = tid / 16;
-  const int m0 = blockIdx.y * kTile;
-  const int n0 = blockIdx.x * kTile;
-  const int nsteps = (K + kBK - 1) / kBK;
-
-  auto load = [&](int st, int k0) {
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {   // 128 rows x 4 chunks of 16 B, for A and for B
-      const int idx = tid + h * kThreads;
-      const int r = idx / 4, c = (idx % 4) * 4;
-      const bool oka = m0 + r < M && k0 + c < K;
-      cp_async16(&as[st][r][c], oka ? A + (m0 + r) * lda + k0 + c : A, oka);
-      const bool okb = n0 + r < N && k0 + c < K;
-      cp_async16(&bs[st][r][c], okb ? B + (n0 + r) * ldb + k0 + c : B, okb);
-    }
-    asm volatile("cp.async.commit_group;" ::: "memory");
-  };
-
-  float acc[8][8] = {};
-  if (nsteps > 0) load(0, 0);
-  for (int step = 0; step < nsteps; ++step) {
-    const int st = step & 1;
-    if (step + 1 < nsteps) {
-      load(st ^ 1, (step + 1) * kBK);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < kBK; kk += 4) {
-      float4 a[8], b[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) a[i] = *reinterpret_cast<const float4*>(&as[st][ty + 16 * i][kk]);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) b[j] = *reinterpret_cast<const float4*>(&bs[st][tx + 16 * j][kk]);
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          acc[i][j] = fmaf(a[i].x, b[j].x, acc[i][j]);
-          acc[i][j] = fmaf(a[i].y, b[j].y, acc[i][j]);
-          acc[i][j] = fmaf(a[i].z, b[j].z, acc[i][j]);
-          acc[i][j] = fmaf(a[i].w, b[j].w, acc[i][j]);
-        }
-    }
-    __syncthreads();
-  }
-  const float al = alpha_s != nullptr ? alpha * *alpha_s : alpha;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int m = m0 + ty + 16 * i;
-    if (m >= M) continue;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int n = n0 + tx + 16 * j;
-      if (n >= N) continue;
-      float v = al * acc[i][j];
-      if (beta != 0.0f) v = fmaf(beta, C[m * ldc + n], v);
-      if (m == n) v += gamma;
-      C[m * ldc + n] = v;
-    }
-  }
-}
 
 // xt[k, i] = x[i, k] for i < n, zero for n <= i < n_pad.
 __global__ void transpose_kernel(const float* __restrict__ x, int n, int K, int64_t ldx,
@@ -248,14 +162,34 @@ __global__ void scale_copy_kernel(const float* __restrict__ src, int K,
     dst[(e / K) * ldd + e % K] = src[e] * sc;
 }
 
+// C[m, n] = alpha' sum_k A[m, k] B[n, k] + beta C[m, n] + gamma [m == n] for
+// M x K A and N x K B (alpha' = alpha * (*alpha_s) when alpha_s is given);
+// `ws` holds xgemm_plan(M, N, K).
 cudaError_t gemm_nt(const float* A, int64_t lda, const float* B, int64_t ldb, float* C,
                     int64_t ldc, int M, int N, int K, float alpha, float beta, float gamma,
-                    const float* alpha_s, cudaStream_t s) {
-  dim3 grid((N + kTile - 1) / kTile, (M + kTile - 1) / kTile);
-  gemm_nt_kernel<<<grid, kThreads, 0, s>>>(A, lda, B, ldb, C, ldc, M, N, K, alpha, beta, gamma,
-                                           alpha_s);
-  return cudaGetLastError();
+                    const float* alpha_s, uint8_t* ws, int* status, int sms, cudaStream_t s) {
+  XGemmArgs a;
+  a.x = A;
+  a.ldx = lda;
+  a.y = B;
+  a.ldy = ldb;
+  a.B = M;
+  a.Q = N;
+  a.K = K;
+  a.unit = 0;
+  a.alpha = alpha;
+  a.alpha_s = alpha_s;
+  a.beta = beta;
+  a.gamma = gamma;
+  a.scores = C;
+  a.ld_scores = ldc;
+  a.ws = ws;
+  a.status = status;
+  a.timeout_ns = kWaitTimeoutNs;
+  return xgemm_run(a, sms, s);
 }
+
+size_t round_up256(size_t x) { return (x + 255) / 256 * 256; }
 
 unsigned elementwise_blocks(int64_t n) {
   const int64_t b = (n + 255) / 256;
@@ -266,28 +200,34 @@ unsigned elementwise_blocks(int64_t n) {
 
 size_t fisher_fit_workspace(int64_t n, int64_t K) {
   const int64_t n_pad = (n + 3) / 4 * 4;
-  return static_cast<size_t>(K) * n_pad * sizeof(float);
+  return round_up256(static_cast<size_t>(K) * n_pad * sizeof(float)) +
+         xgemm_plan(K, K, n_pad).total;
 }
 
 cudaError_t launch_fisher_fit(const float* x, int n, int K, int64_t ldx, float* r, int64_t ldr,
-                              float* ws, cudaStream_t s) {
+                              float* ws, int* status, int sms, cudaStream_t s) {
   const int n_pad = (n + 3) / 4 * 4;
   dim3 grid((n_pad + 31) / 32, (K + 31) / 32);
   transpose_kernel<<<grid, dim3(32, 8), 0, s>>>(x, n, K, ldx, ws, n_pad);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  uint8_t* gws = reinterpret_cast<uint8_t*>(ws) +
+                 round_up256(static_cast<size_t>(K) * n_pad * sizeof(float));
   return gemm_nt(ws, n_pad, ws, n_pad, r, ldr, K, K, n_pad, 1.0f / static_cast<float>(n), 0.0f,
-                 0.0f, nullptr, s);
+                 0.0f, nullptr, gws, status, sms, s);
 }
 
 size_t fisher_power_workspace(int64_t K) {
-  return (4 * static_cast<size_t>(K) * K + 64 + kFrobBlocks) * sizeof(float);
+  return round_up256((4 * static_cast<size_t>(K) * K + 64 + kFrobBlocks) * sizeof(float)) +
+         xgemm_plan(K, K, K).total;
 }
 
 cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
                                 float damping, int inverse, int iterations, float* m, int64_t ldm,
-                                float* ws, cudaStream_t s) {
+                                float* ws, int* status, int sms, cudaStream_t s) {
   const int64_t kk = static_cast<int64_t>(K) * K;
+  uint8_t* gws = reinterpret_cast<uint8_t*>(ws) +
+                 round_up256((4 * static_cast<size_t>(K) * K + 64 + kFrobBlocks) * sizeof(float));
   float* a = ws;            // mixed, damped R
   float* y = a + kk;
   float* z = y + kk;
@@ -302,14 +242,17 @@ cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t
   if (e != cudaSuccess) return e;
   for (int it = 0; it < iterations; ++it) {
     // T = 1.5 I - 0.5 Z Y;  Y <- Y T;  Z <- T Z
-    if ((e = gemm_nt(z, K, y, K, t, K, K, K, K, -0.5f, 0.0f, 1.5f, nullptr, s)) != cudaSuccess)
+    if ((e = gemm_nt(z, K, y, K, t, K, K, K, K, -0.5f, 0.0f, 1.5f, nullptr, gws, status, sms,
+                     s)) != cudaSuccess)
       return e;
-    if ((e = gemm_nt(y, K, t, K, a, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, s)) != cudaSuccess)
+    if ((e = gemm_nt(y, K, t, K, a, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, gws, status, sms,
+                     s)) != cudaSuccess)
       return e;
     float* swap = y;      // new Y is in `a`; the old Y buffer becomes scratch
     y = a;
     a = swap;
-    if ((e = gemm_nt(t, K, z, K, a, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, s)) != cudaSuccess)
+    if ((e = gemm_nt(t, K, z, K, a, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, gws, status, sms,
+                     s)) != cudaSuccess)
       return e;
     swap = z;
     z = a;
@@ -318,7 +261,8 @@ cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t
     symmetrize_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(z, K);
   }
   // Z ~ (R/c)^-1/2:  R^-1/2 = Z / sqrt(c);  R^-1 = Z Z / c
-  if (inverse) return gemm_nt(z, K, z, K, m, ldm, K, K, K, 1.0f, 0.0f, 0.0f, scal + 4, s);
+  if (inverse)
+    return gemm_nt(z, K, z, K, m, ldm, K, K, K, 1.0f, 0.0f, 0.0f, scal + 4, gws, status, sms, s);
   scale_copy_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(z, K, scal + 3, m, ldm);
   return cudaGetLastError();
 }

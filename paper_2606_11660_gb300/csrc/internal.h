@@ -15,6 +15,7 @@ constexpr int kChunk = 64;           // bf16 elements per 128-byte swizzled row
 constexpr int kScoreBN = 256;        // store rows per score tile (tcgen05 N)
 constexpr int kScoreQT = 128;        // queries per query tile (tcgen05 M)
 constexpr int kMaxTopk = 1024;
+constexpr uint64_t kWaitTimeoutNs = 4000000000ull;   // bounded device waits: 4 s
 constexpr int kPlanCTAs = 152;   // persistent CTAs work planners assume (one per SM of this part)
 
 // Per-module launch record kept in workspace (global memory).  The tensor maps
@@ -141,11 +142,11 @@ cudaError_t launch_aggregate(const float* rows, int64_t n, int K, int64_t ld,
                              float* out, int64_t ld_out, cudaStream_t s);
 size_t fisher_fit_workspace(int64_t n, int64_t K);
 cudaError_t launch_fisher_fit(const float* x, int n, int K, int64_t ldx, float* r, int64_t ldr,
-                              float* ws, cudaStream_t s);
+                              float* ws, int* status, int sms, cudaStream_t s);
 size_t fisher_power_workspace(int64_t K);
 cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
                                 float damping, int inverse, int iterations, float* m, int64_t ldm,
-                                float* ws, cudaStream_t s);
+                                float* ws, int* status, int sms, cudaStream_t s);
 
 // Skinny fp32 product C[b, q] = <x_b, y_q> on the tensor cores (on-the-fly
 // scores, preconditioner application): plan and workspace layout.
@@ -163,18 +164,26 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K);
 struct XGemmArgs {
   const float* x;          // [B, ldx] fp32, 16-byte aligned rows
   int64_t ldx;
+  const float* y;          // [Q, ldy] fp32, 16-byte aligned rows
+  int64_t ldy;
   int B, Q, K;
-  int unit;                // 1: cosine (scale by both norms), 0: plain products
-  float* scores;           // [B, ld_scores]
+  int unit;                // 1: cosine (scale by both norms), 0: affine (below)
+  float alpha = 1.0f;      // unit == 0: out = alpha' <x_b, y_q> + beta out + gamma [b == q],
+  const float* alpha_s = nullptr;   //   alpha' = alpha * (*alpha_s) when alpha_s is given
+  float beta = 0.0f;
+  float gamma = 0.0f;
+  float* scores;           // out [B, ld_scores]
   int64_t ld_scores;
-  uint8_t* ws;             // workspace laid out by the plan
+  uint8_t* ws;             // workspace laid out by xgemm_plan(B, Q, K)
   int* status;
   uint64_t timeout_ns;
 };
-// tm_y: y [Q, K] fp32, box 32 x 128; tm_xh / tm_xl: the plan's x_hi / x_lo
-// regions [B, K], box 32 x n_pad; all with the 128-byte swizzle.
-cudaError_t launch_xgemm(const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
-                         const CUtensorMap& tm_xl, const XGemmPlan& plan, const XGemmArgs& a,
-                         int sms, cudaStream_t s);
+// Encodes the tensor maps and launches the split, product and finishing
+// kernels.  Returns cudaErrorInvalidValue if a tensor map cannot be encoded.
+cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s);
+
+// 2-D tiled tensor map with the 128-byte swizzle (host; defined with the C ABI).
+CUresult encode_tmap_2d(CUtensorMap* tm, CUtensorMapDataType dt, const void* ptr, int64_t inner,
+                        int64_t outer, int64_t row_bytes, int box_inner, int box_outer);
 
 }  // namespace bergson

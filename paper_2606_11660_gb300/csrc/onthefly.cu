@@ -10,8 +10,8 @@
 // kind::tf32) at fp32 accuracy.  tf32 keeps 10 of fp32's 23 mantissa bits, so
 // every operand is split into two tf32 values, each rounded to nearest:
 //   y ~= y_hi + y_lo,  y_lo = tf32(y - y_hi)   (error <= 2^-22 |y|),
-//   <x, y> ~= <x_hi, y_hi> + <x_lo, y_hi> + <x_hi, y_lo> (+ <x_lo, y_lo>, which
-// comes free here): the 3xTF32 scheme of Ootomo and Yokota (2022).
+//   <x, y> ~= <x_hi, y_hi> + <x_lo, y_hi> + <x_hi, y_lo>, dropping <x_lo, y_lo>
+// (relative size <= 2^-22): the 3xTF32 scheme of Ootomo and Yokota (2022).
 // Round-to-nearest splitting keeps the per-product errors unbiased, so they
 // grow like sqrt(K) rather than K.
 //
@@ -20,12 +20,13 @@
 // ring; the tile itself is y_hi (the tensor cores truncate it), and four
 // converter warps write its y_lo (the swizzle permutes 16-byte chunks, so an
 // elementwise map keeps the layout) and, for cosine scores, accumulate the
-// rows' squared norms from the same tile; one thread issues two MMAs per 8 columns into TMEM (M = 128 rows
-// of y; N = x_hi and x_lo stacked, twice the batch padded to 16), which reads
-// each y part from shared memory once (shared-memory bandwidth, not the
-// tensor pipe, bounds this kernel); four epilogue warps add the four partial
-// products up.  x is small: a pre-pass splits it into x_hi and x_lo
-// (and its norms) in workspace, and its tiles come from L2.
+// rows' squared norms from the same tile.  One thread issues two MMAs per 8
+// columns into TMEM (M = 128 rows of y): y_hi against x_hi and x_lo stacked
+// (N = twice the batch tile) and y_lo against x_hi (N = the batch tile), which
+// reads each y part from shared memory once (for small batches shared-memory
+// bandwidth, not the tensor pipe, bounds this kernel); four epilogue warps
+// add the three partial products up.  x is split by a pre-pass into x_hi and
+// x_lo (and its norms) in workspace, and its tiles come from L2.
 //
 // Work items are (128-row tile of y, batch tile, K slice), handed out
 // round-robin to persistent CTAs (all items have the same cost); every item
@@ -260,7 +261,8 @@ __global__ void __launch_bounds__(kXThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = make_idesc_tf32(kXM, 2 * p.n_pad);
+      const uint32_t idesc = make_idesc_tf32(kXM, 2 * p.n_pad);   // y_hi [x_hi; x_lo]^T
+      const uint32_t idesc_lo = make_idesc_tf32(kXM, p.n_pad);    // y_lo x_hi^T
       int stage = 0;
       uint32_t ph = 0;
       int ab = 0;
@@ -271,10 +273,10 @@ __global__ void __launch_bounds__(kXThreads, 1)
         if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
         tc_fence_after();
         // Set ab: D_hi = y_hi [x_hi; x_lo]^T in columns [0, 2 n_pad), D_lo =
-        // y_lo [x_hi; x_lo]^T in [2 n_pad, 4 n_pad).  x_hi and x_lo land next to
-        // each other, so one B operand of 2 n_pad rows serves both, and y_hi and
-        // y_lo are each read once per K step.
-        const uint32_t d_hi = tmem + ab * 4 * p.n_pad;
+        // y_lo x_hi^T in [2 n_pad, 3 n_pad).  x_hi and x_lo land next to each
+        // other, so one B operand of 2 n_pad rows serves both, and y_hi and y_lo
+        // are each read once per K step.
+        const uint32_t d_hi = tmem + ab * 3 * p.n_pad;
         const uint32_t d_lo = d_hi + 2 * p.n_pad;
         for (int st = it.s0; st < it.s1; ++st) {
           if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
@@ -292,7 +294,7 @@ __global__ void __launch_bounds__(kXThreads, 1)
             const uint64_t o = 2 * kk;
             const uint32_t acc = st != it.s0 || kk != 0;
             umma_tf32(d_hi, dyh + o, dx + o, idesc, acc);
-            umma_tf32(d_lo, dyl + o, dx + o, idesc, acc);
+            umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, acc);
           }
           umma_commit(smem_u32(&empty[stage]));
           if (++stage == p.stages) { stage = 0; ph ^= 1; }
@@ -365,18 +367,15 @@ __global__ void __launch_bounds__(kXThreads, 1)
       const int q = it.mt * kXM + row;
       float* dst = p.partial + static_cast<int64_t>(it.z) * p.B * p.Q + q;
       const uint32_t tbase =
-          tmem + (static_cast<uint32_t>(32 * quarter) << 16) + ab * 4 * p.n_pad;
+          tmem + (static_cast<uint32_t>(32 * quarter) << 16) + ab * 3 * p.n_pad;
       for (int c = 0; c < p.n_pad; c += 16) {
-        // <x_b, y_q> ~= y_hi x_hi + y_hi x_lo + y_lo x_hi (+ y_lo x_lo), in this order
+        // <x_b, y_q> ~= y_hi x_hi + y_hi x_lo + y_lo x_hi, in this order
         float v[16], w[16];
         tmem_ld16(tbase + c, v);
         tmem_ld16(tbase + p.n_pad + c, w);
 #pragma unroll
         for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
         tmem_ld16(tbase + 2 * p.n_pad + c, w);
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
-        tmem_ld16(tbase + 3 * p.n_pad + c, w);
 #pragma unroll
         for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
         if (q < p.Q) {
@@ -402,24 +401,32 @@ __global__ void __launch_bounds__(kXThreads, 1)
   }
 }
 
-// scores[b, q] = (sum over slices z, in order, of partial[z, b, q]) * sx[b] * t_q
-// with t_q = 1/sqrt(sum over z of ynorm[z, q]) (0 for a zero row); unscaled
-// when sx is null.
+// s = sum over slices z (in order) of partial[z, b, q].  Cosine (sx given):
+// scores[b, q] = s * sx[b] * t_q, t_q = 1/sqrt(sum over z of ynorm[z, q]) (0
+// for a zero row).  Otherwise scores[b, q] = alpha' s + beta scores[b, q] +
+// gamma [b == q], alpha' = alpha * (*alpha_s) when alpha_s is given.
 __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, int Q,
                               const float* __restrict__ sx, const float* __restrict__ ynorm,
-                              float* __restrict__ scores, int64_t ld) {
+                              float alpha, const float* __restrict__ alpha_s, float beta,
+                              float gamma, float* scores, int64_t ld) {
   const int64_t n = static_cast<int64_t>(B) * Q;
+  const float al = alpha_s != nullptr ? alpha * *alpha_s : alpha;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     float s = 0.0f;
     for (int z = 0; z < S; ++z) s += partial[z * n + i];
     const int b = static_cast<int>(i / Q), q = static_cast<int>(i % Q);
+    float* dst = scores + b * ld + q;
     if (sx != nullptr) {
       float ny = 0.0f;
       for (int z = 0; z < S; ++z) ny += ynorm[static_cast<int64_t>(z) * Q + q];
-      s *= sx[b] * (ny > 0.0f ? 1.0f / sqrtf(ny) : 0.0f);
+      *dst = s * sx[b] * (ny > 0.0f ? 1.0f / sqrtf(ny) : 0.0f);
+    } else {
+      float v = al * s;
+      if (beta != 0.0f) v = fmaf(beta, *dst, v);
+      if (b == q) v += gamma;
+      *dst = v;
     }
-    scores[b * ld + q] = s;
   }
 }
 
@@ -474,10 +481,17 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   return pl;
 }
 
-cudaError_t launch_xgemm(const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
-                         const CUtensorMap& tm_xl, const XGemmPlan& pl, const XGemmArgs& a,
-                         int sms, cudaStream_t s) {
+cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   if (a.B == 0 || a.Q == 0) return cudaSuccess;
+  const XGemmPlan pl = xgemm_plan(a.B, a.Q, a.K);
+  CUtensorMap tm_y, tm_xh, tm_xl;
+  if (encode_tmap_2d(&tm_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.y, a.K, a.Q, a.ldy * 4, kXK, kXM) !=
+          CUDA_SUCCESS ||
+      encode_tmap_2d(&tm_xh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.ws + pl.xh_off, a.K, a.B,
+                     static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad) != CUDA_SUCCESS ||
+      encode_tmap_2d(&tm_xl, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.ws + pl.xl_off, a.K, a.B,
+                     static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
   float* sx = reinterpret_cast<float*>(a.ws + pl.sx_off);
   float* xh = reinterpret_cast<float*>(a.ws + pl.xh_off);
   float* xl = reinterpret_cast<float*>(a.ws + pl.xl_off);
@@ -494,9 +508,9 @@ cudaError_t launch_xgemm(const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
   p.steps = pl.steps;
   p.stages = pl.stages;
   p.n_items = pl.n_mtiles * pl.n_ntiles * pl.S;
-  p.n_buf = 8 * pl.n_pad <= 512 ? 2 : 1;
+  p.n_buf = 6 * pl.n_pad <= 512 ? 2 : 1;
   int cols = 32;
-  while (cols < p.n_buf * 4 * pl.n_pad) cols <<= 1;
+  while (cols < p.n_buf * 3 * pl.n_pad) cols <<= 1;
   p.tmem_cols = cols;
   p.unit = a.unit;
   p.partial = reinterpret_cast<float*>(a.ws + pl.partial_off);
@@ -520,7 +534,8 @@ cudaError_t launch_xgemm(const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
   const int64_t n = static_cast<int64_t>(a.B) * a.Q;
   const int64_t blocks = (n + 255) / 256;
   finish_kernel<<<static_cast<unsigned>(blocks < 4096 ? blocks : 4096), 256, 0, s>>>(
-      p.partial, pl.S, a.B, a.Q, a.unit ? sx : nullptr, p.ynorm, a.scores, a.ld_scores);
+      p.partial, pl.S, a.B, a.Q, a.unit ? sx : nullptr, p.ynorm, a.alpha, a.alpha_s, a.beta,
+      a.gamma, a.scores, a.ld_scores);
   return cudaGetLastError();
 }
 
