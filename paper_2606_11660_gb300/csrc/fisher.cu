@@ -135,19 +135,26 @@ __global__ void ns_init_kernel(const float* __restrict__ r, int64_t ld, int K,
   }
 }
 
-// x <- (x + x^T) / 2 in place (one thread per pair i < j).  The iterates are
-// symmetric in exact arithmetic, but the products use B^T = B, which turns the
-// rounding's antisymmetric part into a growing error unless it is removed.
-__global__ void symmetrize_kernel(float* __restrict__ x, int K) {
-  const int64_t n = static_cast<int64_t>(K) * K;
-  for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n;
-       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int i = static_cast<int>(e / K), j = static_cast<int>(e % K);
-    if (i < j) {
-      const float v = 0.5f * (x[e] + x[static_cast<int64_t>(j) * K + i]);
-      x[e] = v;
-      x[static_cast<int64_t>(j) * K + i] = v;
-    }
+// x <- (x + x^T) / 2 in place.  The iterates are symmetric in exact
+// arithmetic, but the products use B^T = B, which turns the rounding's
+// antisymmetric part into a growing error unless it is removed.  One CTA per
+// pair of 32 x 32 tiles (ti <= tj): both tiles are read row by row into shared
+// memory and written back row by row, so every global access is coalesced.
+__global__ void __launch_bounds__(256) symmetrize_kernel(float* __restrict__ x, int K) {
+  __shared__ float a[32][33], b[32][33];
+  const int ti = blockIdx.y, tj = blockIdx.x;
+  if (ti > tj) return;
+  const int i0 = ti * 32, j0 = tj * 32, c = threadIdx.x;
+  for (int r = threadIdx.y; r < 32; r += 8) {
+    a[r][c] = (i0 + r < K && j0 + c < K) ? x[static_cast<int64_t>(i0 + r) * K + j0 + c] : 0.0f;
+    b[r][c] = (j0 + r < K && i0 + c < K) ? x[static_cast<int64_t>(j0 + r) * K + i0 + c] : 0.0f;
+  }
+  __syncthreads();
+  for (int r = threadIdx.y; r < 32; r += 8) {
+    if (i0 + r < K && j0 + c < K)
+      x[static_cast<int64_t>(i0 + r) * K + j0 + c] = 0.5f * (a[r][c] + b[c][r]);
+    if (ti != tj && j0 + r < K && i0 + c < K)
+      x[static_cast<int64_t>(j0 + r) * K + i0 + c] = 0.5f * (b[r][c] + a[c][r]);
   }
 }
 
@@ -257,8 +264,9 @@ cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t
     swap = z;
     z = a;
     a = swap;
-    symmetrize_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(y, K);
-    symmetrize_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(z, K);
+    const dim3 tiles((K + 31) / 32, (K + 31) / 32);
+    symmetrize_kernel<<<tiles, dim3(32, 8), 0, s>>>(y, K);
+    symmetrize_kernel<<<tiles, dim3(32, 8), 0, s>>>(z, K);
   }
   // Z ~ (R/c)^-1/2:  R^-1/2 = Z / sqrt(c);  R^-1 = Z Z / c
   if (inverse)

@@ -411,11 +411,12 @@ __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, i
                               float gamma, float* scores, int64_t ld) {
   const int64_t n = static_cast<int64_t>(B) * Q;
   const float al = alpha_s != nullptr ? alpha * *alpha_s : alpha;
-  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  const int q = blockIdx.x * blockDim.x + threadIdx.x;     // grid: (Q / 256, rows of b)
+  if (q >= Q) return;
+  for (int b = blockIdx.y; b < B; b += gridDim.y) {
+    const int64_t i = static_cast<int64_t>(b) * Q + q;
     float s = 0.0f;
     for (int z = 0; z < S; ++z) s += partial[z * n + i];
-    const int b = static_cast<int>(i / Q), q = static_cast<int>(i % Q);
     float* dst = scores + b * ld + q;
     if (sx != nullptr) {
       float ny = 0.0f;
@@ -531,9 +532,8 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
-  const int64_t n = static_cast<int64_t>(a.B) * a.Q;
-  const int64_t blocks = (n + 255) / 256;
-  finish_kernel<<<static_cast<unsigned>(blocks < 4096 ? blocks : 4096), 256, 0, s>>>(
+  const dim3 fgrid((a.Q + 255) / 256, std::min(a.B, 65535));
+  finish_kernel<<<fgrid, 256, 0, s>>>(
       p.partial, pl.S, a.B, a.Q, a.unit ? sx : nullptr, p.ynorm, a.alpha, a.alpha_s, a.beta,
       a.gamma, a.scores, a.ld_scores);
   return cudaGetLastError();
