@@ -45,7 +45,7 @@ constexpr int pow2ceil(int x) {
   return p;
 }
 
-template <int KI, int KO>
+template <int KI, int KO, bool TOKEN = false>
 struct ProjCfg {
   // Tiles sharing one P' slice: each slice is re-read from L2 once per NT
   // tiles, so a larger NT cuts L2 -> SM traffic (NT = 1 -> 2 -> 4 measured
@@ -54,7 +54,11 @@ struct ProjCfg {
   static constexpr int kPRows = 2 * (KI > KO ? KI : KO);         // hi + lo rows
   static constexpr int kPBytes = kPRows * 128;
   static constexpr int kStageBytes = NT * kActBoxBytes + kPBytes;
-  static constexpr int kEpiBytes = kTileTokens * (KI + 4) * 4 + kTileTokens * (KO + 4) * 4;
+  // Epilogue staging: the contraction stages a~ and g~ 64 tokens at a time
+  // (half a tile; the room goes to pipeline stages: 4 -> 5 of them at k = 32);
+  // token mode keeps the whole tile's worth, where it holds the query blocks.
+  static constexpr int kEpiRows = TOKEN ? kTileTokens : kTileTokens / 2;
+  static constexpr int kEpiBytes = kEpiRows * (KI + 4) * 4 + kEpiRows * (KO + 4) * 4;
   static constexpr int kBarBytes = 512;
   static constexpr int kStagesFit = (kSmemBudget - 1024 - kEpiBytes - kBarBytes) / kStageBytes;
   static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
@@ -168,15 +172,15 @@ __device__ __forceinline__ uint32_t tiles_of(uint32_t slices) {
 
 template <int KI, int KO, bool TOKEN>
 __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
-  using C = ProjCfg<KI, KO>;
+  using C = ProjCfg<KI, KO, TOKEN>;
   constexpr int NT = C::NT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
   float* sA = reinterpret_cast<float*>(smem + C::kStages * C::kStageBytes);
-  float* sG = sA + kTileTokens * (KI + 4);
-  uint64_t* full = reinterpret_cast<uint64_t*>(sG + kTileTokens * (KO + 4));
+  float* sG = sA + C::kEpiRows * (KI + 4);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sG + C::kEpiRows * (KO + 4));
   uint64_t* empty = full + C::kStages;
   uint64_t* tfull = empty + C::kStages;
   uint64_t* tempty = tfull + 2;
@@ -501,51 +505,59 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             }
           }
         } else {
+        constexpr int kHalf = kTileTokens / 2;
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
           if (!(vm >> nt & 1)) continue;
           const int t = (g + nt) * kTileTokens + row;
           const bool valid = t < p.T &&
               (p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0);
-          named_bar_sync(1, 128);                    // previous tile's readers are done
-          float4* ra = reinterpret_cast<float4*>(sA + row * (KI + 4));
-          float4* rg = reinterpret_cast<float4*>(sG + row * (KO + 4));
-          const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+          // Two halves of 64 tokens: the half's owners (whole warps) stage their
+          // a~, g~ rows, then all 128 threads accumulate over the half's tokens.
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            named_bar_sync(1, 128);                  // previous half's readers are done
+            if ((row >> 6) == h) {
+              float4* ra = reinterpret_cast<float4*>(sA + (row - h * kHalf) * (KI + 4));
+              float4* rg = reinterpret_cast<float4*>(sG + (row - h * kHalf) * (KO + 4));
+              const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-          for (int x = 0; x < KI / 4; ++x)
-            ra[x] = valid ? make_float4(va[nt][4 * x], va[nt][4 * x + 1], va[nt][4 * x + 2],
-                                        va[nt][4 * x + 3])
-                          : z4;
+              for (int x = 0; x < KI / 4; ++x)
+                ra[x] = valid ? make_float4(va[nt][4 * x], va[nt][4 * x + 1], va[nt][4 * x + 2],
+                                            va[nt][4 * x + 3])
+                              : z4;
 #pragma unroll
-          for (int x = 0; x < KO / 4; ++x)
-            rg[x] = valid ? make_float4(vg[nt][4 * x], vg[nt][4 * x + 1], vg[nt][4 * x + 2],
-                                        vg[nt][4 * x + 3])
-                          : z4;
-          named_bar_sync(1, 128);
-          if (p.bias_partials != nullptr) {      // projected bias gradient: sum_t g~_t
-            const int col = et % KO, r0 = (et / KO) * KO;
+              for (int x = 0; x < KO / 4; ++x)
+                rg[x] = valid ? make_float4(vg[nt][4 * x], vg[nt][4 * x + 1], vg[nt][4 * x + 2],
+                                            vg[nt][4 * x + 3])
+                              : z4;
+            }
+            named_bar_sync(1, 128);
+            if (p.bias_partials != nullptr) {    // projected bias gradient: sum_t g~_t
+              const int col = et % KO, r0 = (et / KO) * (KO / 2);
 #pragma unroll 4
-            for (int i = 0; i < KO; ++i) bias_acc += sG[(r0 + i) * (KO + 4) + col];
-          }
+              for (int i = 0; i < KO / 2; ++i) bias_acc += sG[(r0 + i) * (KO + 4) + col];
+            }
 #pragma unroll 4
-          for (int t2 = 0; t2 < kTileTokens; ++t2) {
-            const float gv = sG[t2 * (KO + 4) + oi];
-            const float* ar = sA + t2 * (KI + 4) + oj;
-            if constexpr (OPT % 4 == 0) {
+            for (int t2 = 0; t2 < kHalf; ++t2) {
+              const float gv = sG[t2 * (KO + 4) + oi];
+              const float* ar = sA + t2 * (KI + 4) + oj;
+              if constexpr (OPT % 4 == 0) {
 #pragma unroll
-              for (int x = 0; x < OPT / 4; ++x) {
-                const float4 a4 = reinterpret_cast<const float4*>(ar)[x];
-                acc[4 * x] = fmaf(gv, a4.x, acc[4 * x]);
-                acc[4 * x + 1] = fmaf(gv, a4.y, acc[4 * x + 1]);
-                acc[4 * x + 2] = fmaf(gv, a4.z, acc[4 * x + 2]);
-                acc[4 * x + 3] = fmaf(gv, a4.w, acc[4 * x + 3]);
-              }
-            } else {
+                for (int x = 0; x < OPT / 4; ++x) {
+                  const float4 a4 = reinterpret_cast<const float4*>(ar)[x];
+                  acc[4 * x] = fmaf(gv, a4.x, acc[4 * x]);
+                  acc[4 * x + 1] = fmaf(gv, a4.y, acc[4 * x + 1]);
+                  acc[4 * x + 2] = fmaf(gv, a4.z, acc[4 * x + 2]);
+                  acc[4 * x + 3] = fmaf(gv, a4.w, acc[4 * x + 3]);
+                }
+              } else {
 #pragma unroll
-              for (int x = 0; x < OPT / 2; ++x) {
-                const float2 a2 = reinterpret_cast<const float2*>(ar)[x];
-                acc[2 * x] = fmaf(gv, a2.x, acc[2 * x]);
-                acc[2 * x + 1] = fmaf(gv, a2.y, acc[2 * x + 1]);
+                for (int x = 0; x < OPT / 2; ++x) {
+                  const float2 a2 = reinterpret_cast<const float2*>(ar)[x];
+                  acc[2 * x] = fmaf(gv, a2.x, acc[2 * x]);
+                  acc[2 * x + 1] = fmaf(gv, a2.y, acc[2 * x + 1]);
+                }
               }
             }
           }
@@ -618,7 +630,7 @@ __global__ void token_reduce_kernel(const float* __restrict__ tp, int n_mods, in
 
 template <int KI, int KO, bool TOKEN>
 cudaError_t launch_project_t(const ProjParams& p, int grid, cudaStream_t s) {
-  using C = ProjCfg<KI, KO>;
+  using C = ProjCfg<KI, KO, TOKEN>;
   static bool attr_set = false;   // per process; the attribute is per function and device
   cudaError_t e = cudaSuccess;
   if (!attr_set) {
@@ -639,7 +651,7 @@ cudaError_t launch_project_mode(bool token, const ProjParams& p, int grid, cudaS
 
 template <int KI, int KO>
 constexpr int token_capacity_of() {
-  const int cap = ProjCfg<KI, KO>::kEpiBytes / (4 * KI * KO);
+  const int cap = ProjCfg<KI, KO, true>::kEpiBytes / (4 * KI * KO);
   return cap > 16 ? 16 : cap;
 }
 
