@@ -1,6 +1,9 @@
 """Shared helpers for the parity tests (test code only)."""
 from __future__ import annotations
 
+import importlib.util
+import os
+
 import numpy as np
 import torch
 
@@ -67,3 +70,20 @@ def check_topk(got_s, got_i, S, k, score_atol=1e-3, tie=1e-4):
         must = set(order[:k][row[order[:k]] > kth + tie].tolist())
         assert must <= set(gi.tolist()), f"query {q}: missing clear top-k members"
         assert np.all(row[gi] >= kth - tie), f"query {q}: returned a row clearly below the k-th"
+
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def golden_lines(name: str):
+    """Non-comment lines of a fixture in tests/golden."""
+    with open(os.path.join(GOLDEN, name)) as f:
+        return [line.strip() for line in f if line.strip() and not line.startswith("#")]
+
+
+def load_make_golden():
+    """tests/golden/make_golden.py as a module (it calls only the oracle)."""
+    spec = importlib.util.spec_from_file_location("make_golden", os.path.join(GOLDEN, "make_golden.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod

@@ -49,6 +49,28 @@ def test_tiny_workload_parity():
     assert err.max() <= TIGHT, f"max rel err {err.max():.2e}"
 
 
+def test_tiny_workload_matches_golden_fixtures():
+    """CUDA path against the stored oracle fixtures of tests/golden (projected
+    rows, then the store and an exact top-4 for 8 queries)."""
+    from tests._util import golden_lines
+    cfg = wl.TINY
+    gl, _, ld = make_layers(cfg.modules, cfg.B, cfg.T, [(16, 16)], rc=True)
+    out = run_project(gl, cfg.B, cfg.T, None, ld)
+    want = np.array([[float(v) for v in line.split()] for line in golden_lines("tiny_projected.txt")])
+    assert rel_frobenius(np32(out).astype(np.float64), want).max() <= TIGHT
+    store = torch.empty((cfg.B, ld), dtype=torch.float16, device=DEV)
+    bg.bergson_build_store(out, cfg.B, ld, True, store, 0)
+    queries = wl.gaussian_rows(cfg.B, ld, seed=3).to(DEV)
+    ws = bg.workspace_tensor(bg.bergson_score_topk_workspace(cfg.B, ld, cfg.B, 4), DEV)
+    s = torch.empty((cfg.B, 4), dtype=torch.float32, device=DEV)
+    i = torch.empty((cfg.B, 4), dtype=torch.int64, device=DEV)
+    bg.bergson_score_topk(store, cfg.B, ld, queries, 4, s, i, ws)
+    assert bg.bergson_sync_status() == bg.BERGSON_OK, bg.bergson_last_error()
+    rows = [[tok.split(":") for tok in line.split()] for line in golden_lines("tiny_topk.txt")]
+    np.testing.assert_array_equal(i.cpu().numpy(), [[int(a) for a, _ in r] for r in rows])
+    np.testing.assert_allclose(np32(s), [[float(b) for _, b in r] for r in rows], atol=1e-3, rtol=0)
+
+
 def test_identity_projection_gives_normalised_gradient():
     spec = wl.ModuleSpec("lin", 64, 64)
     gl, ol, ld = make_layers([spec], 3, 100, [(64, 64)], rc=True, kind=bg.BERGSON_PROJ_IDENTITY)
