@@ -31,6 +31,8 @@ constexpr int kMaxScoreCTAs = 160;                   // upper bound on persisten
 constexpr int kMaxDevices = 64;
 constexpr int64_t kPrefixRowsPerTopk = 512;          // prefix pass: 512 * topk store rows
 constexpr int64_t kPrefixMinFactor = 8;              // ... only when N >= 8 * prefix
+constexpr int64_t kPrefixMinQueries = 129;           // ... and Q > 128 (fewer queries insert
+                                                     // too little into their heaps to repay it)
 
 __device__ int g_status_word;                        // device status word (one per device)
 
@@ -853,7 +855,7 @@ int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store
   // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
   // lands in the outputs, and its k-th score seeds the full pass's threshold.
   const int64_t prefix = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
-  const bool use_prefix = N >= kPrefixMinFactor * prefix;
+  const bool use_prefix = N >= kPrefixMinFactor * prefix && Q >= kPrefixMinQueries;
   for (int pass = 0; pass < n_qg_total; pass += sms) {
     const int n_qg = std::min(sms, n_qg_total - pass);
     const int q_begin = pass * gsize;

@@ -40,6 +40,10 @@ constexpr int kStoreEvictFirst = 1;
 // into its heap after the tile's TMEM buffer is released.
 constexpr int kQueueCap = 8;
 
+// Candidate keys the merge keeps in shared memory for its radix select
+// (26,624 x 8 bytes = 208 KB); larger candidate sets are merged in sorted rounds.
+constexpr int kMergeSmemKeys = 26624;
+
 template <int QT>
 struct ScoreCfg {
   static constexpr int kStageBytes = kStoreBoxBytes + QT * kQBoxBytes;
@@ -340,19 +344,119 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
   }
 }
 
+// Bitonic sort of keys[0, n) (n a power of two) into descending order.
+__device__ __forceinline__ void bitonic_desc(unsigned long long* keys, int n) {
+  for (int kk = 2; kk <= n; kk <<= 1) {
+    for (int j = kk >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const int ixj = i ^ j;
+        if (ixj > i) {
+          const unsigned long long a = keys[i];
+          const unsigned long long b = keys[ixj];
+          const bool desc = (i & kk) == 0;
+          if (desc ? (a < b) : (a > b)) {
+            keys[i] = b;
+            keys[ixj] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+__device__ __forceinline__ void write_topk(const unsigned long long* keys, int q, int topk,
+                                           float* out_scores, int64_t* out_idx) {
+  for (int e = threadIdx.x; e < topk; e += blockDim.x) {
+    const unsigned long long k = keys[e];
+    const uint32_t lo = static_cast<uint32_t>(k);
+    const bool real = lo >= 0x80000000u;          // rows < 2^31 map to ~row >= 2^31
+    out_scores[static_cast<int64_t>(q) * topk + e] =
+        real ? order_to_float(static_cast<uint32_t>(k >> 32)) : -INFINITY;
+    out_idx[static_cast<int64_t>(q) * topk + e] = real ? static_cast<int64_t>(~lo) : -1;
+  }
+}
+
 // Final top-k of one query from the heaps of the CTAs that covered it.
+//
+// select_n > 0: all cpg * topk candidate keys fit in shared memory.  An exact
+// radix select (eight passes over 8-bit digits, most significant first) finds
+// the topk-th largest key T; keys are unique (the low word is the row), so
+// exactly topk keys are >= T.  They are compacted and bitonic-sorted
+// (select_n = a power of two >= topk).  Otherwise (select_n == 0) the keys
+// are sorted in rounds of sort_n, keeping the best topk of each round.
 __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __restrict__ heaps,
                                                     int n_qg, int cpg, int gsize, int topk,
                                                     int q_begin, int q_end, int sort_n,
+                                                    int select_n,
                                                     float* __restrict__ out_scores,
                                                     int64_t* __restrict__ out_idx) {
   extern __shared__ unsigned long long keys[];
+  __shared__ unsigned int hist[256];
+  __shared__ unsigned long long s_prefix;
+  __shared__ int s_need, s_count;
   const int q = q_begin + blockIdx.x;
   if (q >= q_end) return;
   const int local = q - q_begin;
   const int gl = local / gsize;
   const int slot = local % gsize;
   const int64_t total = static_cast<int64_t>(cpg) * topk;
+  if (select_n > 0) {
+    const int n = static_cast<int>(total);
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      const int cta = gl + (i / topk) * n_qg;
+      keys[i] = heaps[(static_cast<int64_t>(cta) * topk + i % topk) * gsize + slot];
+    }
+    if (threadIdx.x == 0) {
+      s_prefix = 0ull;
+      s_need = topk;
+      s_count = 0;
+    }
+    __syncthreads();
+    for (int shift = 56; shift >= 0; shift -= 8) {
+      for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0u;
+      __syncthreads();
+      const unsigned long long prefix = s_prefix;
+      const unsigned long long above = shift == 56 ? 0ull : (~0ull << (shift + 8));
+      // Candidates cluster in score, so most share a digit: lanes of a warp
+      // with the same digit add their count once (one atomic per group).
+      for (int i0 = 0; i0 < n; i0 += blockDim.x) {
+        const int i = i0 + threadIdx.x;
+        const unsigned long long k = i < n ? keys[i] : 0ull;
+        const bool hit = i < n && (k & above) == prefix;
+        const unsigned dig = hit ? static_cast<unsigned>((k >> shift) & 255u) : 256u;
+        const unsigned peers = __match_any_sync(0xffffffffu, dig);
+        if (hit && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[dig], __popc(peers));
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        const int need = s_need;
+        int acc = 0, d = 255;
+        for (; d > 0; --d) {
+          if (acc + static_cast<int>(hist[d]) >= need) break;
+          acc += static_cast<int>(hist[d]);
+        }
+        s_prefix = prefix | (static_cast<unsigned long long>(d) << shift);
+        s_need = need - acc;
+      }
+      __syncthreads();
+    }
+    const unsigned long long T = s_prefix;       // the topk-th largest key
+    unsigned long long* sel = keys + n;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      const unsigned long long k = keys[i];
+      if (k >= T) {
+        const int pos = atomicAdd(&s_count, 1);
+        if (pos < select_n) sel[pos] = k;
+      }
+    }
+    __syncthreads();
+    for (int i = min(s_count, select_n) + threadIdx.x; i < select_n; i += blockDim.x) sel[i] = 0ull;
+    __syncthreads();
+    bitonic_desc(sel, select_n);
+    write_topk(sel, q, topk, out_scores, out_idx);
+    return;
+  }
   int64_t consumed = 0;
   bool first = true;
   while (first || consumed < total) {
@@ -370,32 +474,9 @@ __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __
     consumed += sort_n - start;
     first = false;
     __syncthreads();
-    for (int kk = 2; kk <= sort_n; kk <<= 1) {
-      for (int j = kk >> 1; j > 0; j >>= 1) {
-        for (int i = threadIdx.x; i < sort_n; i += blockDim.x) {
-          const int ixj = i ^ j;
-          if (ixj > i) {
-            const unsigned long long a = keys[i];
-            const unsigned long long b = keys[ixj];
-            const bool desc = (i & kk) == 0;
-            if (desc ? (a < b) : (a > b)) {
-              keys[i] = b;
-              keys[ixj] = a;
-            }
-          }
-        }
-        __syncthreads();
-      }
-    }
+    bitonic_desc(keys, sort_n);
   }
-  for (int e = threadIdx.x; e < topk; e += blockDim.x) {
-    const unsigned long long k = keys[e];
-    const uint32_t lo = static_cast<uint32_t>(k);
-    const bool real = lo >= 0x80000000u;          // rows < 2^31 map to ~row >= 2^31
-    out_scores[static_cast<int64_t>(q) * topk + e] =
-        real ? order_to_float(static_cast<uint32_t>(k >> 32)) : -INFINITY;
-    out_idx[static_cast<int64_t>(q) * topk + e] = real ? static_cast<int64_t>(~lo) : -1;
-  }
+  write_topk(keys, q, topk, out_scores, out_idx);
 }
 
 template <int QT>
@@ -435,16 +516,21 @@ cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, in
   const int64_t total = static_cast<int64_t>(cpg) * topk;
   int sort_n = 2;
   while (sort_n < total && sort_n < 8192) sort_n <<= 1;
-  const size_t smem = static_cast<size_t>(sort_n) * sizeof(unsigned long long);
+  int select_n = 2;
+  while (select_n < topk) select_n <<= 1;
+  const bool radix = total + select_n <= kMergeSmemKeys;
+  if (!radix) select_n = 0;
+  const size_t smem =
+      static_cast<size_t>(radix ? total + select_n : sort_n) * sizeof(unsigned long long);
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         8192 * sizeof(unsigned long long));
+                                         kMergeSmemKeys * sizeof(unsigned long long));
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   merge_kernel<<<nq, 512, smem, s>>>(heaps, n_qg, cpg, qt * kScoreQT, topk, q_begin, q_end, sort_n,
-                                     out_scores, out_idx);
+                                     select_n, out_scores, out_idx);
   return cudaGetLastError();
 }
 
