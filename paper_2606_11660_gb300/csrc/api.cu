@@ -29,7 +29,7 @@ constexpr double kSplitShare = 0.4;
 constexpr int kPiecesPerShare = 2;
 constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
 constexpr int kMaxDevices = 64;
-constexpr int64_t kPrefixRowsPerTopk = 512;          // prefix pass: 512 * topk store rows
+constexpr int64_t kPrefixRowsPerTopk = 128;          // prefix pass: 128 * topk store rows
 constexpr int64_t kPrefixMinFactor = 8;              // ... only when N >= 8 * prefix
 constexpr int64_t kPrefixMinQueries = 129;           // ... and Q > 128 (fewer queries insert
                                                      // too little into their heaps to repay it)

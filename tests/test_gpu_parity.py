@@ -293,10 +293,11 @@ def test_score_topk_random(N, K, Q, topk):
     check_topk(s, i, S, topk)
 
 
-@pytest.mark.parametrize("Q,topk", [(130, 5), (40, 3)])
+@pytest.mark.parametrize("Q,topk", [(130, 5), (200, 3), (40, 3)])
 def test_score_prefix_threshold_pass(Q, topk):
-    # N >= 8 * 512 * topk: the scorer first takes the exact top-k of a prefix of
-    # the store and starts the full pass from its k-th score.
+    # N >= 8 * 128 * topk and Q > 128: the scorer first takes the exact top-k of
+    # a prefix of the store and starts the full pass from its k-th score (Q = 40
+    # takes the single-pass path on the same data).
     N, K = 30_000, 256
     g = wl.generator(Q * 7 + topk, "cpu")
     rows = torch.randn((N, K), generator=g)
