@@ -116,7 +116,6 @@ cudaError_t launch_wait_probe(int* status, uint64_t timeout_ns, cudaStream_t s);
 // per-token scores against p.queries (token_partials).
 cudaError_t launch_project(int k_in, int k_out, bool token, const ProjParams& p, int grid,
                           cudaStream_t s);
-size_t project_smem_bytes(int k_in, int k_out);
 int token_query_capacity(int k_in, int k_out);
 cudaError_t launch_token_reduce(const float* token_partials, int n_mods, int Q, int B, int T,
                                 const uint8_t* mask, float* out, cudaStream_t s);
@@ -130,7 +129,6 @@ cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q,
                                      cudaStream_t s);
 cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
                          const ScoreParams& p, int grid, cudaStream_t s);
-size_t score_smem_bytes(int qt);
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
                          int q_begin, int q_end, int qg_base, float* out_scores, int64_t* out_idx,
                          cudaStream_t s);

@@ -655,11 +655,6 @@ constexpr int token_capacity_of() {
   return cap > 16 ? 16 : cap;
 }
 
-template <int KI, int KO>
-constexpr size_t smem_of() {
-  return ProjCfg<KI, KO>::kSmemBytes;
-}
-
 }  // namespace
 
 #define BERGSON_PROJ_DISPATCH(KI_, KO_, EXPR)        \
@@ -702,19 +697,6 @@ cudaError_t launch_token_reduce(const float* token_partials, int n_mods, int Q, 
   token_reduce_kernel<<<static_cast<unsigned>(blocks < 8192 ? blocks : 8192), 256, 0, s>>>(
       token_partials, n_mods, Q, B, T, mask, out);
   return cudaGetLastError();
-}
-
-size_t project_smem_bytes(int k_in, int k_out) {
-  BERGSON_PROJ_DISPATCH(16, 16, (smem_of<16, 16>()))
-  BERGSON_PROJ_DISPATCH(16, 32, (smem_of<16, 32>()))
-  BERGSON_PROJ_DISPATCH(16, 64, (smem_of<16, 64>()))
-  BERGSON_PROJ_DISPATCH(32, 16, (smem_of<32, 16>()))
-  BERGSON_PROJ_DISPATCH(32, 32, (smem_of<32, 32>()))
-  BERGSON_PROJ_DISPATCH(32, 64, (smem_of<32, 64>()))
-  BERGSON_PROJ_DISPATCH(64, 16, (smem_of<64, 16>()))
-  BERGSON_PROJ_DISPATCH(64, 32, (smem_of<64, 32>()))
-  BERGSON_PROJ_DISPATCH(64, 64, (smem_of<64, 64>()))
-  return 0;
 }
 
 cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, int B,

@@ -503,10 +503,6 @@ cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap&
   return cudaErrorInvalidValue;
 }
 
-size_t score_smem_bytes(int qt) {
-  return qt == 1 ? ScoreCfg<1>::kSmemBytes : ScoreCfg<2>::kSmemBytes;
-}
-
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
                          int q_begin, int q_end, int /*qg_base*/, float* out_scores,
                          int64_t* out_idx, cudaStream_t s) {
