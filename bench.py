@@ -300,7 +300,7 @@ def bench_collection(args, world, dev, peaks, peak_kind):
     return res, (cfg, layers, mask, ws, out, store)
 
 
-def bench_onthefly(args, world, dev, state):
+def bench_onthefly(args, world, dev, state, peaks):
     """On-the-fly scoring step: project the batch, score it against 1024 fixed queries."""
     import torch
 
@@ -341,10 +341,16 @@ def bench_onthefly(args, world, dev, state):
     ms = max_over_ranks(t0.elapsed_time(t1), world)
     score_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
     flops = 2.0 * cfg.B * K * Q
+    alg = 4 * K * (Q + cfg.B)                     # fp32 queries and rows, each read once
+    gbs = alg / (score_ms * 1e-3) / 1e9
     return {"value": round(cfg.B * world * args.steps / (ms * 1e-3), 2), "unit": "examples/s",
             "ms_per_step": round(ms / args.steps, 4), "queries": Q,
             "score_call_ms": round(score_ms, 4),
             "score_gflops": round(flops / (score_ms * 1e-3) / 1e9, 1),
+            "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4),
+                         "kernel": "bergson_score_grads call (split, tcgen05 3xTF32 product, "
+                                   "finish)", "algorithmic_bytes_per_call": alg},
             "gpu_launches": (5 + 3) * args.steps,
             "what": "bergson_project_grads + bergson_score_grads (cosine vs 1024 fp32 queries, "
                     "no store) per batch"}
@@ -390,7 +396,7 @@ def bench_tokens(args, world, dev, state, peaks):
                     "against 4 query rows"}
 
 
-def bench_fisher(args, world, dev, state):
+def bench_fisher(args, world, dev, state, peaks):
     """TrackStar-style preconditioning: fit R on 1024 rows, R^-1/2 once, apply per batch."""
     import torch
 
@@ -435,13 +441,26 @@ def bench_fisher(args, world, dev, state):
     step_ms = ev[3].elapsed_time(ev[4]) / args.steps
     apply_ms = ev[4].elapsed_time(ev[5]) / args.steps
     gemm_flops = 2.0 * K ** 3 * (3 * args.fisher_iters)
+    apply_gbs = 4.0 * K * (K + 2 * cfg.B) / (apply_ms * 1e-3) / 1e9   # M once, rows in and out
+    # fp32-accurate products run three tf32 MMAs each; the tf32 rate is the
+    # measured bf16 peak times the nominal tf32 : bf16 ratio (1.1 : 2.25).
+    tf32_eff = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]) * (1.1 / 2.25) / 3.0
+    ns_tflops = gemm_flops / (pow_ms * 1e-3) / 1e12
     return {"value": round(cfg.B * world / (step_ms * 1e-3), 2), "unit": "examples/s",
             "ms_per_step": round(step_ms, 4), "apply_ms": round(apply_ms, 4),
             "apply_tflops": round(2.0 * cfg.B * K * K / (apply_ms * 1e-3) / 1e12, 2),
             "fit_ms": round(fit_ms, 3), "fit_rows": n_fit,
             "fit_tflops": round(2.0 * K * K * n_fit / (fit_ms * 1e-3) / 1e12, 2),
             "preconditioner_ms": round(pow_ms, 1), "newton_schulz_iterations": args.fisher_iters,
-            "preconditioner_tflops": round(gemm_flops / (pow_ms * 1e-3) / 1e12, 2),
+            "preconditioner_tflops": round(ns_tflops, 2),
+            "roofline_apply": {"bound": "hbm", "achieved": round(apply_gbs, 1),
+                               "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                               "frac": round(apply_gbs / peaks["hbm_gbs"], 4)},
+            "roofline_newton_schulz": {"bound": "tensor", "achieved": round(ns_tflops, 1),
+                                       "peak": round(tf32_eff, 1), "unit": "TFLOP/s",
+                                       "frac": round(ns_tflops / tf32_eff, 4),
+                                       "peak_source": "measured sustained bf16 x 1.1/2.25 "
+                                                      "(nominal tf32:bf16) / 3 tf32 products"},
             "what": "step = project_grads + precondition_rows (R^-1/2, K=12288) + build_store; "
                     "fit and R^-1/2 are one-time costs (3xTF32 tcgen05 GEMMs)"}
 
@@ -751,9 +770,9 @@ def main_ours(args):
     torch.cuda.set_device(dev)
     peaks, peak_kind = load_peaks()
     coll, state = bench_collection(args, world, dev, peaks, peak_kind)
-    onthefly = bench_onthefly(args, world, dev, state)
+    onthefly = bench_onthefly(args, world, dev, state, peaks)
     tokens = bench_tokens(args, world, dev, state, peaks)
-    fisher = bench_fisher(args, world, dev, state) if not args.no_fisher else None
+    fisher = bench_fisher(args, world, dev, state, peaks) if not args.no_fisher else None
     e2e = bench_e2e(args, world, dev, state) if not args.no_e2e else None
     del state
     torch.cuda.empty_cache()
