@@ -56,6 +56,24 @@ def test_multi_module_mask_ragged_mixed_k():
                                rtol=1e-4, atol=1e-4 * np.abs(got.sum(axis=2)).max())
 
 
+def test_shared_input_layers_token_scores():
+    """Token mode with layers that read one A tensor: their items run from a
+    work table (side by side); per-token scores still match the oracle."""
+    specs = [wl.ModuleSpec("gate", 256, 512), wl.ModuleSpec("up", 256, 512, True),
+             wl.ModuleSpec("down", 512, 256)]
+    B, T = 3, 300
+    gl, ol, ld = make_layers(specs, B, T, [(16, 16)] * 3, base_seed=6, data_seed=5, rc=True,
+                             input_scale=True)
+    assert gl[1].A.data_ptr() == gl[0].A.data_ptr()
+    assert bg.bergson_debug_project_plan(gl, B, T)[3] == 2
+    g = wl.generator(8, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.2).to(torch.uint8)
+    queries = torch.randn((4, ld), generator=g)
+    got = _tokens(gl, B, T, mask.to(DEV), queries.to(DEV))
+    want = orc.token_scores(ol, mask.numpy(), queries.numpy())
+    _close(got, want)
+
+
 def test_query_capacity_is_enforced():
     spec = wl.ModuleSpec("lin", 64, 64)
     gl, _, ld = make_layers([spec], 1, 8, [(64, 64)])
