@@ -9,9 +9,10 @@
 //      swizzle; slices whose 32 tokens are all masked are not read) and the
 //      matching 64-column slices of P'^T (hi and lo bf16 rows) into a ring of
 //      shared-memory stages;
-//   2. one thread issues tcgen05.mma (M = 128 tokens, N = k, K = 16) into TMEM:
-//      a~ = A P_in' (k_in columns) and g~ = G P_out' (k_out columns), each as
-//      A*hi + A*lo accumulated in fp32;
+//   2. one thread issues tcgen05.mma (M = 128 tokens, N = 2k, K = 16) into TMEM:
+//      a~ = A P_in' and g~ = G P_out', each as A*[hi|lo] in one MMA whose B
+//      operand is the slice's hi rows followed by its lo rows (fp32
+//      accumulators, the two halves added by the epilogue);
 //   3. four epilogue warps read a~ and g~ out of TMEM (one token per thread),
 //      zero masked tokens, stage them in shared memory and accumulate the
 //      k_out x k_in outer-product sum in fp32 registers.
@@ -63,7 +64,8 @@ struct ProjCfg {
   static constexpr int kStagesFit = (kSmemBudget - 1024 - kEpiBytes - kBarBytes) / kStageBytes;
   static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kEpiBytes + kBarBytes;
-  static constexpr int kTmemPerBuf = NT * (KI + KO);
+  // Per tile: A*[hi|lo] in 2 KI columns, then G*[hi|lo] in 2 KO columns.
+  static constexpr int kTmemPerBuf = NT * 2 * (KI + KO);
   static constexpr int kTmemCols = pow2ceil(2 * kTmemPerBuf);
   static constexpr int kOPT = KO * KI / kTileTokens;            // outputs per epilogue thread
   static_assert(kStages >= 2, "shared memory budget too small");
@@ -130,12 +132,27 @@ __device__ __forceinline__ uint32_t group_slices(const ProjParams& p, int b, int
   return vm;
 }
 
-// Copies this thread's TMEM lane (one token) of N columns to dst (fp32, 16-byte aligned).
+// v[j] = column j + column N + j of this thread's TMEM lane (one token): a
+// projection accumulated as its P'hi part (columns [0, N)) and P'lo part.
+template <int N>
+__device__ __forceinline__ void tmem_ld_hilo(uint32_t taddr, float* v) {
+#pragma unroll
+  for (int c = 0; c < N / 16; ++c) tmem_ld16(taddr + c * 16, &v[c * 16]);
+#pragma unroll
+  for (int c = 0; c < N / 8; ++c) {
+    float lo[8];
+    tmem_ld8(taddr + N + c * 8, lo);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[c * 8 + j] += lo[j];
+  }
+}
+
+// Copies this thread's token projection (N values, hi + lo parts) to dst
+// (fp32, 16-byte aligned).
 template <int N>
 __device__ __forceinline__ void store_token_row(uint32_t taddr, float* dst) {
   float v[N];
-#pragma unroll
-  for (int c = 0; c < N / 16; ++c) tmem_ld16(taddr + c * 16, &v[c * 16]);
+  tmem_ld_hilo<N>(taddr, v);
 #pragma unroll
   for (int x = 0; x < N / 4; ++x)
     reinterpret_cast<float4*>(dst)[x] = make_float4(v[4 * x], v[4 * x + 1], v[4 * x + 2], v[4 * x + 3]);
@@ -312,7 +329,10 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           for (int side = 0; side < 2 && ok; ++side) {
             if (ic.side != 0 && side != ic.side - 1) continue;
             const int N = side ? KO : KI;
-            const uint32_t idesc = make_idesc_f16(kTileTokens, N, true);
+            // B = the P' slice's hi rows then lo rows (2N rows, contiguous): one
+            // MMA gives A*hi in N columns and A*lo in the next N, reading the
+            // activation tile once.
+            const uint32_t idesc = make_idesc_f16(kTileTokens, 2 * N, true);
             const int d = side ? md->d_out : md->d_in;
             const int c0 = ic.side != 0 ? ic.ch_begin : 0;
             const int c1 = ic.side != 0 ? ic.ch_end : (d + kChunk - 1) / kChunk;
@@ -324,13 +344,11 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
 #pragma unroll
               for (int nt = 0; nt < NT; ++nt) {
                 if (!(vm >> nt & 1)) continue;
-                const uint32_t dcol = dbuf + nt * (KI + KO) + (side ? KI : 0);
+                const uint32_t dcol = dbuf + nt * 2 * (KI + KO) + (side ? 2 * KI : 0);
 #pragma unroll
-                for (int kk = 0; kk < kChunk / 16; ++kk) {
-                  const uint64_t ad = sw128_desc(act + nt * kActBoxBytes + kk * 32);
-                  umma_f16(dcol, ad, sw128_desc(pp + kk * 32), idesc, ch != c0 || kk != 0);
-                  umma_f16(dcol, ad, sw128_desc(pp + N * 128 + kk * 32), idesc, 1u);
-                }
+                for (int kk = 0; kk < kChunk / 16; ++kk)
+                  umma_f16(dcol, sw128_desc(act + nt * kActBoxBytes + kk * 32),
+                           sw128_desc(pp + kk * 32), idesc, ch != c0 || kk != 0);
               }
               umma_commit(smem_u32(&empty[stage]));
               if (++stage == C::kStages) { stage = 0; ph ^= 1; }
@@ -400,12 +418,12 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             for (int nt = 0; nt < NT; ++nt) {
               if (!(vm >> nt & 1)) continue;
               const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
-                                     ab * C::kTmemPerBuf + nt * (KI + KO);
+                                     ab * C::kTmemPerBuf + nt * 2 * (KI + KO);
               const int64_t tok = static_cast<int64_t>(g - ic.t_begin + nt) * kTileTokens + row;
               if (ic.side == 1)
                 store_token_row<KI>(taddr, dst + tok * KI);
               else
-                store_token_row<KO>(taddr + KI, dst + tok * KO);
+                store_token_row<KO>(taddr + 2 * KI, dst + tok * KO);
             }
             tc_fence_before();
             __syncwarp();
@@ -439,18 +457,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       for (int g = ic.t_begin; g < ic.t_end; g += NT) {
         const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
         if (vm == 0) continue;
-        float va[NT][KI];
-        float vg[NT][KO];
-        if (finisher) {
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (!(vm >> nt & 1)) continue;
-            const int64_t tok = static_cast<int64_t>(g - ic.t_begin + nt) * kTileTokens + row;
-            sum_token_rows<KI>(p.piece_buf + ic.base + tok * KI, stride_a, ic.n_a, va[nt]);
-            sum_token_rows<KO>(p.piece_buf + ic.base + ic.n_a * stride_a + tok * KO, stride_g,
-                               ic.n_g, vg[nt]);
-          }
-        } else {
+        if (!finisher) {
           if (et == 0) {
             if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
               raise_device_error(p.status, s_abort, kStatusTimeout);
@@ -459,110 +466,112 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           named_bar_sync(1, 128);
           if (*s_epi_stop) { aborted = true; break; }
           tc_fence_after();
+        }
+        // One tile at a time: its a~ and g~ (hi + lo halves summed) are loaded,
+        // used and dropped before the next tile's; the TMEM buffer is released
+        // after the group (the MMA warp fills the other buffer meanwhile).
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (!(vm >> nt & 1)) continue;
+        for (int nt = 0; nt < NT; ++nt) {
+          if (!(vm >> nt & 1)) continue;
+          float va[KI];
+          float vg[KO];
+          if (finisher) {
+            const int64_t tok = static_cast<int64_t>(g - ic.t_begin + nt) * kTileTokens + row;
+            sum_token_rows<KI>(p.piece_buf + ic.base + tok * KI, stride_a, ic.n_a, va);
+            sum_token_rows<KO>(p.piece_buf + ic.base + ic.n_a * stride_a + tok * KO, stride_g,
+                               ic.n_g, vg);
+          } else {
             const uint32_t taddr = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
-                                   ab * C::kTmemPerBuf + nt * (KI + KO);
-#pragma unroll
-            for (int c = 0; c < KI / 16; ++c) tmem_ld16(taddr + c * 16, &va[nt][c * 16]);
-#pragma unroll
-            for (int c = 0; c < KO / 16; ++c) tmem_ld16(taddr + KI + c * 16, &vg[nt][c * 16]);
+                                   ab * C::kTmemPerBuf + nt * 2 * (KI + KO);
+            tmem_ld_hilo<KI>(taddr, va);
+            tmem_ld_hilo<KO>(taddr + 2 * KI, vg);
           }
+          const int t = (g + nt) * kTileTokens + row;
+          if constexpr (TOKEN) {
+            // s[q] = g~^T Q~_q a~ for this thread's token: its share of the
+            // query's score (masked tokens score 0).
+            if (t < p.T) {
+              const bool valid =
+                  p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0;
+              for (int q = 0; q < p.n_queries; ++q) {
+                const float* qm = sA + q * (KO * KI);
+                float sq = 0.0f;
+#pragma unroll
+                for (int i = 0; i < KO; ++i) {
+                  float u = 0.0f;
+#pragma unroll
+                  for (int j = 0; j < KI; j += 4) {
+                    const float4 w = *reinterpret_cast<const float4*>(qm + i * KI + j);
+                    u = fmaf(w.x, va[j], u);
+                    u = fmaf(w.y, va[j + 1], u);
+                    u = fmaf(w.z, va[j + 2], u);
+                    u = fmaf(w.w, va[j + 3], u);
+                  }
+                  sq = fmaf(vg[i], u, sq);
+                }
+                p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q) * p.B + ic.b) *
+                                     p.T + t] = valid ? sq : 0.0f;
+              }
+            }
+          } else {
+            constexpr int kHalf = kTileTokens / 2;
+            const bool valid = t < p.T &&
+                (p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0);
+            // Two halves of 64 tokens: the half's owners (whole warps) stage their
+            // a~, g~ rows, then all 128 threads accumulate over the half's tokens.
+#pragma unroll 1
+            for (int h = 0; h < 2; ++h) {
+              named_bar_sync(1, 128);                // previous half's readers are done
+              if ((row >> 6) == h) {
+                float4* ra = reinterpret_cast<float4*>(sA + (row - h * kHalf) * (KI + 4));
+                float4* rg = reinterpret_cast<float4*>(sG + (row - h * kHalf) * (KO + 4));
+                const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int x = 0; x < KI / 4; ++x)
+                  ra[x] = valid ? make_float4(va[4 * x], va[4 * x + 1], va[4 * x + 2], va[4 * x + 3])
+                                : z4;
+#pragma unroll
+                for (int x = 0; x < KO / 4; ++x)
+                  rg[x] = valid ? make_float4(vg[4 * x], vg[4 * x + 1], vg[4 * x + 2], vg[4 * x + 3])
+                                : z4;
+              }
+              named_bar_sync(1, 128);
+              if (p.bias_partials != nullptr) {  // projected bias gradient: sum_t g~_t
+                const int col = et % KO, r0 = (et / KO) * (KO / 2);
+#pragma unroll 4
+                for (int i = 0; i < KO / 2; ++i) bias_acc += sG[(r0 + i) * (KO + 4) + col];
+              }
+#pragma unroll 4
+              for (int t2 = 0; t2 < kHalf; ++t2) {
+                const float gv = sG[t2 * (KO + 4) + oi];
+                const float* ar = sA + t2 * (KI + 4) + oj;
+                if constexpr (OPT % 4 == 0) {
+#pragma unroll
+                  for (int x = 0; x < OPT / 4; ++x) {
+                    const float4 a4 = reinterpret_cast<const float4*>(ar)[x];
+                    acc[4 * x] = fmaf(gv, a4.x, acc[4 * x]);
+                    acc[4 * x + 1] = fmaf(gv, a4.y, acc[4 * x + 1]);
+                    acc[4 * x + 2] = fmaf(gv, a4.z, acc[4 * x + 2]);
+                    acc[4 * x + 3] = fmaf(gv, a4.w, acc[4 * x + 3]);
+                  }
+                } else {
+#pragma unroll
+                  for (int x = 0; x < OPT / 2; ++x) {
+                    const float2 a2 = reinterpret_cast<const float2*>(ar)[x];
+                    acc[2 * x] = fmaf(gv, a2.x, acc[2 * x]);
+                    acc[2 * x + 1] = fmaf(gv, a2.y, acc[2 * x + 1]);
+                  }
+                }
+              }
+            }
+          }
+        }
+        if (!finisher) {
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
           if (++ab == 2) { ab = 0; aph ^= 1; }
         }
-        if constexpr (TOKEN) {
-          // s[q] = g~^T Q~_q a~ for this thread's token: its share of the
-          // query's score (masked tokens score 0).
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (!(vm >> nt & 1)) continue;
-            const int t = (g + nt) * kTileTokens + row;
-            if (t >= p.T) continue;
-            const bool valid =
-                p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0;
-            for (int q = 0; q < p.n_queries; ++q) {
-              const float* qm = sA + q * (KO * KI);
-              float sq = 0.0f;
-#pragma unroll
-              for (int i = 0; i < KO; ++i) {
-                float u = 0.0f;
-#pragma unroll
-                for (int j = 0; j < KI; j += 4) {
-                  const float4 w = *reinterpret_cast<const float4*>(qm + i * KI + j);
-                  u = fmaf(w.x, va[nt][j], u);
-                  u = fmaf(w.y, va[nt][j + 1], u);
-                  u = fmaf(w.z, va[nt][j + 2], u);
-                  u = fmaf(w.w, va[nt][j + 3], u);
-                }
-                sq = fmaf(vg[nt][i], u, sq);
-              }
-              p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q) * p.B + ic.b) *
-                                   p.T + t] = valid ? sq : 0.0f;
-            }
-          }
-        } else {
-        constexpr int kHalf = kTileTokens / 2;
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          if (!(vm >> nt & 1)) continue;
-          const int t = (g + nt) * kTileTokens + row;
-          const bool valid = t < p.T &&
-              (p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0);
-          // Two halves of 64 tokens: the half's owners (whole warps) stage their
-          // a~, g~ rows, then all 128 threads accumulate over the half's tokens.
-#pragma unroll 1
-          for (int h = 0; h < 2; ++h) {
-            named_bar_sync(1, 128);                  // previous half's readers are done
-            if ((row >> 6) == h) {
-              float4* ra = reinterpret_cast<float4*>(sA + (row - h * kHalf) * (KI + 4));
-              float4* rg = reinterpret_cast<float4*>(sG + (row - h * kHalf) * (KO + 4));
-              const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-              for (int x = 0; x < KI / 4; ++x)
-                ra[x] = valid ? make_float4(va[nt][4 * x], va[nt][4 * x + 1], va[nt][4 * x + 2],
-                                            va[nt][4 * x + 3])
-                              : z4;
-#pragma unroll
-              for (int x = 0; x < KO / 4; ++x)
-                rg[x] = valid ? make_float4(vg[nt][4 * x], vg[nt][4 * x + 1], vg[nt][4 * x + 2],
-                                            vg[nt][4 * x + 3])
-                              : z4;
-            }
-            named_bar_sync(1, 128);
-            if (p.bias_partials != nullptr) {    // projected bias gradient: sum_t g~_t
-              const int col = et % KO, r0 = (et / KO) * (KO / 2);
-#pragma unroll 4
-              for (int i = 0; i < KO / 2; ++i) bias_acc += sG[(r0 + i) * (KO + 4) + col];
-            }
-#pragma unroll 4
-            for (int t2 = 0; t2 < kHalf; ++t2) {
-              const float gv = sG[t2 * (KO + 4) + oi];
-              const float* ar = sA + t2 * (KI + 4) + oj;
-              if constexpr (OPT % 4 == 0) {
-#pragma unroll
-                for (int x = 0; x < OPT / 4; ++x) {
-                  const float4 a4 = reinterpret_cast<const float4*>(ar)[x];
-                  acc[4 * x] = fmaf(gv, a4.x, acc[4 * x]);
-                  acc[4 * x + 1] = fmaf(gv, a4.y, acc[4 * x + 1]);
-                  acc[4 * x + 2] = fmaf(gv, a4.z, acc[4 * x + 2]);
-                  acc[4 * x + 3] = fmaf(gv, a4.w, acc[4 * x + 3]);
-                }
-              } else {
-#pragma unroll
-                for (int x = 0; x < OPT / 2; ++x) {
-                  const float2 a2 = reinterpret_cast<const float2*>(ar)[x];
-                  acc[2 * x] = fmaf(gv, a2.x, acc[2 * x]);
-                  acc[2 * x + 1] = fmaf(gv, a2.y, acc[2 * x + 1]);
-                }
-              }
-            }
-          }
-        }
-        }   // projection mode
       }
       if (aborted) break;
       if constexpr (TOKEN) continue;
