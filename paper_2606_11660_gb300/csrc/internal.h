@@ -155,7 +155,8 @@ struct XGemmPlan {
   int steps = 1;           // ceil(K / 32)
   int S = 1;               // K slices
   int stages = 2;          // shared-memory pipeline depth
-  size_t sx_off = 0, ynorm_off = 0, partial_off = 0, xh_off = 0, xl_off = 0, total = 0;
+  int n_chunks = 1;        // column chunks of x for the row split (norm partials per row)
+  size_t xnorm_off = 0, ynorm_off = 0, partial_off = 0, xh_off = 0, xl_off = 0, total = 0;
 };
 XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K);
 

@@ -43,6 +43,7 @@ namespace bergson {
 namespace {
 
 constexpr int kRowThreads = 256;
+constexpr int kSplitChunk = 2048;          // fp32 columns of x per splitting CTA
 constexpr int kXM = 128;                   // rows of y per tile (MMA M)
 constexpr int kXK = 32;                    // fp32 columns per stage: one 128-byte row
 constexpr int kYBytes = kXM * 128;         // one y tile
@@ -114,31 +115,40 @@ __global__ void __launch_bounds__(kRowThreads) row_scales_kernel(
 
 // Row b of x -> rows of x_hi and x_lo ([B, K], contiguous) and scale[b] as above.
 __global__ void __launch_bounds__(kRowThreads) split_rows_kernel(
-    const float* __restrict__ x, int K, int64_t ld, int unit, float* __restrict__ xh,
-    float* __restrict__ xl, float* __restrict__ scale) {
+    const float* __restrict__ x, int K, int64_t ld, int unit, int n_chunks,
+    float* __restrict__ xh, float* __restrict__ xl, float* __restrict__ xnorm) {
+  // grid: (rows, chunks of kSplitChunk columns); each CTA splits one chunk of
+  // one row and, for cosine scores, writes that chunk's compensated sum of
+  // squares (the finishing kernel adds the chunks of a row in order).
   __shared__ float red[kRowThreads / 32];
   const int64_t b = blockIdx.x;
   const float4* xr = reinterpret_cast<const float4*>(x + b * ld);
   float4* hr = reinterpret_cast<float4*>(xh + b * K);
   float4* lr = reinterpret_cast<float4*>(xl + b * K);
-  KahanSum ks;
-  for (int i = threadIdx.x; i < K / 4; i += kRowThreads) {
-    const float4 v = xr[i];
-    float4 h, l;
-    tf32_split(v, h, l);
-    hr[i] = h;
-    lr[i] = l;
-    ks.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
-  }
-  float s = ks.s;
+  for (int c = blockIdx.y; c < n_chunks; c += gridDim.y) {
+    const int i0 = c * (kSplitChunk / 4);
+    const int i1 = min(K / 4, i0 + kSplitChunk / 4);
+    KahanSum ks;
+    for (int i = i0 + threadIdx.x; i < i1; i += kRowThreads) {
+      const float4 v = xr[i];
+      float4 h, l;
+      tf32_split(v, h, l);
+      hr[i] = h;
+      lr[i] = l;
+      ks.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
+    }
+    if (!unit) continue;
+    float s = ks.s;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float tot = 0.0f;
-    for (int w = 0; w < kRowThreads / 32; ++w) tot += red[w];
-    scale[b] = unit ? (tot > 0.0f ? 1.0f / sqrtf(tot) : 0.0f) : 1.0f;
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      float tot = 0.0f;
+      for (int w = 0; w < kRowThreads / 32; ++w) tot += red[w];
+      xnorm[b * n_chunks + c] = tot;
+    }
+    __syncthreads();
   }
 }
 
@@ -401,12 +411,14 @@ __global__ void __launch_bounds__(kXThreads, 1)
   }
 }
 
-// s = sum over slices z (in order) of partial[z, b, q].  Cosine (sx given):
-// scores[b, q] = s * sx[b] * t_q, t_q = 1/sqrt(sum over z of ynorm[z, q]) (0
-// for a zero row).  Otherwise scores[b, q] = alpha' s + beta scores[b, q] +
+// s = sum over slices z (in order) of partial[z, b, q].  Cosine (xnorm
+// given): scores[b, q] = s / sqrt(nx_b) / sqrt(ny_q), nx_b the sum over the
+// row's chunks (in order) of xnorm[b, c], ny_q the sum over z of ynorm[z, q]
+// (0 when either row is zero).  Otherwise scores[b, q] = alpha' s + beta scores[b, q] +
 // gamma [b == q], alpha' = alpha * (*alpha_s) when alpha_s is given.
 __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, int Q,
-                              const float* __restrict__ sx, const float* __restrict__ ynorm,
+                              const float* __restrict__ xnorm, int n_chunks,
+                              const float* __restrict__ ynorm,
                               float alpha, const float* __restrict__ alpha_s, float beta,
                               float gamma, float* scores, int64_t ld) {
   const int64_t n = static_cast<int64_t>(B) * Q;
@@ -418,10 +430,11 @@ __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, i
     float s = 0.0f;
     for (int z = 0; z < S; ++z) s += partial[z * n + i];
     float* dst = scores + b * ld + q;
-    if (sx != nullptr) {
-      float ny = 0.0f;
+    if (xnorm != nullptr) {
+      float nx = 0.0f, ny = 0.0f;
+      for (int c = 0; c < n_chunks; ++c) nx += xnorm[static_cast<int64_t>(b) * n_chunks + c];
       for (int z = 0; z < S; ++z) ny += ynorm[static_cast<int64_t>(z) * Q + q];
-      *dst = s * sx[b] * (ny > 0.0f ? 1.0f / sqrtf(ny) : 0.0f);
+      *dst = nx > 0.0f && ny > 0.0f ? s * (1.0f / sqrtf(nx)) * (1.0f / sqrtf(ny)) : 0.0f;
     } else {
       float v = al * s;
       if (beta != 0.0f) v = fmaf(beta, *dst, v);
@@ -468,8 +481,9 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
     }
   }
   size_t off = 0;
-  pl.sx_off = off;
-  off += round_up256(sizeof(float) * static_cast<size_t>(b1));
+  pl.n_chunks = static_cast<int>(std::max<int64_t>(1, (K + kSplitChunk - 1) / kSplitChunk));
+  pl.xnorm_off = off;
+  off += round_up256(sizeof(float) * static_cast<size_t>(b1) * pl.n_chunks);
   pl.ynorm_off = off;
   off += round_up256(sizeof(float) * static_cast<size_t>(pl.S) * std::max<int64_t>(Q, 1));
   pl.partial_off = off;
@@ -493,10 +507,12 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
       encode_tmap_2d(&tm_xl, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.ws + pl.xl_off, a.K, a.B,
                      static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  float* sx = reinterpret_cast<float*>(a.ws + pl.sx_off);
+  float* xnorm = reinterpret_cast<float*>(a.ws + pl.xnorm_off);
   float* xh = reinterpret_cast<float*>(a.ws + pl.xh_off);
   float* xl = reinterpret_cast<float*>(a.ws + pl.xl_off);
-  split_rows_kernel<<<a.B, kRowThreads, 0, s>>>(a.x, a.K, a.ldx, a.unit, xh, xl, sx);
+  const dim3 sgrid(a.B, std::min(pl.n_chunks, 65535));
+  split_rows_kernel<<<sgrid, kRowThreads, 0, s>>>(a.x, a.K, a.ldx, a.unit, pl.n_chunks, xh, xl,
+                                                  xnorm);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
@@ -534,7 +550,8 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
 
   const dim3 fgrid((a.Q + 255) / 256, std::min(a.B, 65535));
   finish_kernel<<<fgrid, 256, 0, s>>>(
-      p.partial, pl.S, a.B, a.Q, a.unit ? sx : nullptr, p.ynorm, a.alpha, a.alpha_s, a.beta,
+      p.partial, pl.S, a.B, a.Q, a.unit ? xnorm : nullptr, pl.n_chunks, p.ynorm, a.alpha,
+      a.alpha_s, a.beta,
       a.gamma, a.scores, a.ld_scores);
   return cudaGetLastError();
 }
