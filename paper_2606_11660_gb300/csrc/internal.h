@@ -10,6 +10,25 @@
 
 namespace bergson {
 
+// Launches `kernel` with programmatic stream serialization: it may be
+// scheduled before its predecessor in the stream has finished, and must call
+// griddep_wait() before it touches anything that predecessor writes.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                                    size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 constexpr int kTileTokens = 128;     // tokens per MMA tile (tcgen05 M)
 constexpr int kChunk = 64;           // bf16 elements per 128-byte swizzled row
 constexpr int kScoreBN = 256;        // store rows per score tile (tcgen05 N)

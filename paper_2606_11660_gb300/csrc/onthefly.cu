@@ -50,6 +50,7 @@ constexpr int kYBytes = kXM * 128;         // one y tile
 constexpr int kXThreads = 320;             // producer, MMA, 4 converter, 4 epilogue warps
 constexpr int kXSmemBudget = 232448;       // 227 KB opt-in per CTA
 constexpr int kXBarBytes = 512;
+constexpr int kXMaxStages = 8;
 constexpr int kMaxSlices = 64;
 constexpr uint64_t kXDrainTimeoutNs = 2000000000ull;
 
@@ -121,6 +122,7 @@ __global__ void __launch_bounds__(kRowThreads) split_rows_kernel(
   // one row and, for cosine scores, writes that chunk's compensated sum of
   // squares (the finishing kernel adds the chunks of a row in order).
   __shared__ float red[kRowThreads / 32];
+  griddep_launch_dependents();   // the product kernel may start streaming y meanwhile
   const int64_t b = blockIdx.x;
   const float4* xr = reinterpret_cast<const float4*>(x + b * ld);
   float4* hr = reinterpret_cast<float4*>(xh + b * K);
@@ -244,22 +246,45 @@ __global__ void __launch_bounds__(kXThreads, 1)
       uint32_t ph = 0;
       uint32_t issued = 0, issued_par = 0;
       bool ok = true;
+      // y does not depend on the row split that precedes this grid: the first
+      // round of stages gets its y tiles at once and its x tiles after
+      // griddep_wait() (x_hi / x_lo are the split's output).
+      bool dep = false;
+      int n_def = 0;
+      int def_st[kXMaxStages], def_nt[kXMaxStages];
+      auto load_x = [&](int sg, int st, int nt) {
+        const uint32_t fb = smem_u32(&full[sg]);
+        const uint32_t dst = sbase + sg * stage_bytes + 2 * kYBytes;
+        tma_load_2d_hint(dst, &tm_xh, fb, st * kXK, nt * p.n_pad, pol_x);
+        tma_load_2d_hint(dst + xbytes, &tm_xl, fb, st * kXK, nt * p.n_pad, pol_x);
+      };
+      auto release = [&]() {
+        griddep_wait();
+        dep = true;
+        for (int d = 0; d < n_def; ++d) load_x(d, def_st[d], def_nt[d]);
+        n_def = 0;
+      };
       for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
         const XItem it = decode_xitem(p, item);
         for (int st = it.s0; st < it.s1; ++st) {
           if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_arrive_expect_tx(fb, kYBytes + 2 * xbytes);
-          const uint32_t dst = sbase + stage * stage_bytes;
-          tma_load_2d_hint(dst, &tm_y, fb, st * kXK, it.mt * kXM, pol_y);
-          tma_load_2d_hint(dst + 2 * kYBytes, &tm_xh, fb, st * kXK, it.nt * p.n_pad, pol_x);
-          tma_load_2d_hint(dst + 2 * kYBytes + xbytes, &tm_xl, fb, st * kXK, it.nt * p.n_pad,
-                           pol_x);
+          tma_load_2d_hint(sbase + stage * stage_bytes, &tm_y, fb, st * kXK, it.mt * kXM, pol_y);
+          if (dep) {
+            load_x(stage, st, it.nt);
+          } else {
+            def_st[n_def] = st;                     // first round: stage == n_def
+            def_nt[n_def] = it.nt;
+            if (++n_def == p.stages) release();
+          }
           issued |= 1u << stage;
           issued_par = (issued_par & ~(1u << stage)) | (ph << stage);
           if (++stage == p.stages) { stage = 0; ph ^= 1; }
         }
       }
+      if (!dep) release();
+      griddep_launch_dependents();   // every load issued: the finishing grid may launch
       if (!ok) {
         raise_device_error(p.status, s_abort, kStatusTimeout);
         for (int s = 0; s < p.stages; ++s)
@@ -421,6 +446,7 @@ __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, i
                               const float* __restrict__ ynorm,
                               float alpha, const float* __restrict__ alpha_s, float beta,
                               float gamma, float* scores, int64_t ld) {
+  griddep_wait();                 // partials, norms and alpha_s come from earlier grids
   const int64_t n = static_cast<int64_t>(B) * Q;
   const float al = alpha_s != nullptr ? alpha * *alpha_s : alpha;
   const int q = blockIdx.x * blockDim.x + threadIdx.x;     // grid: (Q / 256, rows of b)
@@ -463,7 +489,7 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   pl.n_mtiles = static_cast<int>(std::max<int64_t>(1, (Q + kXM - 1) / kXM));
   pl.steps = static_cast<int>(std::max<int64_t>(1, (K + kXK - 1) / kXK));
   const int stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
-  pl.stages = std::min(8, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
+  pl.stages = std::min(kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
   // K slices: fewest waves of persistent CTAs for the y stream, plus the
   // partials each slice adds (written and read back once).
   const int64_t tiles = static_cast<int64_t>(pl.n_mtiles) * pl.n_ntiles;
@@ -544,16 +570,14 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   const size_t smem = 1024 + static_cast<size_t>(pl.stages) * (2 * kYBytes + 2 * pl.n_pad * 128) +
                       kXBarBytes;
   const int grid = std::max(1, std::min(sms > 0 ? sms : 1, p.n_items));
-  xgemm_kernel<<<grid, kXThreads, smem, s>>>(tm_y, tm_xh, tm_xl, p);
-  e = cudaGetLastError();
+  e = launch_dependent(xgemm_kernel, dim3(grid), dim3(kXThreads), smem, s, tm_y, tm_xh, tm_xl, p);
   if (e != cudaSuccess) return e;
 
   const dim3 fgrid((a.Q + 255) / 256, std::min(a.B, 65535));
-  finish_kernel<<<fgrid, 256, 0, s>>>(
-      p.partial, pl.S, a.B, a.Q, a.unit ? xnorm : nullptr, pl.n_chunks, p.ynorm, a.alpha,
-      a.alpha_s, a.beta,
-      a.gamma, a.scores, a.ld_scores);
-  return cudaGetLastError();
+  const float* xn = a.unit ? xnorm : nullptr;
+  return launch_dependent(finish_kernel, fgrid, dim3(256), 0, s, p.partial, pl.S, a.B, a.Q, xn,
+                          pl.n_chunks, p.ynorm, a.alpha, a.alpha_s, a.beta, a.gamma, a.scores,
+                          a.ld_scores);
 }
 
 }  // namespace bergson

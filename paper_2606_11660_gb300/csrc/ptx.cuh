@@ -281,4 +281,17 @@ __device__ __forceinline__ void named_bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Programmatic dependent launch.  A grid launched with programmatic stream
+// serialization may start while its predecessor in the stream still runs;
+// griddep_wait() blocks until that predecessor has completed and its memory
+// operations are visible (a no-op for a grid launched without the attribute).
+// griddep_launch_dependents() lets the successor grid be scheduled once every
+// CTA of this grid has issued it or exited.
+__device__ __forceinline__ void griddep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 }  // namespace bergson
