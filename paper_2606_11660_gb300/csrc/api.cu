@@ -683,15 +683,17 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
   if (e != cudaSuccess) return fail_cuda(e, "staging copy");
   const ModDesc* mods_dev = reinterpret_cast<const ModDesc*>(ws + L.mods_off);
   const bool need_tiles = T > 0;
-  if (need_tiles) {
-    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, max_pairs, s);
-    if (e != cudaSuccess) return fail_cuda(e, "prep launch");
-  }
+  // Tile flags first, then P' right before the projection kernel, which is
+  // launched as its dependent and sets itself up while P' is generated.
   uint8_t* tile_valid = nullptr;
   if (mask != nullptr && need_tiles) {
     tile_valid = ws + L.tv_off;
     e = launch_tile_valid(mask, static_cast<int>(B), static_cast<int>(T), L.n_tiles, tile_valid, s);
     if (e != cudaSuccess) return fail_cuda(e, "tile flag launch");
+  }
+  if (need_tiles) {
+    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, max_pairs, s);
+    if (e != cudaSuccess) return fail_cuda(e, "prep launch");
   }
   const int sms = sm_count(dg.dev);
   for (size_t gi = 0; gi < L.groups.size(); ++gi) {

@@ -77,20 +77,31 @@ __device__ __forceinline__ void store_hi_lo(__nv_bfloat16* dst, int64_t hi_idx, 
   dst[lo_idx] = __float2bfloat16_rn(v - __bfloat162float(h));
 }
 
+// Entry pair q = (i, j / 2) of a segment: both values of P'[i, j..j+1] as bf16
+// hi + lo, written transposed.
+__device__ __forceinline__ void prep_pair(const PrepSeg& sg, int i, int j) {
+  float v0, v1;
+  projection_pair(sg.seed, i, j, sg.k, sg.kind, sg.moment, &v0, &v1);
+  const int64_t d = sg.d;
+  store_hi_lo(sg.dst, j * d + i, (sg.k + j) * d + i, v0);
+  store_hi_lo(sg.dst, (j + 1) * d + i, (sg.k + j + 1) * d + i, v1);
+}
+
 // blockIdx.y = segment; threads walk the segment's d*k/2 entry pairs with the
-// input index i fastest, so the transposed bf16 stores are coalesced.
+// input index i fastest, so the transposed bf16 stores are coalesced.  The
+// index arithmetic is 32-bit when the segment allows it (the common case).
 __global__ void prep_kernel(const PrepSeg* __restrict__ segs) {
+  griddep_launch_dependents();   // the projection kernel may set itself up meanwhile
   const PrepSeg sg = segs[blockIdx.y];
   const int64_t npairs = static_cast<int64_t>(sg.d) * sg.k / 2;
-  for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < npairs;
-       q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int i = static_cast<int>(q % sg.d);
-    const int j = 2 * static_cast<int>(q / sg.d);
-    float v0, v1;
-    projection_pair(sg.seed, i, j, sg.k, sg.kind, sg.moment, &v0, &v1);
-    const int64_t d = sg.d;
-    store_hi_lo(sg.dst, j * d + i, (sg.k + j) * d + i, v0);
-    store_hi_lo(sg.dst, (j + 1) * d + i, (sg.k + j + 1) * d + i, v1);
+  if (npairs <= 0x7fffffff) {
+    const uint32_t n = static_cast<uint32_t>(npairs), d = static_cast<uint32_t>(sg.d);
+    for (uint32_t q = blockIdx.x * blockDim.x + threadIdx.x; q < n; q += gridDim.x * blockDim.x)
+      prep_pair(sg, static_cast<int>(q % d), 2 * static_cast<int>(q / d));
+  } else {
+    for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < npairs;
+         q += static_cast<int64_t>(gridDim.x) * blockDim.x)
+      prep_pair(sg, static_cast<int>(q % sg.d), 2 * static_cast<int>(q / sg.d));
   }
 }
 

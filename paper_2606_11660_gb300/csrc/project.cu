@@ -237,6 +237,9 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   const uint64_t tmo = p.timeout_ns;
+  // Everything above overlaps the preceding grid (P' generation); the work
+  // table, item counter, tile flags and P' are its or earlier writes.
+  griddep_wait();
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -293,6 +296,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         }
         if (!ok) break;
       }
+      griddep_launch_dependents();   // all loads issued: the reduction grid may launch
       if (!ok) {
         raise_device_error(p.status, s_abort, kStatusTimeout);
         // Let every copy this thread started land before the CTA can exit.
@@ -599,6 +603,8 @@ __global__ void reduce_kernel(const ModDesc* __restrict__ mods, int B, int blk, 
                               int n_chunks, const float* __restrict__ partials,
                               const float* __restrict__ bias_partials, float* __restrict__ out,
                               int64_t ld_out) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int mb = blockIdx.x;
   const int m = mb / B;
   const int b = mb % B;
@@ -648,8 +654,8 @@ cudaError_t launch_project_t(const ProjParams& p, int grid, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  project_kernel<KI, KO, TOKEN><<<grid, 192, C::kSmemBytes, s>>>(p);
-  return cudaGetLastError();
+  return launch_dependent(project_kernel<KI, KO, TOKEN>, dim3(grid), dim3(192), C::kSmemBytes, s,
+                          p);
 }
 
 template <int KI, int KO>
@@ -714,9 +720,8 @@ cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, 
   const int blocks = n_mods * B;
   if (blocks == 0) return cudaSuccess;
   const int blk = k_in * k_out;
-  reduce_kernel<<<blocks, blk < 1024 ? blk : 1024, 0, s>>>(mods, B, blk, k_out, n_chunks, partials,
-                                                          bias_partials, out, ld_out);
-  return cudaGetLastError();
+  return launch_dependent(reduce_kernel, dim3(blocks), dim3(blk < 1024 ? blk : 1024), 0, s, mods,
+                          B, blk, k_out, n_chunks, partials, bias_partials, out, ld_out);
 }
 
 }  // namespace bergson

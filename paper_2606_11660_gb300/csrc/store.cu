@@ -8,6 +8,7 @@
 // vector stores.
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace bergson {
 
@@ -61,6 +62,7 @@ __global__ void __launch_bounds__(kRowThreads) normalize_rows_kernel(
     const float* __restrict__ x, int K, int64_t ldx, int unit, __half* __restrict__ y,
     int64_t ldy, float* __restrict__ norms) {
   __shared__ float red[kRowThreads / 32];
+  griddep_wait();                // the rows are usually the preceding reduction's output
   const int64_t b = blockIdx.x;
   const float4* xr = reinterpret_cast<const float4*>(x + b * ldx);
   KahanSum ss;
@@ -95,8 +97,8 @@ __global__ void __launch_bounds__(kRowThreads) normalize_queries_kernel(
 cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj, int unit,
                                __half* store, int64_t ld_store, float* norms, cudaStream_t s) {
   if (B == 0) return cudaSuccess;
-  normalize_rows_kernel<<<B, kRowThreads, 0, s>>>(proj, K, ld_proj, unit, store, ld_store, norms);
-  return cudaGetLastError();
+  return launch_dependent(normalize_rows_kernel, dim3(B), dim3(kRowThreads), 0, s, proj, K,
+                          ld_proj, unit, store, ld_store, norms);
 }
 
 cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, __half* qh,
