@@ -351,7 +351,8 @@ def bench_onthefly(args, world, dev, state, peaks):
                          "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4),
                          "kernel": "bergson_score_grads call (split, tcgen05 3xTF32 product, "
                                    "finish)", "algorithmic_bytes_per_call": alg},
-            "gpu_launches": (5 + 3) * args.steps,
+            # tile flags, prep, projection, reduce; row split, product, finish
+            "gpu_launches": (4 + 3) * args.steps,
             "what": "bergson_project_grads + bergson_score_grads (cosine vs 1024 fp32 queries, "
                     "no store) per batch"}
 
@@ -390,8 +391,8 @@ def bench_tokens(args, world, dev, state, peaks):
             "ms_per_step": round(ms, 4), "queries": Q,
             "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"],
                          "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4),
-                         "traffic": profiled_traffic("project_kernel_pythia160m.md", "project.cu")},
-            "gpu_launches": 5 * args.steps,
+                         "traffic": profiled_traffic("token_kernel_pythia160m.md", "project.cu")},
+            "gpu_launches": 4 * args.steps,          # tile flags, prep, projection, token sum
             "what": "bergson_token_scores: per-token scores of all 65,536 tokens x 48 modules "
                     "against 4 query rows"}
 
@@ -667,9 +668,10 @@ def profile_case(args):
     __graft_entry__.build()
     dev = torch.device("cuda", 0)
     if args.profile_case == "tokens":
-        # one block of the Pythia-160M-shaped workload, B=8, T=2048, 4 query rows
+        # one block of the Pythia-160M-shaped workload at the bench's B=32,
+        # T=2048 and padding mask, 4 query rows
         cfg = wl.PYTHIA160M
-        B = 8
+        B = cfg.B
         mask = wl.right_padding_mask(B, cfg.T, cfg.max_pad, seed=1, device=dev)
         layers = []
         for m, spec in enumerate(cfg.block_modules(0)):
