@@ -175,6 +175,10 @@ struct XGemmPlan {
   int S = 1;               // K slices
   int stages = 2;          // shared-memory pipeline depth
   int n_chunks = 1;        // column chunks of x for the row split (norm partials per row)
+  bool tmem_a = false;     // y_hi / y_lo as TMEM A operands (n_pad <= 64)
+  int n_buf = 1;           // accumulator sets in TMEM
+  int a_base = 0;          // TMEM column of the A ring (tmem_a)
+  int tmem_cols = 32;      // TMEM columns allocated per CTA
   size_t xnorm_off = 0, ynorm_off = 0, partial_off = 0, xh_off = 0, xl_off = 0, total = 0;
 };
 XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K);

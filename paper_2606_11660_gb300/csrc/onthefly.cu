@@ -160,6 +160,7 @@ struct XGemmParams {
   int n_buf;          // TMEM accumulator sets (2: epilogue overlaps the next item)
   int n_items;
   int tmem_cols;
+  int a_base;         // TMEM column of the y_hi / y_lo ring (A operands in TMEM)
   int unit;
   float* partial;     // [S, B, Q]
   float* ynorm;       // [S, Q] squared norms of y rows over each slice (unit only)
@@ -190,6 +191,11 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint64_
   return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
 }
 
+// TA = true: the converter warps put y (read by the tensor cores as y_hi) and
+// y_lo into TMEM and both MMAs take A from there, so a y tile passes through
+// shared memory once (TMA write, converter read) instead of five times; used
+// while the accumulators leave room for the A ring (n_pad <= 64).
+template <bool TA>
 __global__ void __launch_bounds__(kXThreads, 1)
     xgemm_kernel(const __grid_constant__ CUtensorMap tm_y, const __grid_constant__ CUtensorMap tm_xh,
                  const __grid_constant__ CUtensorMap tm_xl, const XGemmParams p) {
@@ -198,7 +204,8 @@ __global__ void __launch_bounds__(kXThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
   const int xbytes = p.n_pad * 128;
-  const int stage_bytes = 2 * kYBytes + 2 * xbytes;
+  const int xoff = (TA ? 1 : 2) * kYBytes;      // x_hi, x_lo after y (and y_lo)
+  const int stage_bytes = xoff + 2 * xbytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
   uint64_t* empty = full + p.stages;
   uint64_t* conv = empty + p.stages;
@@ -254,7 +261,7 @@ __global__ void __launch_bounds__(kXThreads, 1)
       int def_st[kXMaxStages], def_nt[kXMaxStages];
       auto load_x = [&](int sg, int st, int nt) {
         const uint32_t fb = smem_u32(&full[sg]);
-        const uint32_t dst = sbase + sg * stage_bytes + 2 * kYBytes;
+        const uint32_t dst = sbase + sg * stage_bytes + xoff;
         tma_load_2d_hint(dst, &tm_xh, fb, st * kXK, nt * p.n_pad, pol_x);
         tma_load_2d_hint(dst + xbytes, &tm_xl, fb, st * kXK, nt * p.n_pad, pol_x);
       };
@@ -321,15 +328,26 @@ __global__ void __launch_bounds__(kXThreads, 1)
           }
           tc_fence_after();
           const uint32_t yh = sbase + stage * stage_bytes;
-          const uint64_t dyh = sw128_desc(yh);
-          const uint64_t dyl = sw128_desc(yh + kYBytes);
-          const uint64_t dx = sw128_desc(yh + 2 * kYBytes);
+          const uint64_t dx = sw128_desc(yh + xoff);
+          if constexpr (TA) {
+            const uint32_t ta = tmem + p.a_base + stage * 2 * kXK;   // y_hi, then y_lo
 #pragma unroll
-          for (int kk = 0; kk < kXK / 8; ++kk) {       // 8 tf32 = 32 bytes: +2 in the address field
-            const uint64_t o = 2 * kk;
-            const uint32_t acc = st != it.s0 || kk != 0;
-            umma_tf32(d_hi, dyh + o, dx + o, idesc, acc);
-            umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, acc);
+            for (int kk = 0; kk < kXK / 8; ++kk) {
+              const uint64_t o = 2 * kk;
+              const uint32_t acc = st != it.s0 || kk != 0;
+              umma_tf32_ta(d_hi, ta + 8 * kk, dx + o, idesc, acc);
+              umma_tf32_ta(d_lo, ta + kXK + 8 * kk, dx + o, idesc_lo, acc);
+            }
+          } else {
+            const uint64_t dyh = sw128_desc(yh);
+            const uint64_t dyl = sw128_desc(yh + kYBytes);
+#pragma unroll
+            for (int kk = 0; kk < kXK / 8; ++kk) {     // 8 tf32 = 32 bytes: +2 in the address field
+              const uint64_t o = 2 * kk;
+              const uint32_t acc = st != it.s0 || kk != 0;
+              umma_tf32(d_hi, dyh + o, dx + o, idesc, acc);
+              umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, acc);
+            }
           }
           umma_commit(smem_u32(&empty[stage]));
           if (++stage == p.stages) { stage = 0; ph ^= 1; }
@@ -343,8 +361,50 @@ __global__ void __launch_bounds__(kXThreads, 1)
       mbar_wait(smem_u32(drain), 0, kXDrainTimeoutNs, nullptr);
     }
     __syncwarp();
+  } else if (warp < 6 && TA) {
+    // ------------------------------------------------------------ converter (A in TMEM)
+    // Thread = row r of the y tile = TMEM lane r (warp w reaches lanes
+    // 32 (w % 4) ..).  Chunk c (columns 4c .. 4c + 3) of row r sits at chunk
+    // c ^ (r % 8) of the 128-byte swizzled row.
+    const int quarter = warp & 3;
+    const int r = 32 * quarter + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(32 * quarter) << 16) + p.a_base;
+    int stage = 0;
+    uint32_t ph = 0;
+    for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
+      const XItem it = decode_xitem(p, item);
+      KahanSum nrm;
+      bool aborted = false;
+      for (int st = it.s0; st < it.s1; ++st) {
+        if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) {
+          raise_device_error(p.status, s_abort, kStatusTimeout);
+          aborted = true;
+          break;
+        }
+        tc_fence_after();          // the MMAs that last read this TMEM slot are done
+        const uint8_t* row = smem + stage * stage_bytes + r * 128;
+        float hv[kXK], lv[kXK];
+#pragma unroll
+        for (int c = 0; c < kXK / 4; ++c) {
+          const float4 v = *reinterpret_cast<const float4*>(row + ((c ^ (r & 7)) << 4));
+          const float4 l = tf32_remainder(v);
+          hv[4 * c] = v.x; hv[4 * c + 1] = v.y; hv[4 * c + 2] = v.z; hv[4 * c + 3] = v.w;
+          lv[4 * c] = l.x; lv[4 * c + 1] = l.y; lv[4 * c + 2] = l.z; lv[4 * c + 3] = l.w;
+          if (p.unit) nrm.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
+        }
+        tmem_st32(trow + stage * 2 * kXK, hv);
+        tmem_st32(trow + stage * 2 * kXK + kXK, lv);
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(smem_u32(&conv[stage]));
+        if (++stage == p.stages) { stage = 0; ph ^= 1; }
+      }
+      if (aborted) break;
+      const int q = it.mt * kXM + r;
+      if (p.unit && it.nt == 0 && q < p.Q) p.ynorm[static_cast<int64_t>(it.z) * p.Q + q] = nrm.s;
+    }
   } else if (warp < 6) {
-    // ------------------------------------------------------------ converter
+    // ------------------------------------------------------------ converter (A in smem)
     // Thread ct owns 16-byte chunks ct + 128 i (i < 8) of each tile: rows
     // ct / 8 + 16 i, whatever the swizzle did to their columns.
     const int ct = threadIdx.x - 64;
@@ -481,6 +541,21 @@ cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit
   return cudaGetLastError();
 }
 
+template <bool TA>
+cudaError_t launch_xgemm(int grid, size_t smem, cudaStream_t s, const CUtensorMap& tm_y,
+                         const CUtensorMap& tm_xh, const CUtensorMap& tm_xl,
+                         const XGemmParams& p) {
+  static bool attr_set = false;   // per process; the attribute is per function and device
+  if (!attr_set) {
+    const cudaError_t e = cudaFuncSetAttribute(
+        xgemm_kernel<TA>, cudaFuncAttributeMaxDynamicSharedMemorySize, kXSmemBudget);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  return launch_dependent(xgemm_kernel<TA>, dim3(grid), dim3(kXThreads), smem, s, tm_y, tm_xh,
+                          tm_xl, p);
+}
+
 XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   XGemmPlan pl;
   const int64_t b1 = B > 0 ? B : 1;
@@ -488,8 +563,24 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   pl.n_ntiles = static_cast<int>((b1 + pl.n_pad - 1) / pl.n_pad);
   pl.n_mtiles = static_cast<int>(std::max<int64_t>(1, (Q + kXM - 1) / kXM));
   pl.steps = static_cast<int>(std::max<int64_t>(1, (K + kXK - 1) / kXK));
-  const int stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
-  pl.stages = std::min(kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
+  // y_hi / y_lo go to TMEM when the accumulators leave room for a ring of at
+  // least 4 stages (64 columns each); otherwise y_lo is written next to y.
+  pl.tmem_a = pl.n_pad <= 64;
+  int stage_bytes;
+  if (pl.tmem_a) {
+    pl.n_buf = (512 - 6 * pl.n_pad) / (2 * kXK) >= 4 ? 2 : 1;
+    pl.a_base = (pl.n_buf * 3 * pl.n_pad + 31) / 32 * 32;
+    pl.tmem_cols = 512;
+    stage_bytes = kYBytes + 2 * pl.n_pad * 128;
+    pl.stages = std::min({kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes,
+                          (512 - pl.a_base) / (2 * kXK)});
+  } else {
+    pl.n_buf = 6 * pl.n_pad <= 512 ? 2 : 1;
+    pl.tmem_cols = 32;
+    while (pl.tmem_cols < pl.n_buf * 3 * pl.n_pad) pl.tmem_cols <<= 1;
+    stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
+    pl.stages = std::min(kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
+  }
   // K slices: fewest waves of persistent CTAs for the y stream, plus the
   // partials each slice adds (written and read back once).
   const int64_t tiles = static_cast<int64_t>(pl.n_mtiles) * pl.n_ntiles;
@@ -551,26 +642,21 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   p.steps = pl.steps;
   p.stages = pl.stages;
   p.n_items = pl.n_mtiles * pl.n_ntiles * pl.S;
-  p.n_buf = 6 * pl.n_pad <= 512 ? 2 : 1;
-  int cols = 32;
-  while (cols < p.n_buf * 3 * pl.n_pad) cols <<= 1;
-  p.tmem_cols = cols;
+  p.n_buf = pl.n_buf;
+  p.tmem_cols = pl.tmem_cols;
+  p.a_base = pl.a_base;
   p.unit = a.unit;
   p.partial = reinterpret_cast<float*>(a.ws + pl.partial_off);
   p.ynorm = reinterpret_cast<float*>(a.ws + pl.ynorm_off);
   p.status = a.status;
   p.timeout_ns = a.timeout_ns;
-  static bool attr_set = false;   // per process; the attribute is per function and device
-  if (!attr_set) {
-    e = cudaFuncSetAttribute(xgemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kXSmemBudget);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
-  const size_t smem = 1024 + static_cast<size_t>(pl.stages) * (2 * kYBytes + 2 * pl.n_pad * 128) +
+  const size_t smem = 1024 +
+                      static_cast<size_t>(pl.stages) *
+                          ((pl.tmem_a ? 1 : 2) * kYBytes + 2 * pl.n_pad * 128) +
                       kXBarBytes;
   const int grid = std::max(1, std::min(sms > 0 ? sms : 1, p.n_items));
-  e = launch_dependent(xgemm_kernel, dim3(grid), dim3(kXThreads), smem, s, tm_y, tm_xh, tm_xl, p);
+  e = pl.tmem_a ? launch_xgemm<true>(grid, smem, s, tm_y, tm_xh, tm_xl, p)
+                : launch_xgemm<false>(grid, smem, s, tm_y, tm_xh, tm_xl, p);
   if (e != cudaSuccess) return e;
 
   const dim3 fgrid((a.Q + 255) / 256, std::min(a.B, 65535));
