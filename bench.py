@@ -694,6 +694,17 @@ def profile_case(args):
         for _ in range(2):
             bg.bergson_score_grads(x, B, K, y, True, out, ws)
         st = bg.bergson_sync_status()
+    elif args.profile_case == "apply":
+        # preconditioner application: 32 rows x 12288 against a 12288 x 12288
+        # fp32 M (604 MB, > L2), the per-batch product of the Fisher leg
+        B, K = 32, 12288
+        x = wl.gaussian_rows(B, K, seed=18, device=dev)
+        M = wl.gaussian_rows(K, K, seed=19, device=dev)
+        aws = bg.workspace_tensor(bg.bergson_score_grads_workspace(B, K, K), dev)
+        pre = torch.empty((B, K), device=dev)
+        for _ in range(2):
+            bg.bergson_precondition_rows(x, B, K, M, pre, aws)
+        st = bg.bergson_sync_status()
     elif args.profile_case == "fisher":
         # one Newton-Schulz iteration at K = 8192 (256 MB per matrix)
         K = 8192
@@ -857,7 +868,7 @@ def parse(argv=None):
     ap.add_argument("--no-fisher", action="store_true")
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--fisher-iters", type=int, default=20)
-    ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "fisher",
+    ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "apply", "fisher",
                              "streamed_pythia1b4", "streamed_llama8b"],
                     default=None,
                     help="run a small case of one kernel for ncu and exit")
