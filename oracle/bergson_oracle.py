@@ -33,7 +33,9 @@ Readings taken where the paper is silent (each is listed in the design doc):
   * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
     stateless counter-based generator (SplitMix64 finaliser of Steele, Lea and
     Flood 2014, then the Box-Muller transform of Box and Muller 1958), entry
-    e = i*k + j of the row-major [d, k] matrix, rounded once to fp32;
+    e = i*k + j of the row-major [d, k] matrix, rounded once to fp32; the
+    Rademacher and uniform projections App. B names take one hash of the same
+    counter per entry and are scaled to the same variance 1/k;
   * second moments divide by sqrt(r c^T) with no 1/sum(r) and no epsilon;
   * a masked token contributes nothing, whatever A and G hold there;
   * a row whose norm is zero stays zero.
@@ -54,6 +56,8 @@ _TWO_M53 = 2.0 ** -53
 
 PROJ_GAUSSIAN = 0
 PROJ_IDENTITY = 1
+PROJ_RADEMACHER = 2
+PROJ_UNIFORM = 3
 
 
 def mix64(x):
@@ -92,18 +96,51 @@ def gaussian_counter(seed: int, n: int) -> np.ndarray:
     return np.where((e & np.uint64(1)) == 0, rho * np.cos(theta), rho * np.sin(theta))
 
 
+def counter_hash(seed: int, n: int) -> np.ndarray:
+    """One 64-bit hash per counter: h_e = mix(seed ^ mix(e)), e = 0 .. n-1."""
+    e = np.arange(n, dtype=np.uint64)
+    return mix64(np.uint64(seed) ^ mix64(e))
+
+
+def rademacher_counter(seed: int, n: int) -> np.ndarray:
+    """Rademacher draws (App. B, "Gradients"): +1 where the top bit of h_e is
+    set, -1 where it is clear (fp64)."""
+    top = counter_hash(seed, n) >> np.uint64(63)
+    return np.where(top == np.uint64(1), 1.0, -1.0)
+
+
+def uniform_counter(seed: int, n: int) -> np.ndarray:
+    """Uniform draws on (-1, 1) (App. B, "Gradients"): the top 24 bits v of h_e
+    give x = (2v + 1 - 2^24) / 2^24, the midpoints of 2^24 equal cells, so the
+    draws are symmetric about 0 and exactly representable in fp32."""
+    v = (counter_hash(seed, n) >> np.uint64(40)).astype(np.float64)
+    return (2.0 * v + 1.0 - 2.0 ** 24) / 2.0 ** 24
+
+
 def projection_matrix(seed: int, d: int, k: int, kind: int = PROJ_GAUSSIAN) -> np.ndarray:
     """Dense projection P in R^{d x k}, stored as fp32 values held in fp64.
 
-    Gaussian: P[i, j] = fl32(z(seed, i*k + j) / sqrt(k)), so E||P^T x||^2 = ||x||^2
-    (Johnson-Lindenstrauss scaling).  Identity (tests only): k == d and P = I.
+    Entry (i, j) takes counter e = i*k + j and has mean 0 and variance 1/k, so
+    E||P^T x||^2 = ||x||^2 (Johnson-Lindenstrauss scaling):
+      Gaussian:   P[i, j] = fl32(z_e / sqrt(k));
+      Rademacher: P[i, j] = fl32(s_e / sqrt(k)), s_e = +-1;
+      uniform:    P[i, j] = fl32(sqrt(3) x_e / sqrt(k)), x_e uniform on (-1, 1)
+                  (variance 1/3, hence the sqrt(3));
+      identity (tests only): k == d and P = I.
     """
     if kind == PROJ_IDENTITY:
         if k != d:
             raise ValueError("identity projection needs k == d")
         return np.eye(d, dtype=np.float64)
-    z = gaussian_counter(seed, d * k).reshape(d, k)
-    return (z / np.sqrt(k)).astype(np.float32).astype(np.float64)
+    if kind == PROJ_GAUSSIAN:
+        z = gaussian_counter(seed, d * k)
+    elif kind == PROJ_RADEMACHER:
+        z = rademacher_counter(seed, d * k)
+    elif kind == PROJ_UNIFORM:
+        z = np.sqrt(3.0) * uniform_counter(seed, d * k)
+    else:
+        raise ValueError(f"unknown projection kind {kind}")
+    return (z.reshape(d, k) / np.sqrt(k)).astype(np.float32).astype(np.float64)
 
 
 def module_seeds(base_seed: int, module_index: int) -> tuple[int, int]:
