@@ -14,7 +14,9 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
   4. concatenation over modules in call order and unit normalisation of the
      whole per-example row (grad-cosine);
   5. an fp16 gradient store, cosine scores against unit-normalised queries and
-     exact top-k, ordered by (score descending, index ascending);
+     exact top-k, ordered by (score descending, index ascending), and the k
+     least influential items (Sec. 3.1), ordered by (score ascending, index
+     ascending);
   6. on-the-fly scores (Sec. 3.1, "bergson score"): training rows scored
      directly against query rows without a store, as cosines (grad-cosine) or
      plain inner products (grad-dot) -- Table 3's two identity-Hessian methods;
@@ -320,9 +322,30 @@ def topk_rows(S: np.ndarray, k: int) -> tuple[np.ndarray, np.ndarray]:
     return val, idx
 
 
+def bottomk_rows(S: np.ndarray, k: int) -> tuple[np.ndarray, np.ndarray]:
+    """Exact bottom-k of each row of S (the k least influential items, Sec. 3.1)
+    by full sort on key (score, index): lowest score first, ties by index."""
+    Q, N = S.shape
+    if k > N:
+        raise ValueError("k > N")
+    idx = np.empty((Q, k), dtype=np.int64)
+    val = np.empty((Q, k), dtype=np.float64)
+    cols = np.arange(N)
+    for qi in range(Q):
+        order = np.lexsort((cols, S[qi]))[:k]
+        idx[qi] = order
+        val[qi] = S[qi, order]
+    return val, idx
+
+
 def score_topk(store: np.ndarray, queries: np.ndarray, k: int):
     """Cosine scores of queries against the store and their exact top-k."""
     return topk_rows(cosine_scores(store, queries), k)
+
+
+def score_bottomk(store: np.ndarray, queries: np.ndarray, k: int):
+    """Cosine scores of queries against the store and their exact bottom-k."""
+    return bottomk_rows(cosine_scores(store, queries), k)
 
 
 def onthefly_scores(rows: np.ndarray, queries: np.ndarray, unit: bool = True) -> np.ndarray:
