@@ -63,9 +63,18 @@ typedef enum {
   BERGSON_LAYER_BIAS = 1          /* also write the layer's projected bias gradient */
 } bergson_layer_flags;
 
+/*
+ * Distribution of the projection entries.  Every kind has mean 0 and variance
+ * 1/k per entry (Johnson-Lindenstrauss scaling); entry (i, j) of P [d, k]
+ * takes counter e = i*k + j of its seed's stream.  App. B ("Gradients") names
+ * Rademacher and uniform projection matrices; Gaussian is the default here.
+ */
 typedef enum {
-  BERGSON_PROJ_GAUSSIAN = 0,      /* seeded Gaussian, entries N(0, 1/k) */
-  BERGSON_PROJ_IDENTITY = 1       /* P = I, requires k == d (testing aid) */
+  BERGSON_PROJ_GAUSSIAN = 0,      /* z_e / sqrt(k), z_e the Box-Muller normal draw */
+  BERGSON_PROJ_IDENTITY = 1,      /* P = I, requires k == d (testing aid) */
+  BERGSON_PROJ_RADEMACHER = 2,    /* +-1 / sqrt(k): sign = top bit of h_e = mix(seed ^ mix(e)) */
+  BERGSON_PROJ_UNIFORM = 3        /* sqrt(3) x_e / sqrt(k), x_e = (2v + 1 - 2^24) 2^-24 uniform
+                                     on (-1, 1), v = top 24 bits of h_e */
 } bergson_proj_kind;
 
 /*
@@ -80,8 +89,9 @@ typedef enum {
  *   k_in, k_out   projection sizes, each one of 16, 32, 64.
  *   seed_in, seed_out   seeds of P_in [d_in, k_in] and P_out [d_out, k_out].
  *          Entry (i, j) of P is z(seed, i*k + j) / sqrt(k), z the counter-based
- *          SplitMix64 + Box-Muller normal draw, rounded to fp32.
- *   proj_kind    bergson_proj_kind.
+ *          SplitMix64 + Box-Muller normal draw, rounded to fp32 (Gaussian kind;
+ *          see bergson_proj_kind for the others).
+ *   proj_kind    bergson_proj_kind, shared by both sides of the layer.
  *   r, c   fp32 [d_out] and [d_in] factored second moments (> 0), or both
  *          NULL for no normalisation.  The gradient is divided elementwise by
  *          sqrt(r_i c_j).
@@ -183,6 +193,25 @@ BERGSON_API int bergson_score_topk(const void* store, int64_t N, int64_t K, int6
                        const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
                        float* out_scores, int64_t* out_idx,
                        void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * The k least influential store rows of each query (Bergson Sec. 3.1: the
+ * query tool returns the k most and least influential training items):
+ *
+ *   out_scores[q, :], out_idx[q, :] = the bottomk smallest S[q, n], ordered by
+ *   score ascending, then index ascending.
+ *
+ * S, the arguments, the limits (bottomk in 1 .. min(N, 1024)) and the errors
+ * are those of bergson_score_topk, and so is the workspace
+ * (bergson_score_topk_workspace with topk = bottomk).  The search runs on the
+ * negated unit query; the scores it returns are exactly the negations of the
+ * scores against -q, i.e. the cosines against q.  If fewer than bottomk scores
+ * are usable the tail holds score +inf and index -1.
+ */
+BERGSON_API int bergson_score_bottomk(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                          const float* queries, int64_t Q, int64_t ld_q, int64_t bottomk,
+                          float* out_scores, int64_t* out_idx,
+                          void* workspace, size_t ws_bytes, void* stream);
 
 /* Bytes of workspace bergson_token_scores needs (n_queries in 1 .. 16). */
 BERGSON_API int bergson_token_scores_workspace(const bergson_layer* layers, int n_layers,

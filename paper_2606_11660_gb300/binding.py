@@ -25,6 +25,8 @@ BERGSON_EDEVICE_TIMEOUT = -6
 
 BERGSON_PROJ_GAUSSIAN = 0
 BERGSON_PROJ_IDENTITY = 1
+BERGSON_PROJ_RADEMACHER = 2
+BERGSON_PROJ_UNIFORM = 3
 
 BERGSON_LAYER_BIAS = 1
 
@@ -42,7 +44,8 @@ STATUS_NAMES = {
 # Every symbol include/bergson.h declares.
 EXPORTED = (
     "bergson_project_grads_workspace", "bergson_project_grads", "bergson_build_store",
-    "bergson_score_topk_workspace", "bergson_score_topk", "bergson_projection_matrix",
+    "bergson_score_topk_workspace", "bergson_score_topk", "bergson_score_bottomk",
+    "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
     "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_debug_project_plan", "bergson_project_grads_noalloc",
     "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
@@ -93,6 +96,8 @@ def lib() -> ctypes.CDLL:
         "bergson_score_topk_workspace": (i32, [i64, i64, i64, i64, szp]),
         "bergson_score_topk": (i32, [vp, i64, i64, i64, vp, i64, i64, i64, vp, vp, vp,
                                      ctypes.c_size_t, vp]),
+        "bergson_score_bottomk": (i32, [vp, i64, i64, i64, vp, i64, i64, i64, vp, vp, vp,
+                                        ctypes.c_size_t, vp]),
         "bergson_projection_matrix": (i32, [u64, i64, i64, i32, vp, vp, vp]),
         "bergson_module_seeds": (None, [u64, i64, ctypes.POINTER(u64), ctypes.POINTER(u64)]),
         "bergson_sync_status": (i32, [vp]),
@@ -237,6 +242,17 @@ def bergson_score_topk(store, N: int, K: int, queries, topk: int, out_scores, ou
                                     _ptr(queries), Q, int(queries.stride(0)), int(topk),
                                     _ptr(out_scores), _ptr(out_idx), _ptr(workspace), ws_bytes,
                                     _stream(stream)))
+
+
+def bergson_score_bottomk(store, N: int, K: int, queries, bottomk: int, out_scores, out_idx,
+                          workspace, stream=None) -> None:
+    """The bottomk least similar store rows per query, lowest score first."""
+    Q = int(queries.shape[0])
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check(lib().bergson_score_bottomk(_ptr(store), int(N), int(K), int(store.stride(0)),
+                                       _ptr(queries), Q, int(queries.stride(0)), int(bottomk),
+                                       _ptr(out_scores), _ptr(out_idx), _ptr(workspace), ws_bytes,
+                                       _stream(stream)))
 
 
 def bergson_token_scores_workspace(layers: Sequence, B: int, T: int, n_queries: int) -> int:

@@ -66,6 +66,10 @@ int injected() {
 }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+bool known_proj_kind(int kind) {
+  return kind == BERGSON_PROJ_GAUSSIAN || kind == BERGSON_PROJ_IDENTITY ||
+         kind == BERGSON_PROJ_RADEMACHER || kind == BERGSON_PROJ_UNIFORM;
+}
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -175,7 +179,7 @@ int validate_layers(const bergson_layer* layers, int n_layers, int64_t B, int64_
       return fail(BERGSON_EINVAL, "layer %d: d_in/d_out must be in [8, 2^24]", i);
     if (L.d_in % 8 != 0 || L.d_out % 8 != 0)
       return fail(BERGSON_EALIGN, "layer %d: d_in and d_out must be multiples of 8", i);
-    if (L.proj_kind != BERGSON_PROJ_GAUSSIAN && L.proj_kind != BERGSON_PROJ_IDENTITY)
+    if (!known_proj_kind(L.proj_kind))
       return fail(BERGSON_EINVAL, "layer %d: unknown proj_kind %d", i, L.proj_kind);
     if (!valid_k(L.k_in) || !valid_k(L.k_out))
       return fail(BERGSON_EUNSUPPORTED, "layer %d: k_in and k_out must be 16, 32 or 64", i);
@@ -811,10 +815,13 @@ int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, 
   return BERGSON_OK;
 }
 
-int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store,
-                       const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
-                       float* out_scores, int64_t* out_idx, void* workspace, size_t ws_bytes,
-                       void* stream) {
+// Top-k (least = false) or bottom-k (least = true: the queries are negated
+// when they are normalised, and the final merge reports the scores against
+// the original queries).
+static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                     const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
+                     float* out_scores, int64_t* out_idx, void* workspace, size_t ws_bytes,
+                     void* stream, bool least) {
   int st = validate_score(store, N, K, ld_store, queries, Q, ld_q, topk);
   if (st != BERGSON_OK) return st;
   if (Q > 0 && (out_scores == nullptr || out_idx == nullptr))
@@ -841,7 +848,7 @@ int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store
   unsigned long long* heaps = reinterpret_cast<unsigned long long*>(ws + L.heap_off);
 
   cudaError_t e = launch_normalize_queries(queries, static_cast<int>(Q), static_cast<int>(K), ld_q,
-                                           qh, s);
+                                           least, qh, s);
   if (e != cudaSuccess) return fail_cuda(e, "query normalisation launch");
 
   CUtensorMap tm_store, tm_q;
@@ -881,12 +888,30 @@ int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store
       p.timeout_ns = kWaitTimeoutNs;
       e = launch_score(L.qt, tm_store, tm_q, p, grid, s);
       if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
+      // The prefix pass's scores seed the full pass's thresholds, so only
+      // the final merge converts them back for a bottom-k search.
       e = launch_merge(heaps, grid, n_qg, L.qt, static_cast<int>(topk), q_begin, q_end, pass,
-                       out_scores, out_idx, s);
+                       least && stage == 1, out_scores, out_idx, s);
       if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
     }
   }
   return BERGSON_OK;
+}
+
+int bergson_score_topk(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                       const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
+                       float* out_scores, int64_t* out_idx, void* workspace, size_t ws_bytes,
+                       void* stream) {
+  return run_score(store, N, K, ld_store, queries, Q, ld_q, topk, out_scores, out_idx, workspace,
+                   ws_bytes, stream, false);
+}
+
+int bergson_score_bottomk(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                          const float* queries, int64_t Q, int64_t ld_q, int64_t bottomk,
+                          float* out_scores, int64_t* out_idx, void* workspace, size_t ws_bytes,
+                          void* stream) {
+  return run_score(store, N, K, ld_store, queries, Q, ld_q, bottomk, out_scores, out_idx,
+                   workspace, ws_bytes, stream, true);
 }
 
 static size_t onthefly_workspace(int64_t B, int64_t K, int64_t Q) {
@@ -1122,8 +1147,7 @@ int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind
                               const float* moment, float* out, void* stream) {
   if (d < 1 || d > (1 << 24)) return fail(BERGSON_EINVAL, "d must be in [1, 2^24]");
   if (!valid_k(k)) return fail(BERGSON_EUNSUPPORTED, "k must be 16, 32 or 64");
-  if (proj_kind != BERGSON_PROJ_GAUSSIAN && proj_kind != BERGSON_PROJ_IDENTITY)
-    return fail(BERGSON_EINVAL, "unknown proj_kind %d", proj_kind);
+  if (!known_proj_kind(proj_kind)) return fail(BERGSON_EINVAL, "unknown proj_kind %d", proj_kind);
   if (proj_kind == BERGSON_PROJ_IDENTITY && k != d)
     return fail(BERGSON_EINVAL, "identity projection needs k == d");
   if (out == nullptr) return fail(BERGSON_EINVAL, "out is NULL");

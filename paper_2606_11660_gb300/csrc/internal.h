@@ -144,13 +144,13 @@ cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, 
 
 cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj, int unit,
                                __half* store, int64_t ld_store, float* norms, cudaStream_t s);
-cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, __half* qh,
-                                     cudaStream_t s);
+cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, bool negate,
+                                     __half* qh, cudaStream_t s);
 cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
                          const ScoreParams& p, int grid, cudaStream_t s);
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
-                         int q_begin, int q_end, int qg_base, float* out_scores, int64_t* out_idx,
-                         cudaStream_t s);
+                         int q_begin, int q_end, int qg_base, bool negate, float* out_scores,
+                         int64_t* out_idx, cudaStream_t s);
 
 cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit, float* scale,
                               cudaStream_t s);

@@ -1,7 +1,7 @@
 // Projection preparation (Fig. 1: random down-projection; App. B, "Gradients":
 // double-sided projection), mask tile flags and the bounded-wait probe.
 //
-// The Gaussian projection is generated on the fly from its seed: entry
+// The projection is generated on the fly from its seed: entry
 // (i, j) of P in R^{d x k} is z(seed, i*k + j) / sqrt(k), where z is a
 // stateless counter-based normal draw: SplitMix64's finaliser (Steele, Lea
 // and Flood, OOPSLA 2014) hashes the pair counter into two 53-bit uniforms
@@ -17,6 +17,7 @@
 // into two bf16 terms hi + lo, so A and G (exact bf16) meet a projection that
 // is accurate to ~2^-16 relative instead of bf16's 2^-8.
 
+#include "bergson.h"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -49,19 +50,35 @@ __device__ __forceinline__ void gaussian_pair(uint64_t seed, uint64_t p, float* 
   *zs = rho * s;
 }
 
+// Rademacher and uniform draws (App. B names both) take one hash per counter,
+// h_e = mix(seed ^ mix(e)).  Rademacher: +1 when the top bit of h_e is set,
+// else -1.  Uniform on (-1, 1): the top 24 bits v of h_e give the cell
+// midpoint (2v + 1 - 2^24) 2^-24, exact in fp32; sqrt(3) brings the variance
+// from 1/3 to 1.
+__device__ __forceinline__ float counter_draw(uint64_t seed, uint64_t e, int kind) {
+  const uint64_t h = mix64(seed ^ mix64(e));
+  if (kind == BERGSON_PROJ_RADEMACHER) return (h >> 63) ? 1.0f : -1.0f;
+  const int v = static_cast<int>(h >> 40);
+  return static_cast<float>(2 * v + 1 - (1 << 24)) * 0x1p-24f * 1.7320508075688772f;
+}
+
 // Entries (i, j) and (i, j + 1), j even, of P' = diag(scale) P, fp32.  They
 // are counters e = i*k + j and e + 1, i.e. both draws of pair e / 2.
 __device__ __forceinline__ void projection_pair(uint64_t seed, int i, int j, int k, int kind,
                                                 const float* moment, float* v0, float* v1) {
-  if (kind == 1) {
+  const float inv_sqrt_k = 1.0f / sqrtf(static_cast<float>(k));
+  const uint64_t e = static_cast<uint64_t>(i) * k + j;
+  if (kind == BERGSON_PROJ_IDENTITY) {
     *v0 = (i == j) ? 1.0f : 0.0f;
     *v1 = (i == j + 1) ? 1.0f : 0.0f;
-  } else {
-    const float inv_sqrt_k = 1.0f / sqrtf(static_cast<float>(k));
+  } else if (kind == BERGSON_PROJ_GAUSSIAN) {
     float zc, zs;
-    gaussian_pair(seed, (static_cast<uint64_t>(i) * k + j) >> 1, &zc, &zs);
+    gaussian_pair(seed, e >> 1, &zc, &zs);
     *v0 = zc * inv_sqrt_k;
     *v1 = zs * inv_sqrt_k;
+  } else {
+    *v0 = counter_draw(seed, e, kind) * inv_sqrt_k;
+    *v1 = counter_draw(seed, e + 1, kind) * inv_sqrt_k;
   }
   if (moment != nullptr) {
     const float sc = 1.0f / sqrtf(moment[i]);

@@ -365,14 +365,16 @@ __device__ __forceinline__ void bitonic_desc(unsigned long long* keys, int n) {
   }
 }
 
+// negate: the scores were taken against -q (a bottom-k search); report them
+// against q, so the list runs from the lowest score up.
 __device__ __forceinline__ void write_topk(const unsigned long long* keys, int q, int topk,
-                                           float* out_scores, int64_t* out_idx) {
+                                           int negate, float* out_scores, int64_t* out_idx) {
   for (int e = threadIdx.x; e < topk; e += blockDim.x) {
     const unsigned long long k = keys[e];
     const uint32_t lo = static_cast<uint32_t>(k);
     const bool real = lo >= 0x80000000u;          // rows < 2^31 map to ~row >= 2^31
-    out_scores[static_cast<int64_t>(q) * topk + e] =
-        real ? order_to_float(static_cast<uint32_t>(k >> 32)) : -INFINITY;
+    const float v = real ? order_to_float(static_cast<uint32_t>(k >> 32)) : -INFINITY;
+    out_scores[static_cast<int64_t>(q) * topk + e] = negate ? -v : v;
     out_idx[static_cast<int64_t>(q) * topk + e] = real ? static_cast<int64_t>(~lo) : -1;
   }
 }
@@ -388,7 +390,7 @@ __device__ __forceinline__ void write_topk(const unsigned long long* keys, int q
 __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __restrict__ heaps,
                                                     int n_qg, int cpg, int gsize, int topk,
                                                     int q_begin, int q_end, int sort_n,
-                                                    int select_n,
+                                                    int select_n, int negate,
                                                     float* __restrict__ out_scores,
                                                     int64_t* __restrict__ out_idx) {
   extern __shared__ unsigned long long keys[];
@@ -454,7 +456,7 @@ __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __
     for (int i = min(s_count, select_n) + threadIdx.x; i < select_n; i += blockDim.x) sel[i] = 0ull;
     __syncthreads();
     bitonic_desc(sel, select_n);
-    write_topk(sel, q, topk, out_scores, out_idx);
+    write_topk(sel, q, topk, negate, out_scores, out_idx);
     return;
   }
   int64_t consumed = 0;
@@ -476,7 +478,7 @@ __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __
     __syncthreads();
     bitonic_desc(keys, sort_n);
   }
-  write_topk(keys, q, topk, out_scores, out_idx);
+  write_topk(keys, q, topk, negate, out_scores, out_idx);
 }
 
 template <int QT>
@@ -504,8 +506,8 @@ cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap&
 }
 
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
-                         int q_begin, int q_end, int /*qg_base*/, float* out_scores,
-                         int64_t* out_idx, cudaStream_t s) {
+                         int q_begin, int q_end, int /*qg_base*/, bool negate,
+                         float* out_scores, int64_t* out_idx, cudaStream_t s) {
   const int nq = q_end - q_begin;
   if (nq <= 0) return cudaSuccess;
   const int cpg = grid / n_qg;
@@ -526,7 +528,7 @@ cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, in
     attr_set = true;
   }
   merge_kernel<<<nq, 512, smem, s>>>(heaps, n_qg, cpg, qt * kScoreQT, topk, q_begin, q_end, sort_n,
-                                     select_n, out_scores, out_idx);
+                                     select_n, negate ? 1 : 0, out_scores, out_idx);
   return cudaGetLastError();
 }
 

@@ -78,16 +78,20 @@ __global__ void __launch_bounds__(kRowThreads) normalize_rows_kernel(
   if (norms != nullptr && threadIdx.x == 0) norms[b] = nrm;
 }
 
-// Queries may have any row stride; they are read with scalar loads.
+// Queries may have any row stride; they are read with scalar loads.  With
+// `negate` the row is written as -q / ||q|| (exactly the negation of the
+// unit row: fp16 rounding is symmetric), which turns a top-k search into a
+// bottom-k one.
 __global__ void __launch_bounds__(kRowThreads) normalize_queries_kernel(
-    const float* __restrict__ q, int K, int64_t ldq, __half* __restrict__ qh) {
+    const float* __restrict__ q, int K, int64_t ldq, int negate, __half* __restrict__ qh) {
   __shared__ float red[kRowThreads / 32];
   const int64_t r = blockIdx.x;
   const float* qr = q + r * ldq;
   KahanSum ss;
   for (int i = threadIdx.x; i < K; i += kRowThreads) ss.add(qr[i] * qr[i]);
   const float tot = block_sum(ss.s, red);
-  const float scale = tot > 0.0f ? 1.0f / sqrtf(tot) : 0.0f;
+  const float inv = tot > 0.0f ? 1.0f / sqrtf(tot) : 0.0f;
+  const float scale = negate ? -inv : inv;
   __half* out = qh + r * K;
   for (int i = threadIdx.x; i < K; i += kRowThreads) out[i] = __float2half_rn(qr[i] * scale);
 }
@@ -101,10 +105,10 @@ cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj,
                           ld_proj, unit, store, ld_store, norms);
 }
 
-cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, __half* qh,
-                                     cudaStream_t s) {
+cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, bool negate,
+                                     __half* qh, cudaStream_t s) {
   if (Q == 0) return cudaSuccess;
-  normalize_queries_kernel<<<Q, kRowThreads, 0, s>>>(q, K, ld_q, qh);
+  normalize_queries_kernel<<<Q, kRowThreads, 0, s>>>(q, K, ld_q, negate ? 1 : 0, qh);
   return cudaGetLastError();
 }
 

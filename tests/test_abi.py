@@ -83,6 +83,14 @@ def test_layer_validation(kw, code):
     assert _proj([_layer(**kw)]) == code
 
 
+def test_every_projection_kind_validates():
+    for kind in (bg.BERGSON_PROJ_GAUSSIAN, bg.BERGSON_PROJ_RADEMACHER, bg.BERGSON_PROJ_UNIFORM):
+        st, n = _ws([_layer(proj_kind=kind)])
+        assert st == bg.BERGSON_OK and n > 0
+    assert _ws([_layer(proj_kind=4)])[0] == bg.BERGSON_EINVAL
+    assert bg.lib().bergson_projection_matrix(1, 64, 16, 4, None, FAKE, None) == bg.BERGSON_EINVAL
+
+
 def test_workspace_query_and_block_checks():
     st, n = _ws([_layer(), _layer(out_col_offset=256, k_in=32)])
     assert st == bg.BERGSON_OK and n > 0 and n % 256 == 0
@@ -128,8 +136,9 @@ def test_store_validation():
     assert call(B=0) == bg.BERGSON_OK
 
 
-def test_score_validation():
-    f = bg.lib().bergson_score_topk
+@pytest.mark.parametrize("entry", ["bergson_score_topk", "bergson_score_bottomk"])
+def test_score_validation(entry):
+    f = getattr(bg.lib(), entry)
     n = ctypes.c_size_t()
     assert bg.lib().bergson_score_topk_workspace(100, 64, 10, 5, ctypes.byref(n)) == bg.BERGSON_OK
     ws = n.value

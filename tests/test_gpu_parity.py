@@ -39,6 +39,46 @@ def test_projection_matrix_matches_generator(seed, d, k, moment):
     assert np.median(err) < 2e-7 and np.quantile(err, 0.999) < 2e-6
 
 
+@pytest.mark.parametrize("kind", [bg.BERGSON_PROJ_RADEMACHER, bg.BERGSON_PROJ_UNIFORM])
+@pytest.mark.parametrize("seed,d,k,moment", [(2**63 + 11, 200, 32, False), (3, 768, 16, True),
+                                              (41, 64, 64, True)])
+def test_rademacher_uniform_matrices_match_generator(kind, seed, d, k, moment):
+    mom = torch.rand(d, generator=wl.generator(seed % 1000, "cpu")) * 1.5 + 0.5 if moment else None
+    out = torch.empty((d, k), dtype=torch.float32, device=DEV)
+    bg.bergson_projection_matrix(seed, d, k, kind, None if mom is None else mom.to(DEV), out)
+    torch.cuda.synchronize()
+    want = orc.projection_matrix(seed, d, k, kind)
+    if mom is not None:
+        want = want / np.sqrt(mom.numpy().astype(np.float64))[:, None]
+    got = np32(out)
+    if kind == bg.BERGSON_PROJ_RADEMACHER and mom is None:
+        np.testing.assert_array_equal(got, want)          # +-fl32(1/sqrt(k)): exact
+    else:
+        # the draw is exact in fp32; only the scalings round (a few ulps)
+        assert np.max(np.abs(got - want) / np.abs(want)) < 1e-6
+    assert np.array_equal(np.sign(got), np.sign(want))
+
+
+@pytest.mark.parametrize("kind", [bg.BERGSON_PROJ_RADEMACHER, bg.BERGSON_PROJ_UNIFORM])
+def test_rademacher_uniform_projection_parity(kind):
+    specs = [wl.ModuleSpec("a", 64, 200), wl.ModuleSpec("b", 136, 64), wl.ModuleSpec("c", 768, 2304)]
+    kp = [(16, 16), (32, 16), (16, 32)]
+    B, T = 3, 300
+    gl, ol, ld = make_layers(specs, B, T, kp, base_seed=11, data_seed=4, rc=True,
+                             input_scale=True, kind=kind)
+    g = wl.generator(8, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.1).to(torch.uint8)
+    out = run_project(gl, B, T, mask.to(DEV), ld)
+    want = orc.project_grads(ol, mask.numpy(), ld)
+    err = rel_frobenius(np32(out).astype(np.float64), want)
+    assert err.max() <= TIGHT
+    # a different distribution really is used: the Gaussian call differs
+    gl_g = [bg.Layer(x.A, x.G, x.k_in, x.k_out, x.seed_in, x.seed_out, x.r, x.c, x.out_col_offset)
+            for x in gl]
+    out_g = run_project(gl_g, B, T, mask.to(DEV), ld)
+    assert rel_frobenius(np32(out_g).astype(np.float64), want).min() > 0.1
+
+
 def test_tiny_workload_parity():
     cfg = wl.TINY
     gl, ol, ld = make_layers(cfg.modules, cfg.B, cfg.T, [(16, 16)], rc=True)
