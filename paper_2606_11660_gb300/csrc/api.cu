@@ -851,16 +851,26 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
                                            least, qh, s);
   if (e != cudaSuccess) return fail_cuda(e, "query normalisation launch");
 
+  // Many queries: clusters of two CTAs share each store tile (128 rows each).
+  const bool pair = Q >= kPairMinQueries;
   CUtensorMap tm_store, tm_q;
   CUresult r1 = encode_2d(&tm_store, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, store, K, N, ld_store * 2,
-                          kChunk, kScoreBN);
+                          kChunk, pair ? kScoreBN / 2 : kScoreBN);
   CUresult r2 = encode_2d(&tm_q, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, qh, K, Q, K * 2, kChunk, kScoreQT);
   if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS)
     return fail(BERGSON_ECUDA, "tensor map encoding failed (%d %d)", (int)r1, (int)r2);
 
-  const int sms = std::max(1, std::min(sm_count(dg.dev), kMaxScoreCTAs));
+  int sms = std::max(1, std::min(sm_count(dg.dev), kMaxScoreCTAs));
+  if (pair) {
+    int ctas = 0;
+    e = score_pair_max_ctas(sms, &ctas);
+    if (e != cudaSuccess) return fail_cuda(e, "score kernel occupancy query");
+    sms = std::min(sms, ctas) & ~1;
+    if (sms < 2) return fail(BERGSON_ECUDA, "no two-SM cluster fits the score kernel");
+  }
   const int gsize = L.qt * kScoreQT;
-  const int n_qg_total = static_cast<int>((Q + gsize - 1) / gsize);
+  int n_qg_total = static_cast<int>((Q + gsize - 1) / gsize);
+  if (pair) n_qg_total = (n_qg_total + 1) & ~1;   // whole pairs of query groups
   // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
   // lands in the outputs, and its k-th score seeds the full pass's threshold.
   const int64_t prefix = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
@@ -886,7 +896,8 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
       p.tau0 = stage == 1 && use_prefix ? out_scores : nullptr;
       p.status = status;
       p.timeout_ns = kWaitTimeoutNs;
-      e = launch_score(L.qt, tm_store, tm_q, p, grid, s);
+      e = pair ? launch_score_pair(tm_store, tm_q, p, grid, s)
+               : launch_score(L.qt, tm_store, tm_q, p, grid, s);
       if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
       // The prefix pass's scores seed the full pass's thresholds, so only
       // the final merge converts them back for a bottom-k search.

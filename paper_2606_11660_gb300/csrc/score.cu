@@ -117,6 +117,106 @@ __device__ __forceinline__ float select32(const float* v, uint32_t pos) {
   return (pos & 1u) ? t2[1] : t2[0];
 }
 
+// Epilogue role (QT x 128 threads, one query per thread): per store tile, wait
+// for the accumulators, read the query's 256 scores from TMEM, keep those above
+// its running k-th best, release TMEM (on the even CTA of a pair when kPair),
+// then insert the parked candidates into the query's heap in global memory.
+template <int QT, int kNBuf, bool kPair>
+__device__ __forceinline__ void score_epilogue(const ScoreParams& p, uint32_t tmem, uint64_t* tfull,
+                                               uint64_t* tempty,
+                                               unsigned long long* cand_queue,
+                                               volatile int* s_abort, volatile int* s_epi_stop,
+                                               int g, int nt0, int cpg, int warp, int lane,
+                                               uint64_t tmo) {
+  constexpr int kEpiThreads = QT * 128;
+  const int et = threadIdx.x - 64;                 // 0 .. QT*128-1
+  const int qt = et >> 7;
+  const int quarter = warp & 3;
+  const int slot = qt * kScoreQT + 32 * quarter + lane;
+  const int stride = kEpiThreads;
+  unsigned long long* heap =
+      p.heaps + static_cast<int64_t>(blockIdx.x) * p.topk * stride + slot;
+  for (int e = 0; e < p.topk; ++e) heap[static_cast<int64_t>(e) * stride] = kSentinelKey;
+  unsigned long long tau_key = kSentinelKey;
+  // Scores below the k-th best of any subset of the rows can never reach the
+  // final top-k, so a threshold from a prefix pass (if any) filters from the start.
+  const int q_global = (g * QT + qt) * kScoreQT + 32 * quarter + lane;
+  const float tau0 = (p.tau0 != nullptr && q_global < p.Q)
+                         ? p.tau0[static_cast<int64_t>(q_global) * p.topk + p.topk - 1]
+                         : -INFINITY;
+  float tau = tau0;
+  int nq = 0;                                       // parked candidates of this lane
+  int ab = 0;
+  uint32_t aph = 0;
+  for (int nt = nt0; nt < p.n_ntiles; nt += cpg) {
+    if (et == 0) {
+      if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
+        raise_device_error(p.status, s_abort, kStatusTimeout);
+      *s_epi_stop = *s_abort;
+    }
+    named_bar_sync(1, kEpiThreads);
+    if (*s_epi_stop) break;
+    tc_fence_after();
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
+                           ab * QT * kScoreBN + qt * kScoreBN;
+    const int row_base = nt * kScoreBN;
+#pragma unroll 1
+    for (int c = 0; c < kScoreBN / 32; ++c) {
+      float v[32];
+      tmem_ld32(tbase + c * 32, v);
+      const int r0 = row_base + c * 32;
+      const int nvalid = min(32, p.N - r0);
+      // Candidate positions of this lane (the comparison also drops NaN).
+      uint32_t cand = 0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nvalid && v[j] >= tau) cand |= 1u << j;
+      // Warp-uniform rounds: in round r every lane inserts its r-th candidate,
+      // so a warp pays for its busiest lane, not for every distinct column.
+      while (__any_sync(0xffffffffu, cand != 0)) {
+        if (cand != 0) {
+          const uint32_t pos = __ffs(cand) - 1;
+          cand &= cand - 1;
+          const unsigned long long key = make_key(select32(v, pos), static_cast<uint32_t>(r0) + pos);
+          if (key > tau_key) {
+            if (nq < kQueueCap) {                 // park it; inserted after TMEM is released
+              cand_queue[nq * stride + slot] = key;
+              ++nq;
+            } else {                              // queue full: insert now
+              heap_replace_root(heap, stride, p.topk, key);
+              tau_key = heap[0];
+              tau = fmaxf(tau0, order_to_float(static_cast<uint32_t>(tau_key >> 32)));
+            }
+          }
+        }
+      }
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) {
+      if (kPair)
+        mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[ab]), 0));
+      else
+        mbar_arrive(smem_u32(&tempty[ab]));
+    }
+    if (++ab == kNBuf) { ab = 0; aph ^= 1; }
+    // The MMA warp is already filling TMEM for the next tile; drain the parked
+    // candidates meanwhile (warp-uniform rounds, as above).
+    while (__any_sync(0xffffffffu, nq > 0)) {
+      if (nq > 0) {
+        --nq;
+        const unsigned long long key = cand_queue[nq * stride + slot];
+        if (key > tau_key) {
+          heap_replace_root(heap, stride, p.topk, key);
+          tau_key = heap[0];
+          tau = fmaxf(tau0, order_to_float(static_cast<uint32_t>(tau_key >> 32)));
+        }
+      }
+    }
+    named_bar_sync(1, kEpiThreads);   // keeps the stop broadcast single-writer
+  }
+}
+
 template <int QT>
 __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap tm_store, const __grid_constant__ CUtensorMap tm_q,
@@ -253,87 +353,8 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
     }
     __syncwarp();
   } else {
-    const int et = threadIdx.x - 64;                 // 0 .. QT*128-1
-    const int qt = et >> 7;
-    const int quarter = warp & 3;
-    const int slot = qt * kScoreQT + 32 * quarter + lane;
-    const int stride = C::kEpiThreads;
-    unsigned long long* heap =
-        p.heaps + static_cast<int64_t>(blockIdx.x) * p.topk * stride + slot;
-    for (int e = 0; e < p.topk; ++e) heap[static_cast<int64_t>(e) * stride] = kSentinelKey;
-    unsigned long long tau_key = kSentinelKey;
-    // Scores below the k-th best of any subset of the rows can never reach the
-    // final top-k, so a threshold from a prefix pass (if any) filters from the start.
-    const int q_global = (g * QT + qt) * kScoreQT + 32 * quarter + lane;
-    const float tau0 = (p.tau0 != nullptr && q_global < p.Q)
-                           ? p.tau0[static_cast<int64_t>(q_global) * p.topk + p.topk - 1]
-                           : -INFINITY;
-    float tau = tau0;
-    int nq = 0;                                       // parked candidates of this lane
-    int ab = 0;
-    uint32_t aph = 0;
-    for (int nt = nt0; nt < p.n_ntiles; nt += cpg) {
-      if (et == 0) {
-        if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
-          raise_device_error(p.status, s_abort, kStatusTimeout);
-        *s_epi_stop = *s_abort;
-      }
-      named_bar_sync(1, C::kEpiThreads);
-      if (*s_epi_stop) break;
-      tc_fence_after();
-      const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
-                             ab * QT * kScoreBN + qt * kScoreBN;
-      const int row_base = nt * kScoreBN;
-#pragma unroll 1
-      for (int c = 0; c < kScoreBN / 32; ++c) {
-        float v[32];
-        tmem_ld32(tbase + c * 32, v);
-        const int r0 = row_base + c * 32;
-        const int nvalid = min(32, p.N - r0);
-        // Candidate positions of this lane (the comparison also drops NaN).
-        uint32_t cand = 0;
-#pragma unroll
-        for (int j = 0; j < 32; ++j)
-          if (j < nvalid && v[j] >= tau) cand |= 1u << j;
-        // Warp-uniform rounds: in round r every lane inserts its r-th candidate,
-        // so a warp pays for its busiest lane, not for every distinct column.
-        while (__any_sync(0xffffffffu, cand != 0)) {
-          if (cand != 0) {
-            const uint32_t pos = __ffs(cand) - 1;
-            cand &= cand - 1;
-            const unsigned long long key = make_key(select32(v, pos), static_cast<uint32_t>(r0) + pos);
-            if (key > tau_key) {
-              if (nq < kQueueCap) {                 // park it; inserted after TMEM is released
-                cand_queue[nq * stride + slot] = key;
-                ++nq;
-              } else {                              // queue full: insert now
-                heap_replace_root(heap, stride, p.topk, key);
-                tau_key = heap[0];
-                tau = fmaxf(tau0, order_to_float(static_cast<uint32_t>(tau_key >> 32)));
-              }
-            }
-          }
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
-      if (++ab == C::kNBuf) { ab = 0; aph ^= 1; }
-      // The MMA warp is already filling TMEM for the next tile; drain the parked
-      // candidates meanwhile (warp-uniform rounds, as above).
-      while (__any_sync(0xffffffffu, nq > 0)) {
-        if (nq > 0) {
-          --nq;
-          const unsigned long long key = cand_queue[nq * stride + slot];
-          if (key > tau_key) {
-            heap_replace_root(heap, stride, p.topk, key);
-            tau_key = heap[0];
-            tau = fmaxf(tau0, order_to_float(static_cast<uint32_t>(tau_key >> 32)));
-          }
-        }
-      }
-      named_bar_sync(1, C::kEpiThreads);   // keeps the stop broadcast single-writer
-    }
+    score_epilogue<QT, C::kNBuf, false>(p, tmem, tfull, tempty, cand_queue, s_abort, s_epi_stop,
+                                        g, nt0, cpg, warp, lane, tmo);
   }
 
   tc_fence_before();
@@ -341,6 +362,183 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
+  }
+}
+
+// Pair variant for many queries (two query tiles per CTA, clusters of two
+// CTAs on two SMs).  One tcgen05.mma of M = 256 (the two CTAs' query tiles of
+// the same index) x N = 256 store rows serves both SMs: each CTA loads only
+// its half of the store tile (128 rows), and the tensor cores of the pair read
+// both halves.  Per SM and 16-column step this moves 12 KB into shared memory
+// and reads 16 KB out of it for two 128 x 256 products, against 16 KB and
+// 24 KB for the single-CTA kernel with the same two query tiles, which is what
+// limits that kernel's tensor pipe at this query count.
+//
+// Synchronisation: the odd CTA's TMA loads complete on the even CTA's `full`
+// barrier, which expects the bytes of both; the even CTA's MMA thread frees a
+// stage in both CTAs (commit multicast to `empty`), and signals both CTAs'
+// epilogues (commit multicast to `tfull`); both epilogues release the TMEM
+// buffer on the even CTA's `tempty`.
+constexpr int kPairStoreRows = kScoreBN / 2;               // store rows each CTA loads
+constexpr int kPairStoreBoxBytes = kPairStoreRows * 128;   // 128 rows x 64 fp16
+
+struct PairCfg {
+  static constexpr int QT = 2;
+  static constexpr int kStageBytes = kPairStoreBoxBytes + QT * kQBoxBytes;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kQueueBytes = kQueueCap * QT * 128 * 8;
+  static constexpr int kStagesFit = (kSmemBudget - 1024 - kBarBytes - kQueueBytes) / kStageBytes;
+  static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kQueueBytes + kBarBytes;
+  static constexpr int kNBuf = 1;
+  static constexpr int kEpiThreads = QT * 128;
+  static constexpr int kThreads = 64 + kEpiThreads;
+  static_assert(kStages >= 3, "pipeline depth");
+  static_assert(2 * kStages + 4 * kNBuf + 1 <= kBarBytes / 8 - 2, "barrier area");
+};
+
+// Bounded wait for this CTA's own TMA loads after an abort: the odd CTA's
+// loads complete on the other CTA's barrier, so it waits out a fixed time.
+__device__ __forceinline__ void pair_settle_loads() {
+  const uint64_t t0 = global_timer_ns();
+  while (global_timer_ns() - t0 < 1000000ull) {
+  }
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1)
+    score_pair_kernel(const __grid_constant__ CUtensorMap tm_store,
+                      const __grid_constant__ CUtensorMap tm_q, const ScoreParams p) {
+  using C = PairCfg;
+  constexpr int QT = C::QT;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  unsigned long long* cand_queue =
+      reinterpret_cast<unsigned long long*>(smem + C::kStages * C::kStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::kStages * C::kStageBytes + C::kQueueBytes);
+  uint64_t* empty = full + C::kStages;
+  uint64_t* tfull = empty + C::kStages;       // [kNBuf]
+  uint64_t* tempty = tfull + 2;               // [kNBuf]
+  uint64_t* drain = tempty + 2;
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+  volatile int* s_epi_stop = s_abort + 1;
+
+  const uint32_t rank = cluster_ctarank();   // 0: issues the MMAs
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int g_local = blockIdx.x % p.n_qg;   // even on rank 0, +1 on rank 1
+  const int g = p.qg_base + g_local;
+  const int cpg = gridDim.x / p.n_qg;
+  const int nt0 = blockIdx.x / p.n_qg;       // the same for both CTAs of the pair
+  const int nK = (p.K + kChunk - 1) / kChunk;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    mbar_init(smem_u32(&tfull[0]), 1);
+    mbar_init(smem_u32(&tempty[0]), 2 * QT * 4);   // every epilogue warp of both CTAs
+    mbar_init(smem_u32(drain), 1);
+    *s_abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(s_tmem), 512);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();              // both CTAs' barriers initialised and TMEM allocated
+  tc_fence_after();
+  const uint32_t tmem = *s_tmem;
+  const uint64_t tmo = p.timeout_ns;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tmap(&tm_store);
+      prefetch_tmap(&tm_q);
+      const uint64_t pol_store = kStoreEvictFirst ? policy_evict_first() : policy_evict_normal();
+      const uint64_t pol_q = policy_evict_last();
+      int stage = 0;
+      uint32_t ph = 0;
+      uint32_t issued = 0, issued_par = 0;
+      bool ok = true;
+      for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
+        for (int kc = 0; kc < nK; ++kc) {
+          if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
+          const uint32_t fb_local = smem_u32(&full[stage]);
+          const uint32_t fb = mapa_shared(fb_local, 0);
+          if (rank == 0) mbar_arrive_expect_tx(fb_local, 2 * C::kStageBytes);
+          const uint32_t dst = sbase + stage * C::kStageBytes;
+          tma_load_2d_pair(dst, &tm_store, fb, kc * kChunk,
+                           nt * kScoreBN + static_cast<int>(rank) * kPairStoreRows, pol_store);
+#pragma unroll
+          for (int qt = 0; qt < QT; ++qt)
+            tma_load_2d_pair(dst + kPairStoreBoxBytes + qt * kQBoxBytes, &tm_q, fb, kc * kChunk,
+                             (g * QT + qt) * kScoreQT, pol_q);
+          issued |= 1u << stage;
+          issued_par = (issued_par & ~(1u << stage)) | (ph << stage);
+          if (++stage == C::kStages) { stage = 0; ph ^= 1; }
+        }
+      }
+      if (!ok) {
+        raise_device_error(p.status, s_abort, kStatusTimeout);
+        if (rank == 0) {
+          for (int s = 0; s < C::kStages; ++s)
+            if (issued >> s & 1)
+              mbar_wait(smem_u32(&full[s]), (issued_par >> s) & 1, kDrainTimeoutNs, nullptr);
+        } else {
+          pair_settle_loads();
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (rank == 0 && lane == 0) {
+      const uint32_t idesc = make_idesc_f16(2 * kScoreQT, kScoreBN, false);
+      int stage = 0;
+      uint32_t ph = 0;
+      uint32_t aph = 0;
+      bool ok = true;
+      for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
+        if (!mbar_wait_cluster(smem_u32(&tempty[0]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+        tc_fence_after();
+        for (int kc = 0; kc < nK; ++kc) {
+          if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sd = sbase + stage * C::kStageBytes;
+          const uint32_t qd = sd + kPairStoreBoxBytes;
+#pragma unroll
+          for (int qt = 0; qt < QT; ++qt) {
+#pragma unroll
+            for (int kk = 0; kk < kChunk / 16; ++kk)
+              umma_f16_pair(tmem + qt * kScoreBN, sw128_desc(qd + qt * kQBoxBytes + kk * 32),
+                            sw128_desc(sd + kk * 32), idesc, (kc | kk) != 0);
+          }
+          umma_commit_pair(smem_u32(&empty[stage]), 0x3);
+          if (++stage == C::kStages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit_pair(smem_u32(&tfull[0]), 0x3);
+        aph ^= 1;
+      }
+      if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
+      umma_commit_pair(smem_u32(drain), 0x1);
+      mbar_wait(smem_u32(drain), 0, kDrainTimeoutNs, nullptr);
+    }
+    __syncwarp();
+  } else {
+    score_epilogue<QT, C::kNBuf, true>(p, tmem, tfull, tempty, cand_queue, s_abort, s_epi_stop, g,
+                                       nt0, cpg, warp, lane, tmo);
+  }
+
+  tc_fence_before();
+  cluster_sync();              // no MMA, commit or remote arrival is still in flight
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, 512);
   }
 }
 
@@ -503,6 +701,37 @@ cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap&
   if (qt == 1) return launch_score_t<1>(tm_store, tm_q, p, grid, s);
   if (qt == 2) return launch_score_t<2>(tm_store, tm_q, p, grid, s);
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_score_pair(const CUtensorMap& tm_store, const CUtensorMap& tm_q,
+                              const ScoreParams& p, int grid, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(score_pair_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         PairCfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  score_pair_kernel<<<grid, PairCfg::kThreads, PairCfg::kSmemBytes, s>>>(tm_store, tm_q, p);
+  return cudaGetLastError();
+}
+
+// CTAs of the pair kernel that can be resident at once (2 x co-resident clusters).
+cudaError_t score_pair_max_ctas(int sms, int* ctas) {
+  cudaError_t e = cudaFuncSetAttribute(score_pair_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       PairCfg::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * (sms / 2));
+  cfg.blockDim = dim3(PairCfg::kThreads);
+  cfg.dynamicSmemBytes = PairCfg::kSmemBytes;
+  int clusters = 0;
+  e = cudaOccupancyMaxActiveClusters(&clusters, score_pair_kernel, &cfg);
+  if (e != cudaSuccess) return e;
+  *ctas = 2 * clusters;
+  return cudaSuccess;
 }
 
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
