@@ -873,12 +873,17 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
   if (pair) n_qg_total = (n_qg_total + 1) & ~1;   // whole pairs of query groups
   // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
   // lands in the outputs, and its k-th score seeds the full pass's threshold.
-  const int64_t prefix = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
-  const bool use_prefix = N >= kPrefixMinFactor * prefix && Q >= kPrefixMinQueries;
+  const int64_t prefix_rows = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
+  const bool use_prefix = N >= kPrefixMinFactor * prefix_rows && Q >= kPrefixMinQueries;
   for (int pass = 0; pass < n_qg_total; pass += sms) {
     const int n_qg = std::min(sms, n_qg_total - pass);
     const int q_begin = pass * gsize;
     const int q_end = static_cast<int>(std::min<int64_t>(Q, static_cast<int64_t>(pass + n_qg) * gsize));
+    // The prefix is cut to whole rounds of store tiles over the CTAs of a
+    // query group (a partial second round would cost as much as a full one).
+    const int64_t round_rows = static_cast<int64_t>(sms / n_qg) * kScoreBN;
+    const int64_t prefix = prefix_rows > round_rows ? prefix_rows / round_rows * round_rows
+                                                    : prefix_rows;
     for (int stage = use_prefix ? 0 : 1; stage < 2; ++stage) {
       const int64_t rows = stage == 0 ? prefix : N;
       const int nt = static_cast<int>((rows + kScoreBN - 1) / kScoreBN);

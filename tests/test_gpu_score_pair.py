@@ -115,3 +115,24 @@ def test_pair_and_single_cta_kernels_agree():
     gap = np.abs(s1[:, :, None] - s1[:, None, :]) + np.eye(20)[None] * 1.0
     clear = gap.min(axis=2) > 1e-5          # entries without a near-tie partner
     assert np.all(i2[:256][clear] == i1[clear])
+
+
+def test_pair_scorer_prefix_cut_to_whole_tile_rounds():
+    # Q = 1024, topk = 100: the 12,800-row prefix is cut to one round of store
+    # tiles over the CTAs of a query group; strong neighbours sit just inside and
+    # just past the cut, and exact ties straddle it.
+    N, K, Q, topk = 110_000, 128, 1024, 100
+    g = wl.generator(91, "cpu")
+    rows = torch.randn((N, K), generator=g)
+    queries = torch.randn((Q, K), generator=g)
+    for q in range(0, Q, 16):
+        rows[9_000 + q] = queries[q] * 3.0 + torch.randn((K,), generator=g)
+        rows[12_000 + q] = queries[q] * 3.0 + torch.randn((K,), generator=g)
+    rows[13_500:13_510] = rows[9_700:9_710]
+    store = _store(rows)
+    s, i = _query(store, queries.to(DEV), topk)
+    S = orc.cosine_scores(store.cpu().numpy(), queries.numpy().astype(np.float64))
+    sample = np.r_[0:1024:16, 1:64]
+    check_topk(s[sample], i[sample], S[sample], topk)
+    for q in range(0, Q, 16):
+        assert {9_000 + q, 12_000 + q} <= set(i[q].tolist())
