@@ -647,7 +647,7 @@ def bench_scoring(args, world, dev, peaks, peak_kind):
                    "store_bytes": N * K * 2},
         "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": peak,
                      "unit": "TFLOP/s", "frac": round(tflops / peak, 4),
-                     "traffic": profiled_traffic("score_kernel_score4m.md", "score.cu"),
+                     "traffic": profiled_traffic("score_pair_kernel_score4m.md", "score.cu"),
                      "peak_source": f"{peak_kind} bf16_tflops (fp16 dense runs at the bf16 rate)",
                      "hbm_gbs_achieved": round(N * K * 2 / (ms * 1e-3) / 1e9, 1)},
         "gpu_launches": 5 * args.score_steps,   # query norm, 2 x (score, merge): prefix + full
