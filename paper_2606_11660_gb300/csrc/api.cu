@@ -479,7 +479,9 @@ struct ScoreLayout {
 
 ScoreLayout plan_score(int64_t K, int64_t Q, int64_t topk) {
   ScoreLayout L;
-  L.qt = Q > kScoreQT ? 2 : 1;
+  // Up to 128 queries: one tile per CTA, single-CTA kernel.  129..256: one
+  // tile per CTA of a pair.  More: two tiles per CTA of a pair.
+  L.qt = Q > 2 * kScoreQT ? 2 : 1;
   L.qh_off = 0;
   L.heap_off = round_up(static_cast<size_t>(Q) * K * sizeof(__half), 256);
   L.total = L.heap_off + round_up(static_cast<size_t>(kMaxScoreCTAs) * topk * L.qt * kScoreQT *
@@ -863,7 +865,7 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
   int sms = std::max(1, std::min(sm_count(dg.dev), kMaxScoreCTAs));
   if (pair) {
     int ctas = 0;
-    e = score_pair_max_ctas(sms, &ctas);
+    e = score_pair_max_ctas(L.qt, sms, &ctas);
     if (e != cudaSuccess) return fail_cuda(e, "score kernel occupancy query");
     sms = std::min(sms, ctas) & ~1;
     if (sms < 2) return fail(BERGSON_ECUDA, "no two-SM cluster fits the score kernel");
@@ -901,7 +903,7 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
       p.tau0 = stage == 1 && use_prefix ? out_scores : nullptr;
       p.status = status;
       p.timeout_ns = kWaitTimeoutNs;
-      e = pair ? launch_score_pair(tm_store, tm_q, p, grid, s)
+      e = pair ? launch_score_pair(L.qt, tm_store, tm_q, p, grid, s)
                : launch_score(L.qt, tm_store, tm_q, p, grid, s);
       if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
       // The prefix pass's scores seed the full pass's thresholds, so only

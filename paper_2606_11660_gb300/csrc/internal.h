@@ -148,12 +148,13 @@ cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q,
                                      __half* qh, cudaStream_t s);
 cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
                          const ScoreParams& p, int grid, cudaStream_t s);
-// Two-SM variant (clusters of two CTAs, 256 queries per CTA, 128 store rows per
-// CTA per tile): the store tensor map has 128-row boxes, grid and n_qg are even.
-cudaError_t launch_score_pair(const CUtensorMap& tm_store, const CUtensorMap& tm_q,
+// Two-SM variant (clusters of two CTAs, qt x 128 queries per CTA, 128 store
+// rows per CTA per tile): the store tensor map has 128-row boxes, grid and
+// n_qg are even.
+cudaError_t launch_score_pair(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
                               const ScoreParams& p, int grid, cudaStream_t s);
-cudaError_t score_pair_max_ctas(int sms, int* ctas);
-constexpr int kPairMinQueries = 257;   // the pair kernel serves Q >= this
+cudaError_t score_pair_max_ctas(int qt, int sms, int* ctas);
+constexpr int kPairMinQueries = 129;   // the pair kernel serves Q >= this
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
                          int q_begin, int q_end, int qg_base, bool negate, float* out_scores,
                          int64_t* out_idx, cudaStream_t s);

@@ -365,14 +365,15 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
   }
 }
 
-// Pair variant for many queries (two query tiles per CTA, clusters of two
-// CTAs on two SMs).  One tcgen05.mma of M = 256 (the two CTAs' query tiles of
-// the same index) x N = 256 store rows serves both SMs: each CTA loads only
+// Pair variant for more than 128 queries (QT query tiles per CTA, clusters of
+// two CTAs on two SMs).  One tcgen05.mma of M = 256 (the two CTAs' query tiles
+// of the same index) x N = 256 store rows serves both SMs: each CTA loads only
 // its half of the store tile (128 rows), and the tensor cores of the pair read
-// both halves.  Per SM and 16-column step this moves 12 KB into shared memory
-// and reads 16 KB out of it for two 128 x 256 products, against 16 KB and
-// 24 KB for the single-CTA kernel with the same two query tiles, which is what
-// limits that kernel's tensor pipe at this query count.
+// both halves.  With QT = 2 (more than 256 queries, tensor-bound) a 16-column
+// step moves 12 KB into shared memory and reads 16 KB out of it per SM for two
+// 128 x 256 products, against 16 KB and 24 KB for the single-CTA kernel.  With
+// QT = 1 (129..256 queries, bound by the store stream) the smaller stages give
+// six of them, i.e. more store bytes in flight per SM, and two TMEM buffers.
 //
 // Synchronisation: the odd CTA's TMA loads complete on the even CTA's `full`
 // barrier, which expects the bytes of both; the even CTA's MMA thread frees a
@@ -382,15 +383,16 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
 constexpr int kPairStoreRows = kScoreBN / 2;               // store rows each CTA loads
 constexpr int kPairStoreBoxBytes = kPairStoreRows * 128;   // 128 rows x 64 fp16
 
+template <int QT_>
 struct PairCfg {
-  static constexpr int QT = 2;
+  static constexpr int QT = QT_;
   static constexpr int kStageBytes = kPairStoreBoxBytes + QT * kQBoxBytes;
   static constexpr int kBarBytes = 256;
   static constexpr int kQueueBytes = kQueueCap * QT * 128 * 8;
   static constexpr int kStagesFit = (kSmemBudget - 1024 - kBarBytes - kQueueBytes) / kStageBytes;
   static constexpr int kStages = kStagesFit > 6 ? 6 : kStagesFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kQueueBytes + kBarBytes;
-  static constexpr int kNBuf = 1;
+  static constexpr int kNBuf = 512 / (QT * kScoreBN);   // TMEM accumulator buffers
   static constexpr int kEpiThreads = QT * 128;
   static constexpr int kThreads = 64 + kEpiThreads;
   static_assert(kStages >= 3, "pipeline depth");
@@ -405,11 +407,11 @@ __device__ __forceinline__ void pair_settle_loads() {
   }
 }
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1)
+template <int QT>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<QT>::kThreads, 1)
     score_pair_kernel(const __grid_constant__ CUtensorMap tm_store,
                       const __grid_constant__ CUtensorMap tm_q, const ScoreParams p) {
-  using C = PairCfg;
-  constexpr int QT = C::QT;
+  using C = PairCfg<QT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -439,8 +441,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
     }
-    mbar_init(smem_u32(&tfull[0]), 1);
-    mbar_init(smem_u32(&tempty[0]), 2 * QT * 4);   // every epilogue warp of both CTAs
+    for (int i = 0; i < C::kNBuf; ++i) {
+      mbar_init(smem_u32(&tfull[i]), 1);
+      mbar_init(smem_u32(&tempty[i]), 2 * QT * 4);   // every epilogue warp of both CTAs
+    }
     mbar_init(smem_u32(drain), 1);
     *s_abort = 0;
     fence_barrier_init();
@@ -500,11 +504,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
       const uint32_t idesc = make_idesc_f16(2 * kScoreQT, kScoreBN, false);
       int stage = 0;
       uint32_t ph = 0;
+      int ab = 0;
       uint32_t aph = 0;
       bool ok = true;
       for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
-        if (!mbar_wait_cluster(smem_u32(&tempty[0]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+        if (!mbar_wait_cluster(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
         tc_fence_after();
+        const uint32_t dbuf = tmem + ab * QT * kScoreBN;
         for (int kc = 0; kc < nK; ++kc) {
           if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) { ok = false; break; }
           tc_fence_after();
@@ -514,15 +520,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg::kThreads, 1
           for (int qt = 0; qt < QT; ++qt) {
 #pragma unroll
             for (int kk = 0; kk < kChunk / 16; ++kk)
-              umma_f16_pair(tmem + qt * kScoreBN, sw128_desc(qd + qt * kQBoxBytes + kk * 32),
+              umma_f16_pair(dbuf + qt * kScoreBN, sw128_desc(qd + qt * kQBoxBytes + kk * 32),
                             sw128_desc(sd + kk * 32), idesc, (kc | kk) != 0);
           }
           umma_commit_pair(smem_u32(&empty[stage]), 0x3);
           if (++stage == C::kStages) { stage = 0; ph ^= 1; }
         }
         if (!ok) break;
-        umma_commit_pair(smem_u32(&tfull[0]), 0x3);
-        aph ^= 1;
+        umma_commit_pair(smem_u32(&tfull[ab]), 0x3);
+        if (++ab == C::kNBuf) { ab = 0; aph ^= 1; }
       }
       if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
       umma_commit_pair(smem_u32(drain), 0x1);
@@ -703,35 +709,50 @@ cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap&
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_score_pair(const CUtensorMap& tm_store, const CUtensorMap& tm_q,
-                              const ScoreParams& p, int grid, cudaStream_t s) {
+template <int QT>
+cudaError_t launch_score_pair_t(const CUtensorMap& tm_store, const CUtensorMap& tm_q,
+                                const ScoreParams& p, int grid, cudaStream_t s) {
+  using C = PairCfg<QT>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(score_pair_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         PairCfg::kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(score_pair_kernel<QT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  score_pair_kernel<<<grid, PairCfg::kThreads, PairCfg::kSmemBytes, s>>>(tm_store, tm_q, p);
+  score_pair_kernel<QT><<<grid, C::kThreads, C::kSmemBytes, s>>>(tm_store, tm_q, p);
   return cudaGetLastError();
 }
 
-// CTAs of the pair kernel that can be resident at once (2 x co-resident clusters).
-cudaError_t score_pair_max_ctas(int sms, int* ctas) {
-  cudaError_t e = cudaFuncSetAttribute(score_pair_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       PairCfg::kSmemBytes);
+template <int QT>
+cudaError_t score_pair_max_ctas_t(int sms, int* ctas) {
+  using C = PairCfg<QT>;
+  cudaError_t e = cudaFuncSetAttribute(score_pair_kernel<QT>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * (sms / 2));
-  cfg.blockDim = dim3(PairCfg::kThreads);
-  cfg.dynamicSmemBytes = PairCfg::kSmemBytes;
+  cfg.blockDim = dim3(C::kThreads);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
   int clusters = 0;
-  e = cudaOccupancyMaxActiveClusters(&clusters, score_pair_kernel, &cfg);
+  e = cudaOccupancyMaxActiveClusters(&clusters, score_pair_kernel<QT>, &cfg);
   if (e != cudaSuccess) return e;
   *ctas = 2 * clusters;
   return cudaSuccess;
+}
+
+cudaError_t launch_score_pair(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
+                              const ScoreParams& p, int grid, cudaStream_t s) {
+  if (qt == 1) return launch_score_pair_t<1>(tm_store, tm_q, p, grid, s);
+  if (qt == 2) return launch_score_pair_t<2>(tm_store, tm_q, p, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+// CTAs of the pair kernel that can be resident at once (2 x co-resident clusters).
+cudaError_t score_pair_max_ctas(int qt, int sms, int* ctas) {
+  if (qt == 1) return score_pair_max_ctas_t<1>(sms, ctas);
+  if (qt == 2) return score_pair_max_ctas_t<2>(sms, ctas);
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,

@@ -1,9 +1,10 @@
-"""GPU parity of the two-SM scorer (queries >= 257: clusters of two CTAs, one
-tcgen05 MMA of M = 256 per pair, each CTA loading half of every store tile)
-against the fp64 oracle.
+"""GPU parity of the two-SM scorer (more than 128 queries: clusters of two
+CTAs, one tcgen05 MMA of M = 256 per pair, each CTA loading half of every
+store tile; one query tile per CTA up to 256 queries, two above) against the
+fp64 oracle.
 
-Cases: the smallest pair count (Q = 257: the odd CTA's second query tile
-and most of the even CTA's are empty), ragged query counts, stores whose
+Cases: the smallest pair counts (Q = 129: one query on the odd CTA; Q = 257:
+the odd CTA's second query tile and most of the even CTA's are empty), ragged query counts, stores whose
 last tile leaves the odd CTA's half partly or wholly past N, K not a
 multiple of 64, topk 1 to 100, the prefix-threshold path with ties across
 the prefix boundary, planted neighbours with known exact sets, the bottom-k
@@ -42,6 +43,8 @@ def _query(store, queries, k, entry=None):
 
 
 @pytest.mark.parametrize("N,K,Q,topk", [
+    (10_100, 1024, 129, 17),     # one query tile per CTA; the odd CTA holds one query
+    (5_020, 520, 256, 5),        # one query tile per CTA, both full
     (10_100, 1024, 257, 17),     # last tile: 100 rows, the odd CTA's half empty
     (5_020, 520, 600, 1),        # K % 64 != 0, ragged query groups
     (7_000 + 200, 256, 1024, 100),   # last tile 200 rows: the odd CTA's half partly valid
@@ -89,8 +92,9 @@ def test_pair_scorer_planted_neighbours_exact_set():
     check_topk(s, i, S, per)
 
 
-def test_pair_scorer_bottomk():
-    N, K, Q, k = 9_000, 384, 400, 10
+@pytest.mark.parametrize("Q", [200, 400])
+def test_pair_scorer_bottomk(Q):
+    N, K, k = 9_000, 384, 10
     g = wl.generator(71, "cpu")
     store = _store(torch.randn((N, K), generator=g))
     queries = torch.randn((Q, K), generator=g)
@@ -102,19 +106,21 @@ def test_pair_scorer_bottomk():
     np.testing.assert_array_equal(s, -ts)
 
 
-def test_pair_and_single_cta_kernels_agree():
-    # Q = 256 runs on the single-CTA kernel, Q = 257 on the pair kernel; the
-    # first 256 queries get the same rows and (to fp32 summation order) scores.
+@pytest.mark.parametrize("q_small,q_big", [(128, 129), (128, 257)])
+def test_pair_and_single_cta_kernels_agree(q_small, q_big):
+    # Q = 128 runs on the single-CTA kernel, Q = 129 on pairs with one query
+    # tile per CTA and Q = 257 on pairs with two; the shared queries get the
+    # same rows and (to fp32 summation order) the same scores.
     N, K = 20_000, 512
     g = wl.generator(81, "cpu")
     store = _store(torch.randn((N, K), generator=g))
-    queries = torch.randn((257, K), generator=g).to(DEV)
-    s1, i1 = _query(store, queries[:256].contiguous(), 20)
+    queries = torch.randn((q_big, K), generator=g).to(DEV)
+    s1, i1 = _query(store, queries[:q_small].contiguous(), 20)
     s2, i2 = _query(store, queries, 20)
-    np.testing.assert_allclose(s2[:256], s1, rtol=0, atol=2e-6)
+    np.testing.assert_allclose(s2[:q_small], s1, rtol=0, atol=2e-6)
     gap = np.abs(s1[:, :, None] - s1[:, None, :]) + np.eye(20)[None] * 1.0
     clear = gap.min(axis=2) > 1e-5          # entries without a near-tie partner
-    assert np.all(i2[:256][clear] == i1[clear])
+    assert np.all(i2[:q_small][clear] == i1[clear])
 
 
 def test_pair_scorer_prefix_cut_to_whole_tile_rounds():
