@@ -145,6 +145,9 @@ __device__ __forceinline__ void score_epilogue(const ScoreParams& p, uint32_t tm
                          ? p.tau0[static_cast<int64_t>(q_global) * p.topk + p.topk - 1]
                          : -INFINITY;
   float tau = tau0;
+  // Slots past the last query (ragged query groups) hold zero rows: they take
+  // no candidates, so their lanes do not walk every score of every tile.
+  const bool live = q_global < p.Q;
   int nq = 0;                                       // parked candidates of this lane
   int ab = 0;
   uint32_t aph = 0;
@@ -170,7 +173,7 @@ __device__ __forceinline__ void score_epilogue(const ScoreParams& p, uint32_t tm
       uint32_t cand = 0;
 #pragma unroll
       for (int j = 0; j < 32; ++j)
-        if (j < nvalid && v[j] >= tau) cand |= 1u << j;
+        if (live && j < nvalid && v[j] >= tau) cand |= 1u << j;
       // Warp-uniform rounds: in round r every lane inserts its r-th candidate,
       // so a warp pays for its busiest lane, not for every distinct column.
       while (__any_sync(0xffffffffu, cand != 0)) {
