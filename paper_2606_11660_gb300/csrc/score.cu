@@ -1,21 +1,25 @@
 // Exact cosine top-k over the gradient store (Bergson Sec. 3.1: exact top-k
 // nearest-neighbour lookup; queries score against unit-normalised rows).
 //
-// Score kernel (persistent, one CTA per SM): CTA c owns one query group of
+// Score kernels (persistent, one CTA per SM): a CTA owns one query group of
 // QT x 128 normalised fp16 queries and streams every (grid / n_qg)-th tile of
 // 256 store rows.  TMA brings 64-column slices of the store tile and of the
 // query tiles into a shared-memory ring; one thread issues tcgen05.mma with
-// M = 128 queries, N = 256 store rows, K = 16 into TMEM (fp32), so that TMEM
-// lane = query and column = store row.  Epilogue warps read their query's 256
+// the queries on M and N = 256 store rows, K = 16, into TMEM (fp32), so that
+// TMEM lane = query and column = store row.  Up to 128 queries one CTA runs
+// M = 128 on its own (score_kernel); above that CTAs run in pairs whose MMAs
+// take M = 256 over both CTAs' query tiles, each CTA loading half of every
+// store tile (score_pair_kernel).  Epilogue warps read their query's 256
 // scores, drop everything not above the query's running k-th best, and keep a
-// per-(CTA, query) binary min-heap of the k best (score, row) pairs in global
+// per-(CTA, query) 4-ary min-heap of the k best (score, row) keys in global
 // memory.  The N x Q score matrix never exists.
-// Merge kernel: one CTA per query sorts the heaps of the CTAs that covered the
-// query (bitonic sort of 64-bit keys in shared memory) and writes the final
-// top-k ordered by score descending, then row ascending.
-// Large stores are scored twice: first a prefix of 512*topk rows, whose exact
-// per-query k-th best is a lower bound of the final k-th best; the full pass
-// then starts with that threshold, so few scores ever reach the heaps.
+// Merge kernel: one CTA per query takes the heaps of the CTAs that covered the
+// query, finds the k-th best key by an exact radix select and sorts the top-k
+// by score descending, then row ascending.
+// Large stores are scored twice: first a prefix of about 128 x topk rows
+// (whole rounds of store tiles), whose exact per-query k-th best is a lower
+// bound of the final k-th best; the full pass then starts from that threshold,
+// so few scores ever reach the heaps.
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -29,10 +33,6 @@ constexpr uint64_t kDrainTimeoutNs = 2000000000ull;
 constexpr int kStoreBoxBytes = kScoreBN * 128;      // 256 rows x 64 fp16
 constexpr int kQBoxBytes = kScoreQT * 128;          // 128 rows x 64 fp16
 constexpr unsigned long long kSentinelKey = 0x007FFFFF00000000ull;   // (-inf, row 0xFFFFFFFF)
-// The first CTA of each group of CTAs that share store tiles pulls store chunks
-// into L2 this many chunks ahead of its own loads, so the shared-memory ring
-// sees L2 rather than DRAM latency (0 = no prefetch).
-constexpr int kStorePrefetchChunks = 0;
 // L2 policy of store-chunk loads: 0 = evict_normal, 1 = evict_first.
 constexpr int kStoreEvictFirst = 1;
 
@@ -277,26 +277,12 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
       prefetch_tmap(&tm_q);
       const uint64_t pol_store = kStoreEvictFirst ? policy_evict_first() : policy_evict_normal();
       const uint64_t pol_q = policy_evict_last();
-      const bool prefetcher = kStorePrefetchChunks > 0 && g_local == 0;
-      const int my_tiles = nt0 < p.n_ntiles ? (p.n_ntiles - nt0 + cpg - 1) / cpg : 0;
-      const int64_t my_chunks = static_cast<int64_t>(my_tiles) * nK;
-      if (prefetcher) {
-        for (int64_t c = 0; c < kStorePrefetchChunks && c < my_chunks; ++c)
-          tma_prefetch_l2_2d(&tm_store, static_cast<int>(c % nK) * kChunk,
-                             (nt0 + static_cast<int>(c / nK) * cpg) * kScoreBN);
-      }
       int stage = 0;
       uint32_t ph = 0;
       uint32_t issued = 0, issued_par = 0;
       bool ok = true;
-      int64_t lin = 0;                       // this CTA's chunk counter
       for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
-        for (int kc = 0; kc < nK; ++kc, ++lin) {
-          if (prefetcher && lin + kStorePrefetchChunks < my_chunks) {
-            const int64_t c = lin + kStorePrefetchChunks;
-            tma_prefetch_l2_2d(&tm_store, static_cast<int>(c % nK) * kChunk,
-                               (nt0 + static_cast<int>(c / nK) * cpg) * kScoreBN);
-          }
+        for (int kc = 0; kc < nK; ++kc) {
           if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_arrive_expect_tx(fb, C::kStageBytes);
