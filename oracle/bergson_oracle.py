@@ -31,7 +31,7 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
  10. bias gradients (App. B, "linear (weight and bias) parameters"):
      sum_t m_t g_t, scaled by r^-1/2 and projected with P_out (k_out values).
 
-Readings taken where the paper is silent (each is listed in the design doc):
+Readings taken where the paper is silent:
   * the projection is Gaussian with entries N(0, 1/k) per side, drawn from a
     stateless counter-based generator (SplitMix64 finaliser of Steele, Lea and
     Flood 2014, then the Box-Muller transform of Box and Muller 1958), entry
