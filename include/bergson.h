@@ -393,6 +393,23 @@ BERGSON_API int bergson_debug_project_plan(const bergson_layer* layers, int n_la
                                            int64_t* n_pieces, int64_t* n_shared);
 
 /*
+ * Test aid for the scorer's launch planner (bergson_score_topk and
+ * bergson_score_bottomk): the launches it would make for a store of N rows,
+ * Q queries and topk, on a device with `ctas` resident CTAs of the score
+ * kernel (the SM count, or for more than 128 queries twice the number of
+ * co-resident two-CTA clusters).  *n_launches receives the number of score
+ * launches (each followed by a merge); the first min(max_launches,
+ * *n_launches) are written to out as rows of 12 int64:
+ *   pass, stage (0 = prefix threshold pass, 1 = full pass), store rows,
+ *   query groups, first query group, CTAs per group, grid, store tiles,
+ *   first query, end query (of the merge), pair (1 = clusters of two CTAs),
+ *   128-query tiles per CTA.
+ * Host only: enqueues nothing.  Errors: EINVAL.
+ */
+BERGSON_API int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_t topk, int ctas,
+                                         int64_t* out, int max_launches, int* n_launches);
+
+/*
  * On-disk gradient store (Bergson Sec. 3.1: gradient stores persisted to disk,
  * read back as memory maps).  The file is N rows of K fp16 values, row-major,
  * with no header (numpy.memmap(path, dtype=float16, shape=(N, K)) opens it).

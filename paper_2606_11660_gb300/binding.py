@@ -47,7 +47,8 @@ EXPORTED = (
     "bergson_score_topk_workspace", "bergson_score_topk", "bergson_score_bottomk",
     "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
-    "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_debug_project_plan", "bergson_project_grads_noalloc",
+    "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_debug_project_plan",
+    "bergson_debug_score_plan", "bergson_project_grads_noalloc",
     "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
     "bergson_token_scores", "bergson_aggregate_rows_workspace", "bergson_aggregate_rows",
     "bergson_fisher_fit_workspace", "bergson_fisher_fit", "bergson_fisher_preconditioner_workspace",
@@ -106,6 +107,8 @@ def lib() -> ctypes.CDLL:
         "bergson_debug_wait_probe": (i32, [u64, vp]),
         "bergson_debug_inject_status": (None, [i32, i32]),
         "bergson_debug_project_plan": (i32, [lp, i32, i64, i64, i64p, i64p, i64p, i64p]),
+        "bergson_debug_score_plan": (i32, [i64, i64, i64, i64, i32, i64p, i32,
+                                           ctypes.POINTER(i32)]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
@@ -390,6 +393,22 @@ def bergson_debug_project_plan(layers, B: int, T: int) -> tuple[int, int, int, i
     _check(lib().bergson_debug_project_plan(arr, len(layers), int(B), int(T),
                                             *(ctypes.byref(x) for x in n)))
     return tuple(x.value for x in n)
+
+
+SCORE_PLAN_COLUMNS = ("pass", "stage", "rows", "n_qg", "qg_base", "cpg", "grid", "n_tiles",
+                      "q_begin", "q_end", "pair", "qt")
+
+
+def bergson_debug_score_plan(N: int, K: int, Q: int, topk: int, ctas: int) -> list[dict]:
+    """The score launches (one dict per launch, keys SCORE_PLAN_COLUMNS) the
+    scorer's planner makes for `ctas` resident CTAs; host only."""
+    n = ctypes.c_int32()
+    _check(lib().bergson_debug_score_plan(int(N), int(K), int(Q), int(topk), int(ctas), None, 0,
+                                          ctypes.byref(n)))
+    buf = (ctypes.c_int64 * (12 * max(1, n.value)))()
+    _check(lib().bergson_debug_score_plan(int(N), int(K), int(Q), int(topk), int(ctas), buf,
+                                          n.value, ctypes.byref(n)))
+    return [dict(zip(SCORE_PLAN_COLUMNS, buf[12 * i:12 * i + 12])) for i in range(n.value)]
 
 
 # ------------------------------------------------------------------ helpers

@@ -490,6 +490,71 @@ ScoreLayout plan_score(int64_t K, int64_t Q, int64_t topk) {
   return L;
 }
 
+// One score-kernel launch and the merge that follows it.
+struct ScoreLaunch {
+  int pass = 0;            // index of the pass over query groups
+  int stage = 1;           // 0 = prefix threshold pass, 1 = full pass
+  int64_t rows = 0;        // store rows this launch scores (a prefix, or N)
+  int n_qg = 0;            // query groups of this pass
+  int qg_base = 0;         // first query group of this pass
+  int cpg = 0;             // CTAs per query group
+  int grid = 0;            // n_qg * cpg
+  int n_tiles = 0;         // 256-row store tiles of `rows`
+  int q_begin = 0, q_end = 0;   // queries this launch's merge writes
+};
+
+struct ScoreLaunchPlan {
+  bool pair = false;       // clusters of two CTAs (more than 128 queries)
+  int qt = 1;              // 128-query tiles per CTA
+  int gsize = 0;           // queries per query group
+  int ctas = 0;            // resident CTAs the launches are sized for
+  bool use_prefix = false;
+  std::vector<ScoreLaunch> launches;
+};
+
+// Launch sequence of bergson_score_topk for `ctas` resident CTAs (for the pair
+// kernel: 2 x its co-resident clusters).  Pure host logic.
+ScoreLaunchPlan plan_score_launches(int64_t N, int64_t Q, int64_t topk, int ctas) {
+  ScoreLaunchPlan P;
+  const ScoreLayout L = plan_score(0, Q, topk);
+  P.pair = Q >= kPairMinQueries;
+  P.qt = L.qt;
+  P.gsize = L.qt * kScoreQT;
+  int sms = std::max(1, std::min(ctas, kMaxScoreCTAs));
+  if (P.pair) sms &= ~1;
+  P.ctas = sms;
+  if (Q <= 0 || (P.pair && sms < 2)) return P;
+  int n_qg_total = static_cast<int>((Q + P.gsize - 1) / P.gsize);
+  if (P.pair) n_qg_total = (n_qg_total + 1) & ~1;   // whole pairs of query groups
+  // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
+  // lands in the outputs, and its k-th score seeds the full pass's threshold.
+  const int64_t prefix_rows = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
+  P.use_prefix = N >= kPrefixMinFactor * prefix_rows && Q >= kPrefixMinQueries;
+  for (int pass = 0; pass < n_qg_total; pass += sms) {
+    const int n_qg = std::min(sms, n_qg_total - pass);
+    // The prefix is cut to whole rounds of store tiles over the CTAs of a
+    // query group (a partial second round would cost as much as a full one).
+    const int64_t round_rows = static_cast<int64_t>(sms / n_qg) * kScoreBN;
+    const int64_t prefix = prefix_rows > round_rows ? prefix_rows / round_rows * round_rows
+                                                    : prefix_rows;
+    for (int stage = P.use_prefix ? 0 : 1; stage < 2; ++stage) {
+      ScoreLaunch l;
+      l.pass = pass;
+      l.stage = stage;
+      l.rows = stage == 0 ? prefix : N;
+      l.n_qg = n_qg;
+      l.qg_base = pass;
+      l.n_tiles = static_cast<int>((l.rows + kScoreBN - 1) / kScoreBN);
+      l.cpg = std::max(1, std::min(sms / n_qg, l.n_tiles));
+      l.grid = n_qg * l.cpg;
+      l.q_begin = pass * P.gsize;
+      l.q_end = static_cast<int>(std::min<int64_t>(Q, static_cast<int64_t>(pass + n_qg) * P.gsize));
+      P.launches.push_back(l);
+    }
+  }
+  return P;
+}
+
 int validate_score(const void* store, int64_t N, int64_t K, int64_t ld_store, const float* queries,
                    int64_t Q, int64_t ld_q, int64_t topk) {
   if (N < 1 || N >= (1ll << 31)) return fail(BERGSON_EINVAL, "N must be in [1, 2^31)");
@@ -571,6 +636,24 @@ int bergson_debug_project_plan(const bergson_layer* layers, int n_layers, int64_
     int64_t sh = 0;
     for (uint8_t f : L.shared) sh += f;
     *n_shared = sh;
+  }
+  return BERGSON_OK;
+}
+
+int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_t topk, int ctas,
+                             int64_t* out, int max_launches, int* n_launches) {
+  if (n_launches == nullptr) return fail(BERGSON_EINVAL, "n_launches is NULL");
+  if (N < 1 || K < 8 || Q < 0 || topk < 1 || topk > kMaxTopk || topk > N || K % 8 != 0)
+    return fail(BERGSON_EINVAL, "invalid sizes for the score plan");
+  if (ctas < 1) return fail(BERGSON_EINVAL, "ctas must be >= 1");
+  const ScoreLaunchPlan P = plan_score_launches(N, Q, topk, ctas);
+  *n_launches = static_cast<int>(P.launches.size());
+  const int n = out == nullptr ? 0 : std::min(max_launches, *n_launches);
+  for (int i = 0; i < n; ++i) {
+    const ScoreLaunch& l = P.launches[i];
+    const int64_t row[12] = {l.pass, l.stage, l.rows, l.n_qg, l.qg_base, l.cpg,
+                             l.grid, l.n_tiles, l.q_begin, l.q_end, P.pair ? 1 : 0, P.qt};
+    for (int c = 0; c < 12; ++c) out[static_cast<int64_t>(i) * 12 + c] = row[c];
   }
   return BERGSON_OK;
 }
@@ -862,56 +945,36 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
   if (r1 != CUDA_SUCCESS || r2 != CUDA_SUCCESS)
     return fail(BERGSON_ECUDA, "tensor map encoding failed (%d %d)", (int)r1, (int)r2);
 
-  int sms = std::max(1, std::min(sm_count(dg.dev), kMaxScoreCTAs));
+  int ctas = sm_count(dg.dev);
   if (pair) {
-    int ctas = 0;
-    e = score_pair_max_ctas(L.qt, sms, &ctas);
+    int resident = 0;
+    e = score_pair_max_ctas(L.qt, std::max(1, std::min(ctas, kMaxScoreCTAs)), &resident);
     if (e != cudaSuccess) return fail_cuda(e, "score kernel occupancy query");
-    sms = std::min(sms, ctas) & ~1;
-    if (sms < 2) return fail(BERGSON_ECUDA, "no two-SM cluster fits the score kernel");
+    ctas = std::min(ctas, resident);
   }
-  const int gsize = L.qt * kScoreQT;
-  int n_qg_total = static_cast<int>((Q + gsize - 1) / gsize);
-  if (pair) n_qg_total = (n_qg_total + 1) & ~1;   // whole pairs of query groups
-  // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
-  // lands in the outputs, and its k-th score seeds the full pass's threshold.
-  const int64_t prefix_rows = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
-  const bool use_prefix = N >= kPrefixMinFactor * prefix_rows && Q >= kPrefixMinQueries;
-  for (int pass = 0; pass < n_qg_total; pass += sms) {
-    const int n_qg = std::min(sms, n_qg_total - pass);
-    const int q_begin = pass * gsize;
-    const int q_end = static_cast<int>(std::min<int64_t>(Q, static_cast<int64_t>(pass + n_qg) * gsize));
-    // The prefix is cut to whole rounds of store tiles over the CTAs of a
-    // query group (a partial second round would cost as much as a full one).
-    const int64_t round_rows = static_cast<int64_t>(sms / n_qg) * kScoreBN;
-    const int64_t prefix = prefix_rows > round_rows ? prefix_rows / round_rows * round_rows
-                                                    : prefix_rows;
-    for (int stage = use_prefix ? 0 : 1; stage < 2; ++stage) {
-      const int64_t rows = stage == 0 ? prefix : N;
-      const int nt = static_cast<int>((rows + kScoreBN - 1) / kScoreBN);
-      const int cpg = std::max(1, std::min(sms / n_qg, nt));
-      const int grid = n_qg * cpg;
-      ScoreParams p;
-      p.N = static_cast<int>(rows);
-      p.K = static_cast<int>(K);
-      p.Q = static_cast<int>(Q);
-      p.topk = static_cast<int>(topk);
-      p.n_qg = n_qg;
-      p.qg_base = pass;
-      p.n_ntiles = nt;
-      p.heaps = heaps;
-      p.tau0 = stage == 1 && use_prefix ? out_scores : nullptr;
-      p.status = status;
-      p.timeout_ns = kWaitTimeoutNs;
-      e = pair ? launch_score_pair(L.qt, tm_store, tm_q, p, grid, s)
-               : launch_score(L.qt, tm_store, tm_q, p, grid, s);
-      if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
-      // The prefix pass's scores seed the full pass's thresholds, so only
-      // the final merge converts them back for a bottom-k search.
-      e = launch_merge(heaps, grid, n_qg, L.qt, static_cast<int>(topk), q_begin, q_end, pass,
-                       least && stage == 1, out_scores, out_idx, s);
-      if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
-    }
+  const ScoreLaunchPlan P = plan_score_launches(N, Q, topk, ctas);
+  if (P.launches.empty()) return fail(BERGSON_ECUDA, "no two-SM cluster fits the score kernel");
+  for (const ScoreLaunch& l : P.launches) {
+    ScoreParams p;
+    p.N = static_cast<int>(l.rows);
+    p.K = static_cast<int>(K);
+    p.Q = static_cast<int>(Q);
+    p.topk = static_cast<int>(topk);
+    p.n_qg = l.n_qg;
+    p.qg_base = l.qg_base;
+    p.n_ntiles = l.n_tiles;
+    p.heaps = heaps;
+    p.tau0 = l.stage == 1 && P.use_prefix ? out_scores : nullptr;
+    p.status = status;
+    p.timeout_ns = kWaitTimeoutNs;
+    e = pair ? launch_score_pair(L.qt, tm_store, tm_q, p, l.grid, s)
+             : launch_score(L.qt, tm_store, tm_q, p, l.grid, s);
+    if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
+    // The prefix pass's scores seed the full pass's thresholds, so only
+    // the final merge converts them back for a bottom-k search.
+    e = launch_merge(heaps, l.grid, l.n_qg, L.qt, static_cast<int>(topk), l.q_begin, l.q_end,
+                     l.pass, least && l.stage == 1, out_scores, out_idx, s);
+    if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
   }
   return BERGSON_OK;
 }

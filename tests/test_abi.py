@@ -299,3 +299,71 @@ def test_planner_groups_layers_that_share_an_input():
     c = _layer(A=a.A, d_in=64, d_out=64, k_in=32, out_col_offset=512)
     assert _plan([a, b, c], 2, 32)[3] == 0
     assert _plan([a, _layer(A=a.A, d_in=64, d_out=64, out_col_offset=256)], 2, 32)[3] == 2
+
+
+# --- scorer launch planning (host only) ---------------------------------------
+
+@pytest.mark.parametrize("N,Q,topk,ctas", [
+    (4_000_000, 1024, 100, 152),     # the score4m workload: pairs, two tiles, prefix cut
+    (4_000_000, 1024, 100, 148),     # fewer co-resident clusters
+    (4_000_000, 256, 100, 152),      # pairs with one tile per CTA
+    (4_000_000, 16, 100, 152),       # single-CTA kernel, no prefix
+    (110_000, 1024, 100, 152),       # prefix cut to one round of tiles
+    (10_000, 129, 17, 152),
+    (30_000, 300, 3, 151),           # odd resident count: pairs use 150 CTAs
+    (1000, 39_012, 5, 152),          # more query groups than CTAs: several passes
+    (1000, 39_012, 5, 150),
+    (60_000, 300, 1024, 152),        # the largest topk
+    (300, 511, 300, 152),            # topk = N
+    (5000, 256, 5, 7),               # few resident CTAs
+    (1, 1, 1, 1),
+])
+def test_score_planner_invariants(N, Q, topk, ctas):
+    K = 64
+    plan = bg.bergson_debug_score_plan(N, K, Q, topk, ctas)
+    assert plan
+    pair, qt = Q >= 129, (2 if Q > 256 else 1)
+    gsize = qt * 128
+    limit = min(ctas, 160) & (~1 if pair else ~0)
+    n_qg_total = -(-Q // gsize)
+    if pair:
+        n_qg_total += n_qg_total % 2
+    covered = []
+    passes = sorted({l["pass"] for l in plan})
+    assert passes == list(range(0, n_qg_total, limit))
+    for l in plan:
+        assert (l["pair"], l["qt"]) == (int(pair), qt)
+        assert l["grid"] == l["n_qg"] * l["cpg"] <= limit
+        assert l["n_tiles"] == -(-l["rows"] // 256) and 1 <= l["cpg"] <= l["n_tiles"]
+        assert l["qg_base"] == l["pass"] and l["q_begin"] == l["pass"] * gsize
+        assert 0 < l["q_end"] - l["q_begin"] <= l["n_qg"] * gsize
+        if pair:                             # whole clusters, pairs of query groups
+            assert l["grid"] % 2 == 0 and l["n_qg"] % 2 == 0 and l["qg_base"] % 2 == 0
+        if l["stage"] == 1:
+            assert l["rows"] == N
+            covered += range(l["q_begin"], l["q_end"])
+        else:                                # prefix: enough rows for a real k-th best
+            round_rows = (limit // l["n_qg"]) * 256
+            want = -(-128 * topk // 256) * 256
+            assert topk <= l["rows"] <= want and l["rows"] % 256 == 0
+            assert l["rows"] == want or l["rows"] % round_rows == 0
+            assert 8 * want <= N and Q >= 129
+    assert covered == list(range(Q))         # every query merged exactly once
+    stages = [(l["pass"], l["stage"]) for l in plan]
+    assert stages == sorted(stages)          # prefix (if any) before its full pass
+    n = ctypes.c_size_t()
+    assert bg.lib().bergson_score_topk_workspace(N, K, Q, topk, ctypes.byref(n)) == bg.BERGSON_OK
+    heaps = max(l["grid"] for l in plan) * topk * gsize * 8
+    assert n.value >= heaps + Q * K * 2
+
+
+def test_score_planner_edges():
+    # a single resident CTA cannot host a two-CTA cluster: no launches (the
+    # scoring call reports it as an error)
+    assert bg.bergson_debug_score_plan(10_000, 64, 200, 5, 1) == []
+    assert len(bg.bergson_debug_score_plan(10_000, 64, 100, 5, 1)) == 1
+    assert bg.bergson_debug_score_plan(10_000, 64, 0, 5, 152) == []
+    with pytest.raises(bg.BergsonError):
+        bg.bergson_debug_score_plan(10, 64, 4, 11, 152)      # topk > N
+    with pytest.raises(bg.BergsonError):
+        bg.bergson_debug_score_plan(10_000, 64, 4, 5, 0)
