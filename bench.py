@@ -933,7 +933,7 @@ def parse(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--score-steps", type=int, default=5)
     ap.add_argument("--score-warmup", type=int, default=2)
-    ap.add_argument("--cpu-examples", type=int, default=4)
+    ap.add_argument("--cpu-examples", type=int, default=12)
     ap.add_argument("--no-fisher", action="store_true")
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
