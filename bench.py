@@ -822,8 +822,10 @@ def profile_case(args):
         st = bg.bergson_sync_status()
     else:
         # 409,600-row fp16 store x 8192 (6.7 GB, large enough for the prefix
-        # threshold pass), 1024 queries, top-100
-        N, K, Q, topk = 409_600, 8192, 1024, 100
+        # threshold pass), 1024 queries (score) or 256 queries (score_mid: the
+        # pair kernel with one query tile per CTA), top-100
+        N, K, topk = 409_600, 8192, 100
+        Q = 256 if args.profile_case == "score_mid" else 1024
         store = torch.empty((N, K), dtype=torch.float16, device=dev)
         for n0 in range(0, N, 1 << 16):
             n1 = min(N, n0 + (1 << 16))
@@ -938,7 +940,8 @@ def parse(argv=None):
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--fisher-iters", type=int, default=20)
-    ap.add_argument("--profile-case", choices=["collect", "score", "tokens", "onthefly", "apply", "fisher",
+    ap.add_argument("--profile-case", choices=["collect", "score", "score_mid", "tokens", "onthefly",
+                                               "apply", "fisher",
                              "streamed_pythia1b4", "streamed_llama8b"],
                     default=None,
                     help="run a small case of one kernel for ncu and exit")
