@@ -14,7 +14,8 @@ from .binding import (  # noqa: F401
     BERGSON_EWORKSPACE, BERGSON_OK, BERGSON_PROJ_GAUSSIAN, BERGSON_PROJ_IDENTITY,
     BERGSON_PROJ_RADEMACHER, BERGSON_PROJ_UNIFORM, BergsonError,
     EXPORTED, LIB_PATH, Layer, bergson_build_store, bergson_debug_inject_status,
-    bergson_debug_project_plan, bergson_debug_score_plan, bergson_debug_wait_probe, bergson_last_error, bergson_module_seeds, bergson_project_grads,
+    bergson_debug_project_plan, bergson_debug_score_plan, bergson_debug_xgemm_plan,
+    bergson_debug_wait_probe, bergson_last_error, bergson_module_seeds, bergson_project_grads,
     bergson_project_grads_noalloc, bergson_project_grads_workspace, bergson_projection_matrix, bergson_score_topk,
     bergson_score_bottomk,
     bergson_score_topk_workspace, bergson_score_grads, bergson_score_grads_workspace,

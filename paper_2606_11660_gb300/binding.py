@@ -48,7 +48,7 @@ EXPORTED = (
     "bergson_projection_matrix",
     "bergson_module_seeds", "bergson_sync_status", "bergson_last_error", "bergson_version",
     "bergson_debug_wait_probe", "bergson_debug_inject_status", "bergson_debug_project_plan",
-    "bergson_debug_score_plan", "bergson_project_grads_noalloc",
+    "bergson_debug_score_plan", "bergson_debug_xgemm_plan", "bergson_project_grads_noalloc",
     "bergson_score_grads_workspace", "bergson_score_grads", "bergson_token_scores_workspace",
     "bergson_token_scores", "bergson_aggregate_rows_workspace", "bergson_aggregate_rows",
     "bergson_fisher_fit_workspace", "bergson_fisher_fit", "bergson_fisher_preconditioner_workspace",
@@ -109,6 +109,7 @@ def lib() -> ctypes.CDLL:
         "bergson_debug_project_plan": (i32, [lp, i32, i64, i64, i64p, i64p, i64p, i64p]),
         "bergson_debug_score_plan": (i32, [i64, i64, i64, i64, i32, i64p, i32,
                                            ctypes.POINTER(i32)]),
+        "bergson_debug_xgemm_plan": (i32, [i64, i64, i64, i64p, i32]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
@@ -409,6 +410,18 @@ def bergson_debug_score_plan(N: int, K: int, Q: int, topk: int, ctas: int) -> li
     _check(lib().bergson_debug_score_plan(int(N), int(K), int(Q), int(topk), int(ctas), buf,
                                           n.value, ctypes.byref(n)))
     return [dict(zip(SCORE_PLAN_COLUMNS, buf[12 * i:12 * i + 12])) for i in range(n.value)]
+
+
+XGEMM_PLAN_FIELDS = ("n_pad", "n_ntiles", "n_mtiles", "steps", "S", "stages", "n_chunks",
+                     "tmem_a", "n_buf", "a_base", "tmem_cols", "xnorm_off", "ynorm_off",
+                     "partial_off", "xh_off", "xl_off", "total")
+
+
+def bergson_debug_xgemm_plan(B: int, Q: int, K: int) -> dict:
+    """The skinny-product planner's choices for B x rows, Q y rows, length K; host only."""
+    buf = (ctypes.c_int64 * 17)()
+    _check(lib().bergson_debug_xgemm_plan(int(B), int(Q), int(K), buf, 17))
+    return dict(zip(XGEMM_PLAN_FIELDS, buf))
 
 
 # ------------------------------------------------------------------ helpers

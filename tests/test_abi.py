@@ -367,3 +367,57 @@ def test_score_planner_edges():
         bg.bergson_debug_score_plan(10, 64, 4, 11, 152)      # topk > N
     with pytest.raises(bg.BergsonError):
         bg.bergson_debug_score_plan(10_000, 64, 4, 5, 0)
+
+
+# --- skinny-product planning (host only) --------------------------------------
+
+@pytest.mark.parametrize("B,Q,K", [
+    (32, 1024, 12288),      # on-the-fly scores of the bench batch
+    (32, 12288, 12288),     # Fisher preconditioner applied to a batch
+    (1024, 12288, 12288),   # Fisher fit (rows as x)
+    (12288, 12288, 12288),  # Newton-Schulz products
+    (1, 1, 8), (16, 1, 4), (64, 100, 400), (65, 100, 400), (129, 300, 4096),
+    (1000, 7, 520), ((1 << 20), 3, 64),
+])
+def test_xgemm_planner_invariants(B, Q, K):
+    p = bg.bergson_debug_xgemm_plan(B, Q, K)
+    # tiles cover the operands
+    assert p["n_pad"] % 16 == 0 and 16 <= p["n_pad"] <= 128
+    assert p["n_ntiles"] * p["n_pad"] >= B > (p["n_ntiles"] - 1) * p["n_pad"]
+    assert p["n_mtiles"] * 128 >= Q > (p["n_mtiles"] - 1) * 128
+    assert p["steps"] * 32 >= K > (p["steps"] - 1) * 32
+    # every K slice is a nonempty, contiguous range of steps
+    S, steps = p["S"], p["steps"]
+    assert 1 <= S <= min(steps, 64)
+    bounds = [z * steps // S for z in range(S + 1)]
+    assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
+    # TMEM: accumulators (3 n_pad columns per buffer) and, with y in TMEM, the
+    # 64-column operand ring, within 512 columns
+    acc = p["n_buf"] * 3 * p["n_pad"]
+    assert p["tmem_a"] == (p["n_pad"] <= 64) and p["n_buf"] in (1, 2)
+    assert p["tmem_cols"] <= 512 and p["tmem_cols"] & (p["tmem_cols"] - 1) == 0
+    if p["tmem_a"]:
+        assert p["a_base"] >= acc and p["a_base"] % 32 == 0
+        assert p["a_base"] + p["stages"] * 64 <= p["tmem_cols"] == 512
+    else:
+        assert acc <= p["tmem_cols"]
+    # shared memory: stages of one y tile (and y_lo unless it is in TMEM) plus x_hi, x_lo
+    stage = (1 if p["tmem_a"] else 2) * 128 * 128 + 2 * p["n_pad"] * 128
+    assert 2 <= p["stages"] <= 8 and 1024 + 512 + p["stages"] * stage <= 232448
+    # workspace: ordered, 256-byte aligned regions of the stated sizes
+    offs = [p[k] for k in ("xnorm_off", "ynorm_off", "partial_off", "xh_off", "xl_off", "total")]
+    assert all(o % 256 == 0 for o in offs) and offs == sorted(offs)
+    assert p["ynorm_off"] - p["xnorm_off"] >= 4 * B * p["n_chunks"]
+    assert p["n_chunks"] == -(-K // 2048)
+    assert p["partial_off"] - p["ynorm_off"] >= 4 * S * Q
+    assert p["xh_off"] - p["partial_off"] >= 4 * S * B * Q
+    assert p["xl_off"] - p["xh_off"] >= 4 * B * K and p["total"] - p["xl_off"] >= 4 * B * K
+    n = ctypes.c_size_t()
+    assert bg.lib().bergson_score_grads_workspace(B, K, Q, ctypes.byref(n)) == bg.BERGSON_OK
+    assert n.value == p["total"]
+
+
+def test_xgemm_planner_validation():
+    for args in [(0, 4, 8), (4, 0, 8), (4, 4, 6), (4, 4, 2), ((1 << 20) + 1, 4, 8)]:
+        with pytest.raises(bg.BergsonError):
+            bg.bergson_debug_xgemm_plan(*args)
