@@ -319,6 +319,10 @@ def test_planner_groups_layers_that_share_an_input():
     (1, 1, 1, 1),
 ])
 def test_score_planner_invariants(N, Q, topk, ctas):
+    check_score_plan(N, Q, topk, ctas)
+
+
+def check_score_plan(N, Q, topk, ctas):
     K = 64
     plan = bg.bergson_debug_score_plan(N, K, Q, topk, ctas)
     assert plan
@@ -380,6 +384,10 @@ def test_score_planner_edges():
     (1000, 7, 520), ((1 << 20), 3, 64),
 ])
 def test_xgemm_planner_invariants(B, Q, K):
+    check_xgemm_plan(B, Q, K)
+
+
+def check_xgemm_plan(B, Q, K):
     p = bg.bergson_debug_xgemm_plan(B, Q, K)
     # tiles cover the operands
     assert p["n_pad"] % 16 == 0 and 16 <= p["n_pad"] <= 128
@@ -421,3 +429,26 @@ def test_xgemm_planner_validation():
     for args in [(0, 4, 8), (4, 0, 8), (4, 4, 6), (4, 4, 2), ((1 << 20) + 1, 4, 8)]:
         with pytest.raises(bg.BergsonError):
             bg.bergson_debug_xgemm_plan(*args)
+
+
+def test_planners_on_random_shapes():
+    """The same invariants over a few hundred random shapes (host only)."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=300, deadline=None, derandomize=True)
+    @hyp.given(N=st.integers(1, 5_000_000), Q=st.integers(1, 50_000), topk=st.integers(1, 1024),
+               ctas=st.integers(1, 200))
+    def score(N, Q, topk, ctas):
+        hyp.assume(topk <= N)
+        pair_ok = Q < 129 or min(ctas, 160) >= 2
+        if pair_ok:
+            check_score_plan(N, Q, topk, ctas)
+
+    @hyp.settings(max_examples=300, deadline=None, derandomize=True)
+    @hyp.given(B=st.integers(1, 1 << 20), Q=st.integers(1, 1 << 16), K4=st.integers(1, 1 << 16))
+    def xgemm(B, Q, K4):
+        check_xgemm_plan(B, Q, 4 * K4)
+
+    score()
+    xgemm()
