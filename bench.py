@@ -6,7 +6,11 @@ bergson_project_grads over every module, then bergson_build_store appends the
 32 unit-normalised fp16 rows.  value = examples/s over all ranks.
 
 The scoring phase of the same path (fp16 store of 4,000,000 x 8192 rows,
-1,024 queries, top-100) is timed separately and reported under "scoring".
+1,024 queries, top-100) is timed separately and reported under "scoring",
+with a sweep over 1-512 queries on the same store ("q_sweep").  The other
+rows of the path (on-the-fly scores, per-token scores, the Fisher
+preconditioner, one-block-per-call Pythia-1.4B and Llama-8B shapes) and an
+end-to-end leg from pinned host memory are reported beside it.
 
 --impl reference times the fp64 CPU oracle on the host cores instead (a
 bounded sample of the same workload per step).  Under torchrun every rank runs
