@@ -166,6 +166,57 @@ def cpu_worker(n_examples: int, repeat: int, out_path: str):
         json.dump({"times": times, "n_examples": n_examples}, f)
 
 
+def cpu_score_worker(n_rows: int, n_queries: int, budget_s: float, out_path: str):
+    """Times the oracle's brute-force scoring (fp64 cosines of every query
+    against every row, then the full-sort top-100) on a sample of the score4m
+    workload: n_rows unit-normalised N(0, I_8192) fp16 rows and n_queries
+    N(0, I) queries.  Repeats the call until budget_s has passed (at least twice)."""
+    import numpy as np
+
+    from oracle import bergson_oracle as orc
+    from paper_2606_11660_gb300 import workloads as wl
+
+    sw = wl.SCORE4M
+    store, _ = orc.build_store(wl.gaussian_rows(n_rows, sw.K, seed=7).numpy())
+    queries = wl.gaussian_rows(n_queries, sw.K, seed=8).numpy().astype(np.float64)
+    times = []
+    t_start = time.perf_counter()
+    while len(times) < 2 or time.perf_counter() - t_start < budget_s:
+        t0 = time.perf_counter()
+        orc.score_topk(store, queries, sw.topk)
+        times.append(time.perf_counter() - t0)
+    with open(out_path, "w") as f:
+        json.dump({"times": times, "n_rows": n_rows, "n_queries": n_queries}, f)
+
+
+def run_cpu_score_oracle(n_rows: int, n_queries: int, budget_s: float):
+    cores = len(os.sched_getaffinity(0))
+    env = dict(os.environ)
+    for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = str(cores)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    out = os.path.join("/tmp", f"bergson_cpu_score_{os.getpid()}.json")
+    subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-score-worker", str(n_rows),
+                    str(n_queries), str(budget_s), out], env=env, check=True)
+    with open(out) as f:
+        res = json.load(f)
+    os.unlink(out)
+    return res["times"], cores
+
+
+def scoring_cpu_baseline(n_rows: int = 65_536, n_queries: int = 8, budget_s: float = 10.0):
+    """The oracle's scoring rate on the host cores, as (row x query)/s measured
+    and as store rows/s extrapolated linearly to the bench's 1,024 queries."""
+    times, cores = run_cpu_score_oracle(n_rows, n_queries, budget_s)
+    t = statistics.median(times)
+    rq = n_rows * n_queries / t
+    return {"value": round(rq / 1024, 1), "unit": "store rows/s",
+            "row_query_per_s": round(rq), "cores": cores, "kind": "oracle",
+            "sample": f"{n_queries} queries x {n_rows} unit-normalised N(0, I_8192) fp16 rows: "
+                      f"fp64 cosines + full-sort top-100, median of {len(times)} calls "
+                      f"({t:.2f} s each); value extrapolated linearly to 1024 queries"}
+
+
 def run_cpu_oracle(n_examples: int, repeat: int):
     cores = len(os.sched_getaffinity(0))
     env = dict(os.environ)
@@ -871,6 +922,12 @@ def main_ours(args):
         streamed = {n: bench_streamed(args, world, dev, n, peaks) for n in ("pythia1b4", "llama8b")}
     scoring = bench_scoring(args, world, dev, peaks, peak_kind) if not args.no_score else None
     cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu and scoring is not None:
+        try:
+            scoring["cpu_baseline"] = scoring_cpu_baseline(budget_s=6.0)
+        except (OSError, subprocess.SubprocessError, ValueError) as exc:
+            scoring["cpu_baseline"] = {"value": None, "kind": "oracle",
+                                       "error": f"{type(exc).__name__}: {exc}"[:300]}
     if rank == 0 and world == 1 and not args.no_cpu:
         times, cores = run_cpu_oracle(args.cpu_examples, 1)
         cpu = {"value": args.cpu_examples / times[0], "unit": "examples/s", "cores": cores,
@@ -955,6 +1012,9 @@ def parse(argv=None):
 if __name__ == "__main__":
     if len(sys.argv) > 1 and sys.argv[1] == "--cpu-worker":
         cpu_worker(int(sys.argv[2]), int(sys.argv[3]), sys.argv[4])
+        sys.exit(0)
+    if len(sys.argv) > 1 and sys.argv[1] == "--cpu-score-worker":
+        cpu_score_worker(int(sys.argv[2]), int(sys.argv[3]), float(sys.argv[4]), sys.argv[5])
         sys.exit(0)
     a = parse()
     if a.profile_case is not None:
