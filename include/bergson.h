@@ -166,7 +166,8 @@ BERGSON_API int bergson_build_store(const float* proj, int64_t B, int64_t K, int
                         int unit_normalize, void* store, int64_t ld_store,
                         int64_t row_offset, int64_t N_cap, float* norms_out, void* stream);
 
-/* Bytes of workspace bergson_score_topk needs. */
+/* Bytes of workspace bergson_score_topk (and bergson_score_bottomk) needs;
+ * N, K, Q and topk follow the calls' size rules (EINVAL, EALIGN, EUNSUPPORTED). */
 BERGSON_API int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes);
 
 /*

@@ -555,8 +555,8 @@ ScoreLaunchPlan plan_score_launches(int64_t N, int64_t Q, int64_t topk, int ctas
   return P;
 }
 
-int validate_score(const void* store, int64_t N, int64_t K, int64_t ld_store, const float* queries,
-                   int64_t Q, int64_t ld_q, int64_t topk) {
+// Size rules shared by the scoring calls and their workspace query.
+int validate_score_sizes(int64_t N, int64_t K, int64_t Q, int64_t topk) {
   if (N < 1 || N >= (1ll << 31)) return fail(BERGSON_EINVAL, "N must be in [1, 2^31)");
   if (K < 8 || K > (1ll << 24)) return fail(BERGSON_EINVAL, "K must be in [8, 2^24]");
   if (K % 8 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 8");
@@ -564,6 +564,13 @@ int validate_score(const void* store, int64_t N, int64_t K, int64_t ld_store, co
   if (topk < 1 || topk > kMaxTopk)
     return fail(BERGSON_EUNSUPPORTED, "topk must be in [1, %d]", kMaxTopk);
   if (topk > N) return fail(BERGSON_EINVAL, "topk (%lld) > N (%lld)", (long long)topk, (long long)N);
+  return BERGSON_OK;
+}
+
+int validate_score(const void* store, int64_t N, int64_t K, int64_t ld_store, const float* queries,
+                   int64_t Q, int64_t ld_q, int64_t topk) {
+  const int st = validate_score_sizes(N, K, Q, topk);
+  if (st != BERGSON_OK) return st;
   if (ld_store < K || ld_store % 8 != 0)
     return fail(ld_store < K ? BERGSON_EINVAL : BERGSON_EALIGN,
                 "ld_store must be >= K and a multiple of 8");
@@ -643,8 +650,8 @@ int bergson_debug_project_plan(const bergson_layer* layers, int n_layers, int64_
 int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_t topk, int ctas,
                              int64_t* out, int max_launches, int* n_launches) {
   if (n_launches == nullptr) return fail(BERGSON_EINVAL, "n_launches is NULL");
-  if (N < 1 || K < 8 || Q < 0 || topk < 1 || topk > kMaxTopk || topk > N || K % 8 != 0)
-    return fail(BERGSON_EINVAL, "invalid sizes for the score plan");
+  const int st = validate_score_sizes(N, K, Q, topk);
+  if (st != BERGSON_OK) return st;
   if (ctas < 1) return fail(BERGSON_EINVAL, "ctas must be >= 1");
   const ScoreLaunchPlan P = plan_score_launches(N, Q, topk, ctas);
   *n_launches = static_cast<int>(P.launches.size());
@@ -908,8 +915,8 @@ int bergson_build_store(const float* proj, int64_t B, int64_t K, int64_t ld_proj
 
 int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes) {
   if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
-  if (N < 1 || K < 8 || Q < 0 || topk < 1 || topk > kMaxTopk || topk > N || K % 8 != 0)
-    return fail(BERGSON_EINVAL, "invalid sizes for the score workspace");
+  const int st = validate_score_sizes(N, K, Q, topk);
+  if (st != BERGSON_OK) return st;
   *ws_bytes = plan_score(K, Q, topk).total;
   return BERGSON_OK;
 }

@@ -452,3 +452,43 @@ def test_planners_on_random_shapes():
 
     score()
     xgemm()
+
+
+# --- documented size limits of the workspace queries --------------------------
+
+def _ws_query(fn, *args):
+    n = ctypes.c_size_t()
+    st = getattr(bg.lib(), fn)(*args, ctypes.byref(n))
+    return st, n.value
+
+
+def test_workspace_queries_at_their_size_limits():
+    L = bg.lib()
+    # projection: B * T up to 2^37 tokens
+    arr = (bg.bergson_layer * 1)(_layer(d_in=8, d_out=8))
+    n = ctypes.c_size_t()
+    assert L.bergson_project_grads_workspace(arr, 1, 1 << 20, 1 << 17, ctypes.byref(n)) == bg.BERGSON_OK
+    assert 0 < n.value < (1 << 40)
+    assert L.bergson_project_grads_workspace(arr, 1, (1 << 20) + 1, 1 << 17, ctypes.byref(n)) == \
+        bg.BERGSON_EUNSUPPORTED
+    # scoring: N < 2^31, Q <= 2^24, topk <= 1024
+    st, n_big = _ws_query("bergson_score_topk_workspace", (1 << 31) - 1, 8192, 1 << 24, 1024)
+    assert st == bg.BERGSON_OK and n_big >= (1 << 24) * 8192 * 2
+    assert _ws_query("bergson_score_topk_workspace", 1 << 31, 8192, 16, 8)[0] == bg.BERGSON_EINVAL
+    assert _ws_query("bergson_score_topk_workspace", 1 << 20, 8192, 16, 1025)[0] == \
+        bg.BERGSON_EUNSUPPORTED
+    assert _ws_query("bergson_score_topk_workspace", 1 << 20, 8192, (1 << 24) + 1, 8)[0] == \
+        bg.BERGSON_EINVAL
+    assert _ws_query("bergson_score_topk_workspace", 1 << 20, 8196, 16, 8)[0] == bg.BERGSON_EALIGN
+    # on-the-fly scores / preconditioner application: B <= 2^20, Q <= 2^24, K <= 2^26
+    st, n_otf = _ws_query("bergson_score_grads_workspace", 1 << 20, 1 << 12, 1 << 10)
+    assert st == bg.BERGSON_OK and n_otf >= 2 * 4 * (1 << 20) * (1 << 12)   # x_hi and x_lo
+    assert _ws_query("bergson_score_grads_workspace", (1 << 20) + 1, 64, 64)[0] == bg.BERGSON_EINVAL
+    # Fisher: n <= 2^24 rows, K <= 65536; the preconditioner holds 4 K^2 floats
+    assert _ws_query("bergson_fisher_fit_workspace", 1 << 24, 1 << 16)[0] == bg.BERGSON_OK
+    assert _ws_query("bergson_fisher_fit_workspace", 1 << 24, (1 << 16) + 4)[0] == bg.BERGSON_EINVAL
+    st, n_pre = _ws_query("bergson_fisher_preconditioner_workspace", 1 << 16)
+    assert st == bg.BERGSON_OK and n_pre >= 4 * 4 * (1 << 32)
+    # aggregation: n < 2^31 rows
+    assert _ws_query("bergson_aggregate_rows_workspace", (1 << 31) - 1)[0] == bg.BERGSON_OK
+    assert _ws_query("bergson_aggregate_rows_workspace", 1 << 31)[0] == bg.BERGSON_EINVAL
