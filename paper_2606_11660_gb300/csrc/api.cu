@@ -1072,8 +1072,12 @@ static int validate_onthefly(const float* proj, int64_t B, int64_t K, int64_t ld
 
 int bergson_score_grads_workspace(int64_t B, int64_t K, int64_t Q, size_t* ws_bytes) {
   if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
-  if (B < 0 || B > (1 << 20) || Q < 0 || Q > (1 << 24) || K < 4 || K > (1 << 26))
-    return fail(BERGSON_EINVAL, "invalid sizes for the on-the-fly score workspace");
+  // the calls' size rules (no pointers to check here)
+  const int st = validate_onthefly(nullptr, 0, K, K, nullptr, 0, K, nullptr, 0);
+  if (st != BERGSON_OK) return st;
+  if (B < 0 || B > (1 << 20) || Q < 0 || Q > (1 << 24))
+    return fail(BERGSON_EINVAL, "B must be in [0, 2^20] and Q in [0, 2^24]");
+  if (B * Q > (1ll << 34)) return fail(BERGSON_EUNSUPPORTED, "B*Q too large");
   *ws_bytes = onthefly_workspace(B, K, Q);
   return BERGSON_OK;
 }
@@ -1159,6 +1163,7 @@ int bergson_fisher_fit_workspace(int64_t n, int64_t K, size_t* ws_bytes) {
   if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
   if (n < 1 || n > (1 << 24) || K < 4 || K > (1 << 16))
     return fail(BERGSON_EINVAL, "n must be in [1, 2^24] and K in [4, 65536]");
+  if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
   *ws_bytes = round_up(fisher_fit_workspace(n, K), 256);
   return BERGSON_OK;
 }
@@ -1192,6 +1197,7 @@ int bergson_fisher_fit(const float* rows, int64_t n, int64_t K, int64_t ld, floa
 int bergson_fisher_preconditioner_workspace(int64_t K, size_t* ws_bytes) {
   if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
   if (K < 4 || K > (1 << 16)) return fail(BERGSON_EINVAL, "K must be in [4, 65536]");
+  if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
   *ws_bytes = round_up(fisher_power_workspace(K), 256);
   return BERGSON_OK;
 }

@@ -421,8 +421,11 @@ def check_xgemm_plan(B, Q, K):
     assert p["xh_off"] - p["partial_off"] >= 4 * S * B * Q
     assert p["xl_off"] - p["xh_off"] >= 4 * B * K and p["total"] - p["xl_off"] >= 4 * B * K
     n = ctypes.c_size_t()
-    assert bg.lib().bergson_score_grads_workspace(B, K, Q, ctypes.byref(n)) == bg.BERGSON_OK
-    assert n.value == p["total"]
+    st = bg.lib().bergson_score_grads_workspace(B, K, Q, ctypes.byref(n))
+    if B * Q > (1 << 34):                    # beyond what the calls accept
+        assert st == bg.BERGSON_EUNSUPPORTED
+    else:
+        assert st == bg.BERGSON_OK and n.value == p["total"]
 
 
 def test_xgemm_planner_validation():
@@ -489,6 +492,12 @@ def test_workspace_queries_at_their_size_limits():
     assert _ws_query("bergson_fisher_fit_workspace", 1 << 24, (1 << 16) + 4)[0] == bg.BERGSON_EINVAL
     st, n_pre = _ws_query("bergson_fisher_preconditioner_workspace", 1 << 16)
     assert st == bg.BERGSON_OK and n_pre >= 4 * 4 * (1 << 32)
+    # the queries apply their calls' alignment rules too
+    assert _ws_query("bergson_score_grads_workspace", 32, 4098, 16)[0] == bg.BERGSON_EALIGN
+    assert _ws_query("bergson_score_grads_workspace", 1 << 20, 64, 1 << 24)[0] == \
+        bg.BERGSON_EUNSUPPORTED
+    assert _ws_query("bergson_fisher_fit_workspace", 64, 258)[0] == bg.BERGSON_EALIGN
+    assert _ws_query("bergson_fisher_preconditioner_workspace", 258)[0] == bg.BERGSON_EALIGN
     # aggregation: n < 2^31 rows
     assert _ws_query("bergson_aggregate_rows_workspace", (1 << 31) - 1)[0] == bg.BERGSON_OK
     assert _ws_query("bergson_aggregate_rows_workspace", 1 << 31)[0] == bg.BERGSON_EINVAL
