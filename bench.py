@@ -692,6 +692,7 @@ def score_sweep(args, store, N, K, topk, dev, peaks):
         for _ in range(2):
             bg.bergson_score_topk(store, N, K, queries, topk, s, i, ws, stream)
         torch.cuda.synchronize()
+        time.sleep(0.3)       # the power-capped 1024-query leg runs just before
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
         ev[0].record(stream)
         for _ in range(3):
