@@ -477,8 +477,11 @@ def bench_fisher(args, world, dev, state, peaks):
     ev[0].record(stream)
     bg.bergson_fisher_fit(fit_rows, n_fit, K, R, fws, stream)
     ev[1].record(stream)
-    bg.bergson_fisher_preconditioner(R, None, K, 1.0, 0.1, bg.BERGSON_FISHER_INV_SQRT,
-                                     args.fisher_iters, M, pws, stream)
+    # The iteration count comes from the residual: updates stop at the first
+    # iterate with ||I - Z Y||_F / sqrt(K) <= fisher_tol (at most fisher_iters).
+    iters_done, ns_res = bg.bergson_fisher_preconditioner_tol(
+        R, None, K, 1.0, 0.1, bg.BERGSON_FISHER_INV_SQRT, args.fisher_iters, args.fisher_tol, M,
+        pws, stream)
     ev[2].record(stream)
     for _ in range(args.warmup):
         bg.bergson_precondition_rows(out, cfg.B, K, M, pre, aws, stream)
@@ -498,7 +501,23 @@ def bench_fisher(args, world, dev, state, peaks):
     pow_ms = ev[1].elapsed_time(ev[2])
     step_ms = ev[3].elapsed_time(ev[4]) / args.steps
     apply_ms = ev[4].elapsed_time(ev[5]) / args.steps
-    gemm_flops = 2.0 * K ** 3 * (3 * args.fisher_iters)
+    # ||M R M - I||_F / sqrt(K) of the M in use, formed by the library's own
+    # product (rows of M against R give M R, those rows against M give M R M).
+    del fws, pws
+    torch.cuda.empty_cache()
+    kws = bg.workspace_tensor(bg.bergson_score_grads_workspace(K, K, K), dev)
+    MR = torch.empty((K, K), device=dev)
+    bg.bergson_precondition_rows(M, K, K, R, MR, kws, stream)
+    MRM = torch.empty((K, K), device=dev)
+    bg.bergson_precondition_rows(MR, K, K, M, MRM, kws, stream)
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    del MR, kws
+    MRM.diagonal().sub_(1.0)
+    true_res = float(torch.linalg.norm(MRM.double())) / K ** 0.5
+    del MRM
+    torch.cuda.empty_cache()
+    gemm_flops = 2.0 * K ** 3 * (3 * iters_done + len(ns_res) - iters_done)
     apply_gbs = 4.0 * K * (K + 2 * cfg.B) / (apply_ms * 1e-3) / 1e9   # M once, rows in and out
     # fp32-accurate products run three tf32 MMAs each; the tf32 rate is the
     # measured bf16 peak times the nominal tf32 : bf16 ratio (1.1 : 2.25).
@@ -509,7 +528,12 @@ def bench_fisher(args, world, dev, state, peaks):
             "apply_tflops": round(2.0 * cfg.B * K * K / (apply_ms * 1e-3) / 1e12, 2),
             "fit_ms": round(fit_ms, 3), "fit_rows": n_fit,
             "fit_tflops": round(2.0 * K * K * n_fit / (fit_ms * 1e-3) / 1e12, 2),
-            "preconditioner_ms": round(pow_ms, 1), "newton_schulz_iterations": args.fisher_iters,
+            "preconditioner_ms": round(pow_ms, 1), "newton_schulz_iterations": iters_done,
+            "newton_schulz_tol": args.fisher_tol, "newton_schulz_max_iterations": args.fisher_iters,
+            "newton_schulz_residuals": [float(f"{r:.3e}") for r in ns_res],
+            "residual_MRM": float(f"{true_res:.3e}"),
+            "residual_definition": "||M R M - I||_F / sqrt(K) of the M in use (library products); "
+                                   "the stopping rule reads ||I - Z Y||_F / sqrt(K) per iterate",
             "preconditioner_tflops": round(ns_tflops, 2),
             "roofline_apply": {"bound": "hbm", "achieved": round(apply_gbs, 1),
                                "peak": peaks["hbm_gbs"], "unit": "GB/s",
@@ -1001,7 +1025,10 @@ def parse(argv=None):
     ap.add_argument("--no-fisher", action="store_true")
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
-    ap.add_argument("--fisher-iters", type=int, default=20)
+    ap.add_argument("--fisher-iters", type=int, default=30,
+                    help="at most this many Newton-Schulz updates")
+    ap.add_argument("--fisher-tol", type=float, default=1e-5,
+                    help="stop at the first iterate whose residual is below this")
     ap.add_argument("--profile-case", choices=["collect", "score", "score_mid", "tokens", "onthefly",
                                                "apply", "fisher",
                              "streamed_pythia1b4", "streamed_llama8b"],

@@ -46,7 +46,9 @@ typedef enum {
   BERGSON_EUNSUPPORTED = -3,      /* valid request outside what this build implements */
   BERGSON_EWORKSPACE = -4,        /* workspace smaller than the *_workspace query */
   BERGSON_ECUDA = -5,             /* a CUDA runtime/driver call failed */
-  BERGSON_EDEVICE_TIMEOUT = -6    /* a bounded device wait gave up (see bergson_sync_status) */
+  BERGSON_EDEVICE_TIMEOUT = -6,   /* a bounded device wait gave up (see bergson_sync_status) */
+  BERGSON_EMOMENT = -7            /* a second-moment entry r_i or c_j was not > 0 (recorded by
+                                     the device; see bergson_sync_status) */
 } bergson_status;
 
 typedef enum {
@@ -94,7 +96,10 @@ typedef enum {
  *   proj_kind    bergson_proj_kind, shared by both sides of the layer.
  *   r, c   fp32 [d_out] and [d_in] factored second moments (> 0), or both
  *          NULL for no normalisation.  The gradient is divided elementwise by
- *          sqrt(r_i c_j).
+ *          sqrt(r_i c_j).  The values live on the device, so the host cannot
+ *          check them: an entry that is not > 0 (zero, negative, NaN) is
+ *          recorded as BERGSON_EMOMENT in the device status word (reported by
+ *          bergson_sync_status) and the outputs that depend on it are inf/NaN.
  *   out_col_offset   first column of this module's k_out*k_in block in `out`.
  *   flags  0 or BERGSON_LAYER_BIAS.  With BERGSON_LAYER_BIAS the projected
  *          bias gradient P_out^T (sum over valid tokens of g_t / sqrt(r)) --
@@ -166,6 +171,31 @@ BERGSON_API int bergson_build_store(const float* proj, int64_t B, int64_t K, int
                         int unit_normalize, void* store, int64_t ld_store,
                         int64_t row_offset, int64_t N_cap, float* norms_out, void* stream);
 
+/*
+ * Gradient-store rows with per-module unit normalisation (Sec. 3.1: the
+ * store is indexed by module; Fig. 1 "unit normalization"), the option beside
+ * the whole-row normalisation of bergson_build_store:
+ *
+ *   store[row_offset + b, o_j:o_{j+1}] = fp16( proj[b, o_j:o_{j+1}] / ||proj[b, o_j:o_{j+1}]||_2 )
+ *
+ * for every block j (typically one module's k_out*k_in block); a zero block
+ * is stored as zeros.  Each stored block then has unit norm, so a row has
+ * norm sqrt(n_blocks) and bergson_score_topk's score of a unit query q is
+ * sum_j q[o_j:o_{j+1}] . s_j, every module weighted alike.
+ *   block_offsets  HOST int64 [n_blocks + 1]: 0 = o_0 < o_1 < ... < o_n = K,
+ *                  each a multiple of 8.   n_blocks in 1 .. 2048.
+ *   norms_out      optional fp32 [B, n_blocks]: the blocks' l2 norms before
+ *                  normalisation.
+ * Other arguments and rules as for bergson_build_store; with n_blocks = 1 the
+ * result equals bergson_build_store with unit_normalize = 1.
+ * Errors: EINVAL, EALIGN, ECUDA.
+ */
+BERGSON_API int bergson_build_store_blocks(const float* proj, int64_t B, int64_t K,
+                                           int64_t ld_proj, const int64_t* block_offsets,
+                                           int n_blocks, void* store, int64_t ld_store,
+                                           int64_t row_offset, int64_t N_cap, float* norms_out,
+                                           void* stream);
+
 /* Bytes of workspace bergson_score_topk (and bergson_score_bottomk) needs;
  * N, K, Q and topk follow the calls' size rules (EINVAL, EALIGN, EUNSUPPORTED). */
 BERGSON_API int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes);
@@ -213,6 +243,75 @@ BERGSON_API int bergson_score_bottomk(const void* store, int64_t N, int64_t K, i
                           const float* queries, int64_t Q, int64_t ld_q, int64_t bottomk,
                           float* out_scores, int64_t* out_idx,
                           void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Exact top-k (bottom-k) over a store scored piece by piece (Bergson Sec. 3.1:
+ * gradient stores persisted to disk and queried with exact top-k; a store can
+ * be far larger than device memory).  One call scores the rows of one chunk,
+ *   store[0, N) = rows [row_base, row_base + N) of the whole store,
+ * and merges them into a running result held by the caller:
+ *   init != 0:  scores/idx <- the top-k of this chunk (contents on entry ignored);
+ *   init == 0:  scores/idx <- the top-k of (scores/idx on entry  U  this chunk).
+ * Indices are global (row_base + row).  After calls over chunks that cover
+ * rows [0, N_total) once each, in any order, scores/idx equal
+ * bergson_score_topk over the whole store: the same rows, the same scores
+ * bit for bit (every score is computed the same way whatever chunk holds
+ * its row), the same order (score descending, index ascending; bottom-k:
+ * ascending, index ascending).  With init == 0 the chunk's pass starts from
+ * the running k-th score, so chunks after the first cost little beyond
+ * streaming them.
+ *   N          1 .. 2^31-1 rows in this chunk (may be fewer than topk).
+ *   row_base   >= 0, row_base + N < 2^31.  Chunks must not overlap.
+ *   scores, idx  fp32 / int64 [Q, topk], in and out; tail entries of a
+ *              result with fewer than topk rows are (-inf, -1) for top-k and
+ *              (+inf, -1) for bottom-k.
+ * Other arguments and rules as for bergson_score_topk / _bottomk; workspace
+ * from bergson_score_topk_update_workspace (it does not depend on N).
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_score_topk_update_workspace(int64_t K, int64_t Q, int64_t topk,
+                                                    size_t* ws_bytes);
+BERGSON_API int bergson_score_topk_update(const void* store, int64_t N, int64_t K,
+                                          int64_t ld_store, int64_t row_base,
+                                          const float* queries, int64_t Q, int64_t ld_q,
+                                          int64_t topk, int init, float* scores, int64_t* idx,
+                                          void* workspace, size_t ws_bytes, void* stream);
+BERGSON_API int bergson_score_bottomk_update(const void* store, int64_t N, int64_t K,
+                                             int64_t ld_store, int64_t row_base,
+                                             const float* queries, int64_t Q, int64_t ld_q,
+                                             int64_t bottomk, int init, float* scores,
+                                             int64_t* idx, void* workspace, size_t ws_bytes,
+                                             void* stream);
+
+/*
+ * Exact top-k (least == 0) or bottom-k (least != 0) of a store that lives in
+ * HOST memory (Sec. 3.1: on-disk, memory-mapped gradient stores), streamed
+ * to the device in chunks of chunk_rows rows: chunk c + 1 is copied on
+ * `copy_stream` while chunk c is scored on `stream` (two device chunk
+ * buffers in the workspace), each chunk merged into the running result as
+ * bergson_score_topk_update does.  The result equals bergson_score_topk over
+ * the same rows resident on the device.
+ *   host_store  fp16 [N, ld_store] host memory, 16-byte aligned rows.  Pinned
+ *               (page-locked) memory lets the copies overlap the scoring and
+ *               run at the host link's rate; other host memory (e.g. a
+ *               numpy.memmap of a store file) works, with copies staged by
+ *               the driver.
+ *   copy_stream a second stream for the copies, or NULL to copy on `stream`
+ *               (no overlap).  The call orders the two streams with events it
+ *               creates and destroys itself; on return all its work is
+ *               enqueued on `stream` (and copy_stream), nothing is synchronised.
+ *   workspace   bergson_score_topk_host_workspace(chunk_rows, K, Q, topk) bytes.
+ * N, K, Q, topk, queries and outputs as for bergson_score_topk.
+ * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
+ */
+BERGSON_API int bergson_score_topk_host_workspace(int64_t chunk_rows, int64_t K, int64_t Q,
+                                                  int64_t topk, size_t* ws_bytes);
+BERGSON_API int bergson_score_topk_host(const void* host_store, int64_t N, int64_t K,
+                                        int64_t ld_store, const float* queries, int64_t Q,
+                                        int64_t ld_q, int64_t topk, int least,
+                                        int64_t chunk_rows, float* out_scores, int64_t* out_idx,
+                                        void* workspace, size_t ws_bytes, void* stream,
+                                        void* copy_stream);
 
 /* Bytes of workspace bergson_token_scores needs (n_queries in 1 .. 16). */
 BERGSON_API int bergson_token_scores_workspace(const bergson_layer* layers, int n_layers,
@@ -299,6 +398,30 @@ BERGSON_API int bergson_fisher_preconditioner(const float* R1, const float* R2, 
                                               int64_t ldr, float lam, float damping, int power,
                                               int iterations, float* M, int64_t ldm,
                                               void* workspace, size_t ws_bytes, void* stream);
+/*
+ * bergson_fisher_preconditioner with a stopping rule (same reading of Sec. 3.1
+ * and Fig. 2).  Before each Newton-Schulz update the residual of the current
+ * iterate,
+ *
+ *   res_i = ||I - Z_i Y_i||_F / sqrt(K)     (= ||M_i R M_i - I||_F / sqrt(K)
+ *                                            while the iteration keeps Y = R Z / c),
+ *
+ * is read back to the host; the iteration stops at the first i with
+ * res_i <= tol, or after max_iterations updates.  M is formed from that iterate.
+ *   residuals   host fp32 [max_iterations + 1] or NULL: res_0, res_1, ... up to
+ *               the last iterate computed.
+ *   iterations  host int or NULL: the number of updates applied.
+ * Unlike the other calls this one synchronises `stream` once per iterate
+ * (one 4-byte read each; the call is a one-time setup cost).  tol = 0 runs
+ * all max_iterations updates and still records every residual.
+ * Errors: those of bergson_fisher_preconditioner, and EINVAL for tol < 0.
+ */
+BERGSON_API int bergson_fisher_preconditioner_tol(const float* R1, const float* R2, int64_t K,
+                                                  int64_t ldr, float lam, float damping,
+                                                  int power, int max_iterations, float tol,
+                                                  float* M, int64_t ldm, void* workspace,
+                                                  size_t ws_bytes, float* residuals,
+                                                  int* iterations, void* stream);
 BERGSON_API int bergson_precondition_rows(const float* rows, int64_t B, int64_t K, int64_t ld,
                                           const float* M, int64_t ldm, float* out,
                                           int64_t ld_out, void* workspace, size_t ws_bytes,
@@ -341,8 +464,10 @@ BERGSON_API int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, i
 
 /*
  * Synchronises `stream`, then reports and clears the device status word:
- * BERGSON_OK, BERGSON_EDEVICE_TIMEOUT (a bounded device wait gave up) or
- * BERGSON_ECUDA (the stream carried a CUDA error).
+ * BERGSON_OK, BERGSON_EDEVICE_TIMEOUT (a bounded device wait gave up),
+ * BERGSON_EMOMENT (a factored second-moment entry was not > 0) or
+ * BERGSON_ECUDA (the stream carried a CUDA error).  The word keeps the first
+ * status recorded since it was last cleared.
  */
 BERGSON_API int bergson_sync_status(void* stream);
 
@@ -376,6 +501,20 @@ BERGSON_API int bergson_debug_wait_probe(uint64_t timeout_ns, void* stream);
  * validation, without enqueueing anything.  count = 0 clears it.
  */
 BERGSON_API void bergson_debug_inject_status(int status, int count);
+
+/*
+ * Test aid for the per-device record behind every kernel-attribute setting
+ * (one process may drive several GPUs; CUDA keeps a kernel's shared-memory
+ * limit per function and per device).  Runs n_threads host threads that each
+ * ask, three times over, for the setting on each of n_devices simulated
+ * devices, with a slow fake setting in place of the CUDA call; the first
+ * fake setting for fail_device (-1: none) fails.  set_calls[d] receives how
+ * often the setting ran for device d (1 expected, 2 for fail_device: a
+ * failure is retried) and *failures how many requests saw a failure.
+ * Host only: no GPU is touched.  n_threads, n_devices in 1 .. 64.
+ */
+BERGSON_API int bergson_debug_attr_once(int n_threads, int n_devices, int fail_device,
+                                        int64_t* set_calls, int* failures);
 
 /*
  * Test aid for the projection work planner: for the same arguments as
@@ -452,11 +591,21 @@ BERGSON_API int bergson_store_load(const char* path, int64_t file_row_offset, in
  * The scratch is a fixed static device array of BERGSON_NOALLOC_SCRATCH_BYTES
  * that every GPU loading the library keeps until the process exits; requests
  * needing more (see bergson_project_grads_workspace) fail with
- * BERGSON_EWORKSPACE and enqueue nothing.  No allocation of any kind happens.
+ * BERGSON_EWORKSPACE and enqueue nothing.  The call itself allocates nothing
+ * (no cudaMalloc, no workspace, no allocating library routine).
  * All calls share the one array: calls that overlap on the GPU (e.g. on two
- * streams) race and must be ordered by the caller.  The first call on each
- * device looks up the array's device address; make that first call before any
- * stream capture begins.
+ * streams) race and must be ordered by the caller.
+ *
+ * First call on a device: it looks up the array's device address on the
+ * device that owns `out` (the current device when out is NULL).  Under CUDA's
+ * lazy module loading (the default) that lookup is also the moment the driver
+ * loads this part of the library on the device and reserves the array's
+ * 32 MiB there, so the first call can fail with BERGSON_ECUDA when the device
+ * has no 32 MiB left (e.g. a runtime's pool already holds it all).  To take
+ * that step at a time of the caller's choosing, make a warm-up call early:
+ * any valid layer array with B = 0 and out = NULL does the lookup (and the
+ * reservation) on the current device and enqueues nothing.  Make the first
+ * call on each device before any stream capture begins.
  */
 #define BERGSON_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 

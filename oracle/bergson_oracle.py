@@ -12,7 +12,8 @@ What it computes (Bergson, Sec. 3.1 and Fig. 1; App. B, "Gradients"):
   3. the double-sided per-module random projection
      G^_b = P_out^T W~_b P_in                (k_out x k_in, row-major, k_out major);
   4. concatenation over modules in call order and unit normalisation of the
-     whole per-example row (grad-cosine);
+     whole per-example row (grad-cosine), or, as an option, of each module's
+     block on its own (the store is indexed by module, Sec. 3.1);
   5. an fp16 gradient store, cosine scores against unit-normalised queries and
      exact top-k, ordered by (score descending, index ascending), and the k
      least influential items (Sec. 3.1), ordered by (score ascending, index
@@ -289,6 +290,20 @@ def build_store(proj: np.ndarray, unit: bool = True) -> tuple[np.ndarray, np.nda
     rows, norms = unit_normalize(proj) if unit else (np.asarray(proj, np.float64), None)
     if norms is None:
         norms = np.sqrt(np.sum(rows * rows, axis=1))
+    return rows.astype(np.float16), norms
+
+
+def build_store_blocks(proj: np.ndarray, offsets) -> tuple[np.ndarray, np.ndarray]:
+    """Per-module unit normalisation: each column block [o_j, o_{j+1}) of a row
+    (one module's k_out x k_in block, the store being indexed by module,
+    Sec. 3.1) divided by its own l2 norm, a zero block staying zero, then fp16
+    (round to nearest even from fp64).  Returns (rows, norms [B, n_blocks])."""
+    x = np.asarray(proj, dtype=np.float64)
+    o = [int(v) for v in offsets]
+    rows = np.zeros_like(x)
+    norms = np.zeros((x.shape[0], len(o) - 1))
+    for j in range(len(o) - 1):
+        rows[:, o[j]:o[j + 1]], norms[:, j] = unit_normalize(x[:, o[j]:o[j + 1]])
     return rows.astype(np.float16), norms
 
 

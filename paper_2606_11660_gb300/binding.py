@@ -22,6 +22,7 @@ BERGSON_EUNSUPPORTED = -3
 BERGSON_EWORKSPACE = -4
 BERGSON_ECUDA = -5
 BERGSON_EDEVICE_TIMEOUT = -6
+BERGSON_EMOMENT = -7
 
 BERGSON_PROJ_GAUSSIAN = 0
 BERGSON_PROJ_IDENTITY = 1
@@ -39,6 +40,7 @@ BERGSON_FISHER_INV = 1
 STATUS_NAMES = {
     0: "BERGSON_OK", -1: "BERGSON_EINVAL", -2: "BERGSON_EALIGN", -3: "BERGSON_EUNSUPPORTED",
     -4: "BERGSON_EWORKSPACE", -5: "BERGSON_ECUDA", -6: "BERGSON_EDEVICE_TIMEOUT",
+    -7: "BERGSON_EMOMENT",
 }
 
 # Every symbol include/bergson.h declares.
@@ -53,7 +55,10 @@ EXPORTED = (
     "bergson_token_scores", "bergson_aggregate_rows_workspace", "bergson_aggregate_rows",
     "bergson_fisher_fit_workspace", "bergson_fisher_fit", "bergson_fisher_preconditioner_workspace",
     "bergson_fisher_preconditioner", "bergson_precondition_rows", "bergson_store_save",
-    "bergson_store_load",
+    "bergson_store_load", "bergson_fisher_preconditioner_tol", "bergson_debug_attr_once",
+    "bergson_build_store_blocks", "bergson_score_topk_update_workspace",
+    "bergson_score_topk_update", "bergson_score_bottomk_update",
+    "bergson_score_topk_host_workspace", "bergson_score_topk_host",
 )
 
 
@@ -94,11 +99,21 @@ def lib() -> ctypes.CDLL:
         "bergson_project_grads_workspace": (i32, [lp, i32, i64, i64, szp]),
         "bergson_project_grads": (i32, [lp, i32, i64, i64, vp, vp, i64, vp, ctypes.c_size_t, vp]),
         "bergson_build_store": (i32, [vp, i64, i64, i64, i32, vp, i64, i64, i64, vp, vp]),
+        "bergson_build_store_blocks": (i32, [vp, i64, i64, i64, i64p, i32, vp, i64, i64, i64,
+                                             vp, vp]),
         "bergson_score_topk_workspace": (i32, [i64, i64, i64, i64, szp]),
         "bergson_score_topk": (i32, [vp, i64, i64, i64, vp, i64, i64, i64, vp, vp, vp,
                                      ctypes.c_size_t, vp]),
         "bergson_score_bottomk": (i32, [vp, i64, i64, i64, vp, i64, i64, i64, vp, vp, vp,
                                         ctypes.c_size_t, vp]),
+        "bergson_score_topk_update_workspace": (i32, [i64, i64, i64, szp]),
+        "bergson_score_topk_update": (i32, [vp, i64, i64, i64, i64, vp, i64, i64, i64, i32, vp,
+                                            vp, vp, ctypes.c_size_t, vp]),
+        "bergson_score_bottomk_update": (i32, [vp, i64, i64, i64, i64, vp, i64, i64, i64, i32,
+                                               vp, vp, vp, ctypes.c_size_t, vp]),
+        "bergson_score_topk_host_workspace": (i32, [i64, i64, i64, i64, szp]),
+        "bergson_score_topk_host": (i32, [vp, i64, i64, i64, vp, i64, i64, i64, i32, i64, vp,
+                                          vp, vp, ctypes.c_size_t, vp, vp]),
         "bergson_projection_matrix": (i32, [u64, i64, i64, i32, vp, vp, vp]),
         "bergson_module_seeds": (None, [u64, i64, ctypes.POINTER(u64), ctypes.POINTER(u64)]),
         "bergson_sync_status": (i32, [vp]),
@@ -110,6 +125,7 @@ def lib() -> ctypes.CDLL:
         "bergson_debug_score_plan": (i32, [i64, i64, i64, i64, i32, i64p, i32,
                                            ctypes.POINTER(i32)]),
         "bergson_debug_xgemm_plan": (i32, [i64, i64, i64, i64p, i32]),
+        "bergson_debug_attr_once": (i32, [i32, i32, i32, i64p, ctypes.POINTER(i32)]),
         "bergson_project_grads_noalloc": (i32, [lp, i32, i64, i64, vp, vp, i64, vp]),
         "bergson_score_grads_workspace": (i32, [i64, i64, i64, szp]),
         "bergson_token_scores_workspace": (i32, [lp, i32, i64, i64, i64, szp]),
@@ -121,6 +137,11 @@ def lib() -> ctypes.CDLL:
         "bergson_fisher_preconditioner_workspace": (i32, [i64, szp]),
         "bergson_fisher_preconditioner": (i32, [vp, vp, i64, i64, ctypes.c_float, ctypes.c_float,
                                                 i32, i32, vp, i64, vp, ctypes.c_size_t, vp]),
+        "bergson_fisher_preconditioner_tol": (i32, [vp, vp, i64, i64, ctypes.c_float,
+                                                    ctypes.c_float, i32, i32, ctypes.c_float, vp,
+                                                    i64, vp, ctypes.c_size_t,
+                                                    ctypes.POINTER(ctypes.c_float),
+                                                    ctypes.POINTER(i32), vp]),
         "bergson_precondition_rows": (i32, [vp, i64, i64, i64, vp, i64, vp, i64, vp,
                                             ctypes.c_size_t, vp]),
         "bergson_aggregate_rows": (i32, [vp, i64, i64, i64, vp, i64, i32, i32, vp, i64, vp,
@@ -232,6 +253,16 @@ def bergson_build_store(proj, B: int, K: int, unit_normalize: bool, store, row_o
                                      _stream(stream)))
 
 
+def bergson_build_store_blocks(proj, B: int, K: int, block_offsets: Sequence[int], store,
+                               row_offset: int, norms_out=None, stream=None) -> None:
+    """Store rows with each column block [o_j, o_j+1) unit-normalised on its own."""
+    n = len(block_offsets) - 1
+    offs = (ctypes.c_int64 * max(1, n + 1))(*[int(v) for v in block_offsets])
+    _check(lib().bergson_build_store_blocks(_ptr(proj), int(B), int(K), int(proj.stride(0)), offs,
+                                            n, _ptr(store), int(store.stride(0)), int(row_offset),
+                                            int(store.shape[0]), _ptr(norms_out), _stream(stream)))
+
+
 def bergson_score_topk_workspace(N: int, K: int, Q: int, topk: int) -> int:
     n = ctypes.c_size_t()
     _check(lib().bergson_score_topk_workspace(int(N), int(K), int(Q), int(topk), ctypes.byref(n)))
@@ -257,6 +288,44 @@ def bergson_score_bottomk(store, N: int, K: int, queries, bottomk: int, out_scor
                                        _ptr(queries), Q, int(queries.stride(0)), int(bottomk),
                                        _ptr(out_scores), _ptr(out_idx), _ptr(workspace), ws_bytes,
                                        _stream(stream)))
+
+
+def bergson_score_topk_update_workspace(K: int, Q: int, topk: int) -> int:
+    n = ctypes.c_size_t()
+    _check(lib().bergson_score_topk_update_workspace(int(K), int(Q), int(topk), ctypes.byref(n)))
+    return n.value
+
+
+def bergson_score_topk_update(store, N: int, K: int, row_base: int, queries, topk: int, init: bool,
+                              scores, idx, workspace, stream=None, least: bool = False) -> None:
+    """Merge the top-k (least: bottom-k) of store rows [row_base, row_base + N)
+    (store[0:N] on the device) into the running result scores/idx [Q, topk]."""
+    Q = int(queries.shape[0])
+    fn = lib().bergson_score_bottomk_update if least else lib().bergson_score_topk_update
+    _check(fn(_ptr(store), int(N), int(K), int(store.stride(0)), int(row_base), _ptr(queries), Q,
+              int(queries.stride(0)), int(topk), 1 if init else 0, _ptr(scores), _ptr(idx),
+              _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def bergson_score_topk_host_workspace(chunk_rows: int, K: int, Q: int, topk: int) -> int:
+    n = ctypes.c_size_t()
+    _check(lib().bergson_score_topk_host_workspace(int(chunk_rows), int(K), int(Q), int(topk),
+                                                   ctypes.byref(n)))
+    return n.value
+
+
+def bergson_score_topk_host(host_store, N: int, K: int, queries, topk: int, chunk_rows: int,
+                            out_scores, out_idx, workspace, stream=None, copy_stream=None,
+                            least: bool = False) -> None:
+    """Exact top-k (least: bottom-k) of a store in host memory (a CPU tensor,
+    ideally pinned), streamed to the device in chunks of chunk_rows rows."""
+    Q = int(queries.shape[0])
+    cs = None if copy_stream is None else _stream(copy_stream)
+    _check(lib().bergson_score_topk_host(
+        _ptr(host_store), int(N), int(K), int(host_store.stride(0)), _ptr(queries), Q,
+        int(queries.stride(0)), int(topk), 1 if least else 0, int(chunk_rows), _ptr(out_scores),
+        _ptr(out_idx), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream), cs))
 
 
 def bergson_token_scores_workspace(layers: Sequence, B: int, T: int, n_queries: int) -> int:
@@ -322,6 +391,22 @@ def bergson_fisher_preconditioner(R1, R2, K: int, lam: float, damping: float, po
         workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
+def bergson_fisher_preconditioner_tol(R1, R2, K: int, lam: float, damping: float, power: int,
+                                      max_iterations: int, tol: float, M, workspace,
+                                      stream=None) -> tuple[int, list]:
+    """As bergson_fisher_preconditioner, stopping at the first iterate whose
+    residual ||I - Z Y||_F / sqrt(K) is <= tol.  Returns (updates applied,
+    residuals of the iterates computed)."""
+    res = (ctypes.c_float * (int(max_iterations) + 1))(*([float("nan")] * (int(max_iterations) + 1)))
+    done = ctypes.c_int()
+    _check(lib().bergson_fisher_preconditioner_tol(
+        _ptr(R1), _ptr(R2), int(K), int(R1.stride(0)), float(lam), float(damping), int(power),
+        int(max_iterations), float(tol), _ptr(M), int(M.stride(0)), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), res, ctypes.byref(done), _stream(stream)))
+    vals = [float(v) for v in res]
+    return done.value, [v for v in vals if v == v]
+
+
 def bergson_precondition_rows(rows, B: int, K: int, M, out, workspace, stream=None) -> None:
     """out[b] = M rows[b] (M symmetric K x K)."""
     _check(lib().bergson_precondition_rows(_ptr(rows), int(B), int(K), int(rows.stride(0)),
@@ -384,6 +469,16 @@ def bergson_debug_wait_probe(timeout_ns: int, stream=None) -> None:
 
 def bergson_debug_inject_status(status: int, count: int) -> None:
     lib().bergson_debug_inject_status(int(status), int(count))
+
+
+def bergson_debug_attr_once(n_threads: int, n_devices: int, fail_device: int = -1):
+    """(setting runs per simulated device, failed requests) of the per-device
+    attribute record under n_threads concurrent first calls; host only."""
+    calls = (ctypes.c_int64 * int(n_devices))()
+    fails = ctypes.c_int()
+    _check(lib().bergson_debug_attr_once(int(n_threads), int(n_devices), int(fail_device), calls,
+                                         ctypes.byref(fails)))
+    return list(calls), fails.value
 
 
 def bergson_debug_project_plan(layers, B: int, T: int) -> tuple[int, int, int, int]:

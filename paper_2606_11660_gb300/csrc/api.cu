@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <chrono>
 #include <cmath>
 #include <atomic>
 #include <cstdarg>
@@ -11,6 +12,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <thread>
 #include <vector>
 
 #include "bergson.h"
@@ -514,7 +516,8 @@ struct ScoreLaunchPlan {
 
 // Launch sequence of bergson_score_topk for `ctas` resident CTAs (for the pair
 // kernel: 2 x its co-resident clusters).  Pure host logic.
-ScoreLaunchPlan plan_score_launches(int64_t N, int64_t Q, int64_t topk, int ctas) {
+ScoreLaunchPlan plan_score_launches(int64_t N, int64_t Q, int64_t topk, int ctas,
+                                    bool allow_prefix = true) {
   ScoreLaunchPlan P;
   const ScoreLayout L = plan_score(0, Q, topk);
   P.pair = Q >= kPairMinQueries;
@@ -529,7 +532,7 @@ ScoreLaunchPlan plan_score_launches(int64_t N, int64_t Q, int64_t topk, int ctas
   // Prefix pass (large stores only): the exact top-k of the first `prefix` rows
   // lands in the outputs, and its k-th score seeds the full pass's threshold.
   const int64_t prefix_rows = round_up(static_cast<size_t>(kPrefixRowsPerTopk * topk), kScoreBN);
-  P.use_prefix = N >= kPrefixMinFactor * prefix_rows && Q >= kPrefixMinQueries;
+  P.use_prefix = allow_prefix && N >= kPrefixMinFactor * prefix_rows && Q >= kPrefixMinQueries;
   for (int pass = 0; pass < n_qg_total; pass += sms) {
     const int n_qg = std::min(sms, n_qg_total - pass);
     // The prefix is cut to whole rounds of store tiles over the CTAs of a
@@ -679,6 +682,43 @@ int bergson_debug_xgemm_plan(int64_t B, int64_t Q, int64_t K, int64_t* out, int 
   return BERGSON_OK;
 }
 
+int bergson_debug_attr_once(int n_threads, int n_devices, int fail_device, int64_t* set_calls,
+                            int* failures) {
+  if (n_threads < 1 || n_threads > 64 || n_devices < 1 || n_devices > 64)
+    return fail(BERGSON_EINVAL, "n_threads and n_devices must be in [1, 64]");
+  if (set_calls == nullptr || failures == nullptr)
+    return fail(BERGSON_EINVAL, "set_calls or failures is NULL");
+  PerDeviceOnce once;
+  std::vector<std::atomic<int64_t>> calls(n_devices);
+  for (auto& c : calls) c.store(0);
+  std::atomic<int> fails{0}, ready{0};
+  std::atomic<bool> go{false};
+  auto body = [&](int t) {
+    ready.fetch_add(1);
+    while (!go.load()) std::this_thread::yield();
+    for (int rep = 0; rep < 3; ++rep) {
+      for (int j = 0; j < n_devices; ++j) {
+        const int dev = (j + t) % n_devices;
+        const cudaError_t e = once.ensure(dev, [&] {
+          // A slow setting widens the window in which other threads arrive.
+          std::this_thread::sleep_for(std::chrono::milliseconds(2));
+          const int64_t n = calls[dev].fetch_add(1);
+          return dev == fail_device && n == 0 ? cudaErrorInvalidValue : cudaSuccess;
+        });
+        if (e != cudaSuccess) fails.fetch_add(1);
+      }
+    }
+  };
+  std::vector<std::thread> th;
+  for (int t = 0; t < n_threads; ++t) th.emplace_back(body, t);
+  while (ready.load() < n_threads) std::this_thread::yield();
+  go.store(true);
+  for (auto& x : th) x.join();
+  for (int d = 0; d < n_devices; ++d) set_calls[d] = calls[d].load();
+  *failures = fails.load();
+  return BERGSON_OK;
+}
+
 void bergson_debug_inject_status(int status, int count) {
   g_inject_status.store(status);
   g_inject_count.store(count > 0 ? count : 0);
@@ -802,7 +842,8 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
     if (e != cudaSuccess) return fail_cuda(e, "tile flag launch");
   }
   if (need_tiles) {
-    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, max_pairs, s);
+    e = launch_prep(reinterpret_cast<const PrepSeg*>(ws + L.segs_off), 2 * n_layers, max_pairs,
+                    status, s);
     if (e != cudaSuccess) return fail_cuda(e, "prep launch");
   }
   const int sms = sm_count(dg.dev);
@@ -913,6 +954,53 @@ int bergson_build_store(const float* proj, int64_t B, int64_t K, int64_t ld_proj
   return BERGSON_OK;
 }
 
+int bergson_build_store_blocks(const float* proj, int64_t B, int64_t K, int64_t ld_proj,
+                               const int64_t* block_offsets, int n_blocks, void* store,
+                               int64_t ld_store, int64_t row_offset, int64_t N_cap,
+                               float* norms_out, void* stream) {
+  if (B < 0 || B > (1ll << 31) - 1) return fail(BERGSON_EINVAL, "B must be in [0, 2^31)");
+  if (K < 8 || K > (1ll << 28)) return fail(BERGSON_EINVAL, "K must be in [8, 2^28]");
+  if (K % 8 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 8");
+  if (block_offsets == nullptr) return fail(BERGSON_EINVAL, "block_offsets is NULL");
+  if (n_blocks < 1 || n_blocks > kMaxStoreBlocks)
+    return fail(BERGSON_EINVAL, "n_blocks must be in [1, %d]", kMaxStoreBlocks);
+  StoreBlocks sb;
+  sb.n = n_blocks;
+  if (block_offsets[0] != 0 || block_offsets[n_blocks] != K)
+    return fail(BERGSON_EINVAL, "block_offsets must start at 0 and end at K");
+  for (int j = 0; j <= n_blocks; ++j) {
+    if (j > 0 && block_offsets[j] <= block_offsets[j - 1])
+      return fail(BERGSON_EINVAL, "block_offsets must increase (block %d is empty)", j - 1);
+    if (block_offsets[j] % 8 != 0)
+      return fail(BERGSON_EALIGN, "block_offsets must be multiples of 8 (offset %d)", j);
+    sb.offset[j] = static_cast<int32_t>(block_offsets[j]);
+  }
+  if (ld_proj < K) return fail(BERGSON_EINVAL, "ld_proj must be >= K");
+  if (ld_proj % 4 != 0) return fail(BERGSON_EALIGN, "ld_proj must be a multiple of 4");
+  if (ld_store < K) return fail(BERGSON_EINVAL, "ld_store must be >= K");
+  if (ld_store % 8 != 0) return fail(BERGSON_EALIGN, "ld_store must be a multiple of 8");
+  if (row_offset < 0 || N_cap < 0 || row_offset + B > N_cap)
+    return fail(BERGSON_EINVAL, "rows [%lld, %lld) do not fit N_cap=%lld", (long long)row_offset,
+                (long long)(row_offset + B), (long long)N_cap);
+  if (B > 0) {
+    if (proj == nullptr || store == nullptr) return fail(BERGSON_EINVAL, "proj or store is NULL");
+    if (!aligned(proj, 16) || !aligned(store, 16))
+      return fail(BERGSON_EALIGN, "proj and store must be 16-byte aligned");
+    if (norms_out != nullptr && !aligned(norms_out, 4))
+      return fail(BERGSON_EALIGN, "norms_out must be 4-byte aligned");
+  }
+  int st;
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (B == 0) return BERGSON_OK;
+  DeviceGuard dg(store);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "store device lookup");
+  __half* dst = static_cast<__half*>(store) + row_offset * ld_store;
+  cudaError_t e = launch_build_store_blocks(proj, static_cast<int>(B), ld_proj, sb, dst, ld_store,
+                                            norms_out, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail_cuda(e, "store kernel launch");
+  return BERGSON_OK;
+}
+
 int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes) {
   if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
   const int st = validate_score_sizes(N, K, Q, topk);
@@ -924,12 +1012,28 @@ int bergson_score_topk_workspace(int64_t N, int64_t K, int64_t Q, int64_t topk, 
 // Top-k (least = false) or bottom-k (least = true: the queries are negated
 // when they are normalised, and the final merge reports the scores against
 // the original queries).
+//
+// Update mode (update = true): out_scores / out_idx hold on entry the result of
+// earlier calls over other rows (global indices, this call's order); the call
+// scores rows [row_base, row_base + N) of the whole store and leaves in them
+// the top-k of both.  Its threshold starts at the prior k-th score, so it
+// skips the prefix pass.  Rows report row_base + local row in either mode.
 static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
                      const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
                      float* out_scores, int64_t* out_idx, void* workspace, size_t ws_bytes,
-                     void* stream, bool least) {
-  int st = validate_score(store, N, K, ld_store, queries, Q, ld_q, topk);
+                     void* stream, bool least, int64_t row_base = 0, bool update = false,
+                     bool chunk_rules = false) {
+  int st = chunk_rules ? validate_score_sizes(topk, K, Q, topk)
+                       : validate_score(store, N, K, ld_store, queries, Q, ld_q, topk);
   if (st != BERGSON_OK) return st;
+  if (chunk_rules) {
+    if (N < 1) return fail(BERGSON_EINVAL, "the chunk must hold at least one row");
+    if (row_base < 0 || row_base + N > (1ll << 31) - 1)
+      return fail(BERGSON_EINVAL, "rows [row_base, row_base + N) must lie in [0, 2^31 - 1)");
+    if ((st = validate_score(store, std::max(N, topk), K, ld_store, queries, Q, ld_q, topk)) !=
+        BERGSON_OK)
+      return st;
+  }
   if (Q > 0 && (out_scores == nullptr || out_idx == nullptr))
     return fail(BERGSON_EINVAL, "out_scores or out_idx is NULL");
   if ((out_scores && !aligned(out_scores, 4)) || (out_idx && !aligned(out_idx, 8)))
@@ -973,7 +1077,7 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
     if (e != cudaSuccess) return fail_cuda(e, "score kernel occupancy query");
     ctas = std::min(ctas, resident);
   }
-  const ScoreLaunchPlan P = plan_score_launches(N, Q, topk, ctas);
+  const ScoreLaunchPlan P = plan_score_launches(N, Q, topk, ctas, !update);
   if (P.launches.empty()) return fail(BERGSON_ECUDA, "no two-SM cluster fits the score kernel");
   for (const ScoreLaunch& l : P.launches) {
     ScoreParams p;
@@ -985,7 +1089,10 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
     p.qg_base = l.qg_base;
     p.n_ntiles = l.n_tiles;
     p.heaps = heaps;
-    p.tau0 = l.stage == 1 && P.use_prefix ? out_scores : nullptr;
+    p.tau0 = l.stage == 1 && (P.use_prefix || update) ? out_scores : nullptr;
+    // a prefix pass leaves its scores in the search's own order; a prior
+    // bottom-k state holds scores against q
+    p.tau0_negate = update && least ? 1 : 0;
     p.status = status;
     p.timeout_ns = kWaitTimeoutNs;
     e = pair ? launch_score_pair(L.qt, tm_store, tm_q, p, l.grid, s)
@@ -993,8 +1100,11 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
     if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");
     // The prefix pass's scores seed the full pass's thresholds, so only
     // the final merge converts them back for a bottom-k search.
+    const bool final_merge = l.stage == 1;
     e = launch_merge(heaps, l.grid, l.n_qg, L.qt, static_cast<int>(topk), l.q_begin, l.q_end,
-                     l.pass, least && l.stage == 1, out_scores, out_idx, s);
+                     l.pass, least && final_merge, final_merge ? row_base : 0,
+                     update && final_merge ? out_scores : nullptr,
+                     update && final_merge ? out_idx : nullptr, out_scores, out_idx, s);
     if (e != cudaSuccess) return fail_cuda(e, "merge kernel launch");
   }
   return BERGSON_OK;
@@ -1014,6 +1124,128 @@ int bergson_score_bottomk(const void* store, int64_t N, int64_t K, int64_t ld_st
                           void* stream) {
   return run_score(store, N, K, ld_store, queries, Q, ld_q, bottomk, out_scores, out_idx,
                    workspace, ws_bytes, stream, true);
+}
+
+int bergson_score_topk_update_workspace(int64_t K, int64_t Q, int64_t topk, size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  const int st = validate_score_sizes(topk, K, Q, topk);
+  if (st != BERGSON_OK) return st;
+  *ws_bytes = plan_score(K, Q, topk).total;
+  return BERGSON_OK;
+}
+
+int bergson_score_topk_update(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                              int64_t row_base, const float* queries, int64_t Q, int64_t ld_q,
+                              int64_t topk, int init, float* scores, int64_t* idx,
+                              void* workspace, size_t ws_bytes, void* stream) {
+  return run_score(store, N, K, ld_store, queries, Q, ld_q, topk, scores, idx, workspace, ws_bytes,
+                   stream, false, row_base, init == 0, true);
+}
+
+int bergson_score_bottomk_update(const void* store, int64_t N, int64_t K, int64_t ld_store,
+                                 int64_t row_base, const float* queries, int64_t Q, int64_t ld_q,
+                                 int64_t bottomk, int init, float* scores, int64_t* idx,
+                                 void* workspace, size_t ws_bytes, void* stream) {
+  return run_score(store, N, K, ld_store, queries, Q, ld_q, bottomk, scores, idx, workspace,
+                   ws_bytes, stream, true, row_base, init == 0, true);
+}
+
+// Device bytes of one chunk buffer of the host-streaming scorer.
+static size_t host_chunk_bytes(int64_t chunk_rows, int64_t K) {
+  return round_up(static_cast<size_t>(chunk_rows) * K * sizeof(__half), 256);
+}
+
+int bergson_score_topk_host_workspace(int64_t chunk_rows, int64_t K, int64_t Q, int64_t topk,
+                                      size_t* ws_bytes) {
+  if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
+  if (chunk_rows < 1 || chunk_rows > (1ll << 31) - 1)
+    return fail(BERGSON_EINVAL, "chunk_rows must be in [1, 2^31)");
+  const int st = validate_score_sizes(topk, K, Q, topk);
+  if (st != BERGSON_OK) return st;
+  *ws_bytes = 2 * host_chunk_bytes(chunk_rows, K) + plan_score(K, Q, topk).total;
+  return BERGSON_OK;
+}
+
+int bergson_score_topk_host(const void* host_store, int64_t N, int64_t K, int64_t ld_store,
+                            const float* queries, int64_t Q, int64_t ld_q, int64_t topk,
+                            int least, int64_t chunk_rows, float* out_scores, int64_t* out_idx,
+                            void* workspace, size_t ws_bytes, void* stream, void* copy_stream) {
+  int st = validate_score_sizes(N, K, Q, topk);
+  if (st != BERGSON_OK) return st;
+  if (chunk_rows < 1 || chunk_rows > (1ll << 31) - 1)
+    return fail(BERGSON_EINVAL, "chunk_rows must be in [1, 2^31)");
+  if (host_store == nullptr) return fail(BERGSON_EINVAL, "host_store is NULL");
+  if (ld_store < K) return fail(BERGSON_EINVAL, "ld_store must be >= K");
+  if (ld_store % 8 != 0 || !aligned(host_store, 16))
+    return fail(BERGSON_EALIGN, "host_store needs 16-byte aligned rows");
+  if (Q > 0 && (queries == nullptr || out_scores == nullptr || out_idx == nullptr))
+    return fail(BERGSON_EINVAL, "queries, out_scores or out_idx is NULL");
+  const size_t chunk_bytes = host_chunk_bytes(chunk_rows, K);
+  const size_t need = 2 * chunk_bytes + plan_score(K, Q, topk).total;
+  if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(BERGSON_EWORKSPACE, "workspace too small: %zu < %zu bytes", ws_bytes, need);
+  if ((st = injected()) != BERGSON_OK) return st;
+  if (Q == 0) return BERGSON_OK;
+  DeviceGuard dg(workspace);
+  if (dg.err != cudaSuccess) return fail_cuda(dg.err, "workspace device lookup");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaStream_t cs = copy_stream != nullptr ? static_cast<cudaStream_t>(copy_stream) : s;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  uint8_t* buf[2] = {ws, ws + chunk_bytes};
+  uint8_t* score_ws = ws + 2 * chunk_bytes;
+  const size_t score_ws_bytes = ws_bytes - 2 * chunk_bytes;
+  // Events order the two streams: a chunk is scored once its copy landed, and
+  // a buffer is refilled once the chunk scored from it is done.
+  cudaEvent_t ev[5] = {};
+  cudaError_t e = cudaSuccess;
+  for (int i = 0; i < 5 && e == cudaSuccess; ++i)
+    e = cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming);
+  cudaEvent_t* copied = ev;          // [2]
+  cudaEvent_t* used = ev + 2;        // [2]
+  cudaEvent_t start = ev[4];
+  int rc = BERGSON_OK;
+  if (e != cudaSuccess) rc = fail_cuda(e, "event creation");
+  if (rc == BERGSON_OK && cs != s) {
+    // the buffers may still be read by work enqueued on `stream` before this call
+    if ((e = cudaEventRecord(start, s)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(cs, start, 0)) != cudaSuccess)
+      rc = fail_cuda(e, "stream ordering");
+  }
+  const int64_t n_chunks = (N + chunk_rows - 1) / chunk_rows;
+  for (int64_t c = 0; c < n_chunks && rc == BERGSON_OK; ++c) {
+    const int b = static_cast<int>(c & 1);
+    const int64_t r0 = c * chunk_rows;
+    const int64_t rows = std::min(chunk_rows, N - r0);
+    if (c >= 2 && (e = cudaStreamWaitEvent(cs, used[b], 0)) != cudaSuccess) {
+      rc = fail_cuda(e, "stream ordering");
+      break;
+    }
+    e = cudaMemcpy2DAsync(buf[b], static_cast<size_t>(K) * sizeof(__half),
+                          static_cast<const __half*>(host_store) + r0 * ld_store,
+                          static_cast<size_t>(ld_store) * sizeof(__half),
+                          static_cast<size_t>(K) * sizeof(__half), static_cast<size_t>(rows),
+                          cudaMemcpyHostToDevice, cs);
+    if (e != cudaSuccess) {
+      rc = fail_cuda(e, "chunk copy");
+      break;
+    }
+    if ((e = cudaEventRecord(copied[b], cs)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(s, copied[b], 0)) != cudaSuccess) {
+      rc = fail_cuda(e, "stream ordering");
+      break;
+    }
+    rc = run_score(buf[b], rows, K, K, queries, Q, ld_q, topk, out_scores, out_idx, score_ws,
+                   score_ws_bytes, stream, least != 0, r0, c > 0, true);
+    if (rc != BERGSON_OK) break;
+    if ((e = cudaEventRecord(used[b], s)) != cudaSuccess) rc = fail_cuda(e, "stream ordering");
+  }
+  // Destroying an event whose work is still pending is allowed: its
+  // resources are released once that work completes.
+  for (int i = 0; i < 5; ++i)
+    if (ev[i] != nullptr) cudaEventDestroy(ev[i]);
+  return rc;
 }
 
 static size_t onthefly_workspace(int64_t B, int64_t K, int64_t Q) {
@@ -1202,9 +1434,11 @@ int bergson_fisher_preconditioner_workspace(int64_t K, size_t* ws_bytes) {
   return BERGSON_OK;
 }
 
-int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K, int64_t ldr,
-                                  float lam, float damping, int power, int iterations, float* M,
-                                  int64_t ldm, void* workspace, size_t ws_bytes, void* stream) {
+static int run_fisher_preconditioner(const float* R1, const float* R2, int64_t K, int64_t ldr,
+                                     float lam, float damping, int power, int iterations,
+                                     float tol, float* residuals, int* iterations_done, float* M,
+                                     int64_t ldm, void* workspace, size_t ws_bytes,
+                                     void* stream) {
   if (K < 4 || K > (1 << 16)) return fail(BERGSON_EINVAL, "K must be in [4, 65536]");
   if (K % 4 != 0) return fail(BERGSON_EALIGN, "K must be a multiple of 4");
   int st = check_square(R1, K, ldr, "R1");
@@ -1216,6 +1450,7 @@ int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K, i
   if (power != BERGSON_FISHER_INV_SQRT && power != BERGSON_FISHER_INV)
     return fail(BERGSON_EINVAL, "unknown power %d", power);
   if (iterations < 1 || iterations > 100) return fail(BERGSON_EINVAL, "iterations in [1, 100]");
+  if (!(tol >= 0.0f)) return fail(BERGSON_EINVAL, "tol must be >= 0");
   const size_t need = round_up(fisher_power_workspace(K), 256);
   if (workspace == nullptr) return fail(BERGSON_EINVAL, "workspace is NULL");
   if (!aligned(workspace, 256)) return fail(BERGSON_EALIGN, "workspace must be 256-byte aligned");
@@ -1227,11 +1462,28 @@ int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K, i
   int* status = status_word(dg.dev);
   if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
   cudaError_t e = launch_fisher_power(R1, R2, static_cast<int>(K), ldr, lam, damping,
-                                      power == BERGSON_FISHER_INV ? 1 : 0, iterations, M, ldm,
+                                      power == BERGSON_FISHER_INV ? 1 : 0, iterations, tol,
+                                      residuals, iterations_done, M, ldm,
                                       static_cast<float*>(workspace), status, sm_count(dg.dev),
                                       static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return fail_cuda(e, "Fisher preconditioner launch");
   return BERGSON_OK;
+}
+
+int bergson_fisher_preconditioner(const float* R1, const float* R2, int64_t K, int64_t ldr,
+                                  float lam, float damping, int power, int iterations, float* M,
+                                  int64_t ldm, void* workspace, size_t ws_bytes, void* stream) {
+  return run_fisher_preconditioner(R1, R2, K, ldr, lam, damping, power, iterations, 0.0f, nullptr,
+                                   nullptr, M, ldm, workspace, ws_bytes, stream);
+}
+
+int bergson_fisher_preconditioner_tol(const float* R1, const float* R2, int64_t K, int64_t ldr,
+                                      float lam, float damping, int power, int max_iterations,
+                                      float tol, float* M, int64_t ldm, void* workspace,
+                                      size_t ws_bytes, float* residuals, int* iterations,
+                                      void* stream) {
+  return run_fisher_preconditioner(R1, R2, K, ldr, lam, damping, power, max_iterations, tol,
+                                   residuals, iterations, M, ldm, workspace, ws_bytes, stream);
 }
 
 int bergson_precondition_rows(const float* rows, int64_t B, int64_t K, int64_t ld, const float* M,
@@ -1265,8 +1517,10 @@ int bergson_projection_matrix(uint64_t seed, int64_t d, int64_t k, int proj_kind
   if ((st = injected()) != BERGSON_OK) return st;
   DeviceGuard dg(out);
   if (dg.err != cudaSuccess) return fail_cuda(dg.err, "output device lookup");
+  int* status = status_word(dg.dev);
+  if (status == nullptr) return fail(BERGSON_ECUDA, "device status word unavailable");
   cudaError_t e = launch_projection_matrix(seed, static_cast<int>(d), static_cast<int>(k),
-                                           proj_kind, moment, out,
+                                           proj_kind, moment, status, out,
                                            static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return fail_cuda(e, "projection matrix launch");
   return BERGSON_OK;
@@ -1287,6 +1541,9 @@ int bergson_sync_status(void* stream) {
   if (v != 0) {
     const int zero = 0;
     cudaMemcpy(w, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (v == BERGSON_EMOMENT)
+      return fail(v, "a factored second-moment entry (r or c) was not > 0; the projected "
+                     "values computed from it are inf or NaN (device status %d)", v);
     return fail(v, "a bounded device wait gave up (device status %d)", v);
   }
   return BERGSON_OK;

@@ -78,15 +78,17 @@ __global__ void mix_kernel(const float* __restrict__ r1, const float* __restrict
 
 constexpr int kFrobBlocks = 512;
 
-// part[blockIdx] = compensated sum of squares over a grid-stride slice of R.
-__global__ void frob_partial_kernel(const float* __restrict__ r, int64_t ld, int K,
+// part[blockIdx] = compensated sum of squares of (R - shift I) over a
+// grid-stride slice of R.
+__global__ void frob_partial_kernel(const float* __restrict__ r, int64_t ld, int K, float shift,
                                     float* __restrict__ part) {
   __shared__ float red[32];
   float s = 0.0f, comp = 0.0f;
   const int64_t n = static_cast<int64_t>(K) * K;
   for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n;
        e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const float x = r[(e / K) * ld + e % K];
+    const int64_t i = e / K, j = e % K;
+    const float x = r[i * ld + j] - (i == j ? shift : 0.0f);
     const float y = x * x - comp;
     const float t = s + y;
     comp = (t - s) - y;
@@ -119,6 +121,20 @@ __global__ void frob_final_kernel(const float* __restrict__ part, int n_part,
   scal[2] = 1.0f / c;
   scal[3] = 1.0f / sqrtf(c);
   scal[4] = 1.0f / c;
+}
+
+// *out = scale * sqrt(fixed-order compensated sum of part[0, n_part))
+__global__ void frob_norm_kernel(const float* __restrict__ part, int n_part, float scale,
+                                 float* __restrict__ out) {
+  if (threadIdx.x != 0) return;
+  float t = 0.0f, comp = 0.0f;
+  for (int i = 0; i < n_part; ++i) {
+    const float y = part[i] - comp;
+    const float u = t + y;
+    comp = (u - t) - y;
+    t = u;
+  }
+  *out = scale * sqrtf(t);
 }
 
 // y = r * scal[2] (R / c); z = I
@@ -155,6 +171,26 @@ __global__ void __launch_bounds__(256) symmetrize_kernel(float* __restrict__ x, 
       x[static_cast<int64_t>(i0 + r) * K + j0 + c] = 0.5f * (a[r][c] + b[c][r]);
     if (ti != tj && j0 + r < K && i0 + c < K)
       x[static_cast<int64_t>(j0 + r) * K + i0 + c] = 0.5f * (b[r][c] + a[c][r]);
+  }
+}
+
+// x <- x^T in place (K x K, leading dimension K).  One CTA per pair of 32 x 32
+// tiles (ti <= tj), both read row by row into shared memory and written back
+// swapped, so every global access is coalesced.
+__global__ void __launch_bounds__(256) transpose_inplace_kernel(float* __restrict__ x, int K) {
+  __shared__ float a[32][33], b[32][33];
+  const int ti = blockIdx.y, tj = blockIdx.x;
+  if (ti > tj) return;
+  const int i0 = ti * 32, j0 = tj * 32, c = threadIdx.x;
+  for (int r = threadIdx.y; r < 32; r += 8) {
+    a[r][c] = (i0 + r < K && j0 + c < K) ? x[static_cast<int64_t>(i0 + r) * K + j0 + c] : 0.0f;
+    b[r][c] = (j0 + r < K && i0 + c < K) ? x[static_cast<int64_t>(j0 + r) * K + i0 + c] : 0.0f;
+  }
+  __syncthreads();
+  for (int r = threadIdx.y; r < 32; r += 8) {
+    if (i0 + r < K && j0 + c < K) x[static_cast<int64_t>(i0 + r) * K + j0 + c] = b[c][r];
+    if (ti != tj && j0 + r < K && i0 + c < K)
+      x[static_cast<int64_t>(j0 + r) * K + i0 + c] = a[c][r];
   }
 }
 
@@ -230,7 +266,8 @@ size_t fisher_power_workspace(int64_t K) {
 }
 
 cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
-                                float damping, int inverse, int iterations, float* m, int64_t ldm,
+                                float damping, int inverse, int iterations, float tol,
+                                float* residuals, int* iterations_done, float* m, int64_t ldm,
                                 float* ws, int* status, int sms, cudaStream_t s) {
   const int64_t kk = static_cast<int64_t>(K) * K;
   uint8_t* gws = reinterpret_cast<uint8_t*>(ws) +
@@ -239,34 +276,62 @@ cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t
   float* y = a + kk;
   float* z = y + kk;
   float* t = z + kk;
-  float* scal = t + kk;     // trace, ||R||_F, 1/c, 1/sqrt(c), 1/c; [64, 64 + 512): partial sums
+  float* scal = t + kk;     // trace, ||R||_F, 1/c, 1/sqrt(c), 1/c, residual;
+                            // [64, 64 + 512): partial sums
+  const bool track = residuals != nullptr || tol > 0.0f;
+  if (iterations_done != nullptr) *iterations_done = 0;
   mixed_trace_kernel<<<1, 1024, 0, s>>>(r1, r2, ldr, K, lam, scal);
   mix_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(r1, r2, ldr, K, lam, damping, scal, a, K);
-  frob_partial_kernel<<<kFrobBlocks, 256, 0, s>>>(a, K, K, scal + 64);
+  frob_partial_kernel<<<kFrobBlocks, 256, 0, s>>>(a, K, K, 0.0f, scal + 64);
   frob_final_kernel<<<1, 32, 0, s>>>(scal + 64, kFrobBlocks, scal);
   ns_init_kernel<<<elementwise_blocks(kk), 256, 0, s>>>(a, K, K, scal, y, z);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  for (int it = 0; it < iterations; ++it) {
-    // T = 1.5 I - 0.5 Z Y;  Y <- Y T;  Z <- T Z
+  const dim3 tiles((K + 31) / 32, (K + 31) / 32);
+  for (int it = 0;; ++it) {
+    if (!track && it == iterations) break;
+    // T = 1.5 I - 0.5 Z Y;  Z <- T Z;  Y <- Y T.
+    // Z Y is not symmetric in floating point, so T != T^T: the Y update must
+    // use T itself.  The products are NT (C = A B^T), so T Z = nt(T, Z) (Z is
+    // symmetric) and Y T = nt(Y, T^T): T is transposed in place between them.
+    // (Taking Y T^T instead is unstable: to first order, a symmetric
+    // perturbation of the iterates along eigenvectors i, j of R grows by
+    // (rho - 1) / 2 per step, rho = (s_i / s_j + s_j / s_i) / 2 with s the
+    // eigenvalues of R^1/2, so once R's condition number exceeds ~34
+    // (s_i / s_j > 3 + sqrt(8)) the converged iterates drift away again.
+    // With Y T the same perturbation maps to a fixed point: stable.)
     if ((e = gemm_nt(z, K, y, K, t, K, K, K, K, -0.5f, 0.0f, 1.5f, nullptr, gws, status, sms,
                      s)) != cudaSuccess)
       return e;
-    if ((e = gemm_nt(y, K, t, K, a, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, gws, status, sms,
-                     s)) != cudaSuccess)
-      return e;
-    float* swap = y;      // new Y is in `a`; the old Y buffer becomes scratch
-    y = a;
-    a = swap;
+    if (track) {
+      // ||I - Z Y||_F / sqrt(K) = 2 ||T - I||_F / sqrt(K): the current iterate's
+      // residual (Z Y = Z (R/c) Z = M R M while the iteration keeps Y = (R/c) Z).
+      frob_partial_kernel<<<kFrobBlocks, 256, 0, s>>>(t, K, K, 1.0f, scal + 64);
+      frob_norm_kernel<<<1, 32, 0, s>>>(scal + 64, kFrobBlocks,
+                                        2.0f / sqrtf(static_cast<float>(K)), scal + 5);
+      float res = 0.0f;
+      if ((e = cudaMemcpyAsync(&res, scal + 5, sizeof(float), cudaMemcpyDeviceToHost, s)) !=
+              cudaSuccess ||
+          (e = cudaStreamSynchronize(s)) != cudaSuccess)
+        return e;
+      if (residuals != nullptr) residuals[it] = res;
+      if (res <= tol) break;
+    }
+    if (it == iterations) break;
     if ((e = gemm_nt(t, K, z, K, a, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, gws, status, sms,
-                     s)) != cudaSuccess)
+                     s)) != cudaSuccess)            // a = T Z (new Z)
       return e;
-    swap = z;
+    transpose_inplace_kernel<<<tiles, dim3(32, 8), 0, s>>>(t, K);     // t = T^T
+    if ((e = gemm_nt(y, K, t, K, z, K, K, K, K, 1.0f, 0.0f, 0.0f, nullptr, gws, status, sms,
+                     s)) != cudaSuccess)            // old Z buffer = Y T (new Y)
+      return e;
+    float* old_y = y;
+    y = z;
     z = a;
-    a = swap;
-    const dim3 tiles((K + 31) / 32, (K + 31) / 32);
+    a = old_y;
     symmetrize_kernel<<<tiles, dim3(32, 8), 0, s>>>(y, K);
     symmetrize_kernel<<<tiles, dim3(32, 8), 0, s>>>(z, K);
+    if (iterations_done != nullptr) *iterations_done = it + 1;
   }
   // Z ~ (R/c)^-1/2:  R^-1/2 = Z / sqrt(c);  R^-1 = Z Z / c
   if (inverse)

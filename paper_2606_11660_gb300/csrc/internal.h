@@ -8,7 +8,48 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 namespace bergson {
+
+// A per-device "done once" record for settings that CUDA keeps per function
+// and per device (the dynamic shared-memory limit of a kernel): ensure(dev,
+// set) runs set() the first time it is asked for device `dev` and remembers
+// success, so that one process can drive several GPUs and two host threads
+// making their first calls at the same time neither skip nor repeat it.  A
+// failed set() is not remembered (the next call tries again).  Devices past
+// the first 64 are not cached: set() runs on every call.
+class PerDeviceOnce {
+ public:
+  template <typename Set>
+  cudaError_t ensure(int dev, Set&& set) {
+    const bool cached = dev >= 0 && dev < 64;
+    const uint64_t bit = cached ? (uint64_t{1} << dev) : 0;
+    if (cached && (done_.load(std::memory_order_acquire) & bit) != 0) return cudaSuccess;
+    std::lock_guard<std::mutex> lk(mu_);
+    if (cached && (done_.load(std::memory_order_relaxed) & bit) != 0) return cudaSuccess;
+    const cudaError_t e = set();
+    if (e == cudaSuccess && cached) done_.fetch_or(bit, std::memory_order_release);
+    return e;
+  }
+
+ private:
+  std::atomic<uint64_t> done_{0};
+  std::mutex mu_;
+};
+
+// Sets `kernel`'s dynamic shared-memory limit to `bytes` on the current
+// device, once per device (see PerDeviceOnce).
+template <typename Kernel>
+cudaError_t smem_attr_once(PerDeviceOnce& once, Kernel kernel, int bytes) {
+  int dev = -1;
+  const cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  return once.ensure(dev, [&] {
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  });
+}
 
 // Launches `kernel` with programmatic stream serialization: it may be
 // scheduled before its predecessor in the stream has finished, and must call
@@ -115,6 +156,8 @@ struct ScoreParams {
   int n_ntiles;         // ceil(N / 256)
   unsigned long long* heaps;  // [grid, topk, QT*128]
   const float* tau0;    // per query starting threshold at tau0[q * topk + topk - 1], or nullptr
+  int tau0_negate;      // 1: the threshold is -tau0[...] (tau0 holds scores against q while
+                        //    the search runs on -q: a bottom-k state)
   int* status;
   uint64_t timeout_ns;
 };
@@ -124,9 +167,11 @@ int record_error(int code, const char* fmt, ...);
 
 // ---- launchers (return the launch error, if any) ----
 
-cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, cudaStream_t s);
+// Both record BERGSON_EMOMENT in *status when a second-moment entry is not > 0.
+cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, int* status,
+                        cudaStream_t s);
 cudaError_t launch_projection_matrix(uint64_t seed, int d, int k, int kind, const float* moment,
-                                     float* out, cudaStream_t s);
+                                     int* status, float* out, cudaStream_t s);
 cudaError_t launch_tile_valid(const uint8_t* mask, int B, int T, int n_tiles, uint8_t* tile_valid,
                               cudaStream_t s);
 cudaError_t launch_wait_probe(int* status, uint64_t timeout_ns, cudaStream_t s);
@@ -144,6 +189,15 @@ cudaError_t launch_reduce(const ModDesc* mods, int n_mods, int k_in, int k_out, 
 
 cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj, int unit,
                                __half* store, int64_t ld_store, float* norms, cudaStream_t s);
+// Column blocks of a store row normalised separately (one module each).
+constexpr int kMaxStoreBlocks = 2048;
+struct StoreBlocks {
+  int32_t offset[kMaxStoreBlocks + 1];   // 0 = offset[0] < ... < offset[n] = K, multiples of 8
+  int32_t n;
+};
+cudaError_t launch_build_store_blocks(const float* proj, int B, int64_t ld_proj,
+                                      const StoreBlocks& blocks, __half* store, int64_t ld_store,
+                                      float* norms, cudaStream_t s);
 cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, bool negate,
                                      __half* qh, cudaStream_t s);
 cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap& tm_q,
@@ -155,8 +209,14 @@ cudaError_t launch_score_pair(int qt, const CUtensorMap& tm_store, const CUtenso
                               const ScoreParams& p, int grid, cudaStream_t s);
 cudaError_t score_pair_max_ctas(int qt, int sms, int* ctas);
 constexpr int kPairMinQueries = 129;   // the pair kernel serves Q >= this
+// Final top-k of queries [q_begin, q_end) from the CTAs' heaps.  Heap rows
+// are local to the scored rows; the results report row_base + row.  With
+// prior_scores / prior_idx (a previous [Q, topk] result over other rows, global
+// indices, ordered as this call's output) the prior entries take part in the
+// selection too; they may alias out_scores / out_idx.
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
-                         int q_begin, int q_end, int qg_base, bool negate, float* out_scores,
+                         int q_begin, int q_end, int qg_base, bool negate, int64_t row_base,
+                         const float* prior_scores, const int64_t* prior_idx, float* out_scores,
                          int64_t* out_idx, cudaStream_t s);
 
 cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit, float* scale,
@@ -168,8 +228,14 @@ size_t fisher_fit_workspace(int64_t n, int64_t K);
 cudaError_t launch_fisher_fit(const float* x, int n, int K, int64_t ldx, float* r, int64_t ldr,
                               float* ws, int* status, int sms, cudaStream_t s);
 size_t fisher_power_workspace(int64_t K);
+// At most `iterations` Newton-Schulz updates.  With residuals != nullptr or
+// tol > 0 the residual ||I - Z Y||_F / sqrt(K) of every iterate is read back
+// (one stream synchronisation per iterate) into residuals[0 ..] and the
+// iteration stops at the first iterate whose residual is <= tol;
+// *iterations_done receives the number of updates applied.
 cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t ldr, float lam,
-                                float damping, int inverse, int iterations, float* m, int64_t ldm,
+                                float damping, int inverse, int iterations, float tol,
+                                float* residuals, int* iterations_done, float* m, int64_t ldm,
                                 float* ws, int* status, int sms, cudaStream_t s);
 
 // Skinny fp32 product C[b, q] = <x_b, y_q> on the tensor cores (on-the-fly

@@ -9,7 +9,8 @@
 // when memory is short or fragmented) is not acceptable.  For them this file
 // keeps a fixed scratch area in static device memory and runs the regular
 // bergson_project_grads path on it.  Nothing here calls cudaMalloc, cudaFree
-// or any allocating library routine.
+// or any allocating library routine; the array's memory is reserved by the
+// CUDA driver when it loads this file's module on a device (see below).
 //
 // Properties a caller must know:
 //   * The scratch is a file-scope __device__ array of BERGSON_NOALLOC_SCRATCH_BYTES
@@ -22,8 +23,16 @@
 //     overlaps on the GPU (e.g. on two streams at once) race on the array and
 //     must be ordered by the caller.
 //   * The device address of the array is looked up once per device, on the
-//     first call that runs on that device (with that device current).  Make
-//     that first call before any stream capture begins.
+//     first call that runs on that device (with that device current).  This
+//     file has no kernels, so under lazy module loading (CUDA's default) that
+//     lookup is what loads its module on the device, and the driver reserves
+//     the 32 MiB array then: the first call can fail with BERGSON_ECUDA when
+//     the device has no 32 MiB left.  A warm-up call with B = 0 and
+//     out = NULL (any valid layer array) does the lookup on the current
+//     device and enqueues nothing, so a caller can take that step early.
+//     Make the first call on each device before any stream capture begins.
+//   * The kernels it runs set their shared-memory limits once per device, so
+//     one process may call this on several GPUs (one scratch array each).
 
 #include <mutex>
 

@@ -545,13 +545,9 @@ template <bool TA>
 cudaError_t launch_xgemm(int grid, size_t smem, cudaStream_t s, const CUtensorMap& tm_y,
                          const CUtensorMap& tm_xh, const CUtensorMap& tm_xl,
                          const XGemmParams& p) {
-  static bool attr_set = false;   // per process; the attribute is per function and device
-  if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(
-        xgemm_kernel<TA>, cudaFuncAttributeMaxDynamicSharedMemorySize, kXSmemBudget);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static PerDeviceOnce attr;
+  const cudaError_t e = smem_attr_once(attr, xgemm_kernel<TA>, kXSmemBudget);
+  if (e != cudaSuccess) return e;
   return launch_dependent(xgemm_kernel<TA>, dim3(grid), dim3(kXThreads), smem, s, tm_y, tm_xh,
                           tm_xl, p);
 }

@@ -63,9 +63,14 @@ __device__ __forceinline__ float counter_draw(uint64_t seed, uint64_t e, int kin
 }
 
 // Entries (i, j) and (i, j + 1), j even, of P' = diag(scale) P, fp32.  They
-// are counters e = i*k + j and e + 1, i.e. both draws of pair e / 2.
+// are counters e = i*k + j and e + 1, i.e. both draws of pair e / 2.  The
+// factored second moments must be positive (the scale is moment_i^-1/2): an
+// entry that is not (zero, negative or NaN) is recorded as BERGSON_EMOMENT in
+// the device status word, and the values computed from it (inf or NaN) are
+// stored as they come.
 __device__ __forceinline__ void projection_pair(uint64_t seed, int i, int j, int k, int kind,
-                                                const float* moment, float* v0, float* v1) {
+                                                const float* moment, int* status, float* v0,
+                                                float* v1) {
   const float inv_sqrt_k = 1.0f / sqrtf(static_cast<float>(k));
   const uint64_t e = static_cast<uint64_t>(i) * k + j;
   if (kind == BERGSON_PROJ_IDENTITY) {
@@ -81,7 +86,9 @@ __device__ __forceinline__ void projection_pair(uint64_t seed, int i, int j, int
     *v1 = counter_draw(seed, e + 1, kind) * inv_sqrt_k;
   }
   if (moment != nullptr) {
-    const float sc = 1.0f / sqrtf(moment[i]);
+    const float m = moment[i];
+    if (!(m > 0.0f) && j == 0 && status != nullptr) atomicCAS(status, 0, kStatusMoment);
+    const float sc = 1.0f / sqrtf(m);
     *v0 = *v0 * sc;
     *v1 = *v1 * sc;
   }
@@ -96,9 +103,9 @@ __device__ __forceinline__ void store_hi_lo(__nv_bfloat16* dst, int64_t hi_idx, 
 
 // Entry pair q = (i, j / 2) of a segment: both values of P'[i, j..j+1] as bf16
 // hi + lo, written transposed.
-__device__ __forceinline__ void prep_pair(const PrepSeg& sg, int i, int j) {
+__device__ __forceinline__ void prep_pair(const PrepSeg& sg, int i, int j, int* status) {
   float v0, v1;
-  projection_pair(sg.seed, i, j, sg.k, sg.kind, sg.moment, &v0, &v1);
+  projection_pair(sg.seed, i, j, sg.k, sg.kind, sg.moment, status, &v0, &v1);
   const int64_t d = sg.d;
   store_hi_lo(sg.dst, j * d + i, (sg.k + j) * d + i, v0);
   store_hi_lo(sg.dst, (j + 1) * d + i, (sg.k + j + 1) * d + i, v1);
@@ -107,30 +114,31 @@ __device__ __forceinline__ void prep_pair(const PrepSeg& sg, int i, int j) {
 // blockIdx.y = segment; threads walk the segment's d*k/2 entry pairs with the
 // input index i fastest, so the transposed bf16 stores are coalesced.  The
 // index arithmetic is 32-bit when the segment allows it (the common case).
-__global__ void prep_kernel(const PrepSeg* __restrict__ segs) {
+__global__ void prep_kernel(const PrepSeg* __restrict__ segs, int* status) {
   griddep_launch_dependents();   // the projection kernel may set itself up meanwhile
   const PrepSeg sg = segs[blockIdx.y];
   const int64_t npairs = static_cast<int64_t>(sg.d) * sg.k / 2;
   if (npairs <= 0x7fffffff) {
     const uint32_t n = static_cast<uint32_t>(npairs), d = static_cast<uint32_t>(sg.d);
     for (uint32_t q = blockIdx.x * blockDim.x + threadIdx.x; q < n; q += gridDim.x * blockDim.x)
-      prep_pair(sg, static_cast<int>(q % d), 2 * static_cast<int>(q / d));
+      prep_pair(sg, static_cast<int>(q % d), 2 * static_cast<int>(q / d), status);
   } else {
     for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < npairs;
          q += static_cast<int64_t>(gridDim.x) * blockDim.x)
-      prep_pair(sg, static_cast<int>(q % sg.d), 2 * static_cast<int>(q / sg.d));
+      prep_pair(sg, static_cast<int>(q % sg.d), 2 * static_cast<int>(q / sg.d), status);
   }
 }
 
 __global__ void projection_matrix_kernel(uint64_t seed, int d, int k, int kind,
-                                         const float* __restrict__ moment, float* __restrict__ out) {
+                                         const float* __restrict__ moment, int* status,
+                                         float* __restrict__ out) {
   const int64_t npairs = static_cast<int64_t>(d) * k / 2;
   for (int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; q < npairs;
        q += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int i = static_cast<int>((2 * q) / k);
     const int j = static_cast<int>((2 * q) % k);
     float v0, v1;
-    projection_pair(seed, i, j, k, kind, moment, &v0, &v1);
+    projection_pair(seed, i, j, k, kind, moment, status, &v0, &v1);
     out[2 * q] = v0;
     out[2 * q + 1] = v1;
   }
@@ -168,23 +176,24 @@ __global__ void wait_probe_kernel(int* status, uint64_t timeout_ns) {
   }
 }
 
-cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, cudaStream_t s) {
+cudaError_t launch_prep(const PrepSeg* segs, int n_segs, int64_t max_pairs, int* status,
+                        cudaStream_t s) {
   if (n_segs <= 0 || max_pairs <= 0) return cudaSuccess;
   const int threads = 256;
   int64_t bx = (max_pairs + 4 * threads - 1) / (4 * threads);   // ~4 pairs per thread
   if (bx > 4096) bx = 4096;
   prep_kernel<<<dim3(static_cast<unsigned>(bx), static_cast<unsigned>(n_segs)), threads, 0, s>>>(
-      segs);
+      segs, status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_projection_matrix(uint64_t seed, int d, int k, int kind, const float* moment,
-                                     float* out, cudaStream_t s) {
+                                     int* status, float* out, cudaStream_t s) {
   const int64_t npairs = static_cast<int64_t>(d) * k / 2;
   const int threads = 256;
   const int64_t blocks = (npairs + threads - 1) / threads;
   projection_matrix_kernel<<<static_cast<unsigned>(blocks < 65535 ? blocks : 65535), threads, 0,
-                             s>>>(seed, d, k, kind, moment, out);
+                             s>>>(seed, d, k, kind, moment, status, out);
   return cudaGetLastError();
 }
 

@@ -646,14 +646,9 @@ __global__ void token_reduce_kernel(const float* __restrict__ tp, int n_mods, in
 template <int KI, int KO, bool TOKEN>
 cudaError_t launch_project_t(const ProjParams& p, int grid, cudaStream_t s) {
   using C = ProjCfg<KI, KO, TOKEN>;
-  static bool attr_set = false;   // per process; the attribute is per function and device
-  cudaError_t e = cudaSuccess;
-  if (!attr_set) {
-    e = cudaFuncSetAttribute(project_kernel<KI, KO, TOKEN>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static PerDeviceOnce attr;
+  const cudaError_t e = smem_attr_once(attr, project_kernel<KI, KO, TOKEN>, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
   return launch_dependent(project_kernel<KI, KO, TOKEN>, dim3(grid), dim3(192), C::kSmemBytes, s,
                           p);
 }

@@ -9,6 +9,7 @@
 namespace bergson {
 
 constexpr int kStatusTimeout = -6;   // BERGSON_EDEVICE_TIMEOUT
+constexpr int kStatusMoment = -7;    // BERGSON_EMOMENT
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

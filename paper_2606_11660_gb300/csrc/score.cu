@@ -141,9 +141,11 @@ __device__ __forceinline__ void score_epilogue(const ScoreParams& p, uint32_t tm
   // Scores below the k-th best of any subset of the rows can never reach the
   // final top-k, so a threshold from a prefix pass (if any) filters from the start.
   const int q_global = (g * QT + qt) * kScoreQT + 32 * quarter + lane;
-  const float tau0 = (p.tau0 != nullptr && q_global < p.Q)
-                         ? p.tau0[static_cast<int64_t>(q_global) * p.topk + p.topk - 1]
-                         : -INFINITY;
+  float tau0 = -INFINITY;
+  if (p.tau0 != nullptr && q_global < p.Q) {
+    const float t = p.tau0[static_cast<int64_t>(q_global) * p.topk + p.topk - 1];
+    tau0 = p.tau0_negate ? -t : t;
+  }
   float tau = tau0;
   // Slots past the last query (ragged query groups) hold zero rows: they take
   // no candidates, so their lanes do not walk every score of every tile.
@@ -559,7 +561,8 @@ __device__ __forceinline__ void bitonic_desc(unsigned long long* keys, int n) {
 }
 
 // negate: the scores were taken against -q (a bottom-k search); report them
-// against q, so the list runs from the lowest score up.
+// against q, so the list runs from the lowest score up.  Key rows are global
+// (row_base already added).
 __device__ __forceinline__ void write_topk(const unsigned long long* keys, int q, int topk,
                                            int negate, float* out_scores, int64_t* out_idx) {
   for (int e = threadIdx.x; e < topk; e += blockDim.x) {
@@ -572,6 +575,36 @@ __device__ __forceinline__ void write_topk(const unsigned long long* keys, int q
   }
 }
 
+// Candidate i of query q for the merge: i < n_heap comes from the heaps (its
+// local row moved to row_base + row), the next topk from the prior result
+// (scores against q, negated back into the search's order for a bottom-k
+// state).  Empty entries become the sentinel-free key 0.
+struct MergeSource {
+  const unsigned long long* heaps;
+  int n_qg, gsize, topk, gl, slot;
+  int64_t n_heap;
+  uint32_t row_base;
+  const float* prior_scores;
+  const int64_t* prior_idx;
+  int q;
+  int negate;
+  __device__ __forceinline__ unsigned long long key(int64_t i) const {
+    if (i < n_heap) {
+      const int cta = gl + static_cast<int>(i / topk) * n_qg;
+      const unsigned long long k =
+          heaps[(static_cast<int64_t>(cta) * topk + i % topk) * gsize + slot];
+      const uint32_t lo = static_cast<uint32_t>(k);
+      if (lo < 0x80000000u || row_base == 0u) return k;      // sentinel, or no offset
+      return (k & 0xFFFFFFFF00000000ull) | static_cast<uint32_t>(~(~lo + row_base));
+    }
+    const int64_t e = static_cast<int64_t>(q) * topk + (i - n_heap);
+    const int64_t idx = prior_idx[e];
+    if (idx < 0) return 0ull;
+    const float v = prior_scores[e];
+    return make_key(negate ? -v : v, static_cast<uint32_t>(idx));
+  }
+};
+
 // Final top-k of one query from the heaps of the CTAs that covered it.
 //
 // select_n > 0: all cpg * topk candidate keys fit in shared memory.  An exact
@@ -583,9 +616,10 @@ __device__ __forceinline__ void write_topk(const unsigned long long* keys, int q
 __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __restrict__ heaps,
                                                     int n_qg, int cpg, int gsize, int topk,
                                                     int q_begin, int q_end, int sort_n,
-                                                    int select_n, int negate,
-                                                    float* __restrict__ out_scores,
-                                                    int64_t* __restrict__ out_idx) {
+                                                    int select_n, int negate, uint32_t row_base,
+                                                    const float* prior_scores,
+                                                    const int64_t* prior_idx, float* out_scores,
+                                                    int64_t* out_idx) {
   extern __shared__ unsigned long long keys[];
   __shared__ unsigned int hist[256];
   __shared__ unsigned long long s_prefix;
@@ -593,15 +627,25 @@ __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __
   const int q = q_begin + blockIdx.x;
   if (q >= q_end) return;
   const int local = q - q_begin;
-  const int gl = local / gsize;
-  const int slot = local % gsize;
-  const int64_t total = static_cast<int64_t>(cpg) * topk;
+  MergeSource src;
+  src.heaps = heaps;
+  src.n_qg = n_qg;
+  src.gsize = gsize;
+  src.topk = topk;
+  src.gl = local / gsize;
+  src.slot = local % gsize;
+  src.n_heap = static_cast<int64_t>(cpg) * topk;
+  src.row_base = row_base;
+  src.prior_scores = prior_scores;
+  src.prior_idx = prior_idx;
+  src.q = q;
+  src.negate = negate;
+  // Every prior entry is read (into shared memory) before any output is
+  // written, so the prior may alias the output.
+  const int64_t total = src.n_heap + (prior_idx != nullptr ? topk : 0);
   if (select_n > 0) {
     const int n = static_cast<int>(total);
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-      const int cta = gl + (i / topk) * n_qg;
-      keys[i] = heaps[(static_cast<int64_t>(cta) * topk + i % topk) * gsize + slot];
-    }
+    for (int i = threadIdx.x; i < n; i += blockDim.x) keys[i] = src.key(i);
     if (threadIdx.x == 0) {
       s_prefix = 0ull;
       s_need = topk;
@@ -658,19 +702,14 @@ __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __
     const int start = first ? 0 : topk;
     for (int i = start + threadIdx.x; i < sort_n; i += blockDim.x) {
       const int64_t ci = consumed + (i - start);
-      unsigned long long k = 0ull;
-      if (ci < total) {
-        const int cta = gl + static_cast<int>(ci / topk) * n_qg;
-        const int e = static_cast<int>(ci % topk);
-        k = heaps[(static_cast<int64_t>(cta) * topk + e) * gsize + slot];
-      }
-      keys[i] = k;
+      keys[i] = ci < total ? src.key(ci) : 0ull;
     }
     consumed += sort_n - start;
     first = false;
     __syncthreads();
     bitonic_desc(keys, sort_n);
   }
+  __syncthreads();
   write_topk(keys, q, topk, negate, out_scores, out_idx);
 }
 
@@ -678,13 +717,9 @@ template <int QT>
 cudaError_t launch_score_t(const CUtensorMap& tms, const CUtensorMap& tmq, const ScoreParams& p,
                            int grid, cudaStream_t s) {
   using C = ScoreCfg<QT>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(score_kernel<QT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static PerDeviceOnce attr;
+  const cudaError_t e = smem_attr_once(attr, score_kernel<QT>, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
   score_kernel<QT><<<grid, C::kThreads, C::kSmemBytes, s>>>(tms, tmq, p);
   return cudaGetLastError();
 }
@@ -699,16 +734,17 @@ cudaError_t launch_score(int qt, const CUtensorMap& tm_store, const CUtensorMap&
 }
 
 template <int QT>
+PerDeviceOnce& pair_attr() {
+  static PerDeviceOnce attr;
+  return attr;
+}
+
+template <int QT>
 cudaError_t launch_score_pair_t(const CUtensorMap& tm_store, const CUtensorMap& tm_q,
                                 const ScoreParams& p, int grid, cudaStream_t s) {
   using C = PairCfg<QT>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(score_pair_kernel<QT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  const cudaError_t e = smem_attr_once(pair_attr<QT>(), score_pair_kernel<QT>, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
   score_pair_kernel<QT><<<grid, C::kThreads, C::kSmemBytes, s>>>(tm_store, tm_q, p);
   return cudaGetLastError();
 }
@@ -716,8 +752,7 @@ cudaError_t launch_score_pair_t(const CUtensorMap& tm_store, const CUtensorMap& 
 template <int QT>
 cudaError_t score_pair_max_ctas_t(int sms, int* ctas) {
   using C = PairCfg<QT>;
-  cudaError_t e = cudaFuncSetAttribute(score_pair_kernel<QT>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  cudaError_t e = smem_attr_once(pair_attr<QT>(), score_pair_kernel<QT>, C::kSmemBytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * (sms / 2));
@@ -745,12 +780,13 @@ cudaError_t score_pair_max_ctas(int qt, int sms, int* ctas) {
 }
 
 cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, int qt, int topk,
-                         int q_begin, int q_end, int /*qg_base*/, bool negate,
-                         float* out_scores, int64_t* out_idx, cudaStream_t s) {
+                         int q_begin, int q_end, int /*qg_base*/, bool negate, int64_t row_base,
+                         const float* prior_scores, const int64_t* prior_idx, float* out_scores,
+                         int64_t* out_idx, cudaStream_t s) {
   const int nq = q_end - q_begin;
   if (nq <= 0) return cudaSuccess;
   const int cpg = grid / n_qg;
-  const int64_t total = static_cast<int64_t>(cpg) * topk;
+  const int64_t total = static_cast<int64_t>(cpg) * topk + (prior_idx != nullptr ? topk : 0);
   int sort_n = 2;
   while (sort_n < total && sort_n < 8192) sort_n <<= 1;
   int select_n = 2;
@@ -759,15 +795,13 @@ cudaError_t launch_merge(const unsigned long long* heaps, int grid, int n_qg, in
   if (!radix) select_n = 0;
   const size_t smem =
       static_cast<size_t>(radix ? total + select_n : sort_n) * sizeof(unsigned long long);
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kMergeSmemKeys * sizeof(unsigned long long));
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static PerDeviceOnce attr;
+  const cudaError_t e = smem_attr_once(
+      attr, merge_kernel, static_cast<int>(kMergeSmemKeys * sizeof(unsigned long long)));
+  if (e != cudaSuccess) return e;
   merge_kernel<<<nq, 512, smem, s>>>(heaps, n_qg, cpg, qt * kScoreQT, topk, q_begin, q_end, sort_n,
-                                     select_n, negate ? 1 : 0, out_scores, out_idx);
+                                     select_n, negate ? 1 : 0, static_cast<uint32_t>(row_base),
+                                     prior_scores, prior_idx, out_scores, out_idx);
   return cudaGetLastError();
 }
 

@@ -78,6 +78,32 @@ __global__ void __launch_bounds__(kRowThreads) normalize_rows_kernel(
   if (norms != nullptr && threadIdx.x == 0) norms[b] = nrm;
 }
 
+// Per-module unit normalisation: CTA (b, j) writes
+//   y[b, o_j:o_{j+1}] = fp16(x[b, o_j:o_{j+1}] / ||x[b, o_j:o_{j+1}]||)
+// (a zero block stays zero) and norms[b * n_blocks + j].  Offsets are
+// multiples of 8, so every block starts on a 16-byte boundary of both rows.
+__global__ void __launch_bounds__(kRowThreads) normalize_blocks_kernel(
+    const float* __restrict__ x, int64_t ldx, const __grid_constant__ StoreBlocks bo,
+    __half* __restrict__ y, int64_t ldy, float* __restrict__ norms) {
+  __shared__ float red[kRowThreads / 32];
+  griddep_wait();                // the rows are usually the preceding reduction's output
+  const int64_t b = blockIdx.x;
+  const int j = blockIdx.y;
+  const int c0 = bo.offset[j], c1 = bo.offset[j + 1];
+  const float4* xr = reinterpret_cast<const float4*>(x + b * ldx + c0);
+  KahanSum ss;
+  for (int i = threadIdx.x; i < (c1 - c0) / 4; i += kRowThreads) {
+    const float4 v = xr[i];
+    ss.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
+  }
+  const float tot = block_sum(ss.s, red);
+  const float scale = tot > 0.0f ? 1.0f / sqrtf(tot) : 0.0f;
+  uint4* yr = reinterpret_cast<uint4*>(y + b * ldy + c0);
+  for (int i = threadIdx.x; i < (c1 - c0) / 8; i += kRowThreads)
+    yr[i] = pack8(xr[2 * i], xr[2 * i + 1], scale);
+  if (norms != nullptr && threadIdx.x == 0) norms[b * bo.n + j] = sqrtf(tot);
+}
+
 // Queries may have any row stride; they are read with scalar loads.  With
 // `negate` the row is written as -q / ||q|| (exactly the negation of the
 // unit row: fp16 rounding is symmetric), which turns a top-k search into a
@@ -103,6 +129,14 @@ cudaError_t launch_build_store(const float* proj, int B, int K, int64_t ld_proj,
   if (B == 0) return cudaSuccess;
   return launch_dependent(normalize_rows_kernel, dim3(B), dim3(kRowThreads), 0, s, proj, K,
                           ld_proj, unit, store, ld_store, norms);
+}
+
+cudaError_t launch_build_store_blocks(const float* proj, int B, int64_t ld_proj,
+                                      const StoreBlocks& blocks, __half* store, int64_t ld_store,
+                                      float* norms, cudaStream_t s) {
+  if (B == 0) return cudaSuccess;
+  return launch_dependent(normalize_blocks_kernel, dim3(B, blocks.n), dim3(kRowThreads), 0, s,
+                          proj, ld_proj, blocks, store, ld_store, norms);
 }
 
 cudaError_t launch_normalize_queries(const float* q, int Q, int K, int64_t ld_q, bool negate,

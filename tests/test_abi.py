@@ -501,3 +501,93 @@ def test_workspace_queries_at_their_size_limits():
     # aggregation: n < 2^31 rows
     assert _ws_query("bergson_aggregate_rows_workspace", (1 << 31) - 1)[0] == bg.BERGSON_OK
     assert _ws_query("bergson_aggregate_rows_workspace", 1 << 31)[0] == bg.BERGSON_EINVAL
+
+
+@pytest.mark.parametrize("n_threads,n_devices", [(2, 1), (16, 4), (32, 64)])
+def test_attribute_record_is_per_device_and_thread_safe(n_threads, n_devices):
+    # Concurrent first calls from several host threads, on several (simulated)
+    # devices: the kernel attribute is set exactly once per device.
+    calls, failures = bg.bergson_debug_attr_once(n_threads, n_devices)
+    assert calls == [1] * n_devices and failures == 0
+
+
+def test_attribute_record_retries_a_failed_setting():
+    calls, failures = bg.bergson_debug_attr_once(8, 3, fail_device=1)
+    assert calls == [1, 2, 1] and failures == 1
+    with pytest.raises(bg.BergsonError):
+        bg.bergson_debug_attr_once(0, 3)
+
+
+def test_moment_status_is_part_of_the_abi():
+    # r_i, c_j > 0 is checked on the device (the values are device memory);
+    # the status it records is a public code with a name and a host message.
+    import re
+    hdr = open(os.path.join(ROOT, "include", "bergson.h")).read()
+    m = re.search(r"BERGSON_EMOMENT\s*=\s*(-?\d+)", hdr)
+    assert m and int(m.group(1)) == bg.BERGSON_EMOMENT == -7
+    assert bg.binding.STATUS_NAMES[bg.BERGSON_EMOMENT] == "BERGSON_EMOMENT"
+    bg.bergson_debug_inject_status(bg.BERGSON_EMOMENT, 1)
+    assert _proj([_layer()], B=0) == bg.BERGSON_EMOMENT
+    assert "injected" in bg.bergson_last_error()
+    assert _proj([_layer()], B=0) == bg.BERGSON_OK
+
+
+def test_store_blocks_validation():
+    f = bg.lib().bergson_build_store_blocks
+
+    def call(offs, B=4, K=64, ld_proj=64, ld_store=64, row_offset=0, N_cap=4, n=None):
+        arr = (ctypes.c_int64 * len(offs))(*offs)
+        return f(FAKE, B, K, ld_proj, arr, len(offs) - 1 if n is None else n, FAKE, ld_store,
+                 row_offset, N_cap, None, None)
+
+    assert call([0, 32, 64], B=0) == bg.BERGSON_OK
+    assert call([0, 64], B=0) == bg.BERGSON_OK
+    assert call([8, 64]) == bg.BERGSON_EINVAL            # must start at 0
+    assert call([0, 32]) == bg.BERGSON_EINVAL            # must end at K
+    assert call([0, 32, 32, 64]) == bg.BERGSON_EINVAL    # empty block
+    assert call([0, 40, 32, 64]) == bg.BERGSON_EINVAL    # decreasing
+    assert call([0, 36, 64]) == bg.BERGSON_EALIGN        # not a multiple of 8
+    assert call([0, 64], n=0) == bg.BERGSON_EINVAL
+    assert call([0, 64], n=2049) == bg.BERGSON_EINVAL
+    assert call([0, 64], ld_store=60) == bg.BERGSON_EINVAL
+    assert call([0, 64], row_offset=1) == bg.BERGSON_EINVAL
+    assert f(FAKE, 4, 64, 64, None, 1, FAKE, 64, 0, 4, None, None) == bg.BERGSON_EINVAL
+
+
+def test_chunked_and_host_scoring_validation():
+    L = bg.lib()
+    ws = ctypes.c_size_t()
+    assert L.bergson_score_topk_update_workspace(256, 8, 5, ctypes.byref(ws)) == 0
+    full = ctypes.c_size_t()
+    assert L.bergson_score_topk_workspace(100_000, 256, 8, 5, ctypes.byref(full)) == 0
+    assert ws.value == full.value                       # independent of the chunk's rows
+    assert L.bergson_score_topk_update_workspace(256, 8, 0, ctypes.byref(ws)) == bg.BERGSON_EINVAL
+    assert L.bergson_score_topk_update_workspace(256, 8, 2000, ctypes.byref(ws)) == bg.BERGSON_EUNSUPPORTED
+
+    def upd(N=10, row_base=0, topk=5, K=256, ld=256, init=1, wsb=1 << 30, fn=L.bergson_score_topk_update):
+        return fn(FAKE, N, K, ld, row_base, FAKE, 8, K, topk, init, FAKE, FAKE, FAKE, wsb, None)
+
+    # a chunk may hold fewer rows than topk; nothing runs without a device
+    assert upd(N=3, topk=5) in (bg.BERGSON_ECUDA, bg.BERGSON_OK)
+    assert upd(N=0) == bg.BERGSON_EINVAL
+    assert upd(row_base=-1) == bg.BERGSON_EINVAL
+    assert upd(row_base=(1 << 31) - 10) == bg.BERGSON_EINVAL
+    assert upd(K=100, ld=104) == bg.BERGSON_EALIGN
+    assert upd(wsb=16) == bg.BERGSON_EWORKSPACE
+    assert upd(fn=L.bergson_score_bottomk_update, topk=2000) == bg.BERGSON_EUNSUPPORTED
+
+    assert L.bergson_score_topk_host_workspace(1000, 256, 8, 5, ctypes.byref(ws)) == 0
+    assert ws.value >= 2 * 1000 * 256 * 2 + full.value
+    assert L.bergson_score_topk_host_workspace(0, 256, 8, 5, ctypes.byref(ws)) == bg.BERGSON_EINVAL
+
+    def host(ptr=FAKE, N=1000, ld=256, chunk=100, topk=5, wsb=1 << 30):
+        return L.bergson_score_topk_host(ptr, N, 256, ld, FAKE, 8, 256, topk, 0, chunk, FAKE, FAKE,
+                                         FAKE, wsb, None, None)
+
+    assert host(ptr=None) == bg.BERGSON_EINVAL
+    assert host(chunk=0) == bg.BERGSON_EINVAL
+    assert host(ld=260) == bg.BERGSON_EALIGN
+    assert host(ptr=FAKE + 8) == bg.BERGSON_EALIGN
+    assert host(topk=2000) == bg.BERGSON_EUNSUPPORTED
+    assert host(N=3) == bg.BERGSON_EINVAL               # the whole store still needs topk rows
+    assert host(wsb=1 << 16) == bg.BERGSON_EWORKSPACE

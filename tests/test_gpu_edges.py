@@ -67,3 +67,32 @@ def test_many_small_layers():
     out = run_project(gl, 2, 40, None, ld)
     want = orc.project_grads(ol, None, ld)
     assert rel_frobenius(np32(out).astype(np.float64), want).max() <= 1e-4
+
+
+@pytest.mark.parametrize("bad", [0.0, -1.0, float("nan")])
+def test_nonpositive_second_moment_is_reported_by_the_device(bad):
+    # r, c live on the device, so only the kernel that reads them can check
+    # r, c > 0: it records BERGSON_EMOMENT in the status word, nothing faults,
+    # and the context stays usable (the word is cleared once reported).
+    spec = wl.ModuleSpec("lin", 64, 128)
+    gl, ol, ld = make_layers([spec], 4, 50, [(16, 16)], rc=True)
+    assert bg.bergson_sync_status() == bg.BERGSON_OK
+    r_bad = gl[0].r.clone()
+    r_bad[17] = bad
+    bad_layer = bg.Layer(gl[0].A, gl[0].G, 16, 16, gl[0].seed_in, gl[0].seed_out, r_bad, gl[0].c,
+                         0)
+    ws = bg.workspace_tensor(bg.bergson_project_grads_workspace([bad_layer], 4, 50), DEV)
+    out = torch.empty((4, ld), device=DEV)
+    bg.bergson_project_grads([bad_layer], 4, 50, None, out, ws)
+    assert bg.bergson_sync_status() == bg.BERGSON_EMOMENT
+    assert "second-moment" in bg.bergson_last_error()
+    assert bg.bergson_sync_status() == bg.BERGSON_OK          # cleared once reported
+    c_bad = gl[0].c.clone()
+    c_bad[3] = bad
+    P = torch.empty((spec.d_in, 16), device=DEV)
+    bg.bergson_projection_matrix(gl[0].seed_in, spec.d_in, 16, bg.BERGSON_PROJ_GAUSSIAN, c_bad, P)
+    assert bg.bergson_sync_status() == bg.BERGSON_EMOMENT
+    # the same call with valid moments still matches the oracle afterwards
+    out = run_project(gl, 4, 50, None, ld)
+    want = orc.project_grads(ol, None, ld)
+    assert rel_frobenius(np32(out).astype(np.float64), want).max() <= 1e-4

@@ -91,3 +91,30 @@ def test_precondition_rows_and_whitened_scores():
     assert _rel(got, want) < 2e-3
     want_store, _ = orc.build_store(want)
     np.testing.assert_allclose(store.float().cpu().numpy(), want_store.astype(np.float32), atol=2e-3)
+
+
+def test_newton_schulz_stays_converged_on_ill_conditioned_R():
+    # rank 64 of K = 1024 with damping 0.01: condition number ~2,500 (far above
+    # the ~34 at which taking Y T^T for Y T made the converged iterates
+    # diverge).  Every residual after convergence stays at the fp32 floor.
+    g = wl.generator(25, "cpu")
+    K = 1024
+    x = torch.randn((64, K), generator=g)
+    R = _fit(x.to(DEV))
+    M = torch.full((K, K), float("nan"), device=DEV)
+    ws = bg.workspace_tensor(bg.bergson_fisher_preconditioner_workspace(K), DEV)
+    done, res = bg.bergson_fisher_preconditioner_tol(R, None, K, 1.0, 0.01,
+                                                     bg.BERGSON_FISHER_INV_SQRT, 60, 0.0, M, ws)
+    assert bg.bergson_sync_status() == bg.BERGSON_OK, bg.bergson_last_error()
+    assert done == 60 and len(res) == 61
+    first = next(i for i, r in enumerate(res) if r <= 1e-4)
+    assert first <= 40 and max(res[first:]) <= 1e-4, res
+    want = orc.fisher_power(orc.fisher_mix(orc.fisher_fit(x.numpy()), None, 1.0, 0.01), -0.5)
+    assert _rel(np32(M).astype(np.float64), want) < 1e-3
+    # the stopping rule ends at the first iterate within tol, with the same M
+    M2 = torch.full((K, K), float("nan"), device=DEV)
+    done2, res2 = bg.bergson_fisher_preconditioner_tol(R, None, K, 1.0, 0.01,
+                                                       bg.BERGSON_FISHER_INV_SQRT, 60, 1e-4, M2,
+                                                       ws)
+    assert done2 == first and len(res2) == first + 1 and res2[-1] <= 1e-4
+    assert _rel(np32(M2).astype(np.float64), want) < 1e-3

@@ -278,6 +278,55 @@ def test_build_store_matches_oracle():
     np.testing.assert_array_equal(store[:9, :264].cpu().numpy(), X.numpy().astype(np.float16))
 
 
+def test_build_store_blocks_matches_oracle():
+    # per-module unit norm: blocks of 256, 512, 1024 and 256 columns (module
+    # blocks k_out x k_in), scaled very differently, one zero block, rows
+    # appended at an offset into a store with padded rows
+    g = wl.generator(12, "cpu")
+    offs = [0, 256, 768, 1792, 2048]
+    scale = torch.cat([torch.full((256,), 30.0), torch.full((512,), 1e-3), torch.ones(1024),
+                       torch.full((256,), 5.0)])
+    X = torch.randn((7, 2048), generator=g) * scale
+    X[3, 256:768] = 0.0
+    proj = torch.full((7, 2052), float("nan"))
+    proj[:, :2048] = X
+    proj = proj.to(DEV)
+    store = torch.full((12, 2056), float("nan"), dtype=torch.float16, device=DEV)
+    norms = torch.empty((7, 4), dtype=torch.float32, device=DEV)
+    bg.bergson_build_store_blocks(proj, 7, 2048, offs, store, 4, norms)
+    assert bg.bergson_sync_status() == bg.BERGSON_OK, bg.bergson_last_error()
+    want, want_norms = orc.build_store_blocks(X.numpy().astype(np.float64), offs)
+    got = store.cpu()
+    assert torch.isnan(got[:4]).all() and torch.isnan(got[11:]).all()
+    assert torch.isnan(got[4:11, 2048:]).all()
+    g16 = got[4:11, :2048].float().numpy()
+    ulp = np.spacing(np.abs(want)).astype(np.float32)           # one fp16 ulp per element
+    assert np.all(np.abs(g16 - want.astype(np.float32)) <= ulp)
+    np.testing.assert_array_equal(g16[3, 256:768], 0.0)
+    np.testing.assert_allclose(np32(norms), want_norms, rtol=1e-6)
+    # one block equals the whole-row store, bit for bit
+    a = torch.empty((7, 2048), dtype=torch.float16, device=DEV)
+    b = torch.empty((7, 2048), dtype=torch.float16, device=DEV)
+    bg.bergson_build_store_blocks(proj, 7, 2048, [0, 2048], a, 0)
+    bg.bergson_build_store(proj, 7, 2048, True, b, 0)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+
+
+def test_build_store_blocks_one_per_module_of_a_llama_block_set():
+    # 160 modules of 256 columns (the Llama-8B-shaped layer set at k = 16)
+    g = wl.generator(13, "cpu")
+    K = 160 * 256
+    X = torch.randn((8, K), generator=g) * torch.rand((1, K), generator=g).mul(10).add(0.1)
+    offs = list(range(0, K + 1, 256))
+    store = torch.empty((8, K), dtype=torch.float16, device=DEV)
+    bg.bergson_build_store_blocks(X.to(DEV), 8, K, offs, store, 0)
+    assert bg.bergson_sync_status() == bg.BERGSON_OK, bg.bergson_last_error()
+    want, _ = orc.build_store_blocks(X.numpy().astype(np.float64), offs)
+    g16 = store.cpu().float().numpy()
+    assert np.all(np.abs(g16 - want.astype(np.float32)) <= np.spacing(np.abs(want)))
+
+
 def _store_from_rows(rows: torch.Tensor) -> torch.Tensor:
     N, K = rows.shape
     store = torch.empty((N, K), dtype=torch.float16, device=DEV)
