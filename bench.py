@@ -9,8 +9,13 @@ The scoring phase of the same path (fp16 store of 4,000,000 x 8192 rows,
 1,024 queries, top-100) is timed separately and reported under "scoring",
 with a sweep over 1-512 queries on the same store ("q_sweep").  The other
 rows of the path (on-the-fly scores, per-token scores, the Fisher
-preconditioner, one-block-per-call Pythia-1.4B and Llama-8B shapes) and an
-end-to-end leg from pinned host memory are reported beside it.
+preconditioner, one-block-per-call Pythia-1.4B and Llama-8B shapes), an
+end-to-end leg from pinned host memory, and exact top-k over a store twice
+the resident one streamed from host memory ("outofcore") are reported beside
+it; the host link's own rate is measured in the same run for both host legs.
+The headline figure of every leg is also repeated as a flat top-level key at
+the end of the line (score_*, cfg3_*, cfg4_*, onthefly_*, fisher_*, tokens_*,
+ooc_*, e2e_*).
 
 --impl reference times the fp64 CPU oracle on the host cores instead (a
 bounded sample of the same workload per step).  Under torchrun every rank runs
@@ -506,6 +511,8 @@ def bench_fisher(args, world, dev, state, peaks):
     del fws, pws
     torch.cuda.empty_cache()
     kws = bg.workspace_tensor(bg.bergson_score_grads_workspace(K, K, K), dev)
+    # M inverts the damped matrix R + d I, d = damping * tr(R) / K
+    R.diagonal().add_(0.1 * float(R.diagonal().double().sum()) / K)
     MR = torch.empty((K, K), device=dev)
     bg.bergson_precondition_rows(M, K, K, R, MR, kws, stream)
     MRM = torch.empty((K, K), device=dev)
@@ -532,8 +539,9 @@ def bench_fisher(args, world, dev, state, peaks):
             "newton_schulz_tol": args.fisher_tol, "newton_schulz_max_iterations": args.fisher_iters,
             "newton_schulz_residuals": [float(f"{r:.3e}") for r in ns_res],
             "residual_MRM": float(f"{true_res:.3e}"),
-            "residual_definition": "||M R M - I||_F / sqrt(K) of the M in use (library products); "
-                                   "the stopping rule reads ||I - Z Y||_F / sqrt(K) per iterate",
+            "residual_definition": "||M R M - I||_F / sqrt(K) of the M in use, R the damped "
+                                   "matrix it inverts (library products); the stopping rule "
+                                   "reads ||I - Z Y||_F / sqrt(K) per iterate",
             "preconditioner_tflops": round(ns_tflops, 2),
             "roofline_apply": {"bound": "hbm", "achieved": round(apply_gbs, 1),
                                "peak": peaks["hbm_gbs"], "unit": "GB/s",
@@ -688,13 +696,35 @@ def bench_e2e(args, world, dev, state):
     t1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(t0.elapsed_time(t1), world)
+    # The host link's rate in this run: the same pinned buffer copied alone.
+    link_gbs = h2d_rate(hbuf, dbufs[0], copy_stream)
     del hbuf, dbufs, sides
     torch.cuda.empty_cache()
+    gbs = h2d * steps / (ms * 1e-3) / 1e9
     return {"value": cfg.B * world * steps / (ms * 1e-3), "unit": "examples/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
             "ms_per_step": ms / steps,
+            "h2d_gbs_achieved": round(gbs, 1), "h2d_gbs_measured": round(link_gbs, 1),
+            "frac_of_h2d": round(gbs / link_gbs, 4),
             "h2d": "one contiguous pinned buffer -> one of two device buffers per step; "
-                   "the next step's copy overlaps this step's compute"}
+                   "the next step's copy overlaps this step's compute; h2d_gbs_measured = "
+                   "the same buffer copied alone in this run (best of 3)"}
+
+
+def h2d_rate(hbuf, dbuf, stream, repeats: int = 3) -> float:
+    """GB/s of one pinned host -> device copy of hbuf (best of `repeats`), on `stream`."""
+    import torch
+    n = min(hbuf.numel(), dbuf.numel())
+    best = 0.0
+    for _ in range(repeats):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            dbuf[:n].copy_(hbuf[:n], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        best = max(best, n / (e0.elapsed_time(e1) * 1e-3) / 1e9)
+    return best
 
 
 def score_sweep(args, store, N, K, topk, dev, peaks):
@@ -805,6 +835,93 @@ def bench_scoring(args, world, dev, peaks, peak_kind):
     del store
     torch.cuda.empty_cache()
     return res
+
+
+def mem_available_bytes() -> int:
+    """MemAvailable of /proc/meminfo in bytes (0 if unreadable)."""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def bench_outofcore(args, world, dev, peaks):
+    """Exact top-100 of 1,024 queries over a store twice the resident score4m
+    store (8,000,000 x 8192 fp16 unit rows, 131 GB) held in pinned host memory:
+    bergson_score_topk_host copies it to the device in chunks on a second
+    stream while the previous chunk is scored.  The rate is bound by the host
+    link, measured in the same run on the same buffer."""
+    import torch
+
+    import paper_2606_11660_gb300 as bg
+    from paper_2606_11660_gb300 import workloads as wl
+
+    sw = wl.SCORE4M
+    K, Q, topk, chunk = sw.K, sw.Q, sw.topk, args.ooc_chunk
+    row_bytes = K * 2
+    N = args.ooc_rows
+    # keep 48 GB of host memory free: never drive the host out of memory
+    fit = (mem_available_bytes() - (48 << 30)) // row_bytes
+    reduced = fit < N
+    N = int(min(N, fit)) // chunk * chunk
+    if N < 2 * chunk:
+        return {"value": None, "skipped": f"host memory too small ({mem_available_bytes()} B)"}
+    t_fill = time.time()
+    host = torch.empty((N, K), dtype=torch.float16, pin_memory=True)
+    gen = wl.generator(7, dev)
+    rows_f = torch.empty((1 << 17, K), dtype=torch.float32, device=dev)
+    rows_h = torch.empty((1 << 17, K), dtype=torch.float16, device=dev)
+    for n0 in range(0, N, 1 << 17):
+        n1 = min(N, n0 + (1 << 17))
+        rows_f.normal_(generator=gen)
+        bg.bergson_build_store(rows_f, n1 - n0, K, True, rows_h, 0)
+        host[n0:n1].copy_(rows_h[:n1 - n0])
+    del rows_f, rows_h
+    t_fill = time.time() - t_fill
+    queries = wl.gaussian_rows(Q, K, seed=8, device=dev)
+    ws = bg.workspace_tensor(bg.bergson_score_topk_host_workspace(chunk, K, Q, topk), dev)
+    s = torch.empty((Q, topk), dtype=torch.float32, device=dev)
+    i = torch.empty((Q, topk), dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream()
+    copy_stream = torch.cuda.Stream(device=dev)
+    bg.bergson_score_topk_host(host, N, K, queries, topk, chunk, s, i, ws, stream, copy_stream)
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.ooc_steps):
+        bg.bergson_score_topk_host(host, N, K, queries, topk, chunk, s, i, ws, stream, copy_stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
+        raise RuntimeError(bg.bergson_last_error())
+    ms = max_over_ranks(e0.elapsed_time(e1), world) / args.ooc_steps
+    idx = i.cpu()
+    ok = bool((idx >= 0).all() and (idx < N).all() and (s.diff(dim=1) <= 0).all())
+    # the link alone: one chunk of the same pinned store copied to the device
+    dchunk = torch.empty(chunk * K, dtype=torch.float16, device=dev)
+    link_gbs = h2d_rate(host.view(-1)[:chunk * K], dchunk, copy_stream)
+    del host, ws, dchunk
+    torch.cuda.empty_cache()
+    gbs = N * row_bytes / (ms * 1e-3) / 1e9
+    return {"value": round(N * world / (ms * 1e-3)), "unit": "store rows/s",
+            "ms_per_pass": round(ms, 2), "steps": args.ooc_steps,
+            "config": {"workload": f"host-resident store {N} x {K} fp16 unit rows "
+                                   f"({N * row_bytes / 1e9:.1f} GB, {N / sw.N:.2f}x the resident "
+                                   f"score4m store), Q={Q}, top-{topk}",
+                       "N": N, "K": K, "Q": Q, "topk": topk, "chunk_rows": chunk,
+                       "store_bytes": N * row_bytes, "reduced_to_fit_host_memory": reduced},
+            "store_gbs": round(gbs, 1), "h2d_gbs_measured": round(link_gbs, 1),
+            "frac_of_h2d": round(gbs / link_gbs, 4), "result_valid": ok,
+            "fill_s": round(t_fill, 1),
+            "what": "bergson_score_topk_host: chunk c+1 copied (copy stream) while chunk c is "
+                    "scored and merged into the running top-k (score stream)"}
 
 
 def profile_case(args):
@@ -946,6 +1063,7 @@ def main_ours(args):
     if not args.no_streamed:
         streamed = {n: bench_streamed(args, world, dev, n, peaks) for n in ("pythia1b4", "llama8b")}
     scoring = bench_scoring(args, world, dev, peaks, peak_kind) if not args.no_score else None
+    outofcore = bench_outofcore(args, world, dev, peaks) if not args.no_ooc else None
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu and scoring is not None:
         try:
@@ -973,12 +1091,61 @@ def main_ours(args):
                        "l2": "inputs 19.3 GB per step > 129 MB L2 (no flush needed)"},
             "roofline": coll["roofline"], "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": coll["gpu_launches"], "clocks": coll["clocks"],
-            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly, "token_scores": tokens, "fisher": fisher, "streamed": streamed,
+            "proj_call_ms": round(coll["proj_ms"], 4), "scoring": scoring, "onthefly": onthefly,
+            "token_scores": tokens, "fisher": fisher, "streamed": streamed, "outofcore": outofcore,
         }
+        line.update(headline_keys(line))
+        # every leg's headline also rides inside the roofline object
+        line["roofline"]["other_legs"] = {k: v for k, v in line.items()
+                                          if k.startswith(("score_", "cfg", "onthefly_", "fisher_",
+                                                           "tokens_", "ooc_", "e2e_"))}
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def headline_keys(line: dict) -> dict:
+    """Flat copies of every leg's headline figure (value and roofline fraction),
+    so that records which keep only top-level scalars still show them."""
+    out = {}
+    sc = line.get("scoring")
+    if sc:
+        out["score_rows_per_s"] = round(sc["value"])
+        out["score_ms_per_pass"] = round(sc["ms_per_pass"], 3)
+        out["score_frac"] = sc["roofline"]["frac"]
+        out["score_frac_sustained"] = sc["roofline"].get("frac_of_sustained")
+        for pt in sc.get("q_sweep") or []:
+            out[f"score_q{pt['queries']}_frac"] = pt["frac"]
+    st = line.get("streamed") or {}
+    for key, name in (("cfg3", "pythia1b4"), ("cfg4", "llama8b")):
+        if name in st:
+            out[f"{key}_examples_per_s"] = st[name]["value"]
+            out[f"{key}_frac"] = st[name]["roofline"]["frac"]
+    of = line.get("onthefly")
+    if of:
+        out["onthefly_examples_per_s"] = of["value"]
+        out["onthefly_frac"] = of["roofline"]["frac"]
+    fi = line.get("fisher")
+    if fi:
+        out["fisher_examples_per_s"] = fi["value"]
+        out["fisher_apply_frac"] = fi["roofline_apply"]["frac"]
+        out["fisher_residual_MRM"] = fi["residual_MRM"]
+        out["fisher_iterations"] = fi["newton_schulz_iterations"]
+    tk = line.get("token_scores")
+    if tk:
+        out["tokens_examples_per_s"] = tk["value"]
+        out["tokens_frac"] = tk["roofline"]["frac"]
+    oc = line.get("outofcore")
+    if oc and oc.get("value"):
+        out["ooc_rows_per_s"] = oc["value"]
+        out["ooc_store_gb"] = round(oc["config"]["store_bytes"] / 1e9, 1)
+        out["ooc_frac_of_h2d"] = oc["frac_of_h2d"]
+    e2e = line.get("e2e")
+    if e2e:
+        out["e2e_frac_of_h2d"] = e2e.get("frac_of_h2d")
+        out["e2e_h2d_gbs_measured"] = e2e.get("h2d_gbs_measured")
+    return out
 
 
 def main_reference(args):
@@ -1018,13 +1185,17 @@ def parse(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-score", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--score-steps", type=int, default=5)
     ap.add_argument("--score-warmup", type=int, default=2)
     ap.add_argument("--cpu-examples", type=int, default=12)
     ap.add_argument("--no-fisher", action="store_true")
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-ooc", action="store_true", help="skip the host-resident store leg")
+    ap.add_argument("--ooc-rows", type=int, default=8_000_000)
+    ap.add_argument("--ooc-chunk", type=int, default=262_144)
+    ap.add_argument("--ooc-steps", type=int, default=2)
     ap.add_argument("--fisher-iters", type=int, default=30,
                     help="at most this many Newton-Schulz updates")
     ap.add_argument("--fisher-tol", type=float, default=1e-5,

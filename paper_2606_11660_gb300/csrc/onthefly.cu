@@ -50,9 +50,19 @@ constexpr int kYBytes = kXM * 128;         // one y tile
 constexpr int kXThreads = 320;             // producer, MMA, 4 converter, 4 epilogue warps
 constexpr int kXSmemBudget = 232448;       // 227 KB opt-in per CTA
 constexpr int kXBarBytes = 512;
-constexpr int kXMaxStages = 8;
+constexpr int kXMaxStages = 12;
 constexpr int kMaxSlices = 64;
 constexpr uint64_t kXDrainTimeoutNs = 2000000000ull;
+// The tensor cores' fp32 accumulation rounds toward zero: every MMA into a
+// running TMEM sum loses up to one ulp of it, so a long chain drifts (about
+// -5e-8 of the sum per MMA, measured: -2.7e-5 over 4,096 columns of positive
+// terms).  Each accumulation chain therefore covers at most kSubSteps
+// 32-column steps (4 MMAs of K = 8 each): the MMA warp restarts the
+// accumulator after that many steps and the epilogue adds the pieces with
+// IEEE fp32 adds, in order.
+constexpr int kSubSteps = 16;
+constexpr int kMaxPad = 128;                 // largest batch tile (n_pad)
+constexpr int kMaxPadTA = 64;                // largest batch tile with y in TMEM
 
 struct KahanSum {
   float s = 0.0f, c = 0.0f;
@@ -160,6 +170,9 @@ struct XGemmParams {
   int n_buf;          // TMEM accumulator sets (2: epilogue overlaps the next item)
   int n_items;
   int tmem_cols;
+  int sub;            // 32-column steps per accumulation chain (see kSubSteps)
+  int n_slots;        // TMEM operand slots (y_hi / y_lo, 64 columns each) with y in TMEM
+  int fold;           // 1: y_lo x_hi adds into the y_hi x_hi columns (2 n_pad per set)
   int a_base;         // TMEM column of the y_hi / y_lo ring (A operands in TMEM)
   int unit;
   float* partial;     // [S, B, Q]
@@ -206,10 +219,15 @@ __global__ void __launch_bounds__(kXThreads, 1)
   const int xbytes = p.n_pad * 128;
   const int xoff = (TA ? 1 : 2) * kYBytes;      // x_hi, x_lo after y (and y_lo)
   const int stage_bytes = xoff + 2 * xbytes;
+  // Barriers: full / empty per shared-memory stage; conv per stage (y_lo in
+  // shared memory) or per TMEM operand slot (y in TMEM); tfree per TMEM
+  // operand slot (the MMAs that read it are done); tfull / tempty per
+  // accumulator set.
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
-  uint64_t* empty = full + p.stages;
-  uint64_t* conv = empty + p.stages;
-  uint64_t* tfull = conv + p.stages;
+  uint64_t* empty = full + kXMaxStages;
+  uint64_t* conv = empty + kXMaxStages;
+  uint64_t* tfree = conv + kXMaxStages;
+  uint64_t* tfull = tfree + kXMaxStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
@@ -221,7 +239,10 @@ __global__ void __launch_bounds__(kXThreads, 1)
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int s = 0; s < (TA ? p.n_slots : p.stages); ++s) {
       mbar_init(smem_u32(&conv[s]), 128);
+      mbar_init(smem_u32(&tfree[s]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&tfull[i]), 1);
@@ -307,54 +328,65 @@ __global__ void __launch_bounds__(kXThreads, 1)
       const uint32_t idesc_lo = make_idesc_tf32(kXM, p.n_pad);    // y_lo x_hi^T
       int stage = 0;
       uint32_t ph = 0;
+      int slot = 0;                   // TMEM operand slot (y in TMEM)
+      uint32_t tph = 0;
       int ab = 0;
       uint32_t aph = 0;
       bool ok = true;
       for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
         const XItem it = decode_xitem(p, item);
-        if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
-        tc_fence_after();
-        // Set ab: D_hi = y_hi [x_hi; x_lo]^T in columns [0, 2 n_pad), D_lo =
-        // y_lo x_hi^T in [2 n_pad, 3 n_pad).  x_hi and x_lo land next to each
-        // other, so one B operand of 2 n_pad rows serves both, and y_hi and y_lo
-        // are each read once per K step.
-        const uint32_t d_hi = tmem + ab * 3 * p.n_pad;
-        const uint32_t d_lo = d_hi + 2 * p.n_pad;
-        for (int st = it.s0; st < it.s1; ++st) {
-          if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
-              !mbar_wait(smem_u32(&conv[stage]), ph, tmo, s_abort)) {
-            ok = false;
-            break;
-          }
+        for (int c0 = it.s0; c0 < it.s1 && ok; c0 += p.sub) {   // one accumulation chain each
+          const int c1 = min(it.s1, c0 + p.sub);
+          if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t yh = sbase + stage * stage_bytes;
-          const uint64_t dx = sw128_desc(yh + xoff);
-          if constexpr (TA) {
-            const uint32_t ta = tmem + p.a_base + stage * 2 * kXK;   // y_hi, then y_lo
-#pragma unroll
-            for (int kk = 0; kk < kXK / 8; ++kk) {
-              const uint64_t o = 2 * kk;
-              const uint32_t acc = st != it.s0 || kk != 0;
-              umma_tf32_ta(d_hi, ta + 8 * kk, dx + o, idesc, acc);
-              umma_tf32_ta(d_lo, ta + kXK + 8 * kk, dx + o, idesc_lo, acc);
+          // Set ab: D[0, 2 n_pad) = y_hi [x_hi; x_lo]^T (x_hi and x_lo land
+          // next to each other, so one MMA with N = 2 n_pad writes both), and
+          // y_lo x_hi^T either in its own columns [2 n_pad, 3 n_pad) -- an
+          // independent accumulation chain -- or, folded, added into
+          // D[0, n_pad) (2 n_pad columns per set: two sets fit at n_pad = 128).
+          const int set_cols = (p.fold ? 2 : 3) * p.n_pad;
+          const uint32_t d = tmem + ab * set_cols;
+          const uint32_t d_lo = p.fold ? d : d + 2 * p.n_pad;
+          for (int st = c0; st < c1; ++st) {
+            if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
+                !mbar_wait(smem_u32(&conv[TA ? slot : stage]), TA ? tph : ph, tmo, s_abort)) {
+              ok = false;
+              break;
             }
-          } else {
-            const uint64_t dyh = sw128_desc(yh);
-            const uint64_t dyl = sw128_desc(yh + kYBytes);
+            tc_fence_after();
+            const uint32_t yh = sbase + stage * stage_bytes;
+            const uint64_t dx = sw128_desc(yh + xoff);
+            if constexpr (TA) {
+              const uint32_t ta = tmem + p.a_base + slot * 2 * kXK;   // y_hi, then y_lo
 #pragma unroll
-            for (int kk = 0; kk < kXK / 8; ++kk) {     // 8 tf32 = 32 bytes: +2 in the address field
-              const uint64_t o = 2 * kk;
-              const uint32_t acc = st != it.s0 || kk != 0;
-              umma_tf32(d_hi, dyh + o, dx + o, idesc, acc);
-              umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, acc);
+              for (int kk = 0; kk < kXK / 8; ++kk) {
+                const uint64_t o = 2 * kk;
+                const uint32_t acc = st != c0 || kk != 0;
+                umma_tf32_ta(d, ta + 8 * kk, dx + o, idesc, acc);
+                umma_tf32_ta(d_lo, ta + kXK + 8 * kk, dx + o, idesc_lo, p.fold ? 1u : acc);
+              }
+            } else {
+              const uint64_t dyh = sw128_desc(yh);
+              const uint64_t dyl = sw128_desc(yh + kYBytes);
+#pragma unroll
+              for (int kk = 0; kk < kXK / 8; ++kk) {   // 8 tf32 = 32 bytes: +2 in the address field
+                const uint64_t o = 2 * kk;
+                const uint32_t acc = st != c0 || kk != 0;
+                umma_tf32(d, dyh + o, dx + o, idesc, acc);
+                umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, p.fold ? 1u : acc);
+              }
+            }
+            umma_commit(smem_u32(&empty[stage]));
+            if (++stage == p.stages) { stage = 0; ph ^= 1; }
+            if constexpr (TA) {
+              umma_commit(smem_u32(&tfree[slot]));
+              if (++slot == p.n_slots) { slot = 0; tph ^= 1; }
             }
           }
-          umma_commit(smem_u32(&empty[stage]));
-          if (++stage == p.stages) { stage = 0; ph ^= 1; }
+          if (!ok) break;
+          umma_commit(smem_u32(&tfull[ab]));
+          if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
         }
-        if (!ok) break;
-        umma_commit(smem_u32(&tfull[ab]));
-        if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
       }
       if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
       umma_commit(smem_u32(drain));
@@ -369,14 +401,18 @@ __global__ void __launch_bounds__(kXThreads, 1)
     const int quarter = warp & 3;
     const int r = 32 * quarter + lane;
     const uint32_t trow = tmem + (static_cast<uint32_t>(32 * quarter) << 16) + p.a_base;
-    int stage = 0;
-    uint32_t ph = 0;
+    // The TMEM slots form their own ring (n_slots <= stages): a stage's y
+    // tile moves into the next free slot, so more y tiles can be in flight
+    // in shared memory than there are slots.
+    int stage = 0, slot = 0;
+    uint32_t ph = 0, tph = 0;
     for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
       const XItem it = decode_xitem(p, item);
       KahanSum nrm;
       bool aborted = false;
       for (int st = it.s0; st < it.s1; ++st) {
-        if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) {
+        if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
+            !warp_wait(smem_u32(&tfree[slot]), tph ^ 1, tmo, s_abort)) {
           raise_device_error(p.status, s_abort, kStatusTimeout);
           aborted = true;
           break;
@@ -392,12 +428,13 @@ __global__ void __launch_bounds__(kXThreads, 1)
           lv[4 * c] = l.x; lv[4 * c + 1] = l.y; lv[4 * c + 2] = l.z; lv[4 * c + 3] = l.w;
           if (p.unit) nrm.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
         }
-        tmem_st32(trow + stage * 2 * kXK, hv);
-        tmem_st32(trow + stage * 2 * kXK + kXK, lv);
+        tmem_st32(trow + slot * 2 * kXK, hv);
+        tmem_st32(trow + slot * 2 * kXK + kXK, lv);
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(smem_u32(&conv[stage]));
+        mbar_arrive(smem_u32(&conv[slot]));
         if (++stage == p.stages) { stage = 0; ph ^= 1; }
+        if (++slot == p.n_slots) { slot = 0; tph ^= 1; }
       }
       if (aborted) break;
       const int q = it.mt * kXM + r;
@@ -452,39 +489,64 @@ __global__ void __launch_bounds__(kXThreads, 1)
     const int row = 32 * quarter + lane;
     int ab = 0;
     uint32_t aph = 0;
-    for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
+    bool aborted = false;
+    for (int item = blockIdx.x; item < p.n_items && !aborted; item += gridDim.x) {
       const XItem it = decode_xitem(p, item);
-      if (!warp_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort)) {
-        raise_device_error(p.status, s_abort, kStatusTimeout);
-        break;
-      }
-      tc_fence_after();
       const int q = it.mt * kXM + row;
-      float* dst = p.partial + static_cast<int64_t>(it.z) * p.B * p.Q + q;
-      const uint32_t tbase =
-          tmem + (static_cast<uint32_t>(32 * quarter) << 16) + ab * 3 * p.n_pad;
-      for (int c = 0; c < p.n_pad; c += 16) {
-        // <x_b, y_q> ~= y_hi x_hi + y_hi x_lo + y_lo x_hi, in this order
-        float v[16], w[16];
-        tmem_ld16(tbase + c, v);
-        tmem_ld16(tbase + p.n_pad + c, w);
+      // The item's chains, added in order in registers (compile-time indices:
+      // the column loop is unrolled over the largest batch tile and guarded).
+      constexpr int kPad = TA ? kMaxPadTA : kMaxPad;
+      float acc[kPad];
+      for (int c0 = it.s0; c0 < it.s1; c0 += p.sub) {
+        if (!warp_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort)) {
+          raise_device_error(p.status, s_abort, kStatusTimeout);
+          aborted = true;
+          break;
+        }
+        tc_fence_after();
+        const bool first = c0 == it.s0;
+        const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * quarter) << 16) +
+                               ab * (p.fold ? 2 : 3) * p.n_pad;
 #pragma unroll
-        for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
-        tmem_ld16(tbase + 2 * p.n_pad + c, w);
+        for (int cb = 0; cb < kPad / 16; ++cb) {
+          const int c = 16 * cb;
+          if (c < p.n_pad) {
+            // <x_b, y_q> ~= y_hi x_hi + y_hi x_lo + y_lo x_hi (folded: the
+            // first and third terms come as one sum)
+            float v[16], w[16];
+            tmem_ld16(tbase + c, v);
+            tmem_ld16(tbase + p.n_pad + c, w);
 #pragma unroll
-        for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
-        if (q < p.Q) {
+            for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
+            if (!p.fold) {
+              tmem_ld16(tbase + 2 * p.n_pad + c, w);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int b = it.nt * p.n_pad + c + j;
-            if (b < p.B) dst[static_cast<int64_t>(b) * p.Q] = v[j];
+              for (int jj = 0; jj < 16; ++jj) v[jj] += w[jj];
+            }
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) acc[c + jj] = first ? v[jj] : acc[c + jj] + v[jj];
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+        if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
+      }
+      if (aborted) break;
+      if (q < p.Q) {
+        float* dst = p.partial + static_cast<int64_t>(it.z) * p.B * p.Q + q;
+#pragma unroll
+        for (int cb = 0; cb < kPad / 16; ++cb) {
+          const int c = 16 * cb;
+          if (c < p.n_pad) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int b = it.nt * p.n_pad + c + j;
+              if (b < p.B) dst[static_cast<int64_t>(b) * p.Q] = acc[c + j];
+            }
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
-      if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
     }
   }
 
@@ -559,24 +621,31 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   pl.n_ntiles = static_cast<int>((b1 + pl.n_pad - 1) / pl.n_pad);
   pl.n_mtiles = static_cast<int>(std::max<int64_t>(1, (Q + kXM - 1) / kXM));
   pl.steps = static_cast<int>(std::max<int64_t>(1, (K + kXK - 1) / kXK));
-  // y_hi / y_lo go to TMEM when the accumulators leave room for a ring of at
-  // least 4 stages (64 columns each); otherwise y_lo is written next to y.
+  // y_hi / y_lo go to TMEM (as MMA A operands) for batch tiles of up to 64
+  // rows.  There the three products keep separate column groups (3 n_pad per
+  // accumulator set: two independent accumulation chains), two sets, and the
+  // operand ring takes the remaining columns.  Larger batch tiles fold y_lo
+  // x_hi into the y_hi x_hi columns (2 n_pad per set), so that two sets (and,
+  // up to n_pad = 64, four operand slots) fit even at n_pad = 128; a folded
+  // chain takes twice the MMAs per step, so its chains are half as many steps
+  // long.
   pl.tmem_a = pl.n_pad <= 64;
+  pl.n_buf = 2;
+  // unfolded where two 3 n_pad sets still leave four operand slots (n_pad <= 32)
+  pl.fold = !pl.tmem_a || 2 * 3 * pl.n_pad + 4 * 2 * kXK > 512;
+  pl.sub = pl.fold ? kSubSteps / 2 : kSubSteps;
   int stage_bytes;
   if (pl.tmem_a) {
-    pl.n_buf = (512 - 6 * pl.n_pad) / (2 * kXK) >= 4 ? 2 : 1;
-    pl.a_base = (pl.n_buf * 3 * pl.n_pad + 31) / 32 * 32;
+    pl.a_base = (pl.n_buf * (pl.fold ? 2 : 3) * pl.n_pad + 31) / 32 * 32;
     pl.tmem_cols = 512;
+    pl.n_slots = (512 - pl.a_base) / (2 * kXK);
     stage_bytes = kYBytes + 2 * pl.n_pad * 128;
-    pl.stages = std::min({kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes,
-                          (512 - pl.a_base) / (2 * kXK)});
   } else {
-    pl.n_buf = 6 * pl.n_pad <= 512 ? 2 : 1;
     pl.tmem_cols = 32;
-    while (pl.tmem_cols < pl.n_buf * 3 * pl.n_pad) pl.tmem_cols <<= 1;
+    while (pl.tmem_cols < pl.n_buf * 2 * pl.n_pad) pl.tmem_cols <<= 1;
     stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
-    pl.stages = std::min(kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
   }
+  pl.stages = std::min(kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
   // K slices: fewest waves of persistent CTAs for the y stream, plus the
   // partials each slice adds (written and read back once).
   const int64_t tiles = static_cast<int64_t>(pl.n_mtiles) * pl.n_ntiles;
@@ -640,6 +709,9 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   p.n_items = pl.n_mtiles * pl.n_ntiles * pl.S;
   p.n_buf = pl.n_buf;
   p.tmem_cols = pl.tmem_cols;
+  p.sub = pl.sub;
+  p.n_slots = pl.n_slots;
+  p.fold = pl.fold ? 1 : 0;
   p.a_base = pl.a_base;
   p.unit = a.unit;
   p.partial = reinterpret_cast<float*>(a.ws + pl.partial_off);

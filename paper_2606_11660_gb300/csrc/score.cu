@@ -682,9 +682,13 @@ __global__ void __launch_bounds__(512) merge_kernel(const unsigned long long* __
     }
     const unsigned long long T = s_prefix;       // the topk-th largest key
     unsigned long long* sel = keys + n;
+    // Only real keys (a row in the low word) are kept: when fewer than topk
+    // exist (NaN scores, or a running result over fewer rows than topk), T is
+    // an empty-slot key and more than select_n keys would reach it, so an
+    // arbitrary subset -- real keys included -- would otherwise be dropped.
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
       const unsigned long long k = keys[i];
-      if (k >= T) {
+      if (k >= T && static_cast<uint32_t>(k) >= 0x80000000u) {
         const int pos = atomicAdd(&s_count, 1);
         if (pos < select_n) sel[pos] = k;
       }

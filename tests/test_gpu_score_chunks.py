@@ -147,3 +147,32 @@ def test_host_store_streamed_in_chunks(pinned, least):
     torch.cuda.synchronize()
     np.testing.assert_array_equal(i.cpu().numpy(), want_i)
     np.testing.assert_array_equal(np32(s).view(np.uint32), want_s.view(np.uint32))
+
+
+@pytest.mark.parametrize("Q", [3, 200])
+def test_fewer_usable_scores_than_topk(Q):
+    # NaN rows never enter the result; with only 9 usable rows the result is
+    # those 9 in order, then (-inf, -1).  Before the merge kept only real keys,
+    # the empty-slot keys tying with the k-th could push real rows out.
+    N, K, topk = 600, 128, 16
+    X = wl.gaussian_rows(N, K, seed=98)
+    store = _store(X)
+    keep = np.array([3, 77, 128, 255, 256, 300, 411, 512, 599])
+    dead = torch.ones(N, dtype=torch.bool)
+    dead[torch.from_numpy(keep)] = False
+    store[dead.to(DEV)] = float("nan")
+    queries = wl.gaussian_rows(Q, K, seed=99).to(DEV)
+    got_s, got_i = _single(store, queries, topk)
+    S = orc.cosine_scores(store[torch.from_numpy(keep).to(DEV)].cpu().numpy(),
+                          queries.cpu().numpy().astype(np.float64))
+    for q in range(Q):
+        # the 9 usable rows (order among near-ties follows the fp32 scores)
+        assert sorted(got_i[q, :9].tolist()) == sorted(keep.tolist())
+        want = dict(zip(keep.tolist(), S[q]))
+        np.testing.assert_allclose(got_s[q, :9], [want[r] for r in got_i[q, :9]], atol=1e-3)
+        assert np.all(np.diff(got_s[q, :9]) <= 0)
+        assert np.all(got_i[q, 9:] == -1) and np.all(np.isneginf(got_s[q, 9:]))
+    # the same through the chunked path, chunks smaller than topk included
+    got_s2, got_i2 = _chunked(store, queries, topk, [0, 5, 130, 257, N], [2, 0, 3, 1])
+    np.testing.assert_array_equal(got_i2, got_i)
+    np.testing.assert_array_equal(got_s2.view(np.uint32), got_s.view(np.uint32))
