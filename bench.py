@@ -664,14 +664,20 @@ def bench_e2e(args, world, dev, state):
     copied = [torch.cuda.Event() for _ in range(2)]
     consumed = [None, None]
 
+    copy_ev = []
+
     def step(i, start_event=None):
         b = i % 2
         if start_event is not None:
             copy_stream.wait_event(start_event)
         if consumed[b] is not None:
             copy_stream.wait_event(consumed[b])      # the step two back is done with it
+        ca, cb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ca.record(copy_stream)
         with torch.cuda.stream(copy_stream):
             dbufs[b].copy_(hbuf, non_blocking=True)
+        cb.record(copy_stream)
+        copy_ev.append((ca, cb))
         copied[b].record(copy_stream)
         stream.wait_event(copied[b])
         e2e_layers, dmask = sides[b]
@@ -688,6 +694,7 @@ def bench_e2e(args, world, dev, state):
     torch.cuda.synchronize()
     barrier(world)
     consumed[0] = consumed[1] = None
+    copy_ev.clear()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
@@ -696,19 +703,33 @@ def bench_e2e(args, world, dev, state):
     t1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(t0.elapsed_time(t1), world)
+    # each step's copy: its duration, and the idle gap before it on the copy stream
+    copy_ms = [a.elapsed_time(b) for a, b in copy_ev]
+    gaps = [copy_ev[k - 1][1].elapsed_time(copy_ev[k][0]) for k in range(1, len(copy_ev))]
     # The host link's rate in this run: the same pinned buffer copied alone.
     link_gbs = h2d_rate(hbuf, dbufs[0], copy_stream)
     del hbuf, dbufs, sides
     torch.cuda.empty_cache()
+    release_pinned_cache()
     gbs = h2d * steps / (ms * 1e-3) / 1e9
     return {"value": cfg.B * world * steps / (ms * 1e-3), "unit": "examples/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
             "ms_per_step": ms / steps,
             "h2d_gbs_achieved": round(gbs, 1), "h2d_gbs_measured": round(link_gbs, 1),
             "frac_of_h2d": round(gbs / link_gbs, 4),
+            "copy_ms_per_step": [round(x, 1) for x in copy_ms],
+            "copy_gap_ms": [round(x, 1) for x in gaps],
             "h2d": "one contiguous pinned buffer -> one of two device buffers per step; "
                    "the next step's copy overlaps this step's compute; h2d_gbs_measured = "
                    "the same buffer copied alone in this run (best of 3)"}
+
+
+def release_pinned_cache():
+    """Return torch's cached pinned host blocks to the system (when torch offers it)."""
+    import torch
+    fn = getattr(torch._C, "_host_emptyCache", None)
+    if fn is not None:
+        fn()
 
 
 def h2d_rate(hbuf, dbuf, stream, repeats: int = 3) -> float:
@@ -854,7 +875,8 @@ def bench_outofcore(args, world, dev, peaks):
     store (8,000,000 x 8192 fp16 unit rows, 131 GB) held in pinned host memory:
     bergson_score_topk_host copies it to the device in chunks on a second
     stream while the previous chunk is scored.  The rate is bound by the host
-    link, measured in the same run on the same buffer."""
+    link: the reference is the same chunked copies of the whole store with no
+    scoring, in the same run."""
     import torch
 
     import paper_2606_11660_gb300 as bg
@@ -904,11 +926,27 @@ def bench_outofcore(args, world, dev, peaks):
     ms = max_over_ranks(e0.elapsed_time(e1), world) / args.ooc_steps
     idx = i.cpu()
     ok = bool((idx >= 0).all() and (idx < N).all() and (s.diff(dim=1) <= 0).all())
-    # the link alone: one chunk of the same pinned store copied to the device
-    dchunk = torch.empty(chunk * K, dtype=torch.float16, device=dev)
-    link_gbs = h2d_rate(host.view(-1)[:chunk * K], dchunk, copy_stream)
-    del host, ws, dchunk
+    # the link alone: the same chunked copies of the whole store into two
+    # device buffers, with no scoring (best of 2)
+    del ws
     torch.cuda.empty_cache()
+    bufs = [torch.empty((chunk, K), dtype=torch.float16, device=dev) for _ in range(2)]
+    copy_ms = None
+    for _ in range(2):
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record(copy_stream)
+        with torch.cuda.stream(copy_stream):
+            for c, r0 in enumerate(range(0, N, chunk)):
+                r1 = min(N, r0 + chunk)
+                bufs[c % 2][:r1 - r0].copy_(host[r0:r1], non_blocking=True)
+        c1.record(copy_stream)
+        torch.cuda.synchronize()
+        t = c0.elapsed_time(c1)
+        copy_ms = t if copy_ms is None else min(copy_ms, t)
+    link_gbs = N * row_bytes / (copy_ms * 1e-3) / 1e9
+    del host, bufs
+    torch.cuda.empty_cache()
+    release_pinned_cache()
     gbs = N * row_bytes / (ms * 1e-3) / 1e9
     return {"value": round(N * world / (ms * 1e-3)), "unit": "store rows/s",
             "ms_per_pass": round(ms, 2), "steps": args.ooc_steps,
@@ -918,6 +956,7 @@ def bench_outofcore(args, world, dev, peaks):
                        "N": N, "K": K, "Q": Q, "topk": topk, "chunk_rows": chunk,
                        "store_bytes": N * row_bytes, "reduced_to_fit_host_memory": reduced},
             "store_gbs": round(gbs, 1), "h2d_gbs_measured": round(link_gbs, 1),
+            "copy_only_ms_per_pass": round(copy_ms, 2),
             "frac_of_h2d": round(gbs / link_gbs, 4), "result_valid": ok,
             "fill_s": round(t_fill, 1),
             "what": "bergson_score_topk_host: chunk c+1 copied (copy stream) while chunk c is "
@@ -1018,10 +1057,11 @@ def profile_case(args):
             bg.bergson_project_grads(layers, B, cfg.T, mask, out, ws)
         st = bg.bergson_sync_status()
     else:
-        # 409,600-row fp16 store x 8192 (6.7 GB, large enough for the prefix
-        # threshold pass), 1024 queries (score) or 256 queries (score_mid: the
-        # pair kernel with one query tile per CTA), top-100
-        N, K, topk = 409_600, 8192, 100
+        # 196,608-row fp16 store x 8192 (3.2 GB: a full ncu capture stays at a
+        # few GB on the device; still large enough for the prefix threshold
+        # pass), 1024 queries (score) or 256 queries (score_mid: the pair
+        # kernel with one query tile per CTA), top-100
+        N, K, topk = 196_608, 8192, 100
         Q = 256 if args.profile_case == "score_mid" else 1024
         store = torch.empty((N, K), dtype=torch.float16, device=dev)
         for n0 in range(0, N, 1 << 16):
