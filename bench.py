@@ -420,14 +420,14 @@ def bench_onthefly(args, world, dev, state, peaks):
 
 
 def bench_tokens(args, world, dev, state, peaks):
-    """Per-token scores of the batch against 4 query rows (one fused pass over A and G)."""
+    """Per-token scores of the batch against 64 query rows (one fused pass over A and G)."""
     import torch
 
     import paper_2606_11660_gb300 as bg
     from paper_2606_11660_gb300 import workloads as wl
 
     cfg, layers, mask, ws, out, store = state
-    Q = 4
+    Q = args.token_queries
     queries = wl.gaussian_rows(Q, cfg.k_total, seed=13, device=dev)
     tws = bg.workspace_tensor(bg.bergson_token_scores_workspace(layers, cfg.B, cfg.T, Q), dev)
     tout = torch.empty((Q, cfg.B, cfg.T), dtype=torch.float32, device=dev)
@@ -455,8 +455,8 @@ def bench_tokens(args, world, dev, state, peaks):
                          "unit": "GB/s", "frac": round(gbs / peaks["hbm_gbs"], 4),
                          "traffic": profiled_traffic("token_kernel_pythia160m.md", "project.cu")},
             "gpu_launches": 4 * args.steps,          # tile flags, prep, projection, token sum
-            "what": "bergson_token_scores: per-token scores of all 65,536 tokens x 48 modules "
-                    "against 4 query rows"}
+            "what": f"bergson_token_scores: per-token scores of all 65,536 tokens x 48 modules "
+                    f"against {Q} query rows in one pass over A and G"}
 
 
 def bench_fisher(args, world, dev, state, peaks):
@@ -974,7 +974,7 @@ def profile_case(args):
     dev = torch.device("cuda", 0)
     if args.profile_case == "tokens":
         # one block of the Pythia-160M-shaped workload at the bench's B=32,
-        # T=2048 and padding mask, 4 query rows
+        # T=2048 and padding mask, --token-queries query rows
         cfg = wl.PYTHIA160M
         B = cfg.B
         mask = wl.right_padding_mask(B, cfg.T, cfg.max_pad, seed=1, device=dev)
@@ -983,9 +983,10 @@ def profile_case(args):
             A, G = wl.layer_inputs(spec, B, cfg.T, seed=10_000 + m, device=dev, input_scale=True)
             s_in, s_out = bg.bergson_module_seeds(0, m)
             layers.append(bg.Layer(A, G, cfg.k, cfg.k, s_in, s_out, None, None, cfg.col_offset(m)))
-        queries = wl.gaussian_rows(4, 4 * cfg.k * cfg.k, seed=13, device=dev)
-        ws = bg.workspace_tensor(bg.bergson_token_scores_workspace(layers, B, cfg.T, 4), dev)
-        out = torch.empty((4, B, cfg.T), dtype=torch.float32, device=dev)
+        nq = args.token_queries
+        queries = wl.gaussian_rows(nq, 4 * cfg.k * cfg.k, seed=13, device=dev)
+        ws = bg.workspace_tensor(bg.bergson_token_scores_workspace(layers, B, cfg.T, nq), dev)
+        out = torch.empty((nq, B, cfg.T), dtype=torch.float32, device=dev)
         for _ in range(2):
             bg.bergson_token_scores(layers, B, cfg.T, mask, queries, out, ws)
         st = bg.bergson_sync_status()
@@ -1233,6 +1234,7 @@ def parse(argv=None):
     ap.add_argument("--no-streamed", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-ooc", action="store_true", help="skip the host-resident store leg")
+    ap.add_argument("--token-queries", type=int, default=64)
     ap.add_argument("--ooc-rows", type=int, default=8_000_000)
     ap.add_argument("--ooc-chunk", type=int, default=262_144)
     ap.add_argument("--ooc-steps", type=int, default=2)

@@ -313,7 +313,7 @@ BERGSON_API int bergson_score_topk_host(const void* host_store, int64_t N, int64
                                         void* workspace, size_t ws_bytes, void* stream,
                                         void* copy_stream);
 
-/* Bytes of workspace bergson_token_scores needs (n_queries in 1 .. 16). */
+/* Bytes of workspace bergson_token_scores needs (n_queries in 1 .. 256). */
 BERGSON_API int bergson_token_scores_workspace(const bergson_layer* layers, int n_layers,
                                                int64_t B, int64_t T, int64_t n_queries,
                                                size_t* ws_bytes);
@@ -331,9 +331,13 @@ BERGSON_API int bergson_token_scores_workspace(const bergson_layer* layers, int 
  * per-sequence inner product <out_b, queries_q>.  Masked tokens score 0.
  *   queries  fp32 [n_queries, ld_q], 4-byte aligned; the layers' column
  *            blocks must fit in ld_q and must not overlap.
- *   n_queries  1 .. 16, and at most what the layers' (k_in, k_out) allow
- *            (16 for 16x16, 8 for 32x32, 4 for 64x64).
+ *   n_queries  1 .. 256.  One pass over A and G serves them all: the query
+ *            blocks of a module are streamed through shared memory in groups
+ *            (16 queries for 16x16 blocks, 9 for 32x32, 4 for 64x64) for every
+ *            group of token tiles.
  *   out      fp32 [n_queries, B, T] contiguous.
+ * The workspace holds per-module partial scores (n_layers x n_queries x B x
+ * T floats) that a final pass sums in module order.
  * Other arguments as for bergson_project_grads.  Deterministic.
  * Errors: EINVAL, EALIGN, EUNSUPPORTED, EWORKSPACE, ECUDA.
  */

@@ -31,6 +31,7 @@ constexpr double kSplitShare = 0.4;
 constexpr int kPiecesPerShare = 2;
 constexpr int kMaxScoreCTAs = 160;                   // upper bound on persistent score CTAs
 constexpr int kMaxDevices = 64;
+constexpr int kMaxTokenQueries = 256;                // per-token scores: queries per call
 constexpr int64_t kPrefixRowsPerTopk = 128;          // prefix pass: 128 * topk store rows
 constexpr int64_t kPrefixMinFactor = 8;              // ... only when N >= 8 * prefix
 constexpr int64_t kPrefixMinQueries = 129;           // ... and Q > 128 (fewer queries insert
@@ -744,14 +745,8 @@ static int run_projection(const bergson_layer* layers, int n_layers, int64_t B, 
   int st = validate_layers(layers, n_layers, B, T);
   if (st != BERGSON_OK) return st;
   if (token) {
-    if (n_queries > 16) return fail(BERGSON_EUNSUPPORTED, "at most 16 queries per call");
-    for (int i = 0; i < n_layers; ++i) {
-      const int cap = token_query_capacity(static_cast<int>(layers[i].k_in),
-                                           static_cast<int>(layers[i].k_out));
-      if (n_queries > cap)
-        return fail(BERGSON_EUNSUPPORTED, "layer %d: at most %d queries for k_in=%lld, k_out=%lld",
-                    i, cap, (long long)layers[i].k_in, (long long)layers[i].k_out);
-    }
+    if (n_queries > kMaxTokenQueries)
+      return fail(BERGSON_EUNSUPPORTED, "at most %d queries per call", kMaxTokenQueries);
     if (ld_q < 0) return fail(BERGSON_EINVAL, "ld_q must be >= 0");
     st = validate_blocks(layers, n_layers, ld_q, false);
     if (st != BERGSON_OK) return st;
@@ -904,8 +899,8 @@ int bergson_project_grads(const bergson_layer* layers, int n_layers, int64_t B, 
 int bergson_token_scores_workspace(const bergson_layer* layers, int n_layers, int64_t B, int64_t T,
                                    int64_t n_queries, size_t* ws_bytes) {
   if (ws_bytes == nullptr) return fail(BERGSON_EINVAL, "ws_bytes is NULL");
-  if (n_queries < 1 || n_queries > 16)
-    return fail(BERGSON_EUNSUPPORTED, "n_queries must be in [1, 16]");
+  if (n_queries < 1 || n_queries > kMaxTokenQueries)
+    return fail(BERGSON_EUNSUPPORTED, "n_queries must be in [1, %d]", kMaxTokenQueries);
   int st = validate_layers(layers, n_layers, B, T);
   if (st != BERGSON_OK) return st;
   *ws_bytes = plan_project(layers, n_layers, B, T, n_queries).total;

@@ -180,6 +180,8 @@ cudaError_t launch_wait_probe(int* status, uint64_t timeout_ns, cudaStream_t s);
 // per-token scores against p.queries (token_partials).
 cudaError_t launch_project(int k_in, int k_out, bool token, const ProjParams& p, int grid,
                           cudaStream_t s);
+// Queries whose blocks token mode holds in shared memory at once (more are
+// streamed through in blocks of this many).
 int token_query_capacity(int k_in, int k_out);
 cudaError_t launch_token_reduce(const float* token_partials, int n_mods, int Q, int B, int T,
                                 const uint8_t* mask, float* out, cudaStream_t s);

@@ -68,6 +68,9 @@ struct ProjCfg {
   static constexpr int kTmemPerBuf = NT * 2 * (KI + KO);
   static constexpr int kTmemCols = pow2ceil(2 * kTmemPerBuf);
   static constexpr int kOPT = KO * KI / kTileTokens;            // outputs per epilogue thread
+  // Token mode: queries whose k_out x k_in blocks fit in the staging area at once.
+  static constexpr int kQBFit = kEpiBytes / (4 * KI * KO);
+  static constexpr int kQB = kQBFit > 16 ? 16 : kQBFit;
   static_assert(kStages >= 2, "shared memory budget too small");
   static_assert(kTmemCols <= 512, "TMEM budget exceeded");
   static_assert(kOPT >= 2 && kOPT % 2 == 0, "unsupported projection sizes");
@@ -185,6 +188,16 @@ __device__ __forceinline__ uint32_t tiles_of(uint32_t slices) {
   for (int nt = 0; nt < NT; ++nt)
     if ((slices >> (4 * nt)) & 0xFu) tm |= 1u << nt;
   return tm;
+}
+
+// Token mode: module m's blocks of queries [q0, q0 + n) into sA (128 threads).
+template <int KI, int KO>
+__device__ __forceinline__ void load_query_block(const ProjParams& p, int m, int q0, int n,
+                                                 float* sA, int et) {
+  constexpr int blk = KO * KI;
+  const int64_t off = p.mods[m].col_offset;
+  for (int e = et; e < n * blk; e += 128)
+    sA[e] = p.queries[static_cast<int64_t>(q0 + e / blk) * p.ld_q + off + e % blk];
 }
 
 template <int KI, int KO, bool TOKEN>
@@ -448,15 +461,18 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
 #pragma unroll
       for (int x = 0; x < OPT; ++x) acc[x] = 0.0f;
       bias_acc = 0.0f;
+      constexpr int QB = ProjCfg<KI, KO, true>::kQB;   // queries held in shared memory at once
+      const int n_qblocks = TOKEN ? (p.n_queries + QB - 1) / QB : 0;
       if constexpr (TOKEN) {
-        // This module's k_out x k_in block of every query row, into the
-        // (otherwise unused) staging area.  All threads left the previous
-        // item behind the two barriers above.
-        const int blk = KO * KI;
-        const int64_t off = p.mods[ic.m].col_offset;
-        for (int e = et; e < p.n_queries * blk; e += 128)
-          sA[e] = p.queries[static_cast<int64_t>(e / blk) * p.ld_q + off + e % blk];
-        named_bar_sync(1, 128);
+        // This module's k_out x k_in block of the query rows, into the
+        // (otherwise unused) staging area: all of them when they fit in one
+        // block of QB queries, else block by block for every tile group
+        // below.  All threads left the previous item behind the two barriers
+        // above.
+        if (n_qblocks == 1) {
+          load_query_block<KI, KO>(p, ic.m, 0, p.n_queries, sA, et);
+          named_bar_sync(1, 128);
+        }
       }
       for (int g = ic.t_begin; g < ic.t_end; g += NT) {
         const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
@@ -474,6 +490,17 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         // One tile at a time: its a~ and g~ (hi + lo halves summed) are loaded,
         // used and dropped before the next tile's; the TMEM buffer is released
         // after the group (the MMA warp fills the other buffer meanwhile).
+        // Token mode with more queries than one block: every block is streamed
+        // through shared memory once per tile group, and the group's tiles are
+        // read from TMEM again for each block.
+        for (int qb = 0; qb < (TOKEN ? n_qblocks : 1); ++qb) {
+        const int q0 = qb * QB;
+        const int nqb = TOKEN ? min(QB, p.n_queries - q0) : 0;
+        if (TOKEN && n_qblocks > 1) {
+          named_bar_sync(1, 128);                    // the previous block's readers are done
+          load_query_block<KI, KO>(p, ic.m, q0, nqb, sA, et);
+          named_bar_sync(1, 128);
+        }
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
           if (!(vm >> nt & 1)) continue;
@@ -497,24 +524,35 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             if (t < p.T) {
               const bool valid =
                   p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0;
-              for (int q = 0; q < p.n_queries; ++q) {
+              // u_i = (Q~_q a~)_i for 16 rows i at a time, the k_in loop outermost,
+              // so that the FMAs form 16 independent chains (one warp per SM
+              // sub-partition runs this; a single chain would wait on every
+              // FMA's latency), then s = sum_i g~_i u_i.
+              constexpr int kIG = KO < 16 ? KO : 16;
+              for (int q = 0; q < nqb; ++q) {
                 const float* qm = sA + q * (KO * KI);
                 float sq = 0.0f;
 #pragma unroll
-                for (int i = 0; i < KO; ++i) {
-                  float u = 0.0f;
+                for (int i0 = 0; i0 < KO; i0 += kIG) {
+                  float u[kIG];
+#pragma unroll
+                  for (int ii = 0; ii < kIG; ++ii) u[ii] = 0.0f;
 #pragma unroll
                   for (int j = 0; j < KI; j += 4) {
-                    const float4 w = *reinterpret_cast<const float4*>(qm + i * KI + j);
-                    u = fmaf(w.x, va[j], u);
-                    u = fmaf(w.y, va[j + 1], u);
-                    u = fmaf(w.z, va[j + 2], u);
-                    u = fmaf(w.w, va[j + 3], u);
+#pragma unroll
+                    for (int ii = 0; ii < kIG; ++ii) {
+                      const float4 w = *reinterpret_cast<const float4*>(qm + (i0 + ii) * KI + j);
+                      u[ii] = fmaf(w.x, va[j], u[ii]);
+                      u[ii] = fmaf(w.y, va[j + 1], u[ii]);
+                      u[ii] = fmaf(w.z, va[j + 2], u[ii]);
+                      u[ii] = fmaf(w.w, va[j + 3], u[ii]);
+                    }
                   }
-                  sq = fmaf(vg[i], u, sq);
+#pragma unroll
+                  for (int ii = 0; ii < kIG; ++ii) sq = fmaf(vg[i0 + ii], u[ii], sq);
                 }
-                p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q) * p.B + ic.b) *
-                                     p.T + t] = valid ? sq : 0.0f;
+                p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q0 + q) * p.B +
+                                  ic.b) * p.T + t] = valid ? sq : 0.0f;
               }
             }
           } else {
@@ -570,6 +608,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             }
           }
         }
+        }                                            // query blocks
         if (!finisher) {
           tc_fence_before();
           __syncwarp();
@@ -661,8 +700,7 @@ cudaError_t launch_project_mode(bool token, const ProjParams& p, int grid, cudaS
 
 template <int KI, int KO>
 constexpr int token_capacity_of() {
-  const int cap = ProjCfg<KI, KO, true>::kEpiBytes / (4 * KI * KO);
-  return cap > 16 ? 16 : cap;
+  return ProjCfg<KI, KO, true>::kQB;
 }
 
 }  // namespace

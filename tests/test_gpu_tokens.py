@@ -74,15 +74,33 @@ def test_shared_input_layers_token_scores():
     _close(got, want)
 
 
-def test_query_capacity_is_enforced():
+def test_query_limit_is_enforced():
     spec = wl.ModuleSpec("lin", 64, 64)
     gl, _, ld = make_layers([spec], 1, 8, [(64, 64)])
-    queries = torch.zeros((5, ld), device=DEV)
-    ws = bg.workspace_tensor(1 << 20, DEV)
-    out = torch.empty((5, 1, 8), device=DEV)
+    queries = torch.zeros((257, ld), device=DEV)
+    ws = bg.workspace_tensor(1 << 24, DEV)
+    out = torch.empty((257, 1, 8), device=DEV)
     with pytest.raises(bg.BergsonError) as e:
         bg.bergson_token_scores(gl, 1, 8, None, queries, out, ws)
     assert e.value.status == bg.BERGSON_EUNSUPPORTED
+
+
+@pytest.mark.parametrize("Q", [17, 70, 256])
+def test_many_queries_stream_through_shared_memory_in_blocks(Q):
+    # more queries than one shared-memory block for every (k_in, k_out): the
+    # blocks (16 queries of 16x16, 9 of 32x32, 4 of 64x64) are streamed per
+    # tile group, the last one ragged; one pass over A and G serves them all
+    specs = [wl.ModuleSpec("a", 64, 200), wl.ModuleSpec("b", 136, 64), wl.ModuleSpec("c", 96, 72)]
+    kp = [(16, 16), (32, 32), (64, 64)]
+    B, T = 2, 300
+    gl, ol, ld = make_layers(specs, B, T, kp, base_seed=9, data_seed=7, rc=True)
+    g = wl.generator(10 + Q, "cpu")
+    mask = (torch.rand((B, T), generator=g) > 0.2).to(torch.uint8)
+    queries = torch.randn((Q, ld), generator=g)
+    got = _tokens(gl, B, T, mask.to(DEV), queries.to(DEV))
+    want = orc.token_scores(ol, mask.numpy(), queries.numpy())
+    _close(got, want)
+    assert np.all(got[:, mask.numpy() == 0] == 0.0)
 
 
 @pytest.mark.slow
@@ -90,7 +108,7 @@ def test_pythia160m_full_size_token_scores():
     import bench
     cfg, layers, mask, _, _ = bench.collection_setup(torch.device(DEV))
     K = cfg.k_total
-    Q = 4
+    Q = 64
     queries = wl.gaussian_rows(Q, K, seed=13, device=DEV)
     got = _tokens(layers, cfg.B, cfg.T, mask, queries)
     mask_np = mask.cpu().numpy()
