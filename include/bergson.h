@@ -331,10 +331,12 @@ BERGSON_API int bergson_token_scores_workspace(const bergson_layer* layers, int 
  * per-sequence inner product <out_b, queries_q>.  Masked tokens score 0.
  *   queries  fp32 [n_queries, ld_q], 4-byte aligned; the layers' column
  *            blocks must fit in ld_q and must not overlap.
- *   n_queries  1 .. 256.  One pass over A and G serves them all: the query
- *            blocks of a module are streamed through shared memory in groups
- *            (16 queries for 16x16 blocks, 9 for 32x32, 4 for 64x64) for every
- *            group of token tiles.
+ *   n_queries  1 .. 256.  One pass over A and G serves them all: a module's
+ *            query blocks go through shared memory in groups (up to 16
+ *            queries; fewer for larger k_in x k_out) for every token tile, and
+ *            the inner products a~^T Q~_q^T run on the tensor cores
+ *            (3xTF32, fp32 accuracy) except for (k_in, k_out) = (64, 32) and
+ *            (64, 64), which stay on the CUDA cores.
  *   out      fp32 [n_queries, B, T] contiguous.
  * The workspace holds per-module partial scores (n_layers x n_queries x B x
  * T floats) that a final pass sums in module order.
@@ -556,12 +558,14 @@ BERGSON_API int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_
 /*
  * Test aid for the planner of the skinny tcgen05 product behind
  * bergson_score_grads, bergson_precondition_rows and the Fisher products
- * (C[b, q] = <x_b, y_q> for B rows x, Q rows y of length K).  Writes 17 int64
- * to out (n_out >= 17): batch rows per tile, batch tiles, 128-row y tiles,
- * 32-column steps, K slices, pipeline stages, column chunks of the row split,
- * y operands in TMEM (1/0), accumulator buffers, TMEM column of the operand
- * ring, TMEM columns allocated, and the workspace offsets of the x norms,
- * y norms, partial products, x_hi, x_lo and the total.
+ * (C[b, q] = <x_b, y_q> for B rows x, Q rows y of length K).  Writes 18 int64
+ * to out (n_out >= 18): batch rows per tile, batch tiles, 128-row y tiles,
+ * 32-column steps, K slices, pipeline stages (of y tiles when y goes to
+ * TMEM), column chunks of the row split, y operands in TMEM (1/0),
+ * accumulator buffers, TMEM column of the operand ring, TMEM columns
+ * allocated, the workspace offsets of the x norms, y norms, partial products,
+ * x_hi, x_lo and the total, and the stages of the separate x ring (0 unless y
+ * goes to TMEM).
  * Host only: enqueues nothing.  Errors: EINVAL (B in [1, 2^20], Q in
  * [1, 2^24], K in [4, 2^26] and a multiple of 4).
  */

@@ -48,10 +48,24 @@ constexpr int pow2ceil(int x) {
 
 template <int KI, int KO, bool TOKEN = false>
 struct ProjCfg {
+  // Token mode on the tensor cores (kTC): per tile and block of kTcNQ queries,
+  // U = a~ Q^T (M = 128 tokens, K = k_in, N = kTcNQ k_out rows (q, i)) on
+  // tcgen05 kind::tf32 (3xTF32), then s_q = sum_i g~_i U[q, i] on the CUDA
+  // cores (k_out FMAs per token and query instead of k_out (k_in + 1)).
+  // TMEM with one tile per group: the two projection buffers (4 (k_in + k_out)
+  // columns), a~ hi / lo (2 k_in) and U (kTcN <= 256) must fit in 512 columns.
+  static constexpr int kTcAvail = 512 - 4 * (KI + KO) - 2 * KI;
+  static constexpr int kTcNQa = kTcAvail > 0 ? kTcAvail / KO : 0;
+  static constexpr int kTcNQb = kTcNQa < 256 / KO ? kTcNQa : 256 / KO;
+  static constexpr int kTcNQ = kTcNQb < 16 ? kTcNQb : 16;
+  static constexpr bool kTC = TOKEN && kTcNQ >= 1;
+  static constexpr int kTcN = kTcNQ * KO;
+  static constexpr int kTcAtoms = (KI + 31) / 32;              // 128-byte K atoms of a B row
+  static constexpr int kTcBBytes = kTcN * 128 * kTcAtoms;      // one of B_hi / B_lo
   // Tiles sharing one P' slice: each slice is re-read from L2 once per NT
   // tiles, so a larger NT cuts L2 -> SM traffic (NT = 1 -> 2 -> 4 measured
   // 3.05 -> 2.72 -> 2.59 ms on the 48-module bench call).
-  static constexpr int NT = (KI + KO <= 32) ? 4 : ((KI + KO <= 64) ? 2 : 1);
+  static constexpr int NT = kTC ? 1 : ((KI + KO <= 32) ? 4 : ((KI + KO <= 64) ? 2 : 1));
   static constexpr int kPRows = 2 * (KI > KO ? KI : KO);         // hi + lo rows
   static constexpr int kPBytes = kPRows * 128;
   static constexpr int kStageBytes = NT * kActBoxBytes + kPBytes;
@@ -59,18 +73,22 @@ struct ProjCfg {
   // (half a tile; the room goes to pipeline stages: 4 -> 5 of them at k = 32);
   // token mode keeps the whole tile's worth, where it holds the query blocks.
   static constexpr int kEpiRows = TOKEN ? kTileTokens : kTileTokens / 2;
-  static constexpr int kEpiBytes = kEpiRows * (KI + 4) * 4 + kEpiRows * (KO + 4) * 4;
+  static constexpr int kEpiBytes =
+      kTC ? 2 * kTcBBytes : kEpiRows * (KI + 4) * 4 + kEpiRows * (KO + 4) * 4;
   static constexpr int kBarBytes = 512;
   static constexpr int kStagesFit = (kSmemBudget - 1024 - kEpiBytes - kBarBytes) / kStageBytes;
   static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kEpiBytes + kBarBytes;
   // Per tile: A*[hi|lo] in 2 KI columns, then G*[hi|lo] in 2 KO columns.
   static constexpr int kTmemPerBuf = NT * 2 * (KI + KO);
-  static constexpr int kTmemCols = pow2ceil(2 * kTmemPerBuf);
+  static constexpr int kTmemCols = kTC ? 512 : pow2ceil(2 * kTmemPerBuf);
+  static constexpr int kTmA = 2 * kTmemPerBuf;                  // a~ hi, then lo (kTC)
+  static constexpr int kTmU = kTmA + 2 * KI;                    // U (kTC)
   static constexpr int kOPT = KO * KI / kTileTokens;            // outputs per epilogue thread
-  // Token mode: queries whose k_out x k_in blocks fit in the staging area at once.
+  // Token mode: queries handled per block (held in shared memory at once).
   static constexpr int kQBFit = kEpiBytes / (4 * KI * KO);
-  static constexpr int kQB = kQBFit > 16 ? 16 : kQBFit;
+  static constexpr int kQB = kTC ? kTcNQ : (kQBFit > 16 ? 16 : kQBFit);
+  static_assert(!kTC || (kTcN % 16 == 0 && kTcN <= 256 && kTmU + kTcN <= 512), "token TMEM plan");
   static_assert(kStages >= 2, "shared memory budget too small");
   static_assert(kTmemCols <= 512, "TMEM budget exceeded");
   static_assert(kOPT >= 2 && kOPT % 2 == 0, "unsupported projection sizes");
@@ -200,6 +218,38 @@ __device__ __forceinline__ void load_query_block(const ProjParams& p, int m, int
     sA[e] = p.queries[static_cast<int64_t>(q0 + e / blk) * p.ld_q + off + e % blk];
 }
 
+// Token mode on the tensor cores: module m's blocks of queries [q0, q0 + n)
+// as the B operand of U = a~ Q^T: row r = q * k_out + i holds Q~_q[i, 0:k_in],
+// K-major in 128-byte rows (32 fp32 per K atom, atoms kN rows apart) with the
+// 128-byte swizzle, split into tf32 hi and lo parts (128 threads).
+template <int KI, int KO, int kN>
+__device__ __forceinline__ void load_query_block_tc(const ProjParams& p, int m, int q0, int n,
+                                                    uint8_t* bhi, uint8_t* blo, int et) {
+  constexpr int blk = KO * KI;
+  const int64_t off = p.mods[m].col_offset;
+  for (int e = et; e < n * blk; e += 128) {
+    const int q = e / blk, i = (e / KI) % KO, j = e % KI;
+    const float v = p.queries[static_cast<int64_t>(q0 + q) * p.ld_q + off + i * KI + j];
+    const int r = q * KO + i;
+    const int jj = j & 31;
+    const int byte = (j >> 5) * kN * 128 + r * 128 + (((jj >> 2) ^ (r & 7)) << 4) + (jj & 3) * 4;
+    const float h = tf32_rn(v);
+    *reinterpret_cast<float*>(bhi + byte) = h;
+    *reinterpret_cast<float*>(blo + byte) = tf32_rn(v - h);
+  }
+}
+
+// 32 lanes x N columns of this thread's TMEM row from v (N = 16, 32 or 64).
+template <int N>
+__device__ __forceinline__ void tmem_store_row(uint32_t taddr, const float* v) {
+  if constexpr (N == 16) {
+    tmem_st16(taddr, v);
+  } else {
+#pragma unroll
+    for (int c = 0; c < N; c += 32) tmem_st32(taddr + c, v + c);
+  }
+}
+
 template <int KI, int KO, bool TOKEN>
 __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   using C = ProjCfg<KI, KO, TOKEN>;
@@ -208,16 +258,20 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
-  float* sA = reinterpret_cast<float*>(smem + C::kStages * C::kStageBytes);
+  uint8_t* epi = smem + C::kStages * C::kStageBytes;     // 1024-byte aligned
+  float* sA = reinterpret_cast<float*>(epi);
   float* sG = sA + C::kEpiRows * (KI + 4);
-  uint64_t* full = reinterpret_cast<uint64_t*>(sG + C::kEpiRows * (KO + 4));
+  uint8_t* sBhi = epi;                                  // token mode on the tensor cores:
+  uint8_t* sBlo = epi + C::kTcBBytes;                   //   the query block, tf32 hi / lo
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi + C::kEpiBytes);
   uint64_t* empty = full + C::kStages;
   uint64_t* tfull = empty + C::kStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* sfull = tempty + 2;
   uint64_t* sempty = sfull + 2;
   uint64_t* drain = sempty + 2;
-  int* s_item = reinterpret_cast<int*>(drain + 1);
+  uint64_t* ubar = drain + 1;                           // token U products done (kTC)
+  int* s_item = reinterpret_cast<int*>(ubar + 1);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(s_item + 2);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   volatile int* s_epi_stop = s_abort + 1;   // epilogue leader's broadcast of "stop"
@@ -238,6 +292,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
       mbar_init(smem_u32(&sempty[i]), 2);
     }
     mbar_init(smem_u32(drain), 1);
+    mbar_init(smem_u32(ubar), 1);
     *s_abort = 0;
     fence_barrier_init();
   }
@@ -250,6 +305,8 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   const uint64_t tmo = p.timeout_ns;
+  uint32_t uph = 0;        // token mode on the tensor cores: phase of ubar
+  bool u_pending = false;  // an issued U product not yet waited for (epilogue thread 0)
   // Everything above overlaps the preceding grid (P' generation); the work
   // table, item counter, tile flags and P' are its or earlier writes.
   griddep_wait();
@@ -470,7 +527,12 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         // below.  All threads left the previous item behind the two barriers
         // above.
         if (n_qblocks == 1) {
-          load_query_block<KI, KO>(p, ic.m, 0, p.n_queries, sA, et);
+          if constexpr (C::kTC) {
+            load_query_block_tc<KI, KO, C::kTcN>(p, ic.m, 0, p.n_queries, sBhi, sBlo, et);
+            fence_proxy_async_smem();        // the tensor cores read it through the async proxy
+          } else {
+            load_query_block<KI, KO>(p, ic.m, 0, p.n_queries, sA, et);
+          }
           named_bar_sync(1, 128);
         }
       }
@@ -487,6 +549,95 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           if (*s_epi_stop) { aborted = true; break; }
           tc_fence_after();
         }
+        if constexpr (C::kTC) {
+          // Token scores of tile g (one tile per group) on the tensor cores.
+          // a~ (hi + lo halves summed) and g~ of this thread's token, then a~
+          // split into tf32 hi / lo parts into this lane's A row; the
+          // projection buffer is released at once.
+          const uint32_t lane_base = static_cast<uint32_t>(32 * quarter) << 16;
+          float va[KI];
+          float vg[KO];
+          {
+            const uint32_t taddr = tmem + lane_base + ab * C::kTmemPerBuf;
+            tmem_ld_hilo<KI>(taddr, va);
+            tmem_ld_hilo<KO>(taddr + 2 * KI, vg);
+          }
+          {
+            float ah[KI], al[KI];
+#pragma unroll
+            for (int j = 0; j < KI; ++j) {
+              ah[j] = tf32_rn(va[j]);
+              al[j] = tf32_rn(va[j] - ah[j]);
+            }
+            tmem_store_row<KI>(tmem + lane_base + C::kTmA, ah);
+            tmem_store_row<KI>(tmem + lane_base + C::kTmA + KI, al);
+          }
+          tmem_st_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
+          if (++ab == 2) { ab = 0; aph ^= 1; }
+          const int t = g * kTileTokens + row;
+          const bool in_range = t < p.T;
+          const bool valid =
+              in_range && (p.mask == nullptr || p.mask[static_cast<int64_t>(ic.b) * p.T + t] != 0);
+          for (int qb = 0; qb < n_qblocks; ++qb) {
+            const int q0 = qb * QB;
+            const int nqb = min(QB, p.n_queries - q0);
+            if (n_qblocks > 1) {
+              named_bar_sync(1, 128);          // the previous block's product has completed
+              load_query_block_tc<KI, KO, C::kTcN>(p, ic.m, q0, nqb, sBhi, sBlo, et);
+              fence_proxy_async_smem();
+            }
+            // Every lane's A row, the query block and the previous block's U
+            // reads are complete before one thread issues the products:
+            // U = A_hi B_hi + A_hi B_lo + A_lo B_hi (3xTF32, fp32 accumulation).
+            named_bar_sync(1, 128);
+            if (et == 0) {
+              tc_fence_after();
+              const uint32_t idesc = make_idesc_tf32(kTileTokens, C::kTcN);
+              const uint32_t ua = tmem + C::kTmU;
+              const uint32_t aa = tmem + C::kTmA;
+#pragma unroll
+              for (int kk = 0; kk < KI / 8; ++kk) {
+                const uint32_t boff = (kk >> 2) * C::kTcN * 128;
+                const uint64_t bh = sw128_desc(smem_u32(sBhi) + boff) + 2 * (kk & 3);
+                const uint64_t bl = sw128_desc(smem_u32(sBlo) + boff) + 2 * (kk & 3);
+                umma_tf32_ta(ua, aa + 8 * kk, bh, idesc, kk != 0);
+                umma_tf32_ta(ua, aa + 8 * kk, bl, idesc, 1u);
+                umma_tf32_ta(ua, aa + KI + 8 * kk, bh, idesc, 1u);
+              }
+              umma_commit(smem_u32(ubar));
+              u_pending = true;
+              if (mbar_wait(smem_u32(ubar), uph, tmo, s_abort)) {
+                u_pending = false;
+              } else {
+                raise_device_error(p.status, s_abort, kStatusTimeout);
+              }
+              *s_epi_stop = *s_abort;
+            }
+            named_bar_sync(1, 128);
+            uph ^= 1;
+            if (*s_epi_stop) { aborted = true; break; }
+            tc_fence_after();
+            // s_q = sum_i g~_i U[token, q k_out + i]
+            for (int q = 0; q < nqb; ++q) {
+              float sq = 0.0f;
+#pragma unroll
+              for (int c = 0; c < KO; c += 16) {
+                float u[16];
+                tmem_ld16(tmem + lane_base + C::kTmU + q * KO + c, u);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) sq = fmaf(vg[c + i], u[i], sq);
+              }
+              if (in_range)
+                p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q0 + q) * p.B +
+                                  ic.b) * p.T + t] = valid ? sq : 0.0f;
+            }
+            tc_fence_before();
+          }
+          if (aborted) break;
+        } else {
         // One tile at a time: its a~ and g~ (hi + lo halves summed) are loaded,
         // used and dropped before the next tile's; the TMEM buffer is released
         // after the group (the MMA warp fills the other buffer meanwhile).
@@ -615,6 +766,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           if (lane == 0) mbar_arrive(smem_u32(&tempty[ab]));
           if (++ab == 2) { ab = 0; aph ^= 1; }
         }
+        }                                            // not the tensor-core token path
       }
       if (aborted) break;
       if constexpr (TOKEN) continue;
@@ -627,6 +779,10 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
     }
   }
 
+  if constexpr (C::kTC) {
+    // a U product abandoned after a timeout must finish before TMEM is released
+    if (threadIdx.x == 64 && u_pending) mbar_wait(smem_u32(ubar), uph, kDrainTimeoutNs, nullptr);
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {

@@ -411,9 +411,16 @@ def check_xgemm_plan(B, Q, K):
         assert (512 - p["a_base"]) // 64 >= 4
     else:
         assert acc <= p["tmem_cols"]
-    # shared memory: stages of one y tile (and y_lo unless it is in TMEM) plus x_hi, x_lo
-    stage = (1 if p["tmem_a"] else 2) * 128 * 128 + 2 * p["n_pad"] * 128
-    assert 2 <= p["stages"] <= 12 and 1024 + 512 + p["stages"] * stage <= 232448
+    # shared memory: with y in TMEM a ring of y tiles and a ring of x tiles
+    # (x_hi, x_lo); otherwise stages of y, y_lo, x_hi and x_lo
+    xtile = 2 * p["n_pad"] * 128
+    if p["tmem_a"]:
+        assert 4 <= p["stages"] <= 12 and 2 <= p["xstages"] <= 8
+        ring = p["stages"] * 128 * 128 + p["xstages"] * xtile
+    else:
+        assert 2 <= p["stages"] <= 12 and p["xstages"] == 0
+        ring = p["stages"] * (2 * 128 * 128 + xtile)
+    assert 1024 + 1024 + ring <= 232448
     # workspace: ordered, 256-byte aligned regions of the stated sizes
     offs = [p[k] for k in ("xnorm_off", "ynorm_off", "partial_off", "xh_off", "xl_off", "total")]
     assert all(o % 256 == 0 for o in offs) and offs == sorted(offs)
