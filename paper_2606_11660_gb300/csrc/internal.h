@@ -253,8 +253,6 @@ struct XGemmPlan {
   bool tmem_a = false;     // y_hi / y_lo as TMEM A operands (n_pad <= 64)
   int n_buf = 1;           // accumulator sets in TMEM
   int a_base = 0;          // TMEM column of the A ring (tmem_a)
-  int n_slots = 0;         // 64-column TMEM operand slots of the A ring (tmem_a)
-  int xstages = 0;         // x ring stages (tmem_a: the y ring is `stages`)
   bool fold = false;       // y_lo x_hi accumulates into the y_hi x_hi columns
   int sub = 16;            // 32-column steps per accumulation chain
   int tmem_cols = 32;      // TMEM columns allocated per CTA

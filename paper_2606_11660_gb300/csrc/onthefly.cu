@@ -49,17 +49,17 @@ constexpr int kXK = 32;                    // fp32 columns per stage: one 128-by
 constexpr int kYBytes = kXM * 128;         // one y tile
 constexpr int kXThreads = 320;             // producer, MMA, 4 converter, 4 epilogue warps
 constexpr int kXSmemBudget = 232448;       // 227 KB opt-in per CTA
-constexpr int kXBarBytes = 1024;
-constexpr int kXMaxStages = 12;
+constexpr int kXBarBytes = 512;
+constexpr int kXMaxStages = 8;
 constexpr int kMaxSlices = 64;
 constexpr uint64_t kXDrainTimeoutNs = 2000000000ull;
 // The tensor cores' fp32 accumulation rounds toward zero: every MMA into a
 // running TMEM sum loses up to one ulp of it, so a long chain drifts (about
 // -5e-8 of the sum per MMA, measured: -2.7e-5 over 4,096 columns of positive
 // terms).  Each accumulation chain therefore covers at most kSubSteps
-// 32-column steps (4 MMAs of K = 8 each): the MMA warp restarts the
-// accumulator after that many steps and the epilogue adds the pieces with
-// IEEE fp32 adds, in order.
+// 32-column steps (4 MMAs of K = 8 each; half as many steps when folded, see
+// below): the MMA warp restarts the accumulator after that many steps and the
+// epilogue adds the pieces with IEEE fp32 adds, in order.
 constexpr int kSubSteps = 16;
 constexpr int kMaxPad = 128;                 // largest batch tile (n_pad)
 constexpr int kMaxPadTA = 64;                // largest batch tile with y in TMEM
@@ -170,9 +170,7 @@ struct XGemmParams {
   int n_buf;          // TMEM accumulator sets (2: epilogue overlaps the next item)
   int n_items;
   int tmem_cols;
-  int sub;            // 32-column steps per accumulation chain (see kSubSteps)
-  int n_slots;        // TMEM operand slots (y_hi / y_lo, 64 columns each) with y in TMEM
-  int xstages;        // x ring stages (y in TMEM: x has a ring of its own)
+  int sub;            // 32-column steps per accumulation chain
   int fold;           // 1: y_lo x_hi adds into the y_hi x_hi columns (2 n_pad per set)
   int a_base;         // TMEM column of the y_hi / y_lo ring (A operands in TMEM)
   int unit;
@@ -218,26 +216,12 @@ __global__ void __launch_bounds__(kXThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
   const int xbytes = p.n_pad * 128;
-  // y in TMEM (TA): a ring of y tiles (stage_bytes = one y tile), released by
-  // the converter warps as soon as they have read a tile, and a ring of x
-  // tiles (x_hi, x_lo) after it, released by the MMA commits -- the y tiles
-  // need not wait for the MMAs that use them, so more of them are in flight.
-  // Otherwise one ring of stages [y | y_lo | x_hi | x_lo], released by the MMAs.
   const int xoff = (TA ? 1 : 2) * kYBytes;      // x_hi, x_lo after y (and y_lo)
-  const int stage_bytes = TA ? kYBytes : xoff + 2 * xbytes;
-  const uint32_t xring = sbase + p.stages * stage_bytes;   // TA: x ring
-  const int ring_bytes = p.stages * stage_bytes + (TA ? p.xstages * 2 * xbytes : 0);
-  // Barriers: full / empty per shared-memory stage (of y with TA); conv per
-  // stage (y_lo in shared memory) or per TMEM operand slot (y in TMEM); tfree
-  // per TMEM operand slot (the MMAs that read it are done); xfull / xempty
-  // per x stage (TA); tfull / tempty per accumulator set.
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + ring_bytes);
-  uint64_t* empty = full + kXMaxStages;
-  uint64_t* conv = empty + kXMaxStages;
-  uint64_t* tfree = conv + kXMaxStages;
-  uint64_t* xfull = tfree + kXMaxStages;
-  uint64_t* xempty = xfull + kXMaxStages;
-  uint64_t* tfull = xempty + kXMaxStages;
+  const int stage_bytes = xoff + 2 * xbytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
+  uint64_t* empty = full + p.stages;
+  uint64_t* conv = empty + p.stages;
+  uint64_t* tfull = conv + p.stages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
@@ -248,17 +232,8 @@ __global__ void __launch_bounds__(kXThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), TA ? 4 : 1);   // TA: one arrival per converter warp
-    }
-    for (int s = 0; s < (TA ? p.n_slots : p.stages); ++s) {
+      mbar_init(smem_u32(&empty[s]), 1);
       mbar_init(smem_u32(&conv[s]), 128);
-      mbar_init(smem_u32(&tfree[s]), 1);
-    }
-    if (TA) {
-      for (int s = 0; s < p.xstages; ++s) {
-        mbar_init(smem_u32(&xfull[s]), 1);
-        mbar_init(smem_u32(&xempty[s]), 1);
-      }
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&tfull[i]), 1);
@@ -278,95 +253,7 @@ __global__ void __launch_bounds__(kXThreads, 1)
   const uint32_t tmem = *s_tmem;
   const uint64_t tmo = p.timeout_ns;
 
-  if (warp == 0 && TA) {
-    // ------------------------------------------------------------ producer (two rings)
-    // Two cursors over this CTA's steps: y tiles go out as soon as a y stage
-    // is free, x tiles as soon as an x stage is free (non-blocking tests of
-    // both, so neither ring waits on the other); the first y tiles do not
-    // depend on the row split that precedes this grid, the x tiles do.
-    if (lane == 0) {
-      prefetch_tmap(&tm_y);
-      prefetch_tmap(&tm_xh);
-      prefetch_tmap(&tm_xl);
-      const uint64_t pol_y = policy_evict_first();    // streamed once
-      const uint64_t pol_x = policy_evict_last();     // re-read by every tile
-      struct Cursor {
-        int item, st, s1, mt, nt;
-        bool valid;
-      };
-      auto start = [&](Cursor& c, int item) {
-        c.item = item;
-        c.valid = item < p.n_items;
-        if (!c.valid) return;
-        const XItem it = decode_xitem(p, item);
-        c.st = it.s0;
-        c.s1 = it.s1;
-        c.mt = it.mt;
-        c.nt = it.nt;
-      };
-      auto advance = [&](Cursor& c) {
-        if (++c.st == c.s1) start(c, c.item + gridDim.x);
-      };
-      Cursor cy, cx;
-      start(cy, blockIdx.x);
-      start(cx, blockIdx.x);
-      int ys = 0, xs = 0;
-      uint32_t yph = 0, xph = 0;
-      uint32_t y_issued = 0, y_par = 0, x_issued = 0, x_par = 0;
-      auto issue_y = [&]() {
-        const uint32_t fb = smem_u32(&full[ys]);
-        mbar_arrive_expect_tx(fb, kYBytes);
-        tma_load_2d_hint(sbase + ys * kYBytes, &tm_y, fb, cy.st * kXK, cy.mt * kXM, pol_y);
-        y_issued |= 1u << ys;
-        y_par = (y_par & ~(1u << ys)) | (yph << ys);
-        if (++ys == p.stages) { ys = 0; yph ^= 1; }
-        advance(cy);
-      };
-      auto issue_x = [&]() {
-        const uint32_t fb = smem_u32(&xfull[xs]);
-        const uint32_t dst = xring + xs * 2 * xbytes;
-        mbar_arrive_expect_tx(fb, 2 * xbytes);
-        tma_load_2d_hint(dst, &tm_xh, fb, cx.st * kXK, cx.nt * p.n_pad, pol_x);
-        tma_load_2d_hint(dst + xbytes, &tm_xl, fb, cx.st * kXK, cx.nt * p.n_pad, pol_x);
-        x_issued |= 1u << xs;
-        x_par = (x_par & ~(1u << xs)) | (xph << xs);
-        if (++xs == p.xstages) { xs = 0; xph ^= 1; }
-        advance(cx);
-      };
-      for (int k = 0; k < p.stages && cy.valid; ++k) issue_y();   // the y ring starts empty
-      griddep_wait();                 // x_hi / x_lo are the row split's output
-      bool ok = true;
-      uint64_t t_last = global_timer_ns();
-      while (cx.valid || cy.valid) {
-        bool moved = false;
-        if (cy.valid && mbar_test_wait(smem_u32(&empty[ys]), yph ^ 1)) {
-          issue_y();
-          moved = true;
-        }
-        if (cx.valid && mbar_test_wait(smem_u32(&xempty[xs]), xph ^ 1)) {
-          issue_x();
-          moved = true;
-        }
-        if (moved) {
-          t_last = global_timer_ns();
-        } else if (*s_abort || global_timer_ns() - t_last > tmo) {
-          ok = false;
-          break;
-        }
-      }
-      griddep_launch_dependents();   // every load issued: the finishing grid may launch
-      if (!ok) {
-        raise_device_error(p.status, s_abort, kStatusTimeout);
-        for (int s = 0; s < p.stages; ++s)
-          if (y_issued >> s & 1)
-            mbar_wait(smem_u32(&full[s]), (y_par >> s) & 1, kXDrainTimeoutNs, nullptr);
-        for (int s = 0; s < p.xstages; ++s)
-          if (x_issued >> s & 1)
-            mbar_wait(smem_u32(&xfull[s]), (x_par >> s) & 1, kXDrainTimeoutNs, nullptr);
-      }
-    }
-    __syncwarp();
-  } else if (warp == 0) {
+  if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       prefetch_tmap(&tm_y);
@@ -432,69 +319,59 @@ __global__ void __launch_bounds__(kXThreads, 1)
       const uint32_t idesc_lo = make_idesc_tf32(kXM, p.n_pad);    // y_lo x_hi^T
       int stage = 0;
       uint32_t ph = 0;
-      int slot = 0;                   // TMEM operand slot (y in TMEM)
-      uint32_t tph = 0;
       int ab = 0;
       uint32_t aph = 0;
       bool ok = true;
       for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
         const XItem it = decode_xitem(p, item);
-        for (int c0 = it.s0; c0 < it.s1 && ok; c0 += p.sub) {   // one accumulation chain each
-          const int c1 = min(it.s1, c0 + p.sub);
-          if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+        for (int c0 = it.s0; c0 < it.s1 && ok; c0 += p.sub) {
+        const int c1 = min(it.s1, c0 + p.sub);
+        if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
+        tc_fence_after();
+        // Set ab: D_hi = y_hi [x_hi; x_lo]^T in columns [0, 2 n_pad) (x_hi and
+        // x_lo land next to each other, so one B operand of 2 n_pad rows serves
+        // both, and y_hi and y_lo are each read once per K step), and D_lo =
+        // y_lo x_hi^T either in columns [2 n_pad, 3 n_pad) -- an independent
+        // accumulation chain -- or, folded (large batch tiles), added into
+        // columns [0, n_pad), so that a set takes 2 n_pad columns and two sets
+        // fit at n_pad = 128.
+        const uint32_t d_hi = tmem + ab * (p.fold ? 2 : 3) * p.n_pad;
+        const uint32_t d_lo = p.fold ? d_hi : d_hi + 2 * p.n_pad;
+        for (int st = c0; st < c1; ++st) {
+          if (!mbar_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
+              !mbar_wait(smem_u32(&conv[stage]), ph, tmo, s_abort)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
-          // Set ab: D[0, 2 n_pad) = y_hi [x_hi; x_lo]^T (x_hi and x_lo land
-          // next to each other, so one MMA with N = 2 n_pad writes both), and
-          // y_lo x_hi^T either in its own columns [2 n_pad, 3 n_pad) -- an
-          // independent accumulation chain -- or, folded, added into
-          // D[0, n_pad) (2 n_pad columns per set: two sets fit at n_pad = 128).
-          const int set_cols = (p.fold ? 2 : 3) * p.n_pad;
-          const uint32_t d = tmem + ab * set_cols;
-          const uint32_t d_lo = p.fold ? d : d + 2 * p.n_pad;
-          for (int st = c0; st < c1; ++st) {
-            // TA: `stage` runs over the x ring (x_hi, x_lo) and the y tile
-            // waits in TMEM slot `slot`; otherwise over the one ring of stages.
-            if (!mbar_wait(smem_u32(TA ? &xfull[stage] : &full[stage]), ph, tmo, s_abort) ||
-                !mbar_wait(smem_u32(&conv[TA ? slot : stage]), TA ? tph : ph, tmo, s_abort)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            const uint32_t yh = sbase + stage * stage_bytes;
-            const uint64_t dx = sw128_desc(TA ? xring + stage * 2 * xbytes : yh + xoff);
-            if constexpr (TA) {
-              const uint32_t ta = tmem + p.a_base + slot * 2 * kXK;   // y_hi, then y_lo
+          const uint32_t yh = sbase + stage * stage_bytes;
+          const uint64_t dx = sw128_desc(yh + xoff);
+          if constexpr (TA) {
+            const uint32_t ta = tmem + p.a_base + stage * 2 * kXK;   // y_hi, then y_lo
 #pragma unroll
-              for (int kk = 0; kk < kXK / 8; ++kk) {
-                const uint64_t o = 2 * kk;
-                const uint32_t acc = st != c0 || kk != 0;
-                umma_tf32_ta(d, ta + 8 * kk, dx + o, idesc, acc);
-                umma_tf32_ta(d_lo, ta + kXK + 8 * kk, dx + o, idesc_lo, p.fold ? 1u : acc);
-              }
-            } else {
-              const uint64_t dyh = sw128_desc(yh);
-              const uint64_t dyl = sw128_desc(yh + kYBytes);
-#pragma unroll
-              for (int kk = 0; kk < kXK / 8; ++kk) {   // 8 tf32 = 32 bytes: +2 in the address field
-                const uint64_t o = 2 * kk;
-                const uint32_t acc = st != c0 || kk != 0;
-                umma_tf32(d, dyh + o, dx + o, idesc, acc);
-                umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, p.fold ? 1u : acc);
-              }
+            for (int kk = 0; kk < kXK / 8; ++kk) {
+              const uint64_t o = 2 * kk;
+              const uint32_t acc = st != c0 || kk != 0;
+              umma_tf32_ta(d_hi, ta + 8 * kk, dx + o, idesc, acc);
+              umma_tf32_ta(d_lo, ta + kXK + 8 * kk, dx + o, idesc_lo, p.fold ? 1u : acc);
             }
-            if constexpr (TA) {
-              umma_commit(smem_u32(&xempty[stage]));
-              if (++stage == p.xstages) { stage = 0; ph ^= 1; }
-              umma_commit(smem_u32(&tfree[slot]));
-              if (++slot == p.n_slots) { slot = 0; tph ^= 1; }
-            } else {
-              umma_commit(smem_u32(&empty[stage]));
-              if (++stage == p.stages) { stage = 0; ph ^= 1; }
+          } else {
+            const uint64_t dyh = sw128_desc(yh);
+            const uint64_t dyl = sw128_desc(yh + kYBytes);
+#pragma unroll
+            for (int kk = 0; kk < kXK / 8; ++kk) {     // 8 tf32 = 32 bytes: +2 in the address field
+              const uint64_t o = 2 * kk;
+              const uint32_t acc = st != c0 || kk != 0;
+              umma_tf32(d_hi, dyh + o, dx + o, idesc, acc);
+              umma_tf32(d_lo, dyl + o, dx + o, idesc_lo, p.fold ? 1u : acc);
             }
           }
-          if (!ok) break;
-          umma_commit(smem_u32(&tfull[ab]));
-          if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
+          umma_commit(smem_u32(&empty[stage]));
+          if (++stage == p.stages) { stage = 0; ph ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit(smem_u32(&tfull[ab]));
+        if (++ab == p.n_buf) { ab = 0; aph ^= 1; }
         }
       }
       if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
@@ -510,18 +387,14 @@ __global__ void __launch_bounds__(kXThreads, 1)
     const int quarter = warp & 3;
     const int r = 32 * quarter + lane;
     const uint32_t trow = tmem + (static_cast<uint32_t>(32 * quarter) << 16) + p.a_base;
-    // The TMEM slots form their own ring (n_slots <= stages): a stage's y
-    // tile moves into the next free slot, so more y tiles can be in flight
-    // in shared memory than there are slots.
-    int stage = 0, slot = 0;
-    uint32_t ph = 0, tph = 0;
+    int stage = 0;
+    uint32_t ph = 0;
     for (int item = blockIdx.x; item < p.n_items; item += gridDim.x) {
       const XItem it = decode_xitem(p, item);
       KahanSum nrm;
       bool aborted = false;
       for (int st = it.s0; st < it.s1; ++st) {
-        if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort) ||
-            !warp_wait(smem_u32(&tfree[slot]), tph ^ 1, tmo, s_abort)) {
+        if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) {
           raise_device_error(p.status, s_abort, kStatusTimeout);
           aborted = true;
           break;
@@ -537,16 +410,12 @@ __global__ void __launch_bounds__(kXThreads, 1)
           lv[4 * c] = l.x; lv[4 * c + 1] = l.y; lv[4 * c + 2] = l.z; lv[4 * c + 3] = l.w;
           if (p.unit) nrm.add(v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w);
         }
-        // The tile is in registers: its y stage goes back to the producer now.
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&empty[stage]));
-        tmem_st32(trow + slot * 2 * kXK, hv);
-        tmem_st32(trow + slot * 2 * kXK + kXK, lv);
+        tmem_st32(trow + stage * 2 * kXK, hv);
+        tmem_st32(trow + stage * 2 * kXK + kXK, lv);
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(smem_u32(&conv[slot]));
+        mbar_arrive(smem_u32(&conv[stage]));
         if (++stage == p.stages) { stage = 0; ph ^= 1; }
-        if (++slot == p.n_slots) { slot = 0; tph ^= 1; }
       }
       if (aborted) break;
       const int q = it.mt * kXM + r;
@@ -733,36 +602,27 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   pl.n_ntiles = static_cast<int>((b1 + pl.n_pad - 1) / pl.n_pad);
   pl.n_mtiles = static_cast<int>(std::max<int64_t>(1, (Q + kXM - 1) / kXM));
   pl.steps = static_cast<int>(std::max<int64_t>(1, (K + kXK - 1) / kXK));
-  // y_hi / y_lo go to TMEM (as MMA A operands) for batch tiles of up to 64
-  // rows.  There the three products keep separate column groups (3 n_pad per
-  // accumulator set: two independent accumulation chains), two sets, and the
-  // operand ring takes the remaining columns.  Larger batch tiles fold y_lo
-  // x_hi into the y_hi x_hi columns (2 n_pad per set), so that two sets (and,
-  // up to n_pad = 64, four operand slots) fit even at n_pad = 128; a folded
-  // chain takes twice the MMAs per step, so its chains are half as many steps
-  // long.
+  // y_hi / y_lo go to TMEM when the accumulators leave room for a ring of at
+  // least 4 stages (64 columns each); otherwise y_lo is written next to y,
+  // and y_lo x_hi folds into the y_hi x_hi columns so that two accumulator
+  // sets fit (a folded chain takes twice the MMAs per step: half the steps).
   pl.tmem_a = pl.n_pad <= 64;
-  pl.n_buf = 2;
-  // unfolded where two 3 n_pad sets still leave four operand slots (n_pad <= 32)
-  pl.fold = !pl.tmem_a || 2 * 3 * pl.n_pad + 4 * 2 * kXK > 512;
+  pl.fold = !pl.tmem_a;
   pl.sub = pl.fold ? kSubSteps / 2 : kSubSteps;
   int stage_bytes;
-  const int budget = kXSmemBudget - 1024 - kXBarBytes;
   if (pl.tmem_a) {
-    pl.a_base = (pl.n_buf * (pl.fold ? 2 : 3) * pl.n_pad + 31) / 32 * 32;
+    pl.n_buf = (512 - 6 * pl.n_pad) / (2 * kXK) >= 4 ? 2 : 1;
+    pl.a_base = (pl.n_buf * 3 * pl.n_pad + 31) / 32 * 32;
     pl.tmem_cols = 512;
-    pl.n_slots = (512 - pl.a_base) / (2 * kXK);
-    // a y ring of up to 12 tiles and an x ring of up to 8 (x comes from L2)
-    const int xstage = 2 * pl.n_pad * 128;
-    pl.xstages = std::min(8, (budget - 4 * kYBytes) / xstage);
-    stage_bytes = kYBytes + xstage;                       // (for the slice cost below)
-    pl.stages = std::min(kXMaxStages, (budget - pl.xstages * xstage) / kYBytes);
+    stage_bytes = kYBytes + 2 * pl.n_pad * 128;
+    pl.stages = std::min({kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes,
+                          (512 - pl.a_base) / (2 * kXK)});
   } else {
+    pl.n_buf = 2;
     pl.tmem_cols = 32;
     while (pl.tmem_cols < pl.n_buf * 2 * pl.n_pad) pl.tmem_cols <<= 1;
     stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
-    pl.stages = std::min(kXMaxStages, budget / stage_bytes);
-    pl.xstages = 0;
+    pl.stages = std::min(kXMaxStages, (kXSmemBudget - 1024 - kXBarBytes) / stage_bytes);
   }
   // K slices: fewest waves of persistent CTAs for the y stream, plus the
   // partials each slice adds (written and read back once).
@@ -828,8 +688,6 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   p.n_buf = pl.n_buf;
   p.tmem_cols = pl.tmem_cols;
   p.sub = pl.sub;
-  p.n_slots = pl.n_slots;
-  p.xstages = pl.xstages;
   p.fold = pl.fold ? 1 : 0;
   p.a_base = pl.a_base;
   p.unit = a.unit;
@@ -837,12 +695,10 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   p.ynorm = reinterpret_cast<float*>(a.ws + pl.ynorm_off);
   p.status = a.status;
   p.timeout_ns = a.timeout_ns;
-  const size_t smem =
-      1024 +
-      (pl.tmem_a ? static_cast<size_t>(pl.stages) * kYBytes +
-                       static_cast<size_t>(pl.xstages) * 2 * pl.n_pad * 128
-                 : static_cast<size_t>(pl.stages) * (2 * kYBytes + 2 * pl.n_pad * 128)) +
-      kXBarBytes;
+  const size_t smem = 1024 +
+                      static_cast<size_t>(pl.stages) *
+                          ((pl.tmem_a ? 1 : 2) * kYBytes + 2 * pl.n_pad * 128) +
+                      kXBarBytes;
   const int grid = std::max(1, std::min(sms > 0 ? sms : 1, p.n_items));
   e = pl.tmem_a ? launch_xgemm<true>(grid, smem, s, tm_y, tm_xh, tm_xl, p)
                 : launch_xgemm<false>(grid, smem, s, tm_y, tm_xh, tm_xl, p);

@@ -399,28 +399,22 @@ def check_xgemm_plan(B, Q, K):
     assert 1 <= S <= min(steps, 64)
     bounds = [z * steps // S for z in range(S + 1)]
     assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
-    # TMEM: two accumulator sets (3 n_pad columns each with y in TMEM, 2 n_pad
-    # folded otherwise) and, with y in TMEM, a ring of at least four 64-column
-    # operand slots, within 512 columns
-    fold = not p["tmem_a"] or 6 * p["n_pad"] + 256 > 512
+    # TMEM: accumulator sets of 3 n_pad columns (2 n_pad, two sets, when y_lo
+    # folds into y_hi x_hi for large batch tiles) and, with y in TMEM, the
+    # 64-column operand ring (one slot per stage), within 512 columns
+    fold = not p["tmem_a"]
     acc = p["n_buf"] * (2 if fold else 3) * p["n_pad"]
-    assert p["tmem_a"] == (p["n_pad"] <= 64) and p["n_buf"] == 2
+    assert p["tmem_a"] == (p["n_pad"] <= 64) and p["n_buf"] in (1, 2)
+    assert fold or p["n_buf"] == 2 or 6 * p["n_pad"] + 4 * 64 > 512
     assert p["tmem_cols"] <= 512 and p["tmem_cols"] & (p["tmem_cols"] - 1) == 0
     if p["tmem_a"]:
-        assert p["a_base"] >= acc and p["a_base"] % 32 == 0 and p["tmem_cols"] == 512
-        assert (512 - p["a_base"]) // 64 >= 4
+        assert p["a_base"] >= acc and p["a_base"] % 32 == 0
+        assert p["a_base"] + p["stages"] * 64 <= p["tmem_cols"] == 512
     else:
-        assert acc <= p["tmem_cols"]
-    # shared memory: with y in TMEM a ring of y tiles and a ring of x tiles
-    # (x_hi, x_lo); otherwise stages of y, y_lo, x_hi and x_lo
-    xtile = 2 * p["n_pad"] * 128
-    if p["tmem_a"]:
-        assert 4 <= p["stages"] <= 12 and 2 <= p["xstages"] <= 8
-        ring = p["stages"] * 128 * 128 + p["xstages"] * xtile
-    else:
-        assert 2 <= p["stages"] <= 12 and p["xstages"] == 0
-        ring = p["stages"] * (2 * 128 * 128 + xtile)
-    assert 1024 + 1024 + ring <= 232448
+        assert p["n_buf"] == 2 and acc <= p["tmem_cols"]
+    # shared memory: stages of one y tile (and y_lo unless it is in TMEM) plus x_hi, x_lo
+    stage = (1 if p["tmem_a"] else 2) * 128 * 128 + 2 * p["n_pad"] * 128
+    assert 2 <= p["stages"] <= 8 and 1024 + 512 + p["stages"] * stage <= 232448
     # workspace: ordered, 256-byte aligned regions of the stated sizes
     offs = [p[k] for k in ("xnorm_off", "ynorm_off", "partial_off", "xh_off", "xl_off", "total")]
     assert all(o % 256 == 0 for o in offs) and offs == sorted(offs)
