@@ -508,14 +508,14 @@ def bergson_debug_score_plan(N: int, K: int, Q: int, topk: int, ctas: int) -> li
 
 
 XGEMM_PLAN_FIELDS = ("n_pad", "n_ntiles", "n_mtiles", "steps", "S", "stages", "n_chunks",
-                     "tmem_a", "n_buf", "a_base", "tmem_cols", "xnorm_off", "ynorm_off",
-                     "partial_off", "xh_off", "xl_off", "total")
+                     "n_side", "n_buf", "y_rows", "tmem_cols", "xnorm_off", "ynorm_off",
+                     "partial_off", "xh_off", "xl_off", "total", "lo_slots", "x_slots")
 
 
 def bergson_debug_xgemm_plan(B: int, Q: int, K: int) -> dict:
     """The skinny-product planner's choices for B x rows, Q y rows, length K; host only."""
-    buf = (ctypes.c_int64 * 17)()
-    _check(lib().bergson_debug_xgemm_plan(int(B), int(Q), int(K), buf, 17))
+    buf = (ctypes.c_int64 * 19)()
+    _check(lib().bergson_debug_xgemm_plan(int(B), int(Q), int(K), buf, 19))
     return dict(zip(XGEMM_PLAN_FIELDS, buf))
 
 

@@ -670,16 +670,17 @@ int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_t topk, int 
 }
 
 int bergson_debug_xgemm_plan(int64_t B, int64_t Q, int64_t K, int64_t* out, int n_out) {
-  if (out == nullptr || n_out < 17) return fail(BERGSON_EINVAL, "out needs room for 17 values");
+  if (out == nullptr || n_out < 19) return fail(BERGSON_EINVAL, "out needs room for 19 values");
   if (B < 1 || B > (1 << 20) || Q < 1 || Q > (1 << 24) || K < 4 || K > (1 << 26) || K % 4 != 0)
     return fail(BERGSON_EINVAL, "invalid sizes for the skinny-product plan");
   const XGemmPlan pl = xgemm_plan(B, Q, K);
-  const int64_t v[17] = {pl.n_pad, pl.n_ntiles, pl.n_mtiles, pl.steps, pl.S, pl.stages,
-                         pl.n_chunks, pl.tmem_a ? 1 : 0, pl.n_buf, pl.a_base, pl.tmem_cols,
+  const int64_t v[19] = {pl.n_pad, pl.n_ntiles, pl.n_mtiles, pl.steps, pl.S, pl.stages,
+                         pl.n_chunks, pl.n_side ? 1 : 0, pl.n_buf, pl.y_rows, pl.tmem_cols,
                          static_cast<int64_t>(pl.xnorm_off), static_cast<int64_t>(pl.ynorm_off),
                          static_cast<int64_t>(pl.partial_off), static_cast<int64_t>(pl.xh_off),
-                         static_cast<int64_t>(pl.xl_off), static_cast<int64_t>(pl.total)};
-  for (int i = 0; i < 17; ++i) out[i] = v[i];
+                         static_cast<int64_t>(pl.xl_off), static_cast<int64_t>(pl.total),
+                         pl.lo_slots, pl.x_slots};
+  for (int i = 0; i < 19; ++i) out[i] = v[i];
   return BERGSON_OK;
 }
 

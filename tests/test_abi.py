@@ -389,39 +389,51 @@ def test_xgemm_planner_invariants(B, Q, K):
 
 def check_xgemm_plan(B, Q, K):
     p = bg.bergson_debug_xgemm_plan(B, Q, K)
+    # batches of up to 64 rows put y on the MMA's N side: one batch tile of 32
+    # or 64 rows (MMA M = 64 or 128) against 256-row y tiles; larger batches
+    # use tiles of up to 128 rows against 128-row y tiles
+    n_side = p["n_side"] == 1
+    assert n_side == (B <= 64)
+    if n_side:
+        assert p["n_pad"] == (32 if B <= 32 else 64) and p["y_rows"] == 256
+    else:
+        assert p["n_pad"] % 16 == 0 and 16 <= p["n_pad"] <= 128 and p["y_rows"] == 128
     # tiles cover the operands
-    assert p["n_pad"] % 16 == 0 and 16 <= p["n_pad"] <= 128
     assert p["n_ntiles"] * p["n_pad"] >= B > (p["n_ntiles"] - 1) * p["n_pad"]
-    assert p["n_mtiles"] * 128 >= Q > (p["n_mtiles"] - 1) * 128
+    rows = p["y_rows"]
+    assert p["n_mtiles"] * rows >= Q > (p["n_mtiles"] - 1) * rows
     assert p["steps"] * 32 >= K > (p["steps"] - 1) * 32
     # every K slice is a nonempty, contiguous range of steps
     S, steps = p["S"], p["steps"]
     assert 1 <= S <= min(steps, 64)
     bounds = [z * steps // S for z in range(S + 1)]
     assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
-    # TMEM: accumulator sets of 3 n_pad columns (2 n_pad, two sets, when y_lo
-    # folds into y_hi x_hi for large batch tiles) and, with y in TMEM, the
-    # 64-column operand ring (one slot per stage), within 512 columns
-    fold = not p["tmem_a"]
-    acc = p["n_buf"] * (2 if fold else 3) * p["n_pad"]
-    assert p["tmem_a"] == (p["n_pad"] <= 64) and p["n_buf"] in (1, 2)
-    assert fold or p["n_buf"] == 2 or 6 * p["n_pad"] + 4 * 64 > 512
+    # TMEM: two accumulator sets, 256 columns each on the N side (M = 2 n_pad
+    # rows), 2 n_pad columns each on the M side, within a power of two <= 512
+    assert p["n_buf"] == 2
     assert p["tmem_cols"] <= 512 and p["tmem_cols"] & (p["tmem_cols"] - 1) == 0
-    if p["tmem_a"]:
-        assert p["a_base"] >= acc and p["a_base"] % 32 == 0
-        assert p["a_base"] + p["stages"] * 64 <= p["tmem_cols"] == 512
+    acc = 2 * (256 if n_side else 2 * p["n_pad"])
+    assert acc <= p["tmem_cols"]
+    # shared memory: on the N side rings of y stages, y_lo slots and x slots
+    # (x slots outlive the y stages); on the M side stages of one y tile, its
+    # y_lo and the x_hi, x_lo rows
+    xb = 2 * p["n_pad"] * 128
+    if n_side:
+        assert 2 <= p["stages"] <= 8 and 1 <= p["lo_slots"] <= 4
+        assert p["stages"] < p["x_slots"] <= 8
+        rings = (p["stages"] + p["lo_slots"]) * 256 * 128 + p["x_slots"] * xb
     else:
-        assert p["n_buf"] == 2 and acc <= p["tmem_cols"]
-    # shared memory: stages of one y tile (and y_lo unless it is in TMEM) plus x_hi, x_lo
-    stage = (1 if p["tmem_a"] else 2) * 128 * 128 + 2 * p["n_pad"] * 128
-    assert 2 <= p["stages"] <= 8 and 1024 + 512 + p["stages"] * stage <= 232448
+        assert 2 <= p["stages"] <= 8 and p["lo_slots"] == 0 and p["x_slots"] == 0
+        rings = p["stages"] * (2 * 128 * 128 + xb)
+    assert 1024 + 512 + rings <= 232448
     # workspace: ordered, 256-byte aligned regions of the stated sizes
     offs = [p[k] for k in ("xnorm_off", "ynorm_off", "partial_off", "xh_off", "xl_off", "total")]
     assert all(o % 256 == 0 for o in offs) and offs == sorted(offs)
     assert p["ynorm_off"] - p["xnorm_off"] >= 4 * B * p["n_chunks"]
     assert p["n_chunks"] == -(-K // 2048)
     assert p["partial_off"] - p["ynorm_off"] >= 4 * S * Q
-    assert p["xh_off"] - p["partial_off"] >= 4 * S * B * Q
+    planes = 2 if n_side else 1                  # x_hi and x_lo rows on the N side
+    assert p["xh_off"] - p["partial_off"] >= 4 * planes * S * B * Q
     assert p["xl_off"] - p["xh_off"] >= 4 * B * K and p["total"] - p["xl_off"] >= 4 * B * K
     n = ctypes.c_size_t()
     st = bg.lib().bergson_score_grads_workspace(B, K, Q, ctypes.byref(n))

@@ -23,7 +23,10 @@ def _scores(x, y, unit, ld_pad=0):
 
 
 @pytest.mark.parametrize("B,K,Q", [(37, 12288, 130), (1, 36, 1), (64, 520, 1000), (3, 4096, 7),
-                                   (300, 1000, 200), (16, 4, 129)])
+                                   (300, 1000, 200), (16, 4, 129),
+                                   # K slices of 16 to 26 steps of 32 columns: accumulation
+                                   # chains of 8 steps, then 1 or 2, over 150+ tiles of y
+                                   (64, 1056, 40000), (20, 4128, 39000), (33, 8224, 515)])
 @pytest.mark.parametrize("unit", [True, False])
 def test_random_rows(B, K, Q, unit):
     g = wl.generator(B * 31 + K + Q, "cpu")
