@@ -560,11 +560,12 @@ BERGSON_API int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_
  * bergson_score_grads, bergson_precondition_rows and the Fisher products
  * (C[b, q] = <x_b, y_q> for B rows x, Q rows y of length K).  Writes 19 int64
  * to out (n_out >= 19): batch rows per tile, batch tiles, y tiles, 32-column
- * steps, K slices, pipeline stages (of y), column chunks of the row split, y
- * on the MMA's N side (1/0: batches of up to 64 rows), accumulator buffers,
- * rows of y per tile (256 on the N side, else 128), TMEM columns allocated,
- * the workspace offsets of the x norms, y norms, partial products, x_hi, x_lo
- * and the total, then the N side's y_lo slots and x slots (0 otherwise).
+ * steps, K slices, pipeline stages, column chunks of the row split, CTA pairs
+ * (1/0: batches of up to 64 rows), accumulator buffers, rows of y per tile
+ * (256 on pairs, else 128), TMEM columns allocated, the workspace offsets of
+ * the x norms, y norms, partial products, x_hi, x_lo and the total, then the
+ * TMEM column of the pairs' y operand ring (a 64-column slot per stage; 0
+ * otherwise) and the most 32-column steps per accumulation chain.
  * Host only: enqueues nothing.  Errors: EINVAL (B in [1, 2^20], Q in
  * [1, 2^24], K in [4, 2^26] and a multiple of 4).
  */

@@ -675,11 +675,11 @@ int bergson_debug_xgemm_plan(int64_t B, int64_t Q, int64_t K, int64_t* out, int 
     return fail(BERGSON_EINVAL, "invalid sizes for the skinny-product plan");
   const XGemmPlan pl = xgemm_plan(B, Q, K);
   const int64_t v[19] = {pl.n_pad, pl.n_ntiles, pl.n_mtiles, pl.steps, pl.S, pl.stages,
-                         pl.n_chunks, pl.n_side ? 1 : 0, pl.n_buf, pl.y_rows, pl.tmem_cols,
+                         pl.n_chunks, pl.pair ? 1 : 0, pl.n_buf, pl.y_rows, pl.tmem_cols,
                          static_cast<int64_t>(pl.xnorm_off), static_cast<int64_t>(pl.ynorm_off),
                          static_cast<int64_t>(pl.partial_off), static_cast<int64_t>(pl.xh_off),
                          static_cast<int64_t>(pl.xl_off), static_cast<int64_t>(pl.total),
-                         pl.lo_slots, pl.x_slots};
+                         pl.a_base, pl.sub};
   for (int i = 0; i < 19; ++i) out[i] = v[i];
   return BERGSON_OK;
 }

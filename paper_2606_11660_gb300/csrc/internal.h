@@ -243,22 +243,18 @@ cudaError_t launch_fisher_power(const float* r1, const float* r2, int K, int64_t
 // Skinny fp32 product C[b, q] = <x_b, y_q> on the tensor cores (on-the-fly
 // scores, preconditioner application): plan and workspace layout.
 struct XGemmPlan {
-  int n_pad = 32;          // batch rows per tile (32 or 64 with y on the N side, else a
-                           // multiple of 16 up to 128)
+  int n_pad = 16;          // batch rows per tile (multiple of 16; <= 64 on pairs, <= 128 else)
   int n_ntiles = 1;        // ceil(B / n_pad)
   int n_mtiles = 1;        // ceil(Q / y_rows)
   int steps = 1;           // ceil(K / 32)
   int S = 1;               // K slices
   int stages = 2;          // shared-memory pipeline depth
   int n_chunks = 1;        // column chunks of x for the row split (norm partials per row)
-  bool n_side = false;     // y on the MMA's N side (B <= 64)
+  bool pair = false;       // CTA pairs with y in TMEM (B <= 64)
   int n_buf = 2;           // accumulator sets in TMEM
-  int y_rows = 128;        // rows of y per tile (256 on the N side)
-  int planes = 1;          // partial planes per K slice (2 on the N side: x_hi and x_lo rows)
-  int sub = 8;             // 32-column steps per accumulation chain
-  int lookahead = 2;       // N side: y_hi steps issued ahead of the y_lo step
-  int lo_slots = 0;        // N side: y_lo slots in shared memory
-  int x_slots = 0;         // N side: x slots in shared memory
+  int y_rows = 128;        // rows of y per work item (256 on pairs: 128 per CTA)
+  int a_base = 0;          // pairs: TMEM column of the y_hi / y_lo ring (a slot per stage)
+  int sub = 8;             // 32-column steps per accumulation chain (at most)
   int tmem_cols = 32;      // TMEM columns allocated per CTA
   size_t xnorm_off = 0, ynorm_off = 0, partial_off = 0, xh_off = 0, xl_off = 0, total = 0;
 };

@@ -412,6 +412,15 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
                : "memory");
 }
 
+// Arrive on an mbarrier of either CTA of the cluster with release at CTA
+// scope (no cluster-wide memory barrier).  For signals that order only the
+// arriving thread's tcgen05 operations (after tcgen05.wait::st / ld and
+// tcgen05.fence::before_thread_sync) against the waiting CTA's later tcgen05
+// operations, which is all a per-stage handoff of TMEM operands needs.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -472,6 +481,19 @@ __device__ __forceinline__ void umma_f16_pair(uint32_t d_tmem, uint64_t a_desc, 
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// D (+)= A * B^T over the CTA pair (M = 256, kind::tf32), A from TMEM: rows
+// 0..127 at `a_tmem` in the even CTA's TMEM, rows 128..255 at the same
+// address in the odd CTA's; issued by one thread of the even CTA.
+__device__ __forceinline__ void umma_tf32_pair_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                                  uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::tf32 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 

@@ -389,15 +389,12 @@ def test_xgemm_planner_invariants(B, Q, K):
 
 def check_xgemm_plan(B, Q, K):
     p = bg.bergson_debug_xgemm_plan(B, Q, K)
-    # batches of up to 64 rows put y on the MMA's N side: one batch tile of 32
-    # or 64 rows (MMA M = 64 or 128) against 256-row y tiles; larger batches
-    # use tiles of up to 128 rows against 128-row y tiles
-    n_side = p["n_side"] == 1
-    assert n_side == (B <= 64)
-    if n_side:
-        assert p["n_pad"] == (32 if B <= 32 else 64) and p["y_rows"] == 256
-    else:
-        assert p["n_pad"] % 16 == 0 and 16 <= p["n_pad"] <= 128 and p["y_rows"] == 128
+    # batches of up to 64 rows run on CTA pairs (256 rows of y per item, 128
+    # per CTA); larger batches on single CTAs with tiles of up to 128 rows
+    pair = p["pair"] == 1
+    assert pair == (B <= 64)
+    assert p["n_pad"] % 16 == 0 and 16 <= p["n_pad"] <= (64 if pair else 128)
+    assert p["y_rows"] == (256 if pair else 128)
     # tiles cover the operands
     assert p["n_ntiles"] * p["n_pad"] >= B > (p["n_ntiles"] - 1) * p["n_pad"]
     rows = p["y_rows"]
@@ -408,32 +405,29 @@ def check_xgemm_plan(B, Q, K):
     assert 1 <= S <= min(steps, 64)
     bounds = [z * steps // S for z in range(S + 1)]
     assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
-    # TMEM: two accumulator sets, 256 columns each on the N side (M = 2 n_pad
-    # rows), 2 n_pad columns each on the M side, within a power of two <= 512
+    # TMEM: two accumulator sets of 2 n_pad columns, and on pairs the y_hi /
+    # y_lo ring after them (64 columns a stage), within 512 columns
     assert p["n_buf"] == 2
     assert p["tmem_cols"] <= 512 and p["tmem_cols"] & (p["tmem_cols"] - 1) == 0
-    acc = 2 * (256 if n_side else 2 * p["n_pad"])
-    assert acc <= p["tmem_cols"]
-    # shared memory: on the N side rings of y stages, y_lo slots and x slots
-    # (x slots outlive the y stages); on the M side stages of one y tile, its
-    # y_lo and the x_hi, x_lo rows
-    xb = 2 * p["n_pad"] * 128
-    if n_side:
-        assert 2 <= p["stages"] <= 8 and 1 <= p["lo_slots"] <= 4
-        assert p["stages"] < p["x_slots"] <= 8
-        rings = (p["stages"] + p["lo_slots"]) * 256 * 128 + p["x_slots"] * xb
+    acc = 2 * 2 * p["n_pad"]
+    assert p["sub"] == 8
+    if pair:
+        assert p["a_base"] == acc and p["tmem_cols"] == 512
+        assert p["a_base"] + p["stages"] * 64 <= 512
     else:
-        assert 2 <= p["stages"] <= 8 and p["lo_slots"] == 0 and p["x_slots"] == 0
-        rings = p["stages"] * (2 * 128 * 128 + xb)
-    assert 1024 + 512 + rings <= 232448
+        assert p["a_base"] == 0 and acc <= p["tmem_cols"]
+    # shared memory: stages of one y tile (128 rows) and, on pairs, this CTA's
+    # half of [x_hi; x_lo]; on single CTAs y_lo and both x parts
+    xb = p["n_pad"] * 128
+    stage = 128 * 128 + xb if pair else 2 * 128 * 128 + 2 * xb
+    assert 2 <= p["stages"] <= 8 and 1024 + 512 + p["stages"] * stage <= 232448
     # workspace: ordered, 256-byte aligned regions of the stated sizes
     offs = [p[k] for k in ("xnorm_off", "ynorm_off", "partial_off", "xh_off", "xl_off", "total")]
     assert all(o % 256 == 0 for o in offs) and offs == sorted(offs)
     assert p["ynorm_off"] - p["xnorm_off"] >= 4 * B * p["n_chunks"]
     assert p["n_chunks"] == -(-K // 2048)
     assert p["partial_off"] - p["ynorm_off"] >= 4 * S * Q
-    planes = 2 if n_side else 1                  # x_hi and x_lo rows on the N side
-    assert p["xh_off"] - p["partial_off"] >= 4 * planes * S * B * Q
+    assert p["xh_off"] - p["partial_off"] >= 4 * S * B * Q
     assert p["xl_off"] - p["xh_off"] >= 4 * B * K and p["total"] - p["xl_off"] >= 4 * B * K
     n = ctypes.c_size_t()
     st = bg.lib().bergson_score_grads_workspace(B, K, Q, ctypes.byref(n))
