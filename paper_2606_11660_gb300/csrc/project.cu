@@ -218,26 +218,51 @@ __device__ __forceinline__ void load_query_block(const ProjParams& p, int m, int
     sA[e] = p.queries[static_cast<int64_t>(q0 + e / blk) * p.ld_q + off + e % blk];
 }
 
-// Token mode on the tensor cores: module m's blocks of queries [q0, q0 + n)
-// as the B operand of U = a~ Q^T: row r = q * k_out + i holds Q~_q[i, 0:k_in],
+// Token mode on the tensor cores: a block of module m's query rows [q0, q0 +
+// n) held in registers between its global loads and its split into the B
+// operand of U = a~ Q^T, so that the next block's loads are in flight while
+// the current one is used.  B row r = q * k_out + i holds Q~_q[i, 0:k_in],
 // K-major in 128-byte rows (32 fp32 per K atom, atoms kN rows apart) with the
-// 128-byte swizzle, split into tf32 hi and lo parts (128 threads).
-template <int KI, int KO, int kN>
-__device__ __forceinline__ void load_query_block_tc(const ProjParams& p, int m, int q0, int n,
-                                                    uint8_t* bhi, uint8_t* blo, int et) {
-  constexpr int blk = KO * KI;
-  const int64_t off = p.mods[m].col_offset;
-  for (int e = et; e < n * blk; e += 128) {
-    const int q = e / blk, i = (e / KI) % KO, j = e % KI;
-    const float v = p.queries[static_cast<int64_t>(q0 + q) * p.ld_q + off + i * KI + j];
-    const int r = q * KO + i;
-    const int jj = j & 31;
-    const int byte = (j >> 5) * kN * 128 + r * 128 + (((jj >> 2) ^ (r & 7)) << 4) + (jj & 3) * 4;
-    const float h = tf32_rn(v);
-    *reinterpret_cast<float*>(bhi + byte) = h;
-    *reinterpret_cast<float*>(blo + byte) = tf32_rn(v - h);
+// 128-byte swizzle, split into tf32 hi and lo parts; chunk e of a thread is
+// 16 bytes, columns 4c .. 4c + 3 of row (q, i).
+template <int KI, int KO, int kN, int kNQ>
+struct QueryBlockRegs {
+  static_assert(KI % 4 == 0, "query rows in 16-byte chunks");
+  static constexpr int kPerQ = KO * KI / 4;                  // chunks per query
+  static constexpr int kVec = (kNQ * kPerQ + 127) / 128;     // chunks per thread
+  float4 v[kVec];
+  // vec: the rows are 16-byte aligned (else four 4-byte loads per chunk)
+  __device__ __forceinline__ void load(const ProjParams& p, int m, int q0, int n, int et, bool vec) {
+    const int64_t off = p.mods[m].col_offset;
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      const int e = et + 128 * u;
+      if (e < n * kPerQ) {
+        const int q = e / kPerQ, i = (e % kPerQ) / (KI / 4), c = e % (KI / 4);
+        const float* src = p.queries + static_cast<int64_t>(q0 + q) * p.ld_q + off + i * KI + 4 * c;
+        v[u] = vec ? *reinterpret_cast<const float4*>(src)
+                   : make_float4(src[0], src[1], src[2], src[3]);
+      }
+    }
   }
-}
+  __device__ __forceinline__ void store(uint8_t* bhi, uint8_t* blo, int n, int et) const {
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      const int e = et + 128 * u;
+      if (e < n * kPerQ) {
+        const int q = e / kPerQ, i = (e % kPerQ) / (KI / 4), c = e % (KI / 4);
+        const int r = q * KO + i;
+        const int j = 4 * c, jj = j & 31;
+        const int byte = (j >> 5) * kN * 128 + r * 128 + (((jj >> 2) ^ (r & 7)) << 4);
+        const float4 x = v[u];
+        const float4 h = make_float4(tf32_rn(x.x), tf32_rn(x.y), tf32_rn(x.z), tf32_rn(x.w));
+        *reinterpret_cast<float4*>(bhi + byte) = h;
+        *reinterpret_cast<float4*>(blo + byte) = make_float4(
+            tf32_rn(x.x - h.x), tf32_rn(x.y - h.y), tf32_rn(x.z - h.z), tf32_rn(x.w - h.w));
+      }
+    }
+  }
+};
 
 // 32 lanes x N columns of this thread's TMEM row from v (N = 16, 32 or 64).
 template <int N>
@@ -454,6 +479,9 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
     uint32_t sph = 0;
     float acc[OPT];
     float bias_acc = 0.0f;   // column (et % KO) of g~ summed over rows (et / KO)*KO .. +KO
+    // token mode on the tensor cores: the next query block, in registers
+    QueryBlockRegs<KI, KO, (C::kTC ? C::kTcN : 16), (C::kTC ? C::kTcNQ : 1)> qregs;
+    bool qvec = false;
     for (;;) {
       if (et == 0) {
         if (!mbar_wait(smem_u32(&sfull[ss]), sph, tmo, s_abort))
@@ -526,9 +554,16 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         // block of QB queries, else block by block for every tile group
         // below.  All threads left the previous item behind the two barriers
         // above.
+        if constexpr (C::kTC) {
+          // block 0 of this module into registers (stored below per tile, or
+          // once here when it is the only block)
+          qvec = (reinterpret_cast<uintptr_t>(p.queries) & 15) == 0 && (p.ld_q & 3) == 0 &&
+                 (p.mods[ic.m].col_offset & 3) == 0;
+          qregs.load(p, ic.m, 0, min(QB, p.n_queries), et, qvec);
+        }
         if (n_qblocks == 1) {
           if constexpr (C::kTC) {
-            load_query_block_tc<KI, KO, C::kTcN>(p, ic.m, 0, p.n_queries, sBhi, sBlo, et);
+            qregs.store(sBhi, sBlo, p.n_queries, et);
             fence_proxy_async_smem();        // the tensor cores read it through the async proxy
           } else {
             load_query_block<KI, KO>(p, ic.m, 0, p.n_queries, sA, et);
@@ -586,8 +621,12 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             const int nqb = min(QB, p.n_queries - q0);
             if (n_qblocks > 1) {
               named_bar_sync(1, 128);          // the previous block's product has completed
-              load_query_block_tc<KI, KO, C::kTcN>(p, ic.m, q0, nqb, sBhi, sBlo, et);
+              qregs.store(sBhi, sBlo, nqb, et);
               fence_proxy_async_smem();
+              // the next block (block 0 of the next tile after the last one)
+              // loads while this one is multiplied and reduced
+              const int qn = qb + 1 < n_qblocks ? q0 + QB : 0;
+              qregs.load(p, ic.m, qn, min(QB, p.n_queries - qn), et, qvec);
             }
             // Every lane's A row, the query block and the previous block's U
             // reads are complete before one thread issues the products:
@@ -620,19 +659,27 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             uph ^= 1;
             if (*s_epi_stop) { aborted = true; break; }
             tc_fence_after();
-            // s_q = sum_i g~_i U[token, q k_out + i]
-            for (int q = 0; q < nqb; ++q) {
-              float sq = 0.0f;
+            // s_q = sum_i g~_i U[token, q k_out + i], kLd columns of U (kLd /
+            // k_out queries) per TMEM load; columns past the block's queries
+            // are allocated and read, not used
+            constexpr int kLd = C::kTcN % 64 == 0 ? 64 : (C::kTcN % 32 == 0 ? 32 : 16);
+            constexpr int kQPerLd = kLd / KO;
+            for (int qg = 0; qg < nqb; qg += kQPerLd) {
+              float u[kLd];
+              const uint32_t ua = tmem + lane_base + C::kTmU + qg * KO;
+              if constexpr (kLd == 64) tmem_ld64(ua, u);
+              else if constexpr (kLd == 32) tmem_ld32(ua, u);
+              else tmem_ld16(ua, u);
 #pragma unroll
-              for (int c = 0; c < KO; c += 16) {
-                float u[16];
-                tmem_ld16(tmem + lane_base + C::kTmU + q * KO + c, u);
+              for (int qq = 0; qq < kQPerLd; ++qq) {
+                const int q = qg + qq;
+                float sq = 0.0f;
 #pragma unroll
-                for (int i = 0; i < 16; ++i) sq = fmaf(vg[c + i], u[i], sq);
+                for (int i = 0; i < KO; ++i) sq = fmaf(vg[i], u[qq * KO + i], sq);
+                if (q < nqb && in_range)
+                  p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q0 + q) * p.B +
+                                    ic.b) * p.T + t] = valid ? sq : 0.0f;
               }
-              if (in_range)
-                p.token_partials[((static_cast<int64_t>(ic.m) * p.n_queries + q0 + q) * p.B +
-                                  ic.b) * p.T + t] = valid ? sq : 0.0f;
             }
             tc_fence_before();
           }
