@@ -34,11 +34,12 @@ constexpr int kStoreBoxBytes = kScoreBN * 128;      // 256 rows x 64 fp16
 constexpr int kQBoxBytes = kScoreQT * 128;          // 128 rows x 64 fp16
 constexpr unsigned long long kSentinelKey = 0x007FFFFF00000000ull;   // (-inf, row 0xFFFFFFFF)
 // L2 policy of store-chunk loads: 0 = evict_normal, 1 = evict_first.  The
-// pair kernel with more than one query group keeps the normal policy: every
-// store tile is read once per group, by CTAs that stream the same tiles in
-// the same order, and the later reads hit L2 more often when the first one
-// does not mark the lines for early eviction (DRAM reads 1.33x the store
-// instead of 1.6x at 1024 queries, same time: that pass is tensor-bound).
+// pair kernel with more than one pair of query groups (n_qg counts the
+// CTAs' groups, two per pair) keeps the normal policy: every store half is
+// read once per pair, by CTAs that stream the same tiles in the same order,
+// and the later reads hit L2 more often when the first one does not mark the
+// lines for early eviction (DRAM reads 1.21x the store instead of 1.6x at
+// 1024 queries, same time: that pass is tensor-bound).
 constexpr int kStoreEvictFirst = 1;
 
 // Candidates a lane may park in shared memory per tile before inserting them
@@ -460,7 +461,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<QT>::kThread
       prefetch_tmap(&tm_store);
       prefetch_tmap(&tm_q);
       const uint64_t pol_store =
-          kStoreEvictFirst && p.n_qg == 1 ? policy_evict_first() : policy_evict_normal();
+          kStoreEvictFirst && p.n_qg == 2 ? policy_evict_first() : policy_evict_normal();
       const uint64_t pol_q = policy_evict_last();
       int stage = 0;
       uint32_t ph = 0;
