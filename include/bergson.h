@@ -564,8 +564,8 @@ BERGSON_API int bergson_debug_score_plan(int64_t N, int64_t K, int64_t Q, int64_
  * (1/0: batches of up to 64 rows), accumulator buffers, rows of y per tile
  * (256 on pairs, else 128), TMEM columns allocated, the workspace offsets of
  * the x norms, y norms, partial products, x_hi, x_lo and the total, then the
- * TMEM column of the pairs' y operand ring (a 64-column slot per stage; 0
- * otherwise) and the most 32-column steps per accumulation chain.
+ * TMEM column of the pairs' y operand ring and its 64-column slots (0
+ * otherwise).
  * Host only: enqueues nothing.  Errors: EINVAL (B in [1, 2^20], Q in
  * [1, 2^24], K in [4, 2^26] and a multiple of 4).
  */

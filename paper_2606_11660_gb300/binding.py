@@ -509,7 +509,7 @@ def bergson_debug_score_plan(N: int, K: int, Q: int, topk: int, ctas: int) -> li
 
 XGEMM_PLAN_FIELDS = ("n_pad", "n_ntiles", "n_mtiles", "steps", "S", "stages", "n_chunks",
                      "pair", "n_buf", "y_rows", "tmem_cols", "xnorm_off", "ynorm_off",
-                     "partial_off", "xh_off", "xl_off", "total", "a_base", "sub")
+                     "partial_off", "xh_off", "xl_off", "total", "a_base", "a_slots")
 
 
 def bergson_debug_xgemm_plan(B: int, Q: int, K: int) -> dict:

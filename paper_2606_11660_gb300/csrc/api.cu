@@ -679,7 +679,7 @@ int bergson_debug_xgemm_plan(int64_t B, int64_t Q, int64_t K, int64_t* out, int 
                          static_cast<int64_t>(pl.xnorm_off), static_cast<int64_t>(pl.ynorm_off),
                          static_cast<int64_t>(pl.partial_off), static_cast<int64_t>(pl.xh_off),
                          static_cast<int64_t>(pl.xl_off), static_cast<int64_t>(pl.total),
-                         pl.a_base, pl.sub};
+                         pl.a_base, pl.a_slots};
   for (int i = 0; i < 19; ++i) out[i] = v[i];
   return BERGSON_OK;
 }

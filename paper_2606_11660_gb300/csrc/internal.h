@@ -253,7 +253,9 @@ struct XGemmPlan {
   bool pair = false;       // CTA pairs with y in TMEM (B <= 64)
   int n_buf = 2;           // accumulator sets in TMEM
   int y_rows = 128;        // rows of y per work item (256 on pairs: 128 per CTA)
-  int a_base = 0;          // pairs: TMEM column of the y_hi / y_lo ring (a slot per stage)
+  int a_base = 0;          // pairs: TMEM column of the y operand ring (a slot per stage)
+  int a_slots = 0;         // pairs: slots of that ring (64 columns each; as many as stages)
+  bool two_issuers = false;  // pairs: y_hi and y_lo products issued by two threads (n_pad <= 32)
   int sub = 8;             // 32-column steps per accumulation chain (at most)
   int tmem_cols = 32;      // TMEM columns allocated per CTA
   size_t xnorm_off = 0, ynorm_off = 0, partial_off = 0, xh_off = 0, xl_off = 0, total = 0;

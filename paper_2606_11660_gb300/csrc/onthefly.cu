@@ -48,6 +48,7 @@ constexpr int kXM = 128;                   // rows of y per tile, M side (MMA M)
 constexpr int kXK = 32;                    // fp32 columns per stage: one 128-byte row
 constexpr int kYBytes = kXM * 128;         // one y tile, M side
 constexpr int kXThreads = 320;             // producer, MMA, 4 converter, 4 epilogue warps
+constexpr int kPThreads = 352;             // pairs: the same and a second MMA issuer warp
 constexpr int kXSmemBudget = 232448;       // 227 KB opt-in per CTA
 constexpr int kXBarBytes = 512;
 constexpr int kXMaxStages = 8;
@@ -508,23 +509,26 @@ __host__ __device__ constexpr int chain_start(int L, int n_ch, int k) { return k
 // epilogue warp of both CTAs releases a set on the even CTA's `tempty`.  A
 // stage's TMEM slot is written again only after its `full` barrier
 // completes anew, i.e. after the `empty` commit of the MMAs that read it.
-template <bool kUnit>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
+template <bool kUnit, bool kTwo>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
     xgemm_pair_kernel(const __grid_constant__ CUtensorMap tm_y, const __grid_constant__ CUtensorMap tm_xh,
-                      const __grid_constant__ CUtensorMap tm_xl, const XGemmParams p) {
+                      const __grid_constant__ CUtensorMap tm_xl,
+                      const __grid_constant__ CUtensorMap tm_xh2, const XGemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
   const int xbytes = p.n_pad * 128;
-  const int stage_bytes = kYBytes + xbytes;      // this CTA's y half, then its half of B
+  // this CTA's y half, its half of B = [x_hi; x_lo], and with two issuers its
+  // half of B' = x_hi for the y_lo products (N = n_pad: rows r n_pad / 2 ..)
+  const int stage_bytes = kYBytes + xbytes + (kTwo ? xbytes / 2 : 0);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + p.stages * stage_bytes);
   uint64_t* empty = full + p.stages;
   uint64_t* conv = empty + p.stages;
   uint64_t* tfull = conv + p.stages;
   uint64_t* tempty = tfull + 2;
-  uint64_t* drain = tempty + 2;
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* drain = tempty + 2;                  // one per issuer
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 2);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const uint32_t rank = cluster_ctarank();       // 0: issues the MMAs
@@ -535,14 +539,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), 1);
+      mbar_init(smem_u32(&empty[s]), kTwo ? 2 : 1);   // a commit from each MMA issuer
       mbar_init(smem_u32(&conv[s]), 8);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(smem_u32(&tfull[i]), 1);
+      mbar_init(smem_u32(&tfull[i]), kTwo ? 2 : 1);
       mbar_init(smem_u32(&tempty[i]), 8);
     }
-    mbar_init(smem_u32(drain), 1);
+    mbar_init(smem_u32(&drain[0]), 1);
+    mbar_init(smem_u32(&drain[1]), 1);
     *s_abort = 0;
     fence_barrier_init();
   }
@@ -555,7 +560,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *s_tmem;
   const uint64_t tmo = p.timeout_ns;
-  const int set_cols = 2 * p.n_pad;              // one accumulator set
+  // one accumulator set: y_hi [x_hi; x_lo]^T (2 n_pad columns), then with two
+  // issuers y_lo x_hi^T (n_pad columns)
+  const int set_cols = (kTwo ? 3 : 2) * p.n_pad;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -565,6 +572,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
       prefetch_tmap(&tm_y);
       const CUtensorMap* tm_x = rank == 0 ? &tm_xh : &tm_xl;
       prefetch_tmap(tm_x);
+      if constexpr (kTwo) prefetch_tmap(&tm_xh2);
       const uint64_t pol_y = policy_evict_first();    // streamed once
       const uint64_t pol_x = policy_evict_last();     // re-read by every tile
       int stage = 0;
@@ -576,6 +584,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
       auto load_x = [&](int sg, int st, int nt) {
         tma_load_2d_hint(sbase + sg * stage_bytes + kYBytes, tm_x, smem_u32(&full[sg]), st * kXK,
                          nt * p.n_pad, pol_x);
+        if constexpr (kTwo)
+          tma_load_2d_hint(sbase + sg * stage_bytes + kYBytes + xbytes, &tm_xh2,
+                           smem_u32(&full[sg]), st * kXK,
+                           nt * p.n_pad + static_cast<int>(rank) * (p.n_pad / 2), pol_x);
       };
       auto release = [&]() {
         griddep_wait();
@@ -613,10 +625,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
       }
     }
     __syncwarp();
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer (even CTA)
-    if (rank == 0 && lane == 0) {
-      const uint32_t idesc = make_idesc_tf32(2 * kXM, 2 * p.n_pad);   // y [x_hi; x_lo]^T, M = 256
+  } else if (warp == 1 || warp == 10) {
+    // ------------------------------------------------------------ MMA issuer(s) (even CTA)
+    // kTwo: warp 1 issues the y_hi products into the set's first 2 n_pad
+    // columns and warp 10 the y_lo products into the next 2 n_pad, each in a
+    // fixed order (two issuing threads keep the tensor pipe fed: one stalls
+    // about 115 cycles per MMA instruction at these shapes).
+    if (rank == 0 && lane == 0 && (warp == 1 || kTwo)) {
+      const int who = warp == 10 ? 1 : 0;           // 1: the y_lo issuer
+      // y [x_hi; x_lo]^T, or for the y_lo issuer y_lo x_hi^T; M = 256
+      const uint32_t idesc = make_idesc_tf32(2 * kXM, (who ? 1 : 2) * p.n_pad);
       int stage = 0;
       uint32_t ph = 0;
       int ab = 0;
@@ -630,16 +648,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
           const int c0 = it.s0 + chain_start(L, n_ch, k), c1 = it.s0 + chain_start(L, n_ch, k + 1);
           if (!mbar_wait(smem_u32(&tempty[ab]), aph ^ 1, tmo, s_abort)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t d = tmem + ab * set_cols;
+          const uint32_t d = tmem + ab * set_cols + who * 2 * p.n_pad;   // y_lo part after y_hi
           for (int st = c0; st < c1; ++st) {
             if (!mbar_wait(smem_u32(&conv[stage]), ph, tmo, s_abort)) { ok = false; break; }
             tc_fence_after();
             const uint32_t ta = tmem + p.a_base + stage * 2 * kXK;    // y_hi, then y_lo
-            const uint64_t dx = sw128_desc(sbase + stage * stage_bytes + kYBytes);
+            const uint64_t dx =
+                sw128_desc(sbase + stage * stage_bytes + kYBytes + who * xbytes);   // B or B'
 #pragma unroll
             for (int kk = 0; kk < kXK / 8; ++kk) {   // 8 tf32 = 32 bytes: +2 in the address field
-              umma_tf32_pair_ta(d, ta + 8 * kk, dx + 2 * kk, idesc, st != c0 || kk != 0);
-              umma_tf32_pair_ta(d, ta + kXK + 8 * kk, dx + 2 * kk, idesc, 1u);
+              const uint32_t acc = st != c0 || kk != 0;
+              if constexpr (kTwo) {
+                umma_tf32_pair_ta(d, ta + who * kXK + 8 * kk, dx + 2 * kk, idesc, acc);
+              } else {
+                umma_tf32_pair_ta(d, ta + 8 * kk, dx + 2 * kk, idesc, acc);
+                umma_tf32_pair_ta(d, ta + kXK + 8 * kk, dx + 2 * kk, idesc, 1u);
+              }
             }
             umma_commit_pair(smem_u32(&empty[stage]), 0x3);
             if (++stage == p.stages) { stage = 0; ph ^= 1; }
@@ -650,8 +674,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
         }
       }
       if (!ok) raise_device_error(p.status, s_abort, kStatusTimeout);
-      umma_commit_pair(smem_u32(drain), 0x1);
-      mbar_wait(smem_u32(drain), 0, kXDrainTimeoutNs, nullptr);
+      umma_commit_pair(smem_u32(&drain[who]), 0x1);
+      mbar_wait(smem_u32(&drain[who]), 0, kXDrainTimeoutNs, nullptr);
     }
     __syncwarp();
   } else if (warp < 6) {
@@ -728,12 +752,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kXThreads, 1)
         for (int cb = 0; cb < kMaxPadN / 16; ++cb) {
           const int c = 16 * cb;
           if (c < p.n_pad) {
-            // <x_b, y_q> ~= (y_hi + y_lo) x_hi + (y_hi + y_lo) x_lo
+            // <x_b, y_q> ~= (y_hi + y_lo) x_hi + (y_hi + y_lo) x_lo; with two
+            // issuers y_hi x_hi + y_hi x_lo + y_lo x_hi, the last in the set's
+            // third part
             float v[16], w[16];
             tmem_ld16(tbase + c, v);
             tmem_ld16(tbase + p.n_pad + c, w);
+            if constexpr (kTwo) {
+              float u[16];
+              tmem_ld16(tbase + 2 * p.n_pad + c, u);       // y_lo x_hi
 #pragma unroll
-            for (int jj = 0; jj < 16; ++jj) acc[c + jj] += v[jj] + w[jj];
+              for (int jj = 0; jj < 16; ++jj) acc[c + jj] += (v[jj] + w[jj]) + u[jj];
+            } else {
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj) acc[c + jj] += v[jj] + w[jj];
+            }
           }
         }
         tc_fence_before();
@@ -812,6 +845,16 @@ cudaError_t launch_product(Kernel kernel, PerDeviceOnce& attr, int threads, int 
   return launch_dependent(kernel, dim3(grid), dim3(threads), smem, s, tm_y, tm_xh, tm_xl, p);
 }
 
+template <typename Kernel>
+cudaError_t launch_pair(Kernel kernel, PerDeviceOnce& attr, int grid, size_t smem, cudaStream_t s,
+                        const CUtensorMap& tm_y, const CUtensorMap& tm_xh,
+                        const CUtensorMap& tm_xl, const CUtensorMap& tm_xh2, const XGemmParams& p) {
+  const cudaError_t e = smem_attr_once(attr, kernel, kXSmemBudget);
+  if (e != cudaSuccess) return e;
+  return launch_dependent(kernel, dim3(grid), dim3(kPThreads), smem, s, tm_y, tm_xh, tm_xl, tm_xh2,
+                          p);
+}
+
 }  // namespace
 
 cudaError_t launch_row_scales(const float* x, int n, int K, int64_t ld, int unit, float* scale,
@@ -837,12 +880,15 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
   const int ring_budget = kXSmemBudget - 1024 - kXBarBytes;
   int stage_bytes;
   if (pl.pair) {
-    // two accumulator sets of 2 n_pad columns, then the y_hi / y_lo ring (64
-    // columns a stage)
+    // two accumulator sets of 2 n_pad columns (4 n_pad with two MMA issuers,
+    // batch tiles up to 32 rows), then the y_hi / y_lo ring (64 columns a
+    // stage)
     pl.tmem_cols = 512;
-    pl.a_base = 2 * pl.n_buf * pl.n_pad;
-    stage_bytes = kYBytes + pl.n_pad * 128;
+    pl.two_issuers = pl.n_pad <= 32;
+    pl.a_base = pl.n_buf * (pl.two_issuers ? 3 : 2) * pl.n_pad;
+    stage_bytes = kYBytes + pl.n_pad * 128 + (pl.two_issuers ? pl.n_pad * 64 : 0);
     pl.stages = std::min({kXMaxStages, (512 - pl.a_base) / (2 * kXK), ring_budget / stage_bytes});
+    pl.a_slots = pl.stages;
   } else {
     pl.tmem_cols = 32;
     while (pl.tmem_cols < pl.n_buf * 2 * pl.n_pad) pl.tmem_cols <<= 1;
@@ -886,13 +932,16 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
 cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   if (a.B == 0 || a.Q == 0) return cudaSuccess;
   const XGemmPlan pl = xgemm_plan(a.B, a.Q, a.K);
-  CUtensorMap tm_y, tm_xh, tm_xl;
+  CUtensorMap tm_y, tm_xh, tm_xl, tm_xh2;
   if (encode_tmap_2d(&tm_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.y, a.K, a.Q, a.ldy * 4, kXK, kXM) !=
           CUDA_SUCCESS ||
       encode_tmap_2d(&tm_xh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.ws + pl.xh_off, a.K, a.B,
                      static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad) != CUDA_SUCCESS ||
       encode_tmap_2d(&tm_xl, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.ws + pl.xl_off, a.K, a.B,
-                     static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad) != CUDA_SUCCESS)
+                     static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad) != CUDA_SUCCESS ||
+      (pl.two_issuers &&
+       encode_tmap_2d(&tm_xh2, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, a.ws + pl.xh_off, a.K, a.B,
+                      static_cast<int64_t>(a.K) * 4, kXK, pl.n_pad / 2) != CUDA_SUCCESS))
     return cudaErrorInvalidValue;
   float* xnorm = reinterpret_cast<float*>(a.ws + pl.xnorm_off);
   float* xh = reinterpret_cast<float*>(a.ws + pl.xh_off);
@@ -920,15 +969,24 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   p.ynorm = reinterpret_cast<float*>(a.ws + pl.ynorm_off);
   p.status = a.status;
   p.timeout_ns = a.timeout_ns;
-  const size_t stage_bytes = pl.pair ? kYBytes + pl.n_pad * 128 : 2 * kYBytes + 2 * pl.n_pad * 128;
+  const size_t stage_bytes =
+      pl.pair ? kYBytes + pl.n_pad * 128 + (pl.two_issuers ? pl.n_pad * 64 : 0)
+              : 2 * kYBytes + 2 * pl.n_pad * 128;
   const size_t smem = 1024 + pl.stages * stage_bytes + kXBarBytes;
-  static PerDeviceOnce attr_pair[2], attr_m;
+  static PerDeviceOnce attr_pair[4], attr_m;
   if (pl.pair) {
     const int grid = 2 * std::max(1, std::min(std::max(sms, 2) / 2, p.n_items));
-    e = a.unit ? launch_product(xgemm_pair_kernel<true>, attr_pair[0], kXThreads, grid, smem, s,
-                                tm_y, tm_xh, tm_xl, p)
-               : launch_product(xgemm_pair_kernel<false>, attr_pair[1], kXThreads, grid, smem, s,
-                                tm_y, tm_xh, tm_xl, p);
+    if (!pl.two_issuers) tm_xh2 = tm_xh;        // not read
+    if (pl.two_issuers)
+      e = a.unit ? launch_pair(xgemm_pair_kernel<true, true>, attr_pair[0], grid, smem, s, tm_y,
+                               tm_xh, tm_xl, tm_xh2, p)
+                 : launch_pair(xgemm_pair_kernel<false, true>, attr_pair[1], grid, smem, s, tm_y,
+                               tm_xh, tm_xl, tm_xh2, p);
+    else
+      e = a.unit ? launch_pair(xgemm_pair_kernel<true, false>, attr_pair[2], grid, smem, s, tm_y,
+                               tm_xh, tm_xl, tm_xh2, p)
+                 : launch_pair(xgemm_pair_kernel<false, false>, attr_pair[3], grid, smem, s, tm_y,
+                               tm_xh, tm_xl, tm_xh2, p);
   } else {
     const int grid = std::max(1, std::min(sms > 0 ? sms : 1, p.n_items));
     e = launch_product(xgemm_kernel, attr_m, kXThreads, grid, smem, s, tm_y, tm_xh, tm_xl, p);

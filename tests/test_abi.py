@@ -405,21 +405,24 @@ def check_xgemm_plan(B, Q, K):
     assert 1 <= S <= min(steps, 64)
     bounds = [z * steps // S for z in range(S + 1)]
     assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
-    # TMEM: two accumulator sets of 2 n_pad columns, and on pairs the y_hi /
-    # y_lo ring after them (64 columns a stage), within 512 columns
+    # TMEM: two accumulator sets of 2 n_pad columns (4 n_pad on pairs with two
+    # MMA issuers, batch tiles up to 32 rows), and on pairs the y_hi / y_lo
+    # ring after them (64 columns a stage), within 512 columns
     assert p["n_buf"] == 2
     assert p["tmem_cols"] <= 512 and p["tmem_cols"] & (p["tmem_cols"] - 1) == 0
-    acc = 2 * 2 * p["n_pad"]
-    assert p["sub"] == 8
+    acc = 2 * (3 if pair and p["n_pad"] <= 32 else 2) * p["n_pad"]
     if pair:
+        # a TMEM slot (y_hi, y_lo: 64 columns) per stage
         assert p["a_base"] == acc and p["tmem_cols"] == 512
-        assert p["a_base"] + p["stages"] * 64 <= 512
+        assert p["a_slots"] == p["stages"] and p["a_base"] + p["a_slots"] * 64 <= 512
     else:
-        assert p["a_base"] == 0 and acc <= p["tmem_cols"]
+        assert p["a_base"] == 0 and p["a_slots"] == 0 and acc <= p["tmem_cols"]
     # shared memory: stages of one y tile (128 rows) and, on pairs, this CTA's
-    # half of [x_hi; x_lo]; on single CTAs y_lo and both x parts
+    # half of [x_hi; x_lo] (and, with two issuers, its half of x_hi); on single
+    # CTAs y_lo and both x parts
     xb = p["n_pad"] * 128
-    stage = 128 * 128 + xb if pair else 2 * 128 * 128 + 2 * xb
+    stage = (128 * 128 + xb + (xb // 2 if p["n_pad"] <= 32 else 0) if pair
+             else 2 * 128 * 128 + 2 * xb)
     assert 2 <= p["stages"] <= 8 and 1024 + 512 + p["stages"] * stage <= 232448
     # workspace: ordered, 256-byte aligned regions of the stated sizes
     offs = [p[k] for k in ("xnorm_off", "ynorm_off", "partial_off", "xh_off", "xl_off", "total")]
