@@ -247,7 +247,8 @@ struct XGemmPlan {
   int n_ntiles = 1;        // ceil(B / n_pad)
   int n_mtiles = 1;        // ceil(Q / y_rows)
   int steps = 1;           // ceil(K / 32)
-  int S = 1;               // K slices
+  int S = 1;               // K slices (pairs: the most segments of any y tile)
+  int n_clusters = 0;      // pairs: clusters the (y tile, step) space is split over
   int stages = 2;          // shared-memory pipeline depth
   int n_chunks = 1;        // column chunks of x for the row split (norm partials per row)
   bool pair = false;       // CTA pairs with y in TMEM (B <= 64)

@@ -172,6 +172,7 @@ struct XGemmParams {
   int tmem_cols;
   int sub;            // 32-column steps per accumulation chain
   int a_base;         // pairs: TMEM column of the y_hi / y_lo ring (a slot per stage)
+  int n_clusters;     // pairs: clusters sharing the (y tile, step) space evenly
   int unit;
   float* partial;     // [S, B, Q]
   float* ynorm;       // [S, Q] squared norms of y rows over each slice (unit only)
@@ -193,6 +194,49 @@ __device__ __forceinline__ XItem decode_xitem(const XGemmParams& p, int item) {
   it.s1 = static_cast<int>(static_cast<int64_t>(it.z + 1) * p.steps / p.S);
   return it;
 }
+
+// Pairs split the n_mtiles x steps (y tile, 32-column step) space evenly
+// over the clusters in order: cluster c takes positions [c W / n, (c + 1) W
+// / n), W = n_mtiles steps, cut at tile boundaries into segments.  The
+// segments of a tile are its K slices; a segment's partial plane is its
+// cluster's rank among the clusters that meet the tile.  The cluster that
+// holds position g: ceil((g + 1) n / W) - 1.
+__host__ __device__ __forceinline__ int seg_cluster_of(int64_t g, int64_t W, int n) {
+  return static_cast<int>(((g + 1) * n + W - 1) / W) - 1;
+}
+__host__ __device__ __forceinline__ int seg_planes(int mt, int steps, int64_t W, int n) {
+  const int64_t p0 = static_cast<int64_t>(mt) * steps;
+  return seg_cluster_of(p0 + steps - 1, W, n) - seg_cluster_of(p0, W, n) + 1;
+}
+
+struct SegIter {
+  int64_t g, g1, W;
+  int steps, n, cid;
+  XItem it;
+  __device__ __forceinline__ SegIter(const XGemmParams& p, int c) {
+    steps = p.steps;
+    n = p.n_clusters;
+    cid = c;
+    W = static_cast<int64_t>(p.n_mtiles) * steps;
+    g = c * W / n;
+    g1 = (c + 1) * W / n;
+    load();
+  }
+  __device__ __forceinline__ bool valid() const { return g < g1; }
+  __device__ __forceinline__ void load() {
+    if (g >= g1) return;
+    it.mt = static_cast<int>(g / steps);
+    it.nt = 0;
+    it.s0 = static_cast<int>(g % steps);
+    const int64_t end = it.s0 + (g1 - g);
+    it.s1 = end < steps ? static_cast<int>(end) : steps;
+    it.z = cid - seg_cluster_of(static_cast<int64_t>(it.mt) * steps, W, n);
+  }
+  __device__ __forceinline__ void next() {
+    g += it.s1 - it.s0;
+    load();
+  }
+};
 
 // Lane 0 waits, the warp takes its answer (keeps the warp's control flow
 // uniform).  Inline: the converter and epilogue warps keep running sums in
@@ -533,7 +577,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
 
   const uint32_t rank = cluster_ctarank();       // 0: issues the MMAs
   const int cid = blockIdx.x >> 1;
-  const int n_clusters = gridDim.x >> 1;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -595,8 +638,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
         for (int d = 0; d < n_def; ++d) load_x(d, def_st[d], def_nt[d]);
         n_def = 0;
       };
-      for (int item = cid; item < p.n_items && ok; item += n_clusters) {
-        const XItem it = decode_xitem(p, item);
+      for (SegIter sg(p, cid); sg.valid() && ok; sg.next()) {
+        const XItem& it = sg.it;
         for (int st = it.s0; st < it.s1; ++st) {
           if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
           const uint32_t fb = smem_u32(&full[stage]);
@@ -640,8 +683,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
       int ab = 0;
       uint32_t aph = 0;
       bool ok = true;
-      for (int item = cid; item < p.n_items && ok; item += n_clusters) {
-        const XItem it = decode_xitem(p, item);
+      for (SegIter sg(p, cid); sg.valid() && ok; sg.next()) {
+        const XItem& it = sg.it;
         const int L = it.s1 - it.s0;
         const int n_ch = chain_count(L, p.sub);
         for (int k = 0; k < n_ch && ok; ++k) {
@@ -689,8 +732,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
     int stage = 0;
     uint32_t ph = 0;
     bool aborted = false;
-    for (int item = cid; item < p.n_items && !aborted; item += n_clusters) {
-      const XItem it = decode_xitem(p, item);
+    for (SegIter sg(p, cid); sg.valid() && !aborted; sg.next()) {
+      const XItem& it = sg.it;
       KahanSum nrm;
       for (int st = it.s0; st < it.s1; ++st) {
         if (!warp_wait(smem_u32(&full[stage]), ph, tmo, s_abort)) {
@@ -732,8 +775,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
     int ab = 0;
     uint32_t aph = 0;
     bool aborted = false;
-    for (int item = cid; item < p.n_items && !aborted; item += n_clusters) {
-      const XItem it = decode_xitem(p, item);
+    for (SegIter sg(p, cid); sg.valid() && !aborted; sg.next()) {
+      const XItem& it = sg.it;
       const int q = it.mt * 2 * kXM + static_cast<int>(rank) * kXM + row;
       const int L = it.s1 - it.s0;
       const int n_ch = chain_count(L, p.sub);
@@ -800,30 +843,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
   }
 }
 
-// s = sum over slices z (in order) of partial[z, b, q].  Cosine (xnorm
-// given): scores[b, q] = s / sqrt(nx_b) / sqrt(ny_q), nx_b the sum over the
-// row's chunks (in order) of xnorm[b, c], ny_q the sum over z of ynorm[z, q]
-// (0 when either row is zero).  Otherwise scores[b, q] = alpha' s + beta scores[b, q] +
+// s = sum over slices z (in order) of partial[z, b, q] (on pairs the planes
+// of q's y tile, its segments in K order).  Cosine (xnorm given): scores[b, q]
+// = s / sqrt(nx_b) / sqrt(ny_q), nx_b the sum over the row's chunks (in
+// order) of xnorm[b, c], ny_q the sum over the same planes of ynorm[z, q] (0
+// when either row is zero).  Otherwise scores[b, q] = alpha' s + beta scores[b, q] +
 // gamma [b == q], alpha' = alpha * (*alpha_s) when alpha_s is given.
 __global__ void finish_kernel(const float* __restrict__ partial, int S, int B, int Q,
                               const float* __restrict__ xnorm, int n_chunks,
-                              const float* __restrict__ ynorm,
-                              float alpha, const float* __restrict__ alpha_s, float beta,
-                              float gamma, float* scores, int64_t ld) {
+                              const float* __restrict__ ynorm, int seg_clusters, int steps,
+                              int y_rows, float alpha, const float* __restrict__ alpha_s,
+                              float beta, float gamma, float* scores, int64_t ld) {
   griddep_wait();                 // partials, norms and alpha_s come from earlier grids
   const int64_t n = static_cast<int64_t>(B) * Q;
   const float al = alpha_s != nullptr ? alpha * *alpha_s : alpha;
   const int q = blockIdx.x * blockDim.x + threadIdx.x;     // grid: (Q / 256, rows of b)
   if (q >= Q) return;
+  // planes of this row's y tile: all S, or on pairs the tile's segments
+  const int n_mtiles = (Q + y_rows - 1) / y_rows;
+  const int planes = seg_clusters > 0 ? seg_planes(q / y_rows, steps,
+                                                   static_cast<int64_t>(n_mtiles) * steps,
+                                                   seg_clusters)
+                                      : S;
   for (int b = blockIdx.y; b < B; b += gridDim.y) {
     const int64_t i = static_cast<int64_t>(b) * Q + q;
     float s = 0.0f;
-    for (int z = 0; z < S; ++z) s += partial[z * n + i];
+    for (int z = 0; z < planes; ++z) s += partial[z * n + i];
     float* dst = scores + b * ld + q;
     if (xnorm != nullptr) {
       float nx = 0.0f, ny = 0.0f;
       for (int c = 0; c < n_chunks; ++c) nx += xnorm[static_cast<int64_t>(b) * n_chunks + c];
-      for (int z = 0; z < S; ++z) ny += ynorm[static_cast<int64_t>(z) * Q + q];
+      for (int z = 0; z < planes; ++z) ny += ynorm[static_cast<int64_t>(z) * Q + q];
       *dst = nx > 0.0f && ny > 0.0f ? s * (1.0f / sqrtf(nx)) * (1.0f / sqrtf(ny)) : 0.0f;
     } else {
       float v = al * s;
@@ -896,13 +946,22 @@ XGemmPlan xgemm_plan(int64_t B, int64_t Q, int64_t K) {
     stage_bytes = 2 * kYBytes + 2 * pl.n_pad * 128;
     pl.stages = std::min(kXMaxStages, ring_budget / stage_bytes);
   }
-  const int units = pl.pair ? kPlanCTAs / 2 : kPlanCTAs;    // clusters or CTAs
-  // K slices: fewest waves of persistent CTAs (or pairs) for the y stream,
-  // plus the partials each slice adds (written and read back once).
+  const int units = kPlanCTAs;
+  // Pairs: the (y tile, step) space split evenly over the clusters; S = the
+  // most segments (partial planes) any tile gets.
+  if (pl.pair) {
+    const int64_t W = static_cast<int64_t>(pl.n_mtiles) * pl.steps;
+    pl.n_clusters = static_cast<int>(std::min<int64_t>(kPlanCTAs / 2, W));
+    pl.S = 1;
+    for (int mt = 0; mt < pl.n_mtiles; ++mt)
+      pl.S = std::max(pl.S, seg_planes(mt, pl.steps, W, pl.n_clusters));
+  }
+  // Single CTAs: K slices, the fewest waves of persistent CTAs for the y
+  // stream plus the partials each slice adds (written and read back once).
   const int64_t tiles = static_cast<int64_t>(pl.n_mtiles) * pl.n_ntiles;
   double best = -1.0;
-  pl.S = 1;
-  for (int S = 1; S <= std::min(pl.steps, kMaxSlices); ++S) {
+  if (!pl.pair) pl.S = 1;
+  for (int S = 1; S <= std::min(pl.steps, kMaxSlices) && !pl.pair; ++S) {
     if (tiles * S > (1ll << 30)) break;
     const int64_t waves = (tiles * S + units - 1) / units;
     const int64_t per_item = (pl.steps + S - 1) / S;
@@ -964,6 +1023,7 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   p.tmem_cols = pl.tmem_cols;
   p.sub = pl.sub;
   p.a_base = pl.a_base;
+  p.n_clusters = pl.n_clusters;
   p.unit = a.unit;
   p.partial = reinterpret_cast<float*>(a.ws + pl.partial_off);
   p.ynorm = reinterpret_cast<float*>(a.ws + pl.ynorm_off);
@@ -975,7 +1035,7 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   const size_t smem = 1024 + pl.stages * stage_bytes + kXBarBytes;
   static PerDeviceOnce attr_pair[4], attr_m;
   if (pl.pair) {
-    const int grid = 2 * std::max(1, std::min(std::max(sms, 2) / 2, p.n_items));
+    const int grid = 2 * pl.n_clusters;        // the segmentation assumes exactly these
     if (!pl.two_issuers) tm_xh2 = tm_xh;        // not read
     if (pl.two_issuers)
       e = a.unit ? launch_pair(xgemm_pair_kernel<true, true>, attr_pair[0], grid, smem, s, tm_y,
@@ -996,8 +1056,8 @@ cudaError_t xgemm_run(const XGemmArgs& a, int sms, cudaStream_t s) {
   const dim3 fgrid((a.Q + 255) / 256, std::min(a.B, 65535));
   const float* xn = a.unit ? xnorm : nullptr;
   return launch_dependent(finish_kernel, fgrid, dim3(256), 0, s, p.partial, pl.S, a.B, a.Q, xn,
-                          pl.n_chunks, p.ynorm, a.alpha, a.alpha_s, a.beta, a.gamma, a.scores,
-                          a.ld_scores);
+                          pl.n_chunks, p.ynorm, pl.pair ? pl.n_clusters : 0, pl.steps, pl.y_rows,
+                          a.alpha, a.alpha_s, a.beta, a.gamma, a.scores, a.ld_scores);
 }
 
 }  // namespace bergson

@@ -400,11 +400,24 @@ def check_xgemm_plan(B, Q, K):
     rows = p["y_rows"]
     assert p["n_mtiles"] * rows >= Q > (p["n_mtiles"] - 1) * rows
     assert p["steps"] * 32 >= K > (p["steps"] - 1) * 32
-    # every K slice is a nonempty, contiguous range of steps
     S, steps = p["S"], p["steps"]
-    assert 1 <= S <= min(steps, 64)
-    bounds = [z * steps // S for z in range(S + 1)]
-    assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
+    if pair:
+        # the (y tile, step) space split evenly over min(76, W) clusters:
+        # contiguous nonempty ranges that cover it once; S = the most clusters
+        # (partial planes) that meet one tile
+        W = p["n_mtiles"] * steps
+        n = min(76, W)
+        starts = [c * W // n for c in range(n + 1)]
+        assert starts[0] == 0 and starts[-1] == W and all(a < b for a, b in zip(starts, starts[1:]))
+        owner = lambda g: next(c for c in range(n) if starts[c] <= g < starts[c + 1])
+        planes = max(owner(mt * steps + steps - 1) - owner(mt * steps) + 1
+                     for mt in range(min(p["n_mtiles"], 64)))
+        assert planes <= S <= n
+    else:
+        # every K slice is a nonempty, contiguous range of steps
+        assert 1 <= S <= min(steps, 64)
+        bounds = [z * steps // S for z in range(S + 1)]
+        assert bounds[0] == 0 and bounds[-1] == steps and all(a < b for a, b in zip(bounds, bounds[1:]))
     # TMEM: two accumulator sets of 2 n_pad columns (4 n_pad on pairs with two
     # MMA issuers, batch tiles up to 32 rows), and on pairs the y_hi / y_lo
     # ring after them (64 columns a stage), within 512 columns
