@@ -533,26 +533,35 @@ __host__ __device__ constexpr int chain_start(int L, int n_ch, int k) { return k
 // converts it into its own TMEM (y_hi and y_lo, the tf32 A operands); one
 // tcgen05.mma of M = 256 then covers both halves: B = [x_hi; x_lo] (N = 2
 // n_pad), x_hi from the even CTA's shared memory and x_lo from the odd CTA's.
-// Per 8 columns two MMAs, y_hi B^T and y_lo B^T, into one accumulator:
-// columns [0, n_pad) hold (y_hi + y_lo) x_hi, columns [n_pad, 2 n_pad)
-// (y_hi + y_lo) x_lo, added by the epilogue (the fourth product y_lo x_lo
-// comes for free).  A small-N tcgen05 MMA costs about the same issue time
-// whatever its size, and one pair MMA does the work of two single-CTA MMAs,
-// so a pair issues half the instructions per byte of y that a lone CTA
-// would (measured: 8 MMAs per 16 KB stage cap a lone CTA near half the HBM
-// rate; a pair with 8 per 2 x 16 KB streams at ~0.87 of it).
+// A small-N tcgen05 MMA costs about the same issue time whatever its size,
+// and one pair MMA does the work of two single-CTA MMAs, so a pair issues
+// half the instructions per byte of y that a lone CTA would (measured: 8
+// MMAs per 16 KB stage cap a lone CTA near half the HBM rate).
+//
+// kTwo (batch tiles of up to 32 rows): one issuing thread still stalls about
+// 115 cycles per MMA, so two threads issue.  Warp 1: y_hi [x_hi; x_lo]^T
+// into the set's columns [0, 2 n_pad); warp 10: y_lo x_hi^T into [2 n_pad,
+// 3 n_pad), its B = x_hi split over the pair (each CTA loads its n_pad / 2
+// rows at the same offset).  Each issuer keeps a fixed order into its own
+// columns, so the sums stay deterministic.  Without kTwo, one thread issues
+// y_hi B^T and y_lo B^T into one 2 n_pad-column set (the fourth product
+// y_lo x_lo comes for free).  The epilogue adds the parts.
+//
+// Work: the (y tile, step) space split evenly over the clusters in
+// segments (SegIter); each segment is cut into accumulation chains.
 //
 // Synchronisation: each CTA's loads complete on its own `full` barrier; its
 // converter warps then store the tile's y_hi / y_lo into the TMEM slot of
 // that stage and arrive on the even CTA's `conv` barrier (eight arrivals:
 // four warps of each CTA; CTA-scope release, as these signals only order
 // tcgen05 operations: a cluster-scope release costs a memory barrier per
-// arrival, which halved the stream rate).  The even CTA's MMA thread issues the stage's
-// MMAs, and its commits free the stage in both CTAs (`empty`, multicast) and
-// hand finished accumulator sets to both CTAs' epilogues (`tfull`); every
-// epilogue warp of both CTAs releases a set on the even CTA's `tempty`.  A
-// stage's TMEM slot is written again only after its `full` barrier
-// completes anew, i.e. after the `empty` commit of the MMAs that read it.
+// arrival, which halved the stream rate).  The even CTA's MMA threads issue
+// the stage's MMAs, and their commits free the stage in both CTAs (`empty`,
+// multicast, one arrival per issuer) and hand finished accumulator sets to
+// both CTAs' epilogues (`tfull`, likewise); every epilogue warp of both CTAs
+// releases a set on the even CTA's `tempty`.  A stage's TMEM slot is written
+// again only after its `full` barrier completes anew, i.e. after the `empty`
+// commits of the MMAs that read it.
 template <bool kUnit, bool kTwo>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPThreads, 1)
     xgemm_pair_kernel(const __grid_constant__ CUtensorMap tm_y, const __grid_constant__ CUtensorMap tm_xh,
