@@ -299,8 +299,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
   int* s_item = reinterpret_cast<int*>(ubar + 1);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(s_item + 2);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
-  volatile int* s_epi_stop = s_abort + 1;   // epilogue leader's broadcast of "stop"
-  volatile int* s_last = s_epi_stop + 1;     // epilogue leader's broadcast of "last piece"
+  volatile int* s_last = s_abort + 1;        // epilogue leader's broadcast of "last piece"
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -483,13 +482,15 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
     QueryBlockRegs<KI, KO, (C::kTC ? C::kTcN : 16), (C::kTC ? C::kTcNQ : 1)> qregs;
     bool qvec = false;
     for (;;) {
+      // The leader's wait and the abort flag decide "stop" for all 128
+      // threads at once (the barrier's OR), so no thread can see a later value.
+      bool stop = false;
       if (et == 0) {
         if (!mbar_wait(smem_u32(&sfull[ss]), sph, tmo, s_abort))
           raise_device_error(p.status, s_abort, kStatusTimeout);
-        *s_epi_stop = *s_abort;
+        stop = *s_abort != 0;
       }
-      named_bar_sync(1, 128);
-      if (*s_epi_stop) break;
+      if (named_bar_any(1, 128, stop)) break;
       const int item = s_item[ss];
       named_bar_sync(1, 128);
       if (et == 0) mbar_arrive(smem_u32(&sempty[ss]));
@@ -508,13 +509,13 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
           for (int g = ic.t_begin; g < ic.t_end; g += NT) {
             const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
             if (vm == 0) continue;
+            bool stop = false;
             if (et == 0) {
               if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
                 raise_device_error(p.status, s_abort, kStatusTimeout);
-              *s_epi_stop = *s_abort;
+              stop = *s_abort != 0;
             }
-            named_bar_sync(1, 128);
-            if (*s_epi_stop) { aborted = true; break; }
+            if (named_bar_any(1, 128, stop)) { aborted = true; break; }
             tc_fence_after();
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
@@ -575,13 +576,13 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
         const uint32_t vm = tiles_of<NT>(group_slices<NT>(p, ic.b, g, ic.t_end));
         if (vm == 0) continue;
         if (!finisher) {
+          bool stop = false;
           if (et == 0) {
             if (!mbar_wait(smem_u32(&tfull[ab]), aph, tmo, s_abort))
               raise_device_error(p.status, s_abort, kStatusTimeout);
-            *s_epi_stop = *s_abort;
+            stop = *s_abort != 0;
           }
-          named_bar_sync(1, 128);
-          if (*s_epi_stop) { aborted = true; break; }
+          if (named_bar_any(1, 128, stop)) { aborted = true; break; }
           tc_fence_after();
         }
         if constexpr (C::kTC) {
@@ -620,7 +621,9 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             const int q0 = qb * QB;
             const int nqb = min(QB, p.n_queries - q0);
             if (n_qblocks > 1) {
-              named_bar_sync(1, 128);          // the previous block's product has completed
+              // No barrier first: the previous block's product, the last
+              // reader of sBhi / sBlo, completed before the barrier that
+              // preceded its U reads.
               qregs.store(sBhi, sBlo, nqb, et);
               fence_proxy_async_smem();
               // the next block (block 0 of the next tile after the last one)
@@ -632,6 +635,7 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
             // reads are complete before one thread issues the products:
             // U = A_hi B_hi + A_hi B_lo + A_lo B_hi (3xTF32, fp32 accumulation).
             named_bar_sync(1, 128);
+            bool stop = false;
             if (et == 0) {
               tc_fence_after();
               const uint32_t idesc = make_idesc_tf32(kTileTokens, C::kTcN);
@@ -653,11 +657,10 @@ __global__ void __launch_bounds__(192, 1) project_kernel(const ProjParams p) {
               } else {
                 raise_device_error(p.status, s_abort, kStatusTimeout);
               }
-              *s_epi_stop = *s_abort;
+              stop = *s_abort != 0;
             }
-            named_bar_sync(1, 128);
             uph ^= 1;
-            if (*s_epi_stop) { aborted = true; break; }
+            if (named_bar_any(1, 128, stop)) { aborted = true; break; }
             tc_fence_after();
             // s_q = sum_i g~_i U[token, q k_out + i], kLd columns of U (kLd /
             // k_out queries) per TMEM load; columns past the block's queries

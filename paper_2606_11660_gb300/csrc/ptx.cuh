@@ -502,6 +502,23 @@ __device__ __forceinline__ void named_bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Named barrier over `count` threads that also returns, to each of them,
+// whether any participant passed pred = true (bar.red.or): a decision such
+// as "stop" reaches every thread with the barrier itself, with no shared
+// flag that a later writer could change under a slow reader.
+__device__ __forceinline__ bool named_bar_any(int id, int count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
+}
+
 // Programmatic dependent launch.  A grid launched with programmatic stream
 // serialization may start while its predecessor in the stream still runs;
 // griddep_wait() blocks until that predecessor has completed and its memory
