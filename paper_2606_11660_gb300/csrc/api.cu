@@ -477,7 +477,7 @@ CUresult encode_2d(CUtensorMap* tm, CUtensorMapDataType dt, const void* ptr, int
 
 struct ScoreLayout {
   int qt = 1;
-  size_t qh_off = 0, heap_off = 0, total = 0;
+  size_t qh_off = 0, heap_off = 0, pace_off = 0, total = 0;
 };
 
 ScoreLayout plan_score(int64_t K, int64_t Q, int64_t topk) {
@@ -487,10 +487,22 @@ ScoreLayout plan_score(int64_t K, int64_t Q, int64_t topk) {
   L.qt = Q > 2 * kScoreQT ? 2 : 1;
   L.qh_off = 0;
   L.heap_off = round_up(static_cast<size_t>(Q) * K * sizeof(__half), 256);
-  L.total = L.heap_off + round_up(static_cast<size_t>(kMaxScoreCTAs) * topk * L.qt * kScoreQT *
-                                      sizeof(unsigned long long),
+  L.pace_off = L.heap_off + round_up(static_cast<size_t>(kMaxScoreCTAs) * topk * L.qt * kScoreQT *
+                                         sizeof(unsigned long long),
+                                     256);
+  // the pair kernel's pacing words, one per CTA (timing only: never initialised)
+  L.total = L.pace_off + round_up(static_cast<size_t>(kMaxScoreCTAs) * sizeof(unsigned long long),
                                   256);
   return L;
+}
+
+// A tag per pair-kernel launch for its pacing words (never 0), so that words
+// left by an earlier launch on the same workspace are told apart.
+unsigned int next_pace_tag() {
+  static std::atomic<unsigned int> counter{0};
+  unsigned int t = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+  if (t == 0) t = counter.fetch_add(1, std::memory_order_relaxed) + 1;
+  return t;
 }
 
 // One score-kernel launch and the merge that follows it.
@@ -1091,6 +1103,8 @@ static int run_score(const void* store, int64_t N, int64_t K, int64_t ld_store,
     p.tau0_negate = update && least ? 1 : 0;
     p.status = status;
     p.timeout_ns = kWaitTimeoutNs;
+    p.pace = pair ? reinterpret_cast<unsigned long long*>(ws + L.pace_off) : nullptr;
+    p.pace_tag = pair ? next_pace_tag() : 0;
     e = pair ? launch_score_pair(L.qt, tm_store, tm_q, p, l.grid, s)
              : launch_score(L.qt, tm_store, tm_q, p, l.grid, s);
     if (e != cudaSuccess) return fail_cuda(e, "score kernel launch");

@@ -158,6 +158,9 @@ struct ScoreParams {
   const float* tau0;    // per query starting threshold at tau0[q * topk + topk - 1], or nullptr
   int tau0_negate;      // 1: the threshold is -tau0[...] (tau0 holds scores against q while
                         //    the search runs on -q: a bottom-k state)
+  unsigned long long* pace;   // pair kernel, two or more pair groups: [grid] progress words
+                              //   (launch tag << 32 | chunks issued), or nullptr
+  unsigned int pace_tag;      // this launch's tag (never 0; differs between launches)
   int* status;
   uint64_t timeout_ns;
 };

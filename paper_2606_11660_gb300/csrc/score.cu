@@ -36,10 +36,10 @@ constexpr unsigned long long kSentinelKey = 0x007FFFFF00000000ull;   // (-inf, r
 // L2 policy of store-chunk loads: 0 = evict_normal, 1 = evict_first.  The
 // pair kernel with more than one pair of query groups (n_qg counts the
 // CTAs' groups, two per pair) keeps the normal policy: every store half is
-// read once per pair, by CTAs that stream the same tiles in the same order,
-// and the later reads hit L2 more often when the first one does not mark the
-// lines for early eviction (DRAM reads 1.21x the store instead of 1.6x at
-// 1024 queries, same time: that pass is tensor-bound).
+// read once per pair group, by CTAs that stream the same tiles in the same
+// order (paced, below), and the later reads hit L2 more often when the first
+// one does not mark the lines for early eviction (1.6x the store in DRAM
+// reads with evict_first at 1024 queries).
 constexpr int kStoreEvictFirst = 1;
 
 // Candidates a lane may park in shared memory per tile before inserting them
@@ -380,6 +380,25 @@ __global__ void __launch_bounds__(ScoreCfg<QT>::kThreads, 1)
 constexpr int kPairStoreRows = kScoreBN / 2;               // store rows each CTA loads
 constexpr int kPairStoreBoxBytes = kPairStoreRows * 128;   // 128 rows x 64 fp16
 
+// Pacing of the pair groups that read the same store tiles (two or more pair
+// groups: more than 512 queries).  Each store half is read once per pair
+// group; the second read finds it in L2 only while the groups stay close
+// (left alone they drift apart over a pass, and their re-reads then miss).
+// Each producer publishes its count of issued store chunks every kPaceEvery
+// chunks, tagged with the launch, and before running more than kPaceLead
+// chunks ahead of the next pair group's CTA (same tile sequence, same rank;
+// the groups form a ring) waits for it, at most kPaceWaitNs per wait; a peer
+// that does not catch up in that time ends the pacing for this CTA.  The
+// peer's word is read one check ahead, so a producer that is not ahead does
+// not wait out the load.  A waiting CTA has published its own count, so no
+// ring of CTAs can all wait on one another.  Only timing depends on the
+// words: a stale or foreign word just means a wait that runs out.
+// Measured at 1024 queries (3.2 GB store): DRAM reads 1.08x the store at a
+// lead of 16 (1.07x at 8, but 30% slower; 1.13-1.33x at 32 or unpaced).
+constexpr uint32_t kPaceEvery = 8;
+constexpr uint32_t kPaceLead = 16;                    // an eighth of a 8192-column tile
+constexpr uint64_t kPaceWaitNs = 100000ull;
+
 template <int QT_>
 struct PairCfg {
   static constexpr int QT = QT_;
@@ -467,8 +486,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<QT>::kThread
       uint32_t ph = 0;
       uint32_t issued = 0, issued_par = 0;
       bool ok = true;
+      // pacing against the next pair group's CTA on the same tiles (see kPaceLead)
+      bool pacing = p.pace != nullptr && p.n_qg >= 4;
+      unsigned long long* pace_mine = nullptr;
+      const unsigned long long* pace_peer = nullptr;
+      if (pacing) {
+        const int n_pg = p.n_qg >> 1;
+        const int pg = g_local >> 1;
+        pace_mine = p.pace + blockIdx.x;
+        pace_peer = p.pace + nt0 * p.n_qg + ((pg + 1) % n_pg) * 2 + (g_local & 1);
+      }
+      const unsigned long long tag = static_cast<unsigned long long>(p.pace_tag) << 32;
+      uint32_t n_chunks = 0;
+      unsigned long long peer_next = 0;   // peer word read at the previous check
       for (int nt = nt0; nt < p.n_ntiles && ok; nt += cpg) {
-        for (int kc = 0; kc < nK; ++kc) {
+        for (int kc = 0; kc < nK; ++kc, ++n_chunks) {
+          if (pacing && n_chunks % kPaceEvery == 0) {
+            st_relaxed_u64(pace_mine, tag | n_chunks);
+            if (n_chunks >= kPaceLead) {
+              unsigned long long v = peer_next;
+              const uint64_t t0 = global_timer_ns();
+              while (!((v >> 32) == p.pace_tag && static_cast<uint32_t>(v) + kPaceLead >= n_chunks)) {
+                if (*s_abort || global_timer_ns() - t0 > kPaceWaitNs) {
+                  pacing = false;
+                  break;
+                }
+                v = ld_relaxed_u64(pace_peer);
+              }
+            }
+            peer_next = ld_relaxed_u64(pace_peer);
+          }
           if (!mbar_wait(smem_u32(&empty[stage]), ph ^ 1, tmo, s_abort)) { ok = false; break; }
           const uint32_t fb_local = smem_u32(&full[stage]);
           const uint32_t fb = mapa_shared(fb_local, 0);
@@ -485,6 +532,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<QT>::kThread
           if (++stage == C::kStages) { stage = 0; ph ^= 1; }
         }
       }
+      if (pacing) st_relaxed_u64(pace_mine, tag | n_chunks);   // releases a peer near the end
       if (!ok) {
         raise_device_error(p.status, s_abort, kStatusTimeout);
         if (rank == 0) {

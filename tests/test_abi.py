@@ -358,7 +358,8 @@ def check_score_plan(N, Q, topk, ctas):
     n = ctypes.c_size_t()
     assert bg.lib().bergson_score_topk_workspace(N, K, Q, topk, ctypes.byref(n)) == bg.BERGSON_OK
     heaps = max(l["grid"] for l in plan) * topk * gsize * 8
-    assert n.value >= heaps + Q * K * 2
+    pace_words = max(l["grid"] for l in plan) * 8          # the pair kernel's pacing words
+    assert n.value >= heaps + Q * K * 2 + pace_words
 
 
 def test_score_planner_edges():
