@@ -49,6 +49,7 @@ def _query(store, queries, k, entry=None):
     (5_020, 520, 600, 1),        # K % 64 != 0, ragged query groups
     (7_000 + 200, 256, 1024, 100),   # last tile 200 rows: the odd CTA's half partly valid
     (300, 64, 511, 300),         # topk = N
+    (20_000, 1024, 1300, 10),    # three pair groups: a ring of three paced producers
 ])
 def test_pair_scorer_random(N, K, Q, topk):
     g = wl.generator(N + 7 * Q + K, "cpu")
