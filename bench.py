@@ -777,13 +777,16 @@ def score_sweep(args, store, N, K, topk, dev, peaks):
         if bg.bergson_sync_status(stream) != bg.BERGSON_OK:
             raise RuntimeError(bg.bergson_last_error())
         ms = ev[0].elapsed_time(ev[1]) / 3
+        # which kernel the library chose for this query count (its own planner)
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        plan = bg.bergson_debug_score_plan(N, K, Q, topk, sms)
         t_hbm = N * K * 2 / (peaks["hbm_gbs"] * 1e9) * 1e3
         t_tc = 2.0 * N * K * Q / (peaks["bf16_tflops"] * 1e12) * 1e3
         out.append({"queries": Q, "ms_per_pass": round(ms, 3), "rows_per_s": round(N / (ms * 1e-3)),
                     "bound": "hbm" if t_hbm >= t_tc else "tensor",
                     "floor_ms": round(max(t_hbm, t_tc), 3),
                     "frac": round(max(t_hbm, t_tc) / ms, 4),
-                    "kernel": "score_pair_kernel" if Q >= 257 else "score_kernel"})
+                    "kernel": "score_pair_kernel" if plan and plan[-1]["pair"] else "score_kernel"})
         del queries, ws, s, i
     return out
 
