@@ -362,6 +362,34 @@ def check_score_plan(N, Q, topk, ctas):
     assert n.value >= heaps + Q * K * 2 + pace_words
 
 
+@pytest.mark.parametrize("N,Q", [(20_000, 600), (4_000_000, 1024), (20_000, 1300), (500_000, 4096),
+                                 (3_000, 2000), (10_000_000, 40_000)])
+def test_pair_pacing_peers_stay_in_the_grid(N, Q):
+    # The pair scorer paces each CTA against the same-rank CTA of the next pair
+    # group on the same store tiles: blockIdx = nt0 * n_qg + g_local, g_local =
+    # 2 * pair group + rank.  For every planned launch that peer must be another
+    # CTA of the grid with the same tile sequence and rank, and the workspace
+    # must hold a pacing word per CTA.
+    K, topk = 256, 10
+    plan = bg.bergson_debug_score_plan(N, K, Q, topk, 152)
+    n = ctypes.c_size_t()
+    assert bg.lib().bergson_score_topk_workspace(N, K, Q, topk, ctypes.byref(n)) == bg.BERGSON_OK
+    for l in plan:
+        assert l["pair"] == 1 and l["n_qg"] % 2 == 0 and l["grid"] == l["n_qg"] * l["cpg"]
+        assert l["grid"] <= 160                       # pacing words in the workspace
+        if l["n_qg"] < 4:
+            continue                                  # one pair group: no pacing
+        n_pg = l["n_qg"] // 2
+        peers = set()
+        for b in range(l["grid"]):
+            g_local, nt0 = b % l["n_qg"], b // l["n_qg"]
+            peer = nt0 * l["n_qg"] + ((g_local // 2 + 1) % n_pg) * 2 + (g_local & 1)
+            assert 0 <= peer < l["grid"] and peer != b
+            assert peer // l["n_qg"] == nt0 and (peer % l["n_qg"]) % 2 == g_local % 2
+            peers.add(peer)
+        assert len(peers) == l["grid"]               # a ring: every CTA is someone's peer
+
+
 def test_score_planner_edges():
     # a single resident CTA cannot host a two-CTA cluster: no launches (the
     # scoring call reports it as an error)
